@@ -1,0 +1,74 @@
+"""Dense, non-paged NumPy brute force of Keyless Attention decode (tiny inputs only).
+
+TEST INFRASTRUCTURE, like the rest of ``oracle/``. It shares no code with the C oracle: it
+un-pages the cache with its own indexing, then evaluates, per query head h of value group g,
+
+    q_r = q_h W^R                         (Eq. 2 / Eq. 4, Section 2.2)
+    s   = scale * V_g q_r                 (scores against the cached value rows, Section 3)
+    a   = softmax(s)                      (alpha_{n+1,i}, Section 3)
+    o   = a V_g                           (O_{n+1} = sum_i alpha_{n+1,i} v_i, Section 3)
+
+with NumPy matrix products in fp64.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+
+def bf16_bits_to_f64(bits: np.ndarray) -> np.ndarray:
+    """Exact widening of bf16 bit patterns (uint16) to float64."""
+    bits = np.asarray(bits, dtype=np.uint16)
+    return (bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def unpage(v_cache_bits: np.ndarray, block_table: np.ndarray, seq_lens: np.ndarray):
+    """List over sequences of dense [Hkv, L_b, D] fp64 arrays gathered from the paged cache."""
+    cache = bf16_bits_to_f64(v_cache_bits)          # [num_pages, Hkv, P, D]
+    P = cache.shape[2]
+    seqs = []
+    for b, L in enumerate(np.asarray(seq_lens)):
+        t = np.arange(int(L))
+        pages = np.asarray(block_table)[b, t // P]
+        rows = cache[pages, :, t % P, :]            # [L, Hkv, D]
+        seqs.append(np.transpose(rows, (1, 0, 2)))  # [Hkv, L, D]
+    return seqs
+
+
+def keyless_decode(q_bits, w_r_bits, v_seqs, *, scale: float, wr_per_query_head: bool = False):
+    """Keyless decode over dense value sequences; returns [B, Hq, D] fp64."""
+    q = bf16_bits_to_f64(q_bits)
+    w = bf16_bits_to_f64(w_r_bits)
+    B, Hq, D = q.shape
+    Hkv = v_seqs[0].shape[0] if v_seqs else 1
+    G = Hq // Hkv
+    out = np.zeros((B, Hq, D))
+    for b in range(B):
+        for h in range(Hq):
+            V = v_seqs[b][h // G]                    # [L, D]
+            if V.shape[0] == 0:
+                continue
+            qr = q[b, h] @ w[h if wr_per_query_head else h // G]
+            s = scale * (V @ qr)
+            a = np.exp(s - s.max())
+            a /= a.sum()
+            out[b, h] = a @ V
+    return out
+
+
+def standard_decode(q_bits, k_seqs, v_seqs, *, scale: float):
+    """softmax(q K^T * scale) V over dense K and V sequences (Eq. 1); [B, Hq, D] fp64."""
+    q = bf16_bits_to_f64(q_bits)
+    B, Hq, D = q.shape
+    Hkv = v_seqs[0].shape[0] if v_seqs else 1
+    G = Hq // Hkv
+    out = np.zeros((B, Hq, D))
+    for b in range(B):
+        for h in range(Hq):
+            K, V = k_seqs[b][h // G], v_seqs[b][h // G]
+            if V.shape[0] == 0:
+                continue
+            s = scale * (K @ q[b, h])
+            a = np.exp(s - s.max())
+            a /= a.sum()
+            out[b, h] = a @ V
+    return out

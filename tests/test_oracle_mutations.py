@@ -1,0 +1,81 @@
+"""The oracle's pins are strong enough to catch plausible mistakes (CPU only).
+
+Each case plants one mistake in a private copy of the C oracle (a transposed operand, a
+dropped term, a wrong index, a wrong sign ...), builds it in a temporary directory, and
+checks that at least one pin from ``test_oracle.py``'s families fails against it. The
+committed oracle is never modified.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+
+import numpy as np
+import pytest
+
+import oracle
+from oracle import dense
+from tests import test_oracle as pins
+from tests._inputs import bits, default_scale, tiny
+
+SRC = os.path.join(os.path.dirname(oracle.__file__), "keyless_oracle.c")
+
+MUTATIONS = {
+    "transposed_wr": ("W[(size_t)k * D + j]", "W[(size_t)j * D + k]"),
+    "dropped_first_term": ("for (int k = 0; k < D; ++k) {\n        double qk",
+                           "for (int k = 1; k < D; ++k) {\n        double qk"),
+    "wrong_group_map": ("        int g = h / G;\n        double *qv",
+                        "        int g = h % Hkv;\n        double *qv"),
+    "row_off_by_one": ("(size_t)(t % P)) * D;", "(size_t)((t + 1) % P)) * D;"),
+    "missing_scale": ("s[t - t0] = scale * dot;", "s[t - t0] = dot;"),
+    "flipped_exponent": ("double e = exp(s[t - t0] - m);", "double e = exp(m - s[t - t0]);"),
+    "combine_drops_l": ("double w = ml[2 * s + 1] * exp(ml[2 * s] - M);",
+                        "double w = exp(ml[2 * s] - M);"),
+}
+
+
+def _pin_results():
+    """Run a cross-section of the pins; return {name: passed}."""
+    res = {}
+
+    def run(name, fn, *a):
+        try:
+            fn(*a)
+            res[name] = True
+        except (AssertionError, ValueError):
+            res[name] = False
+
+    run("dense_gqa", pins.test_paged_oracle_equals_dense_bruteforce,
+        dict(B=3, Hq=8, Hkv=2, D=64, P=16, lens=(1, 37, 100)))
+    run("theorem1", pins.test_theorem1_keyless_equals_standard_attention_with_k_equal_v_wr_transposed)
+    run("group_map", pins.test_group_mapping_reads_value_head_h_over_g)
+    run("dominant", pins.test_dominant_score_selects_that_row)
+    run("split_merge", pins.test_split_merge_identity, 33)
+    run("route", pins.test_route_matches_row_times_matrix)
+    return res
+
+
+@pytest.mark.parametrize("name", sorted(MUTATIONS))
+def test_planted_mistake_is_caught(name, tmp_path, monkeypatch):
+    before, after = MUTATIONS[name]
+    src = open(SRC).read()
+    assert src.count(before) == 1, f"mutation anchor for {name} not unique"
+    mutated = tmp_path / "mutated.c"
+    mutated.write_text(src.replace(before, after))
+    so = tmp_path / f"libmut_{name}.so"
+    subprocess.run(["gcc", "-O1", "-fPIC", "-shared", "-std=c11", str(mutated), "-o", str(so),
+                    "-lm"], check=True, capture_output=True)
+    lib = ctypes.CDLL(str(so))
+    real = oracle._load()
+    for f in ("ko_route", "ko_decode", "ko_standard_decode", "ko_attention_weights",
+              "ko_decode_partial", "ko_combine", "ko_append"):
+        getattr(lib, f).argtypes = getattr(real, f).argtypes
+        getattr(lib, f).restype = ctypes.c_int
+    monkeypatch.setattr(oracle, "_lib", lib)
+    res = _pin_results()
+    assert not all(res.values()), f"mutation {name} survived every pin: {res}"
+
+
+def test_unmutated_oracle_passes_the_same_pins():
+    assert all(_pin_results().values())
