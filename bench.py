@@ -1,0 +1,438 @@
+"""Benchmark of one keyless decode step (append + decode attention) on GB300.
+
+A step is one pass of the whole hot path over one batch: kl_append_v writes the current
+token's value rows into the paged Value-Only Cache, then kl_decode_attention runs the routed
+decode (fused routing prologue, split-sequence decode, cross-split combine). Inputs are
+seeded synthetic tensors with the shapes of the selected workload, resident in HBM before the
+timed region; L2 is flushed (a 512 MiB write) between timed steps.
+
+Prints ONE JSON line (rank 0). `--impl reference` times the fp64 CPU oracle instead (the
+reference arm: a slow CPU program, timed on a bounded sample of the same workload).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+DEFAULT_WORKLOAD = "small_gqa"   # batch 8, 32/8 heads, D 128, 4096 tokens, P 16
+METRIC = "decode attention tokens/s and achieved HBM GB/s (% of 8 TB/s) on 1 GB300"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=50)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    p.add_argument("--kernel", default="auto", choices=["auto", "tensor", "simt"])
+    p.add_argument("--num-splits", type=int, default=-1, help="-1: the workload's setting")
+    p.add_argument("--standard", action="store_true",
+                   help="time the same-design K+V decode (comparison) instead of keyless")
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=10.0)
+    return p.parse_args()
+
+
+# ------------------------------------------------------------------------------ helpers --
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_digest() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2606_21848_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith((".cu", ".cuh")):
+            with open(os.path.join(csrc, name), "rb") as f:
+                h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(workload: str, kernel: str):
+    """DRAM bytes per launch from the committed ncu summary, if taken on the current source."""
+    path = os.path.join(ROOT, "profiles", "dram_traffic.md")
+    if not os.path.exists(path):
+        return None
+    digest = kernel_source_digest()
+    for line in open(path):
+        m = re.match(r"\|\s*(\S+)\s*\|\s*(\S+)\s*\|\s*([0-9]+)\s*\|\s*([0-9a-f]+)\s*\|", line)
+        if m and m.group(1) == workload and m.group(2) == kernel and m.group(4) == digest:
+            return int(m.group(3))
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason sampling while the timed region runs."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.idx = device_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100", "-i", str(self.idx)], stdout=subprocess.PIPE,
+                stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        self.lines = []
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+                out = ""
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        if not getattr(self, "lines", None):
+            return None
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for l in self.lines:
+            f = [x.strip() for x in l.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = max(mx, float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() in ("active", "1"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def algorithmic_bytes(x, standard: bool) -> dict:
+    """Bytes the decode must move once: cached rows (V, plus K for the comparison), W^R,
+    q, out (fp32 read by nobody: bf16 written), block table and lengths."""
+    wl = x["workload"]
+    B, Hq, D = x["q"].shape
+    Hkv = x["v_cache"].shape[1]
+    P = x["v_cache"].shape[2]
+    tokens = int(x["seq_lens"].sum())
+    v = tokens * Hkv * D * 2
+    cache = 2 * v if standard else v
+    wr = 0 if standard else x["w_r"].numel() * 2
+    q = B * Hq * D * 2
+    out = B * Hq * D * 2
+    bt = sum(math.ceil(int(L) / P) for L in x["seq_lens"].tolist()) * 4 + B * 4
+    return {"cache": cache, "wr": wr, "total": cache + wr + q + out + bt, "tokens": tokens}
+
+
+# ----------------------------------------------------------------------------- CPU arm --
+
+def cpu_oracle_rate(x, seconds: float, standard: bool):
+    """Time the fp64 oracle (as it stands) on whole sequences until `seconds` pass."""
+    import numpy as np
+
+    import oracle
+    from paper_2606_21848_gb300.workloads import bf16_bits
+
+    q, w, v = bf16_bits(x["q"]), bf16_bits(x["w_r"]), bf16_bits(x["v_cache"])
+    bt, sl = x["block_table"].numpy(), x["seq_lens"].numpy()
+    B, Hq, D = x["q"].shape
+    scale = 1.0 / math.sqrt(D)
+    oracle.build()
+    seqs = 0
+    t0 = time.perf_counter()
+    b = 0
+    while True:
+        heads = np.array([(b, h) for h in range(Hq)], np.int32)
+        if standard:
+            oracle.standard_decode(q, v, v, bt, sl, scale=scale, heads=heads)
+        else:
+            oracle.decode(q, w, v, bt, sl, scale=scale, heads=heads)
+        seqs += 1
+        b = (b + 1) % B
+        el = time.perf_counter() - t0
+        if el >= seconds:
+            break
+    return seqs / el, seqs, el
+
+
+def run_reference(args):
+    rank, world, local = dist_env()
+    if rank != 0:
+        return 0
+    from paper_2606_21848_gb300.workloads import WORKLOADS, generate
+
+    import oracle
+    wl = WORKLOADS[args.workload]
+    x = generate(wl)
+    per_step = max(1.0, args.cpu_seconds / max(1, args.steps))
+    rates = []
+    total_seqs = 0
+    for i in range(args.warmup + args.steps):
+        r, n, _ = cpu_oracle_rate(x, per_step if i >= args.warmup else 0.0, args.standard)
+        if i >= args.warmup:
+            rates.append(r)
+            total_seqs += n
+    value = statistics.mean(rates)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1000.0 * wl.num_seqs / value, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": wl.name, "num_seqs": wl.num_seqs, "q_heads": wl.num_q_heads,
+                   "kv_heads": wl.num_kv_heads, "head_dim": wl.head_dim,
+                   "page_size": wl.page_size, "seq_len": wl.seq_len or list(wl.seq_len_range)},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": oracle.threads(),
+                         "kind": "oracle",
+                         "sample": f"{total_seqs} whole sequences (all heads, decode only) "
+                                   f"of {wl.name}, ~{per_step:.1f}s per step"},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ----------------------------------------------------------------------------- GPU arm --
+
+def run_ours(args):
+    import torch
+
+    import paper_2606_21848_gb300 as kl
+    from paper_2606_21848_gb300.workloads import WORKLOADS, generate
+
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group("nccl", rank=rank, world_size=world)
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    kl.load()
+
+    wl = WORKLOADS[args.workload]
+    x = generate(wl, seed=wl.seed + rank)           # replicas: each rank its own batch
+    B, Hq, D = x["q"].shape
+    num_pages, Hkv, P, _ = x["v_cache"].shape
+    max_pages = x["block_table"].shape[1]
+    sh = kl.make_shape(B, Hq, Hkv, D, P, num_pages, max_pages, wl.wr_per_query_head)
+    kernel = {"auto": kl.KL_KERNEL_AUTO, "tensor": kl.KL_KERNEL_TENSOR,
+              "simt": kl.KL_KERNEL_SIMT}[args.kernel]
+    splits_req = wl.num_splits if args.num_splits < 0 else args.num_splits
+    S = kl.kl_decode_num_splits(sh, splits_req)
+
+    g = {k: x[k].to(dev) for k in ("q", "w_r", "v_cache", "block_table", "seq_lens",
+                                    "positions", "v_new")}
+    k_cache = None
+    if args.standard:
+        # K = V (W^R)^T per value head, so the comparison computes the same attention.
+        k_cache = torch.empty_like(g["v_cache"])
+        for h in range(Hkv):
+            w = g["w_r"][h].float()
+            k_cache[:, h] = (g["v_cache"][:, h].float() @ w.t()).to(torch.bfloat16)
+    out = torch.empty(B, Hq, D, dtype=torch.bfloat16, device=dev)
+    part_o = torch.empty(B, Hq, S, D, dtype=torch.float32, device=dev)
+    part_ml = torch.empty(B, Hq, S, 2, dtype=torch.float32, device=dev)
+    ws = torch.empty(max(256, kl.kl_decode_workspace_size(sh, splits_req)), dtype=torch.uint8,
+                     device=dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    opts_states = kl.decode_options(S, kernel, part_o, part_ml)
+    opts_full = kl.decode_options(splits_req, kernel)
+
+    def decode_states():
+        if args.standard:
+            kl.kl_standard_decode(sh, g["q"], k_cache, g["v_cache"], g["block_table"],
+                                  g["seq_lens"], opts_states, None, kl.KL_BF16, None, err, stream)
+        else:
+            kl.kl_decode_attention_ex(sh, g["q"], g["w_r"], g["v_cache"], g["block_table"],
+                                      g["seq_lens"], opts_states, None, kl.KL_BF16, None, err,
+                                      stream)
+
+    def step_timed(ev):
+        # append | decode kernel | combine, each bracketed by events on the launching stream
+        ev[0].record(stream)
+        kl.kl_append_v(sh, g["v_new"], g["block_table"], g["positions"], g["v_cache"], err,
+                       stream)
+        ev[1].record(stream)
+        decode_states()
+        ev[2].record(stream)
+        kl.kl_combine(sh, part_o, part_ml, S, out, kl.KL_BF16, stream)
+        ev[3].record(stream)
+
+    launches_per_step = 3
+    E = lambda: torch.cuda.Event(enable_timing=True)
+    for _ in range(args.warmup):
+        flush.zero_()
+        step_timed([E() for _ in range(4)])
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0, f"device error flags {int(err.item())}"
+
+    evs = [[E() for _ in range(4)] for _ in range(args.steps)]
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        for i in range(args.steps):
+            flush.zero_()
+            step_timed(evs[i])
+        torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    step_ms = [e[0].elapsed_time(e[3]) for e in evs]
+    dec_ms = [e[1].elapsed_time(e[2]) for e in evs]
+    app_ms = [e[0].elapsed_time(e[1]) for e in evs]
+    comb_ms = [e[2].elapsed_time(e[3]) for e in evs]
+    mean_step = statistics.mean(step_ms)
+    mean_dec = statistics.mean(dec_ms)
+    if world > 1:
+        t = torch.tensor([mean_step, mean_dec], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        mean_step, mean_dec = float(t[0]), float(t[1])
+    assert int(err.item()) == 0, f"device error flags {int(err.item())}"
+
+    ab = algorithmic_bytes(x, args.standard)
+    value = B * world / (mean_step / 1e3)
+    peak, peak_kind = measured_peaks()
+    dec_gbs = ab["total"] / (mean_dec / 1e3) / 1e9
+    step_gbs = ab["total"] / (mean_step / 1e3) / 1e9
+
+    # ---- end to end through the public API with host buffers ----
+    e2e = None
+    if not args.no_e2e:
+        pin = lambda t: t.pin_memory()
+        h_in = {k: pin(x[k]) for k in ("q", "v_new", "positions", "seq_lens", "block_table")}
+        h_out = torch.empty(B, Hq, D, dtype=torch.bfloat16).pin_memory()
+        d_in = {k: torch.empty_like(g[k]) for k in h_in}
+        h2d = sum(t.numel() * t.element_size() for t in h_in.values())
+        d2h = h_out.numel() * h_out.element_size()
+
+        def e2e_step():
+            for k in h_in:
+                d_in[k].copy_(h_in[k], non_blocking=True)
+            kl.kl_append_v(sh, d_in["v_new"], d_in["block_table"], d_in["positions"],
+                           g["v_cache"], err, stream)
+            if args.standard:
+                kl.kl_standard_decode(sh, d_in["q"], k_cache, g["v_cache"], d_in["block_table"],
+                                      d_in["seq_lens"], opts_full, out, kl.KL_BF16, ws, err,
+                                      stream)
+            else:
+                kl.kl_decode_attention(sh, d_in["q"], g["w_r"], g["v_cache"], d_in["block_table"],
+                                       d_in["seq_lens"], splits_req, out, kl.KL_BF16, ws, err,
+                                       stream)
+            h_out.copy_(out, non_blocking=True)
+
+        for _ in range(args.warmup):
+            flush.zero_()
+            e2e_step()
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(args.steps):
+            flush.zero_()
+            a, b = E(), E()
+            a.record(stream)
+            e2e_step()
+            b.record(stream)
+            ts.append((a, b))
+        torch.cuda.synchronize()
+        e2e_ms = statistics.mean(a.elapsed_time(b) for a, b in ts)
+        if world > 1:
+            t = torch.tensor([e2e_ms], device=dev)
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+            e2e_ms = float(t[0])
+        e2e = {"value": B * world / (e2e_ms / 1e3), "unit": "tokens/s",
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms}
+
+    if rank != 0:
+        return 0
+
+    cpu = None
+    if world == 1:
+        rate, n, el = cpu_oracle_rate(x, args.cpu_seconds, args.standard)
+        import oracle
+        cpu = {"value": rate, "unit": "tokens/s", "cores": oracle.threads(), "kind": "oracle",
+               "sample": f"{n} whole sequences of {wl.name} (all {Hq} heads, decode only, "
+                         f"fp64) in {el:.1f}s"}
+
+    kname = "tensor" if kernel == kl.KL_KERNEL_TENSOR or (
+        kernel == kl.KL_KERNEL_AUTO and kl.kl_decode_kernel_available(sh, kl.KL_KERNEL_TENSOR,
+                                                                       args.standard)) else "simt"
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": mean_step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded; inputs resident in HBM)",
+        "config": {"workload": wl.name, "num_seqs": B, "q_heads": Hq, "kv_heads": Hkv,
+                   "head_dim": D, "page_size": P,
+                   "seq_len": wl.seq_len or list(wl.seq_len_range),
+                   "context_tokens": ab["tokens"], "num_splits": S, "kernel": kname,
+                   "decode": "standard K+V (comparison)" if args.standard else "keyless",
+                   "l2": "flushed (512 MiB write) between timed steps",
+                   "parallelism": f"replicas x{world}"},
+        "hbm_gbs_step": step_gbs,
+        "pct_of_8tbs_step": 100.0 * step_gbs / NOMINAL_HBM_GBS,
+        "ms_breakdown": {"append": statistics.mean(app_ms), "decode": mean_dec,
+                         "combine": statistics.mean(comb_ms)},
+        "roofline": {"bound": "hbm", "achieved": dec_gbs, "peak": peak, "unit": "GB/s",
+                     "frac": dec_gbs / peak, "peak_kind": peak_kind,
+                     "pct_of_8tbs": 100.0 * dec_gbs / NOMINAL_HBM_GBS,
+                     "algorithmic_bytes": ab["total"],
+                     "traffic": recorded_traffic(wl.name, kname)},
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clk.summary(),
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,190 @@
+/*
+ * keyless.h -- C ABI of libkeyless: the decode step of Keyless Attention over a paged
+ * Value-Only Cache, as hand-written CUDA for sm_103a (GB300).
+ *
+ * The method ("Keyless Attention: Value-Space Routing and Value-Only Caching for Efficient
+ * Transformers") drops the key projection: a query row is routed into value space by W^R
+ * (Section 2.2, Eq. 4) and scored directly against the cached value rows, and the same rows
+ * form the output (Section 3, decode formula for O_{n+1}):
+ *
+ *     q_r      = q W^R
+ *     alpha_i  = exp(scale * <q_r, v_i>) / sum_i' exp(scale * <q_r, v_i'>),  i = 1 .. n+1
+ *     O_{n+1}  = sum_i alpha_i v_i
+ *
+ * with MHA / MQA / GQA head sharing as in Section 3: query head h reads value head
+ * h / (Hq / Hkv).
+ *
+ * Conventions for every entry point:
+ *   - Pointers are device memory owned by the caller (except `shape` and `opts`, which are
+ *     host structs read during the call). The library never allocates, frees or
+ *     synchronizes; every launch is asynchronous on `stream` (NULL = legacy default stream).
+ *   - bf16 tensors are passed as `const void *` holding IEEE bfloat16 values.
+ *   - The return value reports synchronous host-side validation and launch errors; on any
+ *     error nothing is launched.
+ *   - Data-dependent violations found on the device (a page id outside [0, num_pages), a
+ *     position or length beyond max_pages_per_seq * page_size) skip the offending access
+ *     and OR a KL_FLAG_* bit into the caller's device word `*err` (which may be NULL to
+ *     ignore them). The caller reads `*err` after synchronizing; the kernels never trap.
+ *   - Paging follows PagedAttention: token t of sequence b is row t % P of physical page
+ *     block_table[b * max_pages_per_seq + t / P]; the value cache is laid out as
+ *     [num_pages][Hkv][P][D] bf16, so one (page, head) tile is P * D * 2 contiguous bytes.
+ *     Filling the block table (page allocation) is the caller's job.
+ */
+#ifndef KEYLESS_H
+#define KEYLESS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t. */
+typedef struct CUstream_st *kl_stream_t;
+
+typedef enum kl_status {
+    KL_OK = 0,
+    KL_ERR_INVALID_ARG = 1,  /* null pointer, bad dimension or count */
+    KL_ERR_UNSUPPORTED = 2,  /* valid but not implemented (e.g. head_dim not 64 or 128) */
+    KL_ERR_WORKSPACE = 3,    /* workspace missing or smaller than kl_decode_workspace_size */
+    KL_ERR_CUDA = 4          /* a CUDA runtime call or launch failed */
+} kl_status;
+
+/* Bits OR-ed into the device error word. */
+#define KL_FLAG_BAD_PAGE 0x1     /* block-table entry outside [0, num_pages) */
+#define KL_FLAG_BAD_POSITION 0x2 /* append position outside [0, max_pages_per_seq * P) */
+#define KL_FLAG_BAD_LENGTH 0x4   /* seq_len outside [0, max_pages_per_seq * P] */
+#define KL_FLAG_TIMEOUT 0x8      /* a bounded pipeline wait gave up (output invalid) */
+
+typedef enum kl_dtype { KL_BF16 = 0, KL_FP32 = 1 } kl_dtype;
+
+typedef struct kl_shape {
+    int32_t num_seqs;          /* B */
+    int32_t num_q_heads;       /* Hq */
+    int32_t num_kv_heads;      /* Hkv, the value heads; Hq % Hkv == 0, G = Hq / Hkv */
+    int32_t head_dim;          /* D = d_k; 64 or 128 */
+    int32_t page_size;         /* P tokens per page */
+    int32_t num_pages;         /* pages in the cache pool */
+    int32_t max_pages_per_seq; /* block-table row stride */
+    int32_t wr_per_query_head; /* 0: W^R holds Hkv matrices (index h / G); 1: Hq matrices (index h) */
+    float scale;               /* lambda / sqrt(d_k); <= 0 selects 1 / sqrt(head_dim) (lambda = 1) */
+} kl_shape;
+
+/* Kernel family of the decode. */
+typedef enum kl_kernel {
+    KL_KERNEL_AUTO = 0,   /* tensor-core kernel where supported, else the CUDA-core one */
+    KL_KERNEL_TENSOR = 1, /* tcgen05 + TMA kernel (head_dim 128, group size <= 8) */
+    KL_KERNEL_SIMT = 2    /* CUDA-core kernel (any supported shape) */
+} kl_kernel;
+
+typedef struct kl_decode_options {
+    int32_t num_splits; /* split-sequence count S; 0 = chosen from the shape and the GPU */
+    int32_t kernel;     /* kl_kernel */
+    /* Optional split-state outputs. When both are non-NULL the decode writes every split's
+     * state there -- partial_o [B][Hq][S][D] fp32 (normalized) and partial_ml [B][Hq][S][2]
+     * fp32 ({m, l}, the layout kl_combine reads) -- and neither merges nor writes `out`
+     * (which may be NULL); no workspace is needed. This exposes the states for a later
+     * kl_combine, e.g. after gathering the states of sequence shards from several devices. */
+    float *partial_o;
+    float *partial_ml;
+} kl_decode_options;
+
+/*
+ * Routing projection (Section 2.2, Eq. 4; the composed query of Eq. 2):
+ *   q_r[b][h][j] = sum_k q[b][h][k] * W^R[w(h)][k][j],   fp32 accumulation.
+ * q: [B][Hq][D] bf16. w_r: [Hw][D][D] bf16 row-major (row k = input dimension), Hw = Hkv
+ * (w(h) = h / G) or Hq (w(h) = h) per shape->wr_per_query_head. q_r: [B][Hq][D] fp32 out.
+ */
+kl_status kl_route_query(const kl_shape *shape, const void *q, const void *w_r, float *q_r,
+                         kl_stream_t stream);
+
+/*
+ * Value-Only Cache append (Section 3: the cache holds the value rows of earlier steps and the
+ * row obtained at the current step; no key row is stored):
+ *   v_cache[block_table[b][pos_b / P]][g][pos_b % P][:] = v_new[b][g][:]   for all b, g,
+ * with pos_b = positions[b]. v_new: [B][Hkv][D] bf16; positions: [B] int32; v_cache is
+ * written in place (bit copy). A position outside [0, max_pages_per_seq * P) or a page id
+ * outside the pool skips that sequence and raises KL_FLAG_BAD_POSITION / KL_FLAG_BAD_PAGE.
+ */
+kl_status kl_append_v(const kl_shape *shape, const void *v_new, const int32_t *block_table,
+                      const int32_t *positions, void *v_cache, int32_t *err,
+                      kl_stream_t stream);
+
+/*
+ * Bytes of device workspace kl_decode_attention / kl_standard_decode need for `num_splits`
+ * (0 = the automatic choice); 0 when no workspace is needed. Returns 0 on invalid shapes.
+ */
+size_t kl_decode_workspace_size(const kl_shape *shape, int32_t num_splits);
+
+/* The split count that `num_splits` (0 = automatic) resolves to for this shape. */
+int32_t kl_decode_num_splits(const kl_shape *shape, int32_t num_splits);
+
+/*
+ * Keyless decode attention over the paged Value-Only Cache (Section 3, decode formula for
+ * O_{n+1}; MHA/MQA/GQA head sharing; the routing projection of Section 2.2 is fused into the
+ * kernel's prologue). For every sequence b and query head h:
+ *   q_r = q[b][h] W^R[w(h)],  s_t = scale * <q_r, v_t>,  out[b][h] = sum_t softmax(s)_t v_t,
+ * over the L_b = seq_lens[b] cached rows t = 0 .. L_b - 1 (the current token's row included,
+ * i.e. append first). L_b = 0 writes zeros.
+ * q: [B][Hq][D] bf16; w_r: [Hw][D][D] bf16; v_cache: [num_pages][Hkv][P][D] bf16;
+ * block_table: [B][max_pages_per_seq] int32; seq_lens: [B] int32; out: [B][Hq][D] of
+ * `out_dtype`. The sequence is cut into `num_splits` chunks processed in parallel and merged
+ * as in kl_combine; `workspace` must hold kl_decode_workspace_size(shape, num_splits) bytes
+ * (256-byte aligned). A bad page id or length raises its flag and leaves that output
+ * unspecified.
+ */
+kl_status kl_decode_attention(const kl_shape *shape, const void *q, const void *w_r,
+                              const void *v_cache, const int32_t *block_table,
+                              const int32_t *seq_lens, int32_t num_splits, void *out,
+                              kl_dtype out_dtype, void *workspace, size_t workspace_bytes,
+                              int32_t *err, kl_stream_t stream);
+
+/* kl_decode_attention with an explicit kernel choice (opts may be NULL = defaults). */
+kl_status kl_decode_attention_ex(const kl_shape *shape, const void *q, const void *w_r,
+                                 const void *v_cache, const int32_t *block_table,
+                                 const int32_t *seq_lens, const kl_decode_options *opts,
+                                 void *out, kl_dtype out_dtype, void *workspace,
+                                 size_t workspace_bytes, int32_t *err, kl_stream_t stream);
+
+/*
+ * Merge of split states into one softmax (the decode formula's normalization applied over
+ * the union of the splits). For every (b, h), with split s holding its normalized output
+ * o_s = partial_o[b][h][s][:] and {m_s, l_s} = partial_ml[b][h][s][0..1] (m_s = largest
+ * score of the split, l_s = sum over the split of exp(s_t - m_s); l_s = 0 marks an empty
+ * split):
+ *   M = max_{l_s > 0} m_s,  w_s = l_s exp(m_s - M),  out[b][h] = sum_s w_s o_s / sum_s w_s.
+ * All splits empty writes zeros. partial_o: [B][Hq][S][D] fp32; partial_ml: [B][Hq][S][2]
+ * fp32; out: [B][Hq][D] of out_dtype. Used inside kl_decode_attention and, across devices,
+ * to merge the states of sequence shards.
+ */
+kl_status kl_combine(const kl_shape *shape, const float *partial_o, const float *partial_ml,
+                     int32_t num_splits, void *out, kl_dtype out_dtype, kl_stream_t stream);
+
+/*
+ * Comparison only: standard decode attention softmax(q K^T * scale) V (Eq. 1) over a paged
+ * key cache and a paged value cache of the same layout -- the K+V cache a Value-Only Cache
+ * replaces, read by a kernel of the same design. q is used as given (no routing).
+ * Arguments as in kl_decode_attention_ex with k_cache added.
+ */
+kl_status kl_standard_decode(const kl_shape *shape, const void *q, const void *k_cache,
+                             const void *v_cache, const int32_t *block_table,
+                             const int32_t *seq_lens, const kl_decode_options *opts, void *out,
+                             kl_dtype out_dtype, void *workspace, size_t workspace_bytes,
+                             int32_t *err, kl_stream_t stream);
+
+/*
+ * Whether kernel family `kernel` (kl_kernel) handles this shape: 1 yes, 0 no. For the keyless
+ * decode (standard = 0) or the K+V comparison (standard = 1). A capability query of the
+ * library; the paper has no counterpart.
+ */
+int32_t kl_decode_kernel_available(const kl_shape *shape, int32_t kernel, int32_t standard);
+
+/* Static description of a status code. */
+const char *kl_status_string(kl_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* KEYLESS_H */

@@ -1,0 +1,265 @@
+// C-ABI entry points of libkeyless: host-side validation, split planning, workspace layout
+// and dispatch to the kernels. Nothing here allocates, frees or synchronizes.
+#include <math.h>
+#include <stdint.h>
+
+#include "kl_internal.cuh"
+
+namespace kl {
+
+int device_sm_count() {
+    static int cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+    if (dev >= 0 && dev < 64 && cache[dev] > 0) return cache[dev];
+    int n = 1;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1)
+        n = 1;
+    if (dev >= 0 && dev < 64) cache[dev] = n;
+    return n;
+}
+
+namespace {
+
+constexpr int kChunkQuantum = 128;  // split boundaries fall on multiples of 128 tokens
+constexpr int kMaxSplits = 1024;
+
+bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Validate the shape and resolve the split plan. `num_splits` < 0 skips split planning.
+kl_status resolve(const kl_shape *s, int32_t num_splits, Geometry *g) {
+    if (!s) return KL_ERR_INVALID_ARG;
+    if (s->num_seqs < 0 || s->num_q_heads <= 0 || s->num_kv_heads <= 0 || s->page_size <= 0 ||
+        s->num_pages <= 0 || s->max_pages_per_seq <= 0 || s->head_dim <= 0)
+        return KL_ERR_INVALID_ARG;
+    if (s->num_q_heads % s->num_kv_heads != 0) return KL_ERR_INVALID_ARG;
+    if (s->head_dim != 64 && s->head_dim != 128) return KL_ERR_UNSUPPORTED;
+    if ((int64_t)s->max_pages_per_seq * s->page_size > (int64_t)INT32_MAX / 2)
+        return KL_ERR_INVALID_ARG;
+    if (!(s->scale == s->scale)) return KL_ERR_INVALID_ARG;  // NaN
+    g->B = s->num_seqs;
+    g->Hq = s->num_q_heads;
+    g->Hkv = s->num_kv_heads;
+    g->G = s->num_q_heads / s->num_kv_heads;
+    g->D = s->head_dim;
+    g->P = s->page_size;
+    g->num_pages = s->num_pages;
+    g->max_pages = s->max_pages_per_seq;
+    g->wr_per_qh = s->wr_per_query_head ? 1 : 0;
+    g->scale = s->scale > 0.f ? s->scale : 1.0f / sqrtf((float)s->head_dim);
+    g->S = 1;
+    g->chunk = 0;
+    if (num_splits < 0) return KL_OK;
+    if (num_splits > kMaxSplits) return KL_ERR_INVALID_ARG;
+
+    const int64_t Lmax = (int64_t)g->max_pages * g->P;
+    int64_t S = num_splits;
+    if (S == 0) {
+        // Enough (split, value head, sequence) items to fill every SM about twice, and splits
+        // of at most 4096 tokens so that ragged batches balance; never below 256 tokens.
+        const int64_t units = (int64_t)(g->B > 0 ? g->B : 1) * g->Hkv;
+        const int64_t fill = (2 * (int64_t)device_sm_count() + units - 1) / units;
+        const int64_t cap = (Lmax + 4095) / 4096;
+        S = fill > cap ? fill : cap;
+        const int64_t smax = (Lmax + 255) / 256;
+        if (S > smax) S = smax;
+        if (S > kMaxSplits) S = kMaxSplits;
+        if (S < 1) S = 1;
+    }
+    int64_t chunk = (Lmax + S - 1) / S;
+    chunk = (chunk + kChunkQuantum - 1) / kChunkQuantum * kChunkQuantum;
+    g->chunk = (int)chunk;
+    g->S = (int)((Lmax + chunk - 1) / chunk);
+    if (g->S < 1) g->S = 1;
+    return KL_OK;
+}
+
+struct WorkspaceLayout {
+    size_t part_o, part_ml, total;
+};
+
+WorkspaceLayout layout(const Geometry &g) {
+    WorkspaceLayout w{0, 0, 0};
+    if (g.S <= 1) return w;
+    const size_t rows = (size_t)g.B * g.Hq * g.S;
+    w.part_o = 0;
+    w.part_ml = round_up(rows * g.D * sizeof(float), 256);
+    w.total = w.part_ml + round_up(rows * 2 * sizeof(float), 256);
+    return w;
+}
+
+kl_status from_cuda(cudaError_t e) { return e == cudaSuccess ? KL_OK : KL_ERR_CUDA; }
+
+kl_status decode_common(bool standard, const kl_shape *shape, const void *q, const void *w_r,
+                        const void *k_cache, const void *v_cache, const int32_t *block_table,
+                        const int32_t *seq_lens, const kl_decode_options *opts, void *out,
+                        kl_dtype out_dtype, void *workspace, size_t workspace_bytes,
+                        int32_t *err, kl_stream_t stream) {
+    const int32_t ns = opts ? opts->num_splits : 0;
+    const int32_t kernel = opts ? opts->kernel : KL_KERNEL_AUTO;
+    if (ns < 0 || kernel < KL_KERNEL_AUTO || kernel > KL_KERNEL_SIMT) return KL_ERR_INVALID_ARG;
+    if (out_dtype != KL_BF16 && out_dtype != KL_FP32) return KL_ERR_INVALID_ARG;
+    Geometry g;
+    kl_status st = resolve(shape, ns, &g);
+    if (st != KL_OK) return st;
+    if (g.G > 8) return KL_ERR_UNSUPPORTED;
+    if (g.B == 0) return KL_OK;
+    if (!q || !v_cache || !block_table || !seq_lens) return KL_ERR_INVALID_ARG;
+    if (standard ? !k_cache : !w_r) return KL_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(v_cache, 16) || (w_r && !aligned(w_r, 16)) ||
+        (k_cache && !aligned(k_cache, 16)) || (out && !aligned(out, 16)))
+        return KL_ERR_INVALID_ARG;
+
+    const bool states = opts && opts->partial_o && opts->partial_ml;
+    if (opts && (!opts->partial_o) != (!opts->partial_ml)) return KL_ERR_INVALID_ARG;
+    if (!states && !out) return KL_ERR_INVALID_ARG;
+    if (states && (!aligned(opts->partial_o, 16) || !aligned(opts->partial_ml, 8)))
+        return KL_ERR_INVALID_ARG;
+    const WorkspaceLayout wl = states ? WorkspaceLayout{0, 0, 0} : layout(g);
+    if (wl.total > 0 && (!workspace || workspace_bytes < wl.total || !aligned(workspace, 256)))
+        return KL_ERR_WORKSPACE;
+
+    DecodeArgs a;
+    a.geo = g;
+    a.q = static_cast<const uint16_t *>(q);
+    a.w_r = static_cast<const uint16_t *>(w_r);
+    a.k_cache = static_cast<const uint16_t *>(k_cache);
+    a.v_cache = static_cast<const uint16_t *>(v_cache);
+    a.block_table = block_table;
+    a.seq_lens = seq_lens;
+    char *ws = static_cast<char *>(workspace);
+    a.part_o = states ? opts->partial_o : wl.total ? reinterpret_cast<float *>(ws + wl.part_o) : nullptr;
+    a.part_ml = states ? opts->partial_ml : wl.total ? reinterpret_cast<float *>(ws + wl.part_ml) : nullptr;
+    a.out = out;
+    a.direct_out = !states && g.S == 1;
+    a.out_dtype = out_dtype;
+    a.err = err;
+    a.stream = reinterpret_cast<cudaStream_t>(stream);
+
+    bool use_tc = false;
+    if (kernel == KL_KERNEL_TENSOR) {
+        if (!tc_supported(g, standard)) return KL_ERR_UNSUPPORTED;
+        use_tc = true;
+    } else if (kernel == KL_KERNEL_AUTO) {
+        use_tc = tc_supported(g, standard);
+    }
+    cudaError_t e = use_tc ? launch_decode_tc(a, standard) : launch_decode_simt(a, standard);
+    if (e == cudaSuccess) e = finish_decode(a, states);
+    return from_cuda(e);
+}
+
+}  // namespace
+
+cudaError_t finish_decode(const DecodeArgs &a, bool states_requested) {
+    if (a.direct_out || states_requested) return cudaSuccess;
+    return launch_combine(a.geo.B, a.geo.Hq, a.geo.D, a.geo.S, a.part_o, a.part_ml, a.out,
+                          a.out_dtype, a.stream);
+}
+
+}  // namespace kl
+
+using namespace kl;
+
+extern "C" {
+
+kl_status kl_route_query(const kl_shape *shape, const void *q, const void *w_r, float *q_r,
+                         kl_stream_t stream) {
+    Geometry g;
+    kl_status st = resolve(shape, -1, &g);
+    if (st != KL_OK) return st;
+    if (g.B == 0) return KL_OK;
+    if (!q || !w_r || !q_r) return KL_ERR_INVALID_ARG;
+    return from_cuda(launch_route(g, static_cast<const uint16_t *>(q),
+                                  static_cast<const uint16_t *>(w_r), q_r,
+                                  reinterpret_cast<cudaStream_t>(stream)));
+}
+
+kl_status kl_append_v(const kl_shape *shape, const void *v_new, const int32_t *block_table,
+                      const int32_t *positions, void *v_cache, int32_t *err, kl_stream_t stream) {
+    Geometry g;
+    kl_status st = resolve(shape, -1, &g);
+    if (st != KL_OK) return st;
+    if (g.B == 0) return KL_OK;
+    if (!v_new || !block_table || !positions || !v_cache) return KL_ERR_INVALID_ARG;
+    if (!aligned(v_new, 16) || !aligned(v_cache, 16)) return KL_ERR_INVALID_ARG;
+    return from_cuda(launch_append(g, static_cast<const uint16_t *>(v_new), block_table,
+                                   positions, static_cast<uint16_t *>(v_cache), err,
+                                   reinterpret_cast<cudaStream_t>(stream)));
+}
+
+size_t kl_decode_workspace_size(const kl_shape *shape, int32_t num_splits) {
+    Geometry g;
+    if (num_splits < 0 || resolve(shape, num_splits, &g) != KL_OK) return 0;
+    return layout(g).total;
+}
+
+int32_t kl_decode_num_splits(const kl_shape *shape, int32_t num_splits) {
+    Geometry g;
+    if (num_splits < 0 || resolve(shape, num_splits, &g) != KL_OK) return 0;
+    return g.S;
+}
+
+kl_status kl_decode_attention(const kl_shape *shape, const void *q, const void *w_r,
+                              const void *v_cache, const int32_t *block_table,
+                              const int32_t *seq_lens, int32_t num_splits, void *out,
+                              kl_dtype out_dtype, void *workspace, size_t workspace_bytes,
+                              int32_t *err, kl_stream_t stream) {
+    kl_decode_options o{num_splits, KL_KERNEL_AUTO, nullptr, nullptr};
+    return decode_common(false, shape, q, w_r, nullptr, v_cache, block_table, seq_lens, &o, out,
+                         out_dtype, workspace, workspace_bytes, err, stream);
+}
+
+kl_status kl_decode_attention_ex(const kl_shape *shape, const void *q, const void *w_r,
+                                 const void *v_cache, const int32_t *block_table,
+                                 const int32_t *seq_lens, const kl_decode_options *opts,
+                                 void *out, kl_dtype out_dtype, void *workspace,
+                                 size_t workspace_bytes, int32_t *err, kl_stream_t stream) {
+    return decode_common(false, shape, q, w_r, nullptr, v_cache, block_table, seq_lens, opts,
+                         out, out_dtype, workspace, workspace_bytes, err, stream);
+}
+
+kl_status kl_standard_decode(const kl_shape *shape, const void *q, const void *k_cache,
+                             const void *v_cache, const int32_t *block_table,
+                             const int32_t *seq_lens, const kl_decode_options *opts, void *out,
+                             kl_dtype out_dtype, void *workspace, size_t workspace_bytes,
+                             int32_t *err, kl_stream_t stream) {
+    return decode_common(true, shape, q, nullptr, k_cache, v_cache, block_table, seq_lens, opts,
+                         out, out_dtype, workspace, workspace_bytes, err, stream);
+}
+
+kl_status kl_combine(const kl_shape *shape, const float *partial_o, const float *partial_ml,
+                     int32_t num_splits, void *out, kl_dtype out_dtype, kl_stream_t stream) {
+    Geometry g;
+    kl_status st = resolve(shape, -1, &g);
+    if (st != KL_OK) return st;
+    if (num_splits <= 0 || num_splits > kMaxSplits) return KL_ERR_INVALID_ARG;
+    if (out_dtype != KL_BF16 && out_dtype != KL_FP32) return KL_ERR_INVALID_ARG;
+    if (g.B == 0) return KL_OK;
+    if (!partial_o || !partial_ml || !out) return KL_ERR_INVALID_ARG;
+    if (!aligned(partial_ml, 8)) return KL_ERR_INVALID_ARG;
+    return from_cuda(launch_combine(g.B, g.Hq, g.D, num_splits, partial_o, partial_ml, out,
+                                    out_dtype, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+int32_t kl_decode_kernel_available(const kl_shape *shape, int32_t kernel, int32_t standard) {
+    Geometry g;
+    if (resolve(shape, 1, &g) != KL_OK || g.G > 8) return 0;
+    if (kernel == KL_KERNEL_SIMT || kernel == KL_KERNEL_AUTO) return 1;
+    if (kernel == KL_KERNEL_TENSOR) return tc_supported(g, standard != 0) ? 1 : 0;
+    return 0;
+}
+
+const char *kl_status_string(kl_status s) {
+    switch (s) {
+        case KL_OK: return "ok";
+        case KL_ERR_INVALID_ARG: return "invalid argument";
+        case KL_ERR_UNSUPPORTED: return "unsupported shape or option";
+        case KL_ERR_WORKSPACE: return "workspace missing or too small";
+        case KL_ERR_CUDA: return "CUDA error";
+    }
+    return "unknown status";
+}
+
+}  // extern "C"

@@ -1,0 +1,70 @@
+// Internal declarations shared by the translation units of libkeyless.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "keyless.h"
+
+namespace kl {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+
+// Geometry of one decode call, resolved on the host.
+struct Geometry {
+    int B, Hq, Hkv, G, D, P, num_pages, max_pages, wr_per_qh;
+    float scale;       // lambda / sqrt(d_k)
+    int S;             // split count
+    int chunk;         // tokens per split (a multiple of 128)
+};
+
+// Arguments of a decode launch (keyless or the standard K+V comparison).
+struct DecodeArgs {
+    Geometry geo;
+    const uint16_t *q;        // [B][Hq][D] bf16
+    const uint16_t *w_r;      // [Hw][D][D] bf16 (keyless only)
+    const uint16_t *k_cache;  // [num_pages][Hkv][P][D] bf16 (standard only)
+    const uint16_t *v_cache;  // [num_pages][Hkv][P][D] bf16
+    const int32_t *block_table;
+    const int32_t *seq_lens;
+    float *part_o;            // [B][Hq][S][D]   split states (unless direct_out)
+    float *part_ml;           // [B][Hq][S][2]
+    void *out;                // [B][Hq][D]
+    bool direct_out;          // true: S == 1 and the CTA writes `out` itself (no split states)
+    kl_dtype out_dtype;
+    int32_t *err;
+    cudaStream_t stream;
+};
+
+// bf16 bit helpers (a bf16 value is the upper half of a binary32 value).
+__device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+__device__ __forceinline__ void raise_flag(int32_t *err, int32_t bits) {
+    if (err) atomicOr(err, bits);
+}
+
+// Launchers (each returns cudaGetLastError() of its launch).
+cudaError_t launch_append(const Geometry &g, const uint16_t *v_new, const int32_t *block_table,
+                          const int32_t *positions, uint16_t *v_cache, int32_t *err,
+                          cudaStream_t stream);
+cudaError_t launch_route(const Geometry &g, const uint16_t *q, const uint16_t *w_r, float *q_r,
+                         cudaStream_t stream);
+cudaError_t launch_combine(int B, int Hq, int D, int S, const float *part_o,
+                           const float *part_ml, void *out, kl_dtype out_dtype,
+                           cudaStream_t stream);
+cudaError_t launch_decode_simt(const DecodeArgs &a, bool standard);
+// Merges the split states of a finished decode into `out` unless it wrote `out` directly or
+// the caller asked for the states.
+cudaError_t finish_decode(const DecodeArgs &a, bool states_requested);
+
+// Tensor-core path: whether it supports a geometry, and its launcher.
+bool tc_supported(const Geometry &g, bool standard);
+cudaError_t launch_decode_tc(const DecodeArgs &a, bool standard);
+
+// Number of SMs of the current device (cached per device).
+int device_sm_count();
+
+}  // namespace kl
