@@ -1,10 +1,586 @@
-// Tensor-core (tcgen05 + TMA) decode kernel -- placeholder until the kernel lands.
+// Tensor-core split-sequence decode for sm_103a: TMA page gathers into a shared-memory ring,
+// tcgen05 MMAs with TMEM accumulators, warp-specialized roles.
+//
+// One CTA per (split, value head g, sequence b); head_dim 128, up to 8 query heads per value
+// group. The value-space routing (Section 2.2: q_r = q W^R) runs first, on CUDA cores, into a
+// split-bf16 operand (q_r * scale * log2 e = hi + lo, both bf16) for the G heads of the group.
+// Then each 128-token tile of cached value rows V_t [128 x 128] (Section 3) is used twice by
+// the tensor cores, straight from one shared-memory copy:
+//
+//   scores   S^T = V_t . [q_hi | q_lo]^T        M = 128 tokens, N = 16, K = 128 (A K-major)
+//   output   O^T = V_t^T . [p_hi | p_lo]        M = 128 dims,   N = 16, K = 128 (A MN-major)
+//
+// so every cached row is read from HBM exactly once for both roles. The hi/lo split of the
+// routed query and of the softmax weights keeps about 16 significant bits where a plain bf16
+// operand would keep 8; the tensor cores have ample headroom for the doubled N.
+//
+// Roles (192 threads):
+//   warps 0-3  compute: routing prologue; per tile read S from TMEM (thread = token), online
+//              softmax in base 2 (per-head running max across the CTA), write P^T to shared
+//              memory; read O from TMEM (thread = output dim) and accumulate with rescaling;
+//              epilogue writes the output or the split state.
+//   warp 4     producer: block-table lookups and TMA loads of (page, head) tiles.
+//   warp 5     MMA issuer (one elected lane) and TMEM owner.
+// Every wait is bounded (about one second); a wait that runs out raises KL_FLAG_TIMEOUT,
+// makes every role leave its loop, drains outstanding copies and MMAs and frees TMEM.
+#include <cudaTypedefs.h>
+#include <math.h>
+
 #include "kl_internal.cuh"
+#include "kl_tc_ptx.cuh"
 
 namespace kl {
+namespace {
 
-bool tc_supported(const Geometry &, bool) { return false; }
+constexpr int kD = 128;
+constexpr int kTile = 128;                  // tokens per tile
+constexpr int kNG = 8;                      // query heads per value group (padded)
+constexpr int kN = 2 * kNG;                 // MMA N: hi and lo halves
+constexpr int kComputeWarps = 4;
+constexpr int kProducerWarp = 4;
+constexpr int kMmaWarp = 5;
+constexpr int kThreads = 6 * 32;
+constexpr uint32_t kTileBytes = kTile * kD * 2;   // 32 KiB per cache tile
+constexpr uint32_t kHalfBytes = kTileBytes / 2;   // one 64-dim half: 128 rows x 128 B
+constexpr uint32_t kTmemCols = 64;                // S: 2 x 16 columns, O: 2 x 16 columns
+constexpr uint64_t kTimeoutNs = 1000000000ull;
 
-cudaError_t launch_decode_tc(const DecodeArgs &, bool) { return cudaErrorNotSupported; }
+template <bool kStandard>
+struct Cfg {
+    static constexpr int kStages = 3;
+    static constexpr int kTilesPerStage = kStandard ? 2 : 1;   // K and V, or V only
+};
+
+template <bool kStandard>
+struct __align__(1024) Smem {
+    // Cache tiles, 128B-swizzled: [half (dims 0-63 | 64-127)][128 rows][128 B]. For the
+    // K+V comparison the K tile follows the V tile of the same stage.
+    uint8_t tiles[Cfg<kStandard>::kStages][Cfg<kStandard>::kTilesPerStage][kTileBytes];
+    // Routed query operand [half][16 rows][128 B], 128B-swizzled, K-major.
+    uint8_t qr[2 * kN * 128];
+    // P^T operands, no swizzle, MN-major: [16 groups of 8 tokens][hi | lo][8 tokens][16 B].
+    // During the routing prologue the first one holds the raw query, fp32 [k][8].
+    uint8_t p[2][kTile * kN * 2];
+    float red[2][kComputeWarps][kNG];
+    uint64_t full[Cfg<kStandard>::kStages], empty[Cfg<kStandard>::kStages];
+    uint64_t s_full[2], s_empty[2], p_full[2], o_full[2], o_empty[2], red_bar[2];
+    uint64_t qr_full, q_ready, drain;
+    uint32_t tmem_base;
+    int abort;
+};
+
+// Warp-collective bounded wait: every lane of the warp calls it in uniform control flow and
+// gets the same answer. False when this CTA is aborting or the wait ran out (about 1 s), in
+// which case the caller leaves its loop.
+struct Waiter {
+    volatile int *abort;
+    int32_t *err;
+    __device__ bool operator()(uint64_t *bar, uint32_t parity) const {
+        bool ok = ptx::mbar_try_wait(bar, parity);
+        if (!ok) {
+            const uint64_t t0 = ptx::globaltimer();
+            while (true) {
+                if (ptx::mbar_try_wait(bar, parity)) { ok = true; break; }
+                if (*abort) break;
+                if (ptx::globaltimer() - t0 > kTimeoutNs) {
+                    *abort = 1;
+                    raise_flag(err, KL_FLAG_TIMEOUT);
+                    break;
+                }
+            }
+        }
+        return __all_sync(0xffffffffu, ok);
+    }
+};
+
+struct Heads {
+    float v[8];
+};
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo_half, float hi_half) {
+    const uint32_t a = __bfloat16_as_ushort(__float2bfloat16_rn(lo_half));
+    const uint32_t b = __bfloat16_as_ushort(__float2bfloat16_rn(hi_half));
+    return a | (b << 16);
+}
+
+// Byte offset of element (row n, column k) in a K-major, 128B-swizzled operand of 16 rows
+// and 128 columns laid out as [half][16 rows][128 B].
+__device__ __forceinline__ uint32_t qr_offset(int n, int k) {
+    const int half = k >> 6, kk = k & 63;
+    return half * (kN * 128) + (n >> 3) * 1024 + (n & 7) * 128 + (((kk >> 3) ^ (n & 7)) << 4) +
+           ((kk & 7) << 1);
+}
+
+template <bool kStandard>
+__global__ void __launch_bounds__(kThreads, 1)
+    decode_tc_kernel(const __grid_constant__ CUtensorMap vmap,
+                     const __grid_constant__ CUtensorMap kmap, const DecodeArgs a) {
+    using S = Smem<kStandard>;
+    constexpr int NS = Cfg<kStandard>::kStages;
+    extern __shared__ uint8_t smem_raw[];
+    S &sm = *reinterpret_cast<S *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                   ~uintptr_t(1023));
+
+    const Geometry &geo = a.geo;
+    const int split = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int G = geo.G;
+
+    int L = a.seq_lens[b];
+    if (L < 0 || L > geo.max_pages * geo.P) {
+        if (tid == 0 && split == 0 && g == 0) raise_flag(a.err, KL_FLAG_BAD_LENGTH);
+        L = 0;
+    }
+    const int t_begin = split * geo.chunk;
+    const int t_end = min(t_begin + geo.chunk, L);
+    const int n_tiles = t_end > t_begin ? (t_end - t_begin + kTile - 1) / kTile : 0;
+
+    // Empty split: a zero output or an empty state, no pipeline.
+    if (n_tiles == 0) {
+        if (tid < kD) {
+            for (int h = 0; h < G; ++h) {
+                const size_t bh = (size_t)b * geo.Hq + g * G + h;
+                if (a.direct_out) {
+                    if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * kD + tid] = 0.f;
+                    else static_cast<__nv_bfloat16 *>(a.out)[bh * kD + tid] = __float2bfloat16_rn(0.f);
+                } else {
+                    const size_t slot = bh * geo.S + split;
+                    a.part_o[slot * kD + tid] = 0.f;
+                    if (tid == 0) {
+                        a.part_ml[slot * 2] = -INFINITY;
+                        a.part_ml[slot * 2 + 1] = 0.f;
+                    }
+                }
+            }
+        }
+        return;
+    }
+
+    if (tid == 0) {
+        for (int s = 0; s < NS; ++s) {
+            ptx::mbar_init(&sm.full[s], 1);
+            ptx::mbar_init(&sm.empty[s], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            ptx::mbar_init(&sm.s_full[i], 1);
+            ptx::mbar_init(&sm.s_empty[i], kComputeWarps);
+            ptx::mbar_init(&sm.p_full[i], kComputeWarps);
+            ptx::mbar_init(&sm.o_full[i], 1);
+            ptx::mbar_init(&sm.o_empty[i], kComputeWarps);
+            ptx::mbar_init(&sm.red_bar[i], kComputeWarps);
+        }
+        ptx::mbar_init(&sm.qr_full, kComputeWarps);
+        ptx::mbar_init(&sm.q_ready, kComputeWarps);
+        ptx::mbar_init(&sm.drain, 1);
+        sm.abort = 0;
+        ptx::fence_mbar_init();
+    }
+    if (warp == kMmaWarp) {
+        ptx::tmem_alloc(&sm.tmem_base, kTmemCols);
+        ptx::tmem_relinquish();
+    }
+    if (warp == kProducerWarp && lane == 0) {
+        ptx::prefetch_tensormap(&vmap);
+        if (kStandard) ptx::prefetch_tensormap(&kmap);
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = sm.tmem_base;
+    const Waiter wait{&sm.abort, a.err};
+
+    if (warp == kProducerWarp) {
+        // ------------------------------------------------------------------ producer ----
+        const int P = geo.P;
+        const int ppt = kTile / P;                   // pages per tile (<= 8)
+        const int first_page = t_begin / P;
+        const int end_page = (t_end + P - 1) / P;
+        const int32_t *bt = a.block_table + (size_t)b * geo.max_pages;
+        const uint32_t page_bytes = (uint32_t)P * 128u;   // one half of one page
+        bool bad = false;
+        int issued = 0;
+        for (int i = 0; i < n_tiles; ++i) {
+            const int s = i % NS;
+            const int pidx = first_page + i * ppt + lane;
+            int page = -1;
+            if (lane < ppt && pidx < end_page) page = bt[pidx];
+            if (i >= NS && !wait(&sm.empty[s], ((i / NS) & 1) ^ 1)) break;
+            const bool in_range = page >= 0 && page < geo.num_pages;
+            if (lane < ppt && pidx < end_page && !in_range) bad = true;
+            const unsigned mask = __ballot_sync(0xffffffffu, in_range);
+            if (lane == 0)
+                ptx::mbar_arrive_expect_tx(&sm.full[s], __popc(mask) * page_bytes * 2u *
+                                                            Cfg<kStandard>::kTilesPerStage);
+            __syncwarp();
+            if (in_range) {
+                const int row = (page * geo.Hkv + g) * P;
+                uint8_t *dst = sm.tiles[s][0] + lane * page_bytes;
+                ptx::tma_load_2d(dst, &vmap, &sm.full[s], 0, row);
+                ptx::tma_load_2d(dst + kHalfBytes, &vmap, &sm.full[s], 64, row);
+                if constexpr (kStandard) {
+                    uint8_t *kd = sm.tiles[s][1] + lane * page_bytes;
+                    ptx::tma_load_2d(kd, &kmap, &sm.full[s], 0, row);
+                    ptx::tma_load_2d(kd + kHalfBytes, &kmap, &sm.full[s], 64, row);
+                }
+            }
+            issued = i + 1;
+        }
+        if (__any_sync(0xffffffffu, bad) && lane == 0) raise_flag(a.err, KL_FLAG_BAD_PAGE);
+        // Drain: copies still in flight must land before the CTA's shared memory goes away.
+        if (sm.abort) {
+            const Waiter drain_wait{&sm.abort, a.err};
+            for (int i = max(0, issued - NS); i < issued; ++i) {
+                const uint64_t t0 = ptx::globaltimer();
+                while (!ptx::mbar_try_wait(&sm.full[i % NS], (i / NS) & 1) &&
+                       ptx::globaltimer() - t0 < kTimeoutNs) {
+                }
+            }
+            (void)drain_wait;
+        }
+    } else if (warp == kMmaWarp) {
+        // --------------------------------------------------------------- MMA issuer ----
+        constexpr uint32_t idesc_s = ptx::idesc_bf16(128, kN, false, false);
+        constexpr uint32_t idesc_o = ptx::idesc_bf16(128, kN, true, true);
+        const uint32_t qr_addr = ptx::smem_addr(sm.qr);
+        bool ok = wait(&sm.qr_full, 0);
+        if (ok) ptx::tc_fence_after();
+        for (int i = 0; ok && i <= n_tiles; ++i) {
+            if (i < n_tiles) {
+                const int s = i % NS, sb = i & 1;
+                if (!wait(&sm.full[s], (i / NS) & 1)) break;
+                if (i >= 2 && !wait(&sm.s_empty[sb], ((i >> 1) - 1) & 1)) break;
+                ptx::tc_fence_after();
+                if (lane == 0) {
+                    const uint32_t score_tile =
+                        ptx::smem_addr(sm.tiles[s][Cfg<kStandard>::kTilesPerStage - 1]);
+#pragma unroll
+                    for (int kk = 0; kk < kD / 16; ++kk) {
+                        const uint32_t koff = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
+                        const uint32_t qoff = (kk >> 2) * (kN * 128) + (kk & 3) * 32;
+                        ptx::mma_bf16(tmem + sb * kN,
+                                      ptx::smem_desc(score_tile + koff, 16, 1024, ptx::kSwizzle128B),
+                                      ptx::smem_desc(qr_addr + qoff, 16, 1024, ptx::kSwizzle128B),
+                                      idesc_s, kk > 0);
+                    }
+                    ptx::mma_commit(&sm.s_full[sb]);
+                }
+                __syncwarp();
+            }
+            if (i >= 1) {
+                const int j = i - 1, s = j % NS, pb = j & 1;
+                if (!wait(&sm.p_full[pb], (j >> 1) & 1)) break;
+                if (j >= 2 && !wait(&sm.o_empty[pb], ((j >> 1) - 1) & 1)) break;
+                ptx::tc_fence_after();
+                const int nvalid = min(kTile, t_end - (t_begin + j * kTile));
+                const int ksteps = (nvalid + 15) >> 4;
+                if (lane == 0) {
+                    const uint32_t vt = ptx::smem_addr(sm.tiles[s][0]);
+                    const uint32_t pt = ptx::smem_addr(sm.p[pb]);
+                    for (int kk = 0; kk < ksteps; ++kk) {
+                        // A = V^T: MN-major SW128, 64-dim halves kHalfBytes apart (LBO),
+                        //          8-token row groups 1 KiB apart (SBO); 16 tokens per step.
+                        // B = P^T: MN-major, no swizzle; hi/lo blocks 128 B apart (SBO),
+                        //          8-token groups 256 B apart (LBO).
+                        ptx::mma_bf16(tmem + 2 * kN + pb * kN,
+                                      ptx::smem_desc(vt + kk * 2048, kHalfBytes, 1024, ptx::kSwizzle128B),
+                                      ptx::smem_desc(pt + kk * 512, 256, 128, ptx::kSwizzleNone),
+                                      idesc_o, kk > 0);
+                    }
+                    ptx::mma_commit(&sm.o_full[pb]);
+                    ptx::mma_commit(&sm.empty[s]);
+                }
+                __syncwarp();
+            }
+        }
+        // Drain: every MMA this warp issued completes before TMEM is freed.
+        if (lane == 0) ptx::mma_commit(&sm.drain);
+        __syncwarp();
+        {
+            const uint64_t t0 = ptx::globaltimer();
+            while (!ptx::mbar_try_wait(&sm.drain, 0) && ptx::globaltimer() - t0 < kTimeoutNs) {
+            }
+        }
+    } else {
+        // ------------------------------------------------------------------ compute -----
+        const int t = tid;                                  // 0..127
+        const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+        float *qf = reinterpret_cast<float *>(sm.p[0]);     // [k][8] raw query (prologue only)
+        const float sl2 = geo.scale * kLog2e;
+        bool ok = true;
+
+        // Routing prologue: thread j computes q_r[h][j] for the G heads, fp32.
+        for (int i = t; i < kD * kNG; i += kTile) {
+            const int k = i >> 3, h = i & 7;
+            qf[i] = h < G ? __uint_as_float((uint32_t)a.q[((size_t)b * geo.Hq + g * G + h) * kD + k] << 16)
+                          : 0.f;
+        }
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(&sm.q_ready);
+        ok = wait(&sm.q_ready, 0);
+        if (ok) {
+            float acc[kNG];
+#pragma unroll
+            for (int h = 0; h < kNG; ++h) acc[h] = 0.f;
+            if constexpr (kStandard) {
+#pragma unroll
+                for (int h = 0; h < kNG; ++h) acc[h] = qf[t * kNG + h];
+            } else if (!geo.wr_per_qh) {
+                const uint16_t *W = a.w_r + (size_t)g * kD * kD + t;
+#pragma unroll 4
+                for (int k = 0; k < kD; ++k) {
+                    const float w = __uint_as_float((uint32_t)W[(size_t)k * kD] << 16);
+                    const float4 q0 = *reinterpret_cast<const float4 *>(qf + k * kNG);
+                    const float4 q1 = *reinterpret_cast<const float4 *>(qf + k * kNG + 4);
+                    acc[0] = fmaf(q0.x, w, acc[0]); acc[1] = fmaf(q0.y, w, acc[1]);
+                    acc[2] = fmaf(q0.z, w, acc[2]); acc[3] = fmaf(q0.w, w, acc[3]);
+                    acc[4] = fmaf(q1.x, w, acc[4]); acc[5] = fmaf(q1.y, w, acc[5]);
+                    acc[6] = fmaf(q1.z, w, acc[6]); acc[7] = fmaf(q1.w, w, acc[7]);
+                }
+            } else {
+#pragma unroll
+                for (int h = 0; h < kNG; ++h) {
+                    if (h < G) {
+                        const uint16_t *W = a.w_r + (size_t)(g * G + h) * kD * kD + t;
+                        float s = 0.f;
+#pragma unroll 8
+                        for (int k = 0; k < kD; ++k)
+                            s = fmaf(qf[k * kNG + h], __uint_as_float((uint32_t)W[(size_t)k * kD] << 16), s);
+                        acc[h] = s;
+                    }
+                }
+            }
+            // split-bf16 operand rows: n = h (hi), n = 8 + h (lo); column k = t
+#pragma unroll
+            for (int h = 0; h < kNG; ++h) {
+                const float v = acc[h] * sl2;
+                const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+                const __nv_bfloat16 lo = __float2bfloat16_rn(v - __bfloat162float(hi));
+                *reinterpret_cast<__nv_bfloat16 *>(sm.qr + qr_offset(h, t)) = hi;
+                *reinterpret_cast<__nv_bfloat16 *>(sm.qr + qr_offset(kNG + h, t)) = lo;
+            }
+            ptx::fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&sm.qr_full);
+        }
+
+        float m[kNG], lsum[kNG], o[kNG];
+        Heads alpha_prev;
+#pragma unroll
+        for (int h = 0; h < kNG; ++h) {
+            m[h] = -INFINITY;
+            lsum[h] = 0.f;
+            o[h] = 0.f;
+            alpha_prev.v[h] = 0.f;
+        }
+
+        // O accumulation of tile j: o = o * alpha_j + O_j (thread = output dim t).
+        auto correct = [&](int j, const Heads alpha) -> bool {
+            const int ob = j & 1;
+            if (!wait(&sm.o_full[ob], (j >> 1) & 1)) return false;
+            ptx::tc_fence_after();
+            float ov[16];
+            ptx::tmem_ld16(tmem + 2 * kN + ob * kN + lane_base, ov);
+            ptx::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&sm.o_empty[ob]);
+#pragma unroll
+            for (int h = 0; h < kNG; ++h) o[h] = fmaf(o[h], alpha.v[h], ov[h] + ov[kNG + h]);
+            return true;
+        };
+
+        for (int i = 0; ok && i < n_tiles; ++i) {
+            const int sb = i & 1;
+            if (!wait(&sm.s_full[sb], (i >> 1) & 1)) { ok = false; break; }
+            ptx::tc_fence_after();
+            float sv[16];
+            ptx::tmem_ld16(tmem + sb * kN + lane_base, sv);
+            ptx::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&sm.s_empty[sb]);
+
+            const int nvalid = min(kTile, t_end - (t_begin + i * kTile));
+            const bool valid = t < nvalid;
+            float s[kNG], mx[kNG];
+#pragma unroll
+            for (int h = 0; h < kNG; ++h) {
+                s[h] = (valid && h < G) ? sv[h] + sv[kNG + h] : -INFINITY;
+                mx[h] = s[h];
+            }
+            // per-head maximum over the tile's 128 tokens
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1)
+#pragma unroll
+                for (int h = 0; h < kNG; ++h)
+                    mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], off));
+            if (lane == 0) {
+#pragma unroll
+                for (int h = 0; h < kNG; ++h) sm.red[sb][warp][h] = mx[h];
+                ptx::mbar_arrive(&sm.red_bar[sb]);
+            }
+            if (!wait(&sm.red_bar[sb], (i >> 1) & 1)) { ok = false; break; }
+            Heads alpha;
+            float p[kNG];
+#pragma unroll
+            for (int h = 0; h < kNG; ++h) {
+                float tmax = sm.red[sb][0][h];
+#pragma unroll
+                for (int w = 1; w < kComputeWarps; ++w) tmax = fmaxf(tmax, sm.red[sb][w][h]);
+                const float mn = fmaxf(m[h], tmax);
+                const bool live = h < G;
+                alpha.v[h] = live ? exp2f(m[h] - mn) : 0.f;
+                p[h] = live ? exp2f(s[h] - mn) : 0.f;
+                lsum[h] = fmaf(lsum[h], alpha.v[h], p[h]);
+                m[h] = live ? mn : m[h];
+            }
+            // P^T row of token t: hi and lo halves.
+            {
+                float r[kNG];
+#pragma unroll
+                for (int h = 0; h < kNG; ++h)
+                    r[h] = p[h] - __bfloat162float(__float2bfloat16_rn(p[h]));
+                uint8_t *row = sm.p[sb] + (t >> 3) * 256 + (t & 7) * 16;
+                *reinterpret_cast<uint4 *>(row) =
+                    make_uint4(pack_bf16(p[0], p[1]), pack_bf16(p[2], p[3]),
+                               pack_bf16(p[4], p[5]), pack_bf16(p[6], p[7]));
+                *reinterpret_cast<uint4 *>(row + 128) =
+                    make_uint4(pack_bf16(r[0], r[1]), pack_bf16(r[2], r[3]),
+                               pack_bf16(r[4], r[5]), pack_bf16(r[6], r[7]));
+            }
+            // Rows past the end inside the last 16-token MMA step must be finite: zero them.
+            if (nvalid < kTile) {
+                const int st = i % NS;
+                if (wait(&sm.full[st], (i / NS) & 1) && t >= nvalid && t < ((nvalid + 15) & ~15)) {
+                    uint4 *r0 = reinterpret_cast<uint4 *>(sm.tiles[st][0] + t * 128);
+                    uint4 *r1 = reinterpret_cast<uint4 *>(sm.tiles[st][0] + kHalfBytes + t * 128);
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {
+                        r0[c] = make_uint4(0, 0, 0, 0);
+                        r1[c] = make_uint4(0, 0, 0, 0);
+                    }
+                }
+            }
+            ptx::fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&sm.p_full[sb]);
+
+            if (i >= 1 && !correct(i - 1, alpha_prev)) { ok = false; break; }
+            alpha_prev = alpha;
+        }
+        if (ok) ok = correct(n_tiles - 1, alpha_prev);
+
+        if (ok) {
+            // l totals over the 128 tokens-threads, then the output or the split state
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1)
+#pragma unroll
+                for (int h = 0; h < kNG; ++h) lsum[h] += __shfl_xor_sync(0xffffffffu, lsum[h], off);
+            const int rb = n_tiles & 1;   // red buffer / phase after the tile loop
+            if (lane == 0) {
+#pragma unroll
+                for (int h = 0; h < kNG; ++h) sm.red[rb][warp][h] = lsum[h];
+                ptx::mbar_arrive(&sm.red_bar[rb]);
+            }
+            if (wait(&sm.red_bar[rb], (n_tiles >> 1) & 1)) {
+#pragma unroll
+                for (int h = 0; h < kNG; ++h) {
+                    if (h >= G) continue;
+                    float l = 0.f;
+#pragma unroll
+                    for (int w = 0; w < kComputeWarps; ++w) l += sm.red[rb][w][h];
+                    const float val = o[h] / l;
+                    const size_t bh = (size_t)b * geo.Hq + g * G + h;
+                    if (a.direct_out) {
+                        if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * kD + t] = val;
+                        else static_cast<__nv_bfloat16 *>(a.out)[bh * kD + t] = __float2bfloat16_rn(val);
+                    } else {
+                        const size_t slot = bh * geo.S + split;
+                        a.part_o[slot * kD + t] = val;
+                        if (t == 0) {
+                            a.part_ml[slot * 2] = m[h] * kLn2;
+                            a.part_ml[slot * 2 + 1] = l;
+                        }
+                    }
+                }
+            }
+        }
+    }
+
+    ptx::tc_fence_before();
+    __syncthreads();
+    if (warp == kMmaWarp) {
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+// ------------------------------------------------------------------------ host side ------
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (!fn) {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    }
+    return fn;
+}
+
+// Tensor map of a paged cache viewed as [num_pages * Hkv * P rows][128 dims] bf16; one box is
+// one page of one head, 64 dims wide (one 128-byte swizzle span).
+bool make_cache_map(CUtensorMap *map, const void *base, const Geometry &g) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    const cuuint64_t dims[2] = {(cuuint64_t)kD, (cuuint64_t)g.num_pages * g.Hkv * g.P};
+    const cuuint64_t strides[1] = {(cuuint64_t)kD * 2};
+    const cuuint32_t box[2] = {64, (cuuint32_t)g.P};
+    const cuuint32_t estr[2] = {1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides,
+              box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <bool kStandard>
+cudaError_t launch(const DecodeArgs &a) {
+    const Geometry &g = a.geo;
+    CUtensorMap vmap, kmap;
+    if (!make_cache_map(&vmap, a.v_cache, g)) return cudaErrorInvalidValue;
+    if (kStandard) {
+        if (!make_cache_map(&kmap, a.k_cache, g)) return cudaErrorInvalidValue;
+    } else {
+        kmap = vmap;
+    }
+    const size_t smem = sizeof(Smem<kStandard>) + 1024;
+    static bool configured = false;
+    if (!configured) {
+        cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<kStandard>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
+    decode_tc_kernel<kStandard><<<dim3(g.S, g.Hkv, g.B), kThreads, smem, a.stream>>>(vmap, kmap, a);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+bool tc_supported(const Geometry &g, bool standard) {
+    (void)standard;
+    if (g.D != kD || g.G > kNG) return false;
+    if (g.P != 16 && g.P != 32 && g.P != 64 && g.P != 128) return false;
+    if ((int64_t)g.num_pages * g.Hkv * g.P >= ((int64_t)1 << 31)) return false;
+    int dev = 0, major = 0, minor = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return false;
+    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+    return major == 10 && minor == 3;
+}
+
+cudaError_t launch_decode_tc(const DecodeArgs &a, bool standard) {
+    if (a.geo.B == 0) return cudaSuccess;
+    return standard ? launch<true>(a) : launch<false>(a);
+}
 
 }  // namespace kl
