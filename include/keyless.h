@@ -173,6 +173,31 @@ kl_status kl_standard_decode(const kl_shape *shape, const void *q, const void *k
                              kl_dtype out_dtype, void *workspace, size_t workspace_bytes,
                              int32_t *err, kl_stream_t stream);
 
+/* Size of the fixed device scratch that kl_decode_attention_noalloc uses (32 MiB). */
+#define KL_NOALLOC_SCRATCH_BYTES (32u * 1024u * 1024u)
+
+/*
+ * kl_decode_attention without a workspace argument, for callers that must not allocate device
+ * memory -- for example code running inside a host framework that owns all device memory
+ * through its own pool and does not let its plugins call cudaMalloc, or a latency-critical
+ * path that cannot afford an allocation's implicit synchronization and unpredictable cost.
+ * The paper has no counterpart: this is a deployment convenience of the library.
+ * The split states live in one fixed array of KL_NOALLOC_SCRATCH_BYTES in device memory,
+ * which every GPU that loads the library holds until the process exits. The library looks
+ * up that array's device address during the first call on each device (with that device
+ * current); make that first call before any stream capture. Nothing is allocated and no
+ * allocating routine is called. Every call on a device shares the one array and leaves its
+ * contents behind, so calls that may overlap on the GPU (different streams, or different
+ * host threads without ordering) race and must be serialized by the caller. A shape and
+ * split count whose split states need more than KL_NOALLOC_SCRATCH_BYTES is rejected with
+ * KL_ERR_WORKSPACE before anything is launched (num_splits = 1 needs no scratch). Other
+ * arguments, results and error flags are those of kl_decode_attention.
+ */
+kl_status kl_decode_attention_noalloc(const kl_shape *shape, const void *q, const void *w_r,
+                                      const void *v_cache, const int32_t *block_table,
+                                      const int32_t *seq_lens, int32_t num_splits, void *out,
+                                      kl_dtype out_dtype, int32_t *err, kl_stream_t stream);
+
 /*
  * Whether kernel family `kernel` (kl_kernel) handles this shape: 1 yes, 0 no. For the keyless
  * decode (standard = 0) or the K+V comparison (standard = 1). A capability query of the

@@ -17,6 +17,7 @@ KL_OK, KL_ERR_INVALID_ARG, KL_ERR_UNSUPPORTED, KL_ERR_WORKSPACE, KL_ERR_CUDA = r
 KL_BF16, KL_FP32 = 0, 1
 KL_KERNEL_AUTO, KL_KERNEL_TENSOR, KL_KERNEL_SIMT = 0, 1, 2
 KL_FLAG_BAD_PAGE, KL_FLAG_BAD_POSITION, KL_FLAG_BAD_LENGTH, KL_FLAG_TIMEOUT = 1, 2, 4, 8
+KL_NOALLOC_SCRATCH_BYTES = 32 * 1024 * 1024
 
 HEADER = os.path.join(_build.INCLUDE, "keyless.h")
 
@@ -69,6 +70,7 @@ def load() -> ctypes.CDLL:
         "kl_decode_attention_ex": ([SH, P, P, P, P, P, OP, P, I32, P, SZ, P, P], I32),
         "kl_combine": ([SH, P, P, I32, P, I32, P], I32),
         "kl_standard_decode": ([SH, P, P, P, P, P, OP, P, I32, P, SZ, P, P], I32),
+        "kl_decode_attention_noalloc": ([SH, P, P, P, P, P, I32, P, I32, P, P], I32),
         "kl_decode_kernel_available": ([SH, I32, I32], I32),
         "kl_status_string": ([I32], ctypes.c_char_p),
     }
@@ -172,6 +174,15 @@ def kl_standard_decode(shape, q, k_cache, v_cache, block_table, seq_lens, opts, 
                                      None if opts is None else ctypes.byref(opts), _p(out),
                                      out_dtype, _p(workspace), _nbytes(workspace), _p(err),
                                      _stream(stream)), "kl_standard_decode")
+
+
+def kl_decode_attention_noalloc(shape, q, w_r, v_cache, block_table, seq_lens, num_splits, out,
+                                out_dtype, err=None, stream=None):
+    """The decode with its split states in the library's fixed device scratch (no workspace)."""
+    _check(load().kl_decode_attention_noalloc(ctypes.byref(shape), _p(q), _p(w_r), _p(v_cache),
+                                              _p(block_table), _p(seq_lens), num_splits, _p(out),
+                                              out_dtype, _p(err), _stream(stream)),
+           "kl_decode_attention_noalloc")
 
 
 def kl_decode_kernel_available(shape, kernel, standard=False) -> bool:

@@ -1,0 +1,71 @@
+// kl_decode_attention_noalloc: the keyless decode for callers that cannot allocate device
+// memory. The split states that kl_decode_attention keeps in a caller-provided workspace live
+// here in one fixed, file-scope device array instead.
+#include <mutex>
+
+#include "kl_internal.cuh"
+
+namespace kl {
+namespace {
+
+// Fixed scratch for split states: [B][Hq][S][D] fp32 outputs, then [B][Hq][S][2] fp32 {m, l}.
+// Every GPU that loads this library holds these bytes until the process exits.
+constexpr size_t kScratchBytes = (size_t)KL_NOALLOC_SCRATCH_BYTES;
+static __device__ __align__(256) unsigned char g_split_scratch[kScratchBytes];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_setup_mutex;
+void *g_scratch_ptr[kMaxDevices] = {nullptr};
+
+// Device address of the scratch array on the current device, looked up once per device.
+// Host code cannot use the symbol itself as a device address.
+cudaError_t scratch_for_current_device(void **out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(g_setup_mutex);
+    if (!g_scratch_ptr[dev]) {
+        void *p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_split_scratch);
+        if (e != cudaSuccess) return e;
+        g_scratch_ptr[dev] = p;
+    }
+    *out = g_scratch_ptr[dev];
+    return cudaSuccess;
+}
+
+size_t round_up256(size_t x) { return (x + 255) / 256 * 256; }
+
+}  // namespace
+}  // namespace kl
+
+extern "C" kl_status kl_decode_attention_noalloc(const kl_shape *shape, const void *q,
+                                                 const void *w_r, const void *v_cache,
+                                                 const int32_t *block_table,
+                                                 const int32_t *seq_lens, int32_t num_splits,
+                                                 void *out, kl_dtype out_dtype, int32_t *err,
+                                                 kl_stream_t stream) {
+    using namespace kl;
+    if (!shape || num_splits < 0) return KL_ERR_INVALID_ARG;
+    const int32_t S = kl_decode_num_splits(shape, num_splits);
+    if (S <= 0) return KL_ERR_INVALID_ARG;
+    if (S == 1)   // no split states: the ordinary path needs no workspace either
+        return kl_decode_attention(shape, q, w_r, v_cache, block_table, seq_lens, 1, out,
+                                   out_dtype, nullptr, 0, err, stream);
+    const size_t rows = (size_t)shape->num_seqs * shape->num_q_heads * S;
+    const size_t o_bytes = round_up256(rows * shape->head_dim * sizeof(float));
+    const size_t ml_bytes = round_up256(rows * 2 * sizeof(float));
+    if (o_bytes + ml_bytes > kScratchBytes) return KL_ERR_WORKSPACE;
+    if (!out) return KL_ERR_INVALID_ARG;
+
+    void *base = nullptr;
+    if (scratch_for_current_device(&base) != cudaSuccess) return KL_ERR_CUDA;
+    float *part_o = static_cast<float *>(base);
+    float *part_ml = reinterpret_cast<float *>(static_cast<unsigned char *>(base) + o_bytes);
+    kl_decode_options opts{S, KL_KERNEL_AUTO, part_o, part_ml};
+    kl_status st = kl_decode_attention_ex(shape, q, w_r, v_cache, block_table, seq_lens, &opts,
+                                          nullptr, out_dtype, nullptr, 0, err, stream);
+    if (st != KL_OK) return st;
+    return kl_combine(shape, part_o, part_ml, S, out, out_dtype, stream);
+}
