@@ -4,7 +4,8 @@ A step is one pass of the whole hot path over one batch: kl_append_v writes the 
 token's value rows into the paged Value-Only Cache, then kl_decode_attention runs the routed
 decode (fused routing prologue, split-sequence decode, cross-split combine). Inputs are
 seeded synthetic tensors with the shapes of the selected workload, resident in HBM before the
-timed region; L2 is flushed (a 512 MiB write) between timed steps.
+timed region; L2 is flushed between timed steps (a 512 MiB write, then a read of it, so the
+lines left in L2 are clean).
 
 Prints ONE JSON line (rank 0). `--impl reference` times the fp64 CPU oracle instead (the
 reference arm: a slow CPU program, timed on a bounded sample of the same workload).
@@ -274,6 +275,14 @@ def run_ours(args):
                      device=dev)
     err = torch.zeros(1, dtype=torch.int32, device=dev)
     flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    flush_sink = torch.empty((), dtype=torch.float32, device=dev)
+
+    def flush_l2():
+        # Evict the cache rows from L2: write 512 MiB (4x L2), then read it back so that the
+        # lines left in L2 are clean and their write-back does not land inside the next step.
+        flush.zero_()
+        torch.sum(flush, dim=0, out=flush_sink)
+
     stream = torch.cuda.current_stream(dev)
     opts_states = kl.decode_options(S, kernel, part_o, part_ml)
     opts_full = kl.decode_options(splits_req, kernel)
@@ -287,21 +296,35 @@ def run_ours(args):
                                       g["seq_lens"], opts_states, None, kl.KL_BF16, None, err,
                                       stream)
 
+    def decode_direct():
+        # S == 1: the production call writes the output itself (one kernel, no combine)
+        if args.standard:
+            kl.kl_standard_decode(sh, g["q"], k_cache, g["v_cache"], g["block_table"],
+                                  g["seq_lens"], opts_full, out, kl.KL_BF16, ws, err, stream)
+        else:
+            kl.kl_decode_attention(sh, g["q"], g["w_r"], g["v_cache"], g["block_table"],
+                                   g["seq_lens"], splits_req, out, kl.KL_BF16, ws, err, stream)
+
     def step_timed(ev):
-        # append | decode kernel | combine, each bracketed by events on the launching stream
+        # append | decode kernel | combine, each bracketed by events on the launching stream;
+        # the kernels are the ones kl_decode_attention launches, called one by one
         ev[0].record(stream)
         kl.kl_append_v(sh, g["v_new"], g["block_table"], g["positions"], g["v_cache"], err,
                        stream)
         ev[1].record(stream)
-        decode_states()
-        ev[2].record(stream)
-        kl.kl_combine(sh, part_o, part_ml, S, out, kl.KL_BF16, stream)
+        if S == 1:
+            decode_direct()
+            ev[2].record(stream)
+        else:
+            decode_states()
+            ev[2].record(stream)
+            kl.kl_combine(sh, part_o, part_ml, S, out, kl.KL_BF16, stream)
         ev[3].record(stream)
 
-    launches_per_step = 3
+    launches_per_step = 2 if S == 1 else 3
     E = lambda: torch.cuda.Event(enable_timing=True)
     for _ in range(args.warmup):
-        flush.zero_()
+        flush_l2()
         step_timed([E() for _ in range(4)])
     torch.cuda.synchronize()
     assert int(err.item()) == 0, f"device error flags {int(err.item())}"
@@ -312,7 +335,7 @@ def run_ours(args):
     torch.cuda.synchronize()
     with ClockSampler(local) as clk:
         for i in range(args.steps):
-            flush.zero_()
+            flush_l2()
             step_timed(evs[i])
         torch.cuda.synchronize()
     if world > 1:
@@ -361,12 +384,12 @@ def run_ours(args):
             h_out.copy_(out, non_blocking=True)
 
         for _ in range(args.warmup):
-            flush.zero_()
+            flush_l2()
             e2e_step()
         torch.cuda.synchronize()
         ts = []
         for _ in range(args.steps):
-            flush.zero_()
+            flush_l2()
             a, b = E(), E()
             a.record(stream)
             e2e_step()
@@ -405,7 +428,7 @@ def run_ours(args):
                    "seq_len": wl.seq_len or list(wl.seq_len_range),
                    "context_tokens": ab["tokens"], "num_splits": S, "kernel": kname,
                    "decode": "standard K+V (comparison)" if args.standard else "keyless",
-                   "l2": "flushed (512 MiB write) between timed steps",
+                   "l2": "flushed between timed steps (512 MiB write, then read back)",
                    "parallelism": f"replicas x{world}"},
         "hbm_gbs_step": step_gbs,
         "pct_of_8tbs_step": 100.0 * step_gbs / NOMINAL_HBM_GBS,

@@ -58,10 +58,10 @@ kl_status resolve(const kl_shape *s, int32_t num_splits, Geometry *g) {
     int64_t S = num_splits;
     if (S == 0) {
         // Enough (split, value head, sequence) items to fill every SM about twice, and splits
-        // of at most 4096 tokens so that ragged batches balance; never below 256 tokens.
+        // of at most 8192 tokens so that ragged batches balance; never below 256 tokens.
         const int64_t units = (int64_t)(g->B > 0 ? g->B : 1) * g->Hkv;
         const int64_t fill = (2 * (int64_t)device_sm_count() + units - 1) / units;
-        const int64_t cap = (Lmax + 4095) / 4096;
+        const int64_t cap = (Lmax + 8191) / 8192;
         S = fill > cap ? fill : cap;
         const int64_t smax = (Lmax + 255) / 256;
         if (S > smax) S = smax;

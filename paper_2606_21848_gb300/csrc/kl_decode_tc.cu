@@ -64,7 +64,7 @@ struct __align__(1024) Smem {
     float red[2][kComputeWarps][kNG];
     uint64_t full[Cfg<kStandard>::kStages], empty[Cfg<kStandard>::kStages];
     uint64_t s_full[2], s_empty[2], p_full[2], o_full[2], o_empty[2], red_bar[2];
-    uint64_t qr_full, q_ready, drain;
+    uint64_t qr_full, q_ready, r_full, drain;
     uint32_t tmem_base;
     int abort;
 };
@@ -114,7 +114,9 @@ __device__ __forceinline__ uint32_t qr_offset(int n, int k) {
 template <bool kStandard>
 __global__ void __launch_bounds__(kThreads, 1)
     decode_tc_kernel(const __grid_constant__ CUtensorMap vmap,
-                     const __grid_constant__ CUtensorMap kmap, const DecodeArgs a) {
+                     const __grid_constant__ CUtensorMap kmap,
+                     const __grid_constant__ CUtensorMap wmap,
+                     const __grid_constant__ CUtensorMap qmap, const DecodeArgs a) {
     using S = Smem<kStandard>;
     constexpr int NS = Cfg<kStandard>::kStages;
     extern __shared__ uint8_t smem_raw[];
@@ -134,6 +136,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int t_begin = split * geo.chunk;
     const int t_end = min(t_begin + geo.chunk, L);
     const int n_tiles = t_end > t_begin ? (t_end - t_begin + kTile - 1) / kTile : 0;
+    // With one W^R per value head the routing runs on the tensor cores: W^R[g] and the G query
+    // rows arrive by TMA as ring position 0 and the cache tiles follow at positions 1, 2, ...
+    const bool tc_route = !kStandard && !geo.wr_per_qh;
+    const int ro = tc_route ? 1 : 0;
 
     // Empty split: a zero output or an empty state, no pipeline.
     if (n_tiles == 0) {
@@ -171,6 +177,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         ptx::mbar_init(&sm.qr_full, kComputeWarps);
         ptx::mbar_init(&sm.q_ready, kComputeWarps);
+        ptx::mbar_init(&sm.r_full, 1);
         ptx::mbar_init(&sm.drain, 1);
         sm.abort = 0;
         ptx::fence_mbar_init();
@@ -182,6 +189,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == kProducerWarp && lane == 0) {
         ptx::prefetch_tensormap(&vmap);
         if (kStandard) ptx::prefetch_tensormap(&kmap);
+        if (tc_route) {
+            ptx::prefetch_tensormap(&wmap);
+            ptx::prefetch_tensormap(&qmap);
+        }
     }
     ptx::tc_fence_before();
     __syncthreads();
@@ -199,12 +210,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t page_bytes = (uint32_t)P * 128u;   // one half of one page
         bool bad = false;
         int issued = 0;
+        if (tc_route) {
+            // ring position 0: W^R[g] as the MN-major A operand [j half][128 k rows][128 B] and
+            // the group's query rows as the K-major B operand (rows 0..G-1 of the q_r buffer)
+            if (lane == 0) {
+                ptx::mbar_arrive_expect_tx(&sm.full[0], kTileBytes + 2u * (uint32_t)G * 128u);
+                ptx::tma_load_2d(sm.tiles[0][0], &wmap, &sm.full[0], 0, g * kD);
+                ptx::tma_load_2d(sm.tiles[0][0] + kHalfBytes, &wmap, &sm.full[0], 64, g * kD);
+                ptx::tma_load_2d(sm.qr, &qmap, &sm.full[0], 0, b * geo.Hq + g * G);
+                ptx::tma_load_2d(sm.qr + kN * 128, &qmap, &sm.full[0], 64, b * geo.Hq + g * G);
+            }
+            __syncwarp();
+            issued = 1;
+        }
         for (int i = 0; i < n_tiles; ++i) {
-            const int s = i % NS;
+            const int r = i + ro, s = r % NS;
             const int pidx = first_page + i * ppt + lane;
             int page = -1;
             if (lane < ppt && pidx < end_page) page = bt[pidx];
-            if (i >= NS && !wait(&sm.empty[s], ((i / NS) & 1) ^ 1)) break;
+            if (r >= NS && !wait(&sm.empty[s], ((r / NS) & 1) ^ 1)) break;
             const bool in_range = page >= 0 && page < geo.num_pages;
             if (lane < ppt && pidx < end_page && !in_range) bad = true;
             const unsigned mask = __ballot_sync(0xffffffffu, in_range);
@@ -223,7 +247,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     ptx::tma_load_2d(kd + kHalfBytes, &kmap, &sm.full[s], 64, row);
                 }
             }
-            issued = i + 1;
+            issued = r + 1;
         }
         if (__any_sync(0xffffffffu, bad) && lane == 0) raise_flag(a.err, KL_FLAG_BAD_PAGE);
         // Drain: copies still in flight must land before the CTA's shared memory goes away.
@@ -242,12 +266,36 @@ __global__ void __launch_bounds__(kThreads, 1)
         constexpr uint32_t idesc_s = ptx::idesc_bf16(128, kN, false, false);
         constexpr uint32_t idesc_o = ptx::idesc_bf16(128, kN, true, true);
         const uint32_t qr_addr = ptx::smem_addr(sm.qr);
-        bool ok = wait(&sm.qr_full, 0);
+        bool ok = true;
+        if (tc_route) {
+            // q_r^T[128 j x 16] = W^R^T (MN-major, from ring slot 0) . q^T (K-major rows of the
+            // q_r buffer), into the columns of O buffer 0, which the first output MMA reuses.
+            constexpr uint32_t idesc_r = ptx::idesc_bf16(128, kN, true, false);
+            ok = wait(&sm.full[0], 0);
+            if (ok) {
+                ptx::tc_fence_after();
+                if (lane == 0) {
+                    const uint32_t wt = ptx::smem_addr(sm.tiles[0][0]);
+#pragma unroll
+                    for (int kk = 0; kk < kD / 16; ++kk) {
+                        const uint32_t qoff = (kk >> 2) * (kN * 128) + (kk & 3) * 32;
+                        ptx::mma_bf16(tmem + 2 * kN,
+                                      ptx::smem_desc(wt + kk * 2048, kHalfBytes, 1024, ptx::kSwizzle128B),
+                                      ptx::smem_desc(qr_addr + qoff, 16, 1024, ptx::kSwizzle128B),
+                                      idesc_r, kk > 0);
+                    }
+                    ptx::mma_commit(&sm.r_full);
+                    ptx::mma_commit(&sm.empty[0]);
+                }
+                __syncwarp();
+            }
+        }
+        ok = ok && wait(&sm.qr_full, 0);
         if (ok) ptx::tc_fence_after();
         for (int i = 0; ok && i <= n_tiles; ++i) {
             if (i < n_tiles) {
-                const int s = i % NS, sb = i & 1;
-                if (!wait(&sm.full[s], (i / NS) & 1)) break;
+                const int s = (i + ro) % NS, sb = i & 1;
+                if (!wait(&sm.full[s], ((i + ro) / NS) & 1)) break;
                 if (i >= 2 && !wait(&sm.s_empty[sb], ((i >> 1) - 1) & 1)) break;
                 ptx::tc_fence_after();
                 if (lane == 0) {
@@ -267,7 +315,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 __syncwarp();
             }
             if (i >= 1) {
-                const int j = i - 1, s = j % NS, pb = j & 1;
+                const int j = i - 1, s = (j + ro) % NS, pb = j & 1;
                 if (!wait(&sm.p_full[pb], (j >> 1) & 1)) break;
                 if (j >= 2 && !wait(&sm.o_empty[pb], ((j >> 1) - 1) & 1)) break;
                 ptx::tc_fence_after();
@@ -308,47 +356,59 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float sl2 = geo.scale * kLog2e;
         bool ok = true;
 
-        // Routing prologue: thread j computes q_r[h][j] for the G heads, fp32.
-        for (int i = t; i < kD * kNG; i += kTile) {
-            const int k = i >> 3, h = i & 7;
-            qf[i] = h < G ? __uint_as_float((uint32_t)a.q[((size_t)b * geo.Hq + g * G + h) * kD + k] << 16)
-                          : 0.f;
-        }
-        __syncwarp();
-        if (lane == 0) ptx::mbar_arrive(&sm.q_ready);
-        ok = wait(&sm.q_ready, 0);
-        if (ok) {
-            float acc[kNG];
+        // Routing prologue: thread j obtains q_r[h][j] for the G heads in fp32 -- from the
+        // routing MMA in TMEM (one W^R per value head), or on CUDA cores (one W^R per query
+        // head), or, for the K+V comparison, the unrouted query itself.
+        float acc[kNG];
 #pragma unroll
-            for (int h = 0; h < kNG; ++h) acc[h] = 0.f;
-            if constexpr (kStandard) {
+        for (int h = 0; h < kNG; ++h) acc[h] = 0.f;
+        if (tc_route) {
+            ok = wait(&sm.r_full, 0);
+            if (ok) {
+                ptx::tc_fence_after();
+                float rv[16];
+                ptx::tmem_ld16(tmem + 2 * kN + lane_base, rv);
+                ptx::tc_fence_before();
 #pragma unroll
-                for (int h = 0; h < kNG; ++h) acc[h] = qf[t * kNG + h];
-            } else if (!geo.wr_per_qh) {
-                const uint16_t *W = a.w_r + (size_t)g * kD * kD + t;
-#pragma unroll 4
-                for (int k = 0; k < kD; ++k) {
-                    const float w = __uint_as_float((uint32_t)W[(size_t)k * kD] << 16);
-                    const float4 q0 = *reinterpret_cast<const float4 *>(qf + k * kNG);
-                    const float4 q1 = *reinterpret_cast<const float4 *>(qf + k * kNG + 4);
-                    acc[0] = fmaf(q0.x, w, acc[0]); acc[1] = fmaf(q0.y, w, acc[1]);
-                    acc[2] = fmaf(q0.z, w, acc[2]); acc[3] = fmaf(q0.w, w, acc[3]);
-                    acc[4] = fmaf(q1.x, w, acc[4]); acc[5] = fmaf(q1.y, w, acc[5]);
-                    acc[6] = fmaf(q1.z, w, acc[6]); acc[7] = fmaf(q1.w, w, acc[7]);
-                }
-            } else {
+                for (int h = 0; h < kNG; ++h) acc[h] = h < G ? rv[h] : 0.f;
+                // the q rows in the q_r buffer were read by the routing MMA; now overwrite them
+                ptx::fence_proxy_async_smem();
+            }
+        } else {
+            for (int i = t; i < kD * kNG; i += kTile) {
+                const int k = i >> 3, h = i & 7;
+                qf[i] = h < G ? __uint_as_float(
+                                    (uint32_t)a.q[((size_t)b * geo.Hq + g * G + h) * kD + k] << 16)
+                              : 0.f;
+            }
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&sm.q_ready);
+            ok = wait(&sm.q_ready, 0);
+            if (ok) {
+                if constexpr (kStandard) {
 #pragma unroll
-                for (int h = 0; h < kNG; ++h) {
-                    if (h < G) {
-                        const uint16_t *W = a.w_r + (size_t)(g * G + h) * kD * kD + t;
-                        float s = 0.f;
-#pragma unroll 8
-                        for (int k = 0; k < kD; ++k)
-                            s = fmaf(qf[k * kNG + h], __uint_as_float((uint32_t)W[(size_t)k * kD] << 16), s);
-                        acc[h] = s;
+                    for (int h = 0; h < kNG; ++h) acc[h] = qf[t * kNG + h];
+                } else {
+#pragma unroll
+                    for (int h = 0; h < kNG; ++h) {
+                        if (h < G) {
+                            const uint16_t *W = a.w_r + (size_t)(g * G + h) * kD * kD + t;
+                            float sum = 0.f;
+                            for (int k0 = 0; k0 < kD; k0 += 32) {
+                                uint32_t w[32];
+#pragma unroll
+                                for (int u = 0; u < 32; ++u) w[u] = W[(size_t)(k0 + u) * kD];
+#pragma unroll
+                                for (int u = 0; u < 32; ++u)
+                                    sum = fmaf(qf[(k0 + u) * kNG + h], __uint_as_float(w[u] << 16), sum);
+                            }
+                            acc[h] = sum;
+                        }
                     }
                 }
             }
+        }
+        if (ok) {
             // split-bf16 operand rows: n = h (hi), n = 8 + h (lo); column k = t
 #pragma unroll
             for (int h = 0; h < kNG; ++h) {
@@ -448,8 +508,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             // Rows past the end inside the last 16-token MMA step must be finite: zero them.
             if (nvalid < kTile) {
-                const int st = i % NS;
-                if (wait(&sm.full[st], (i / NS) & 1) && t >= nvalid && t < ((nvalid + 15) & ~15)) {
+                const int st = (i + ro) % NS;
+                if (wait(&sm.full[st], ((i + ro) / NS) & 1) && t >= nvalid && t < ((nvalid + 15) & ~15)) {
                     uint4 *r0 = reinterpret_cast<uint4 *>(sm.tiles[st][0] + t * 128);
                     uint4 *r1 = reinterpret_cast<uint4 *>(sm.tiles[st][0] + kHalfBytes + t * 128);
 #pragma unroll
@@ -528,14 +588,14 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     return fn;
 }
 
-// Tensor map of a paged cache viewed as [num_pages * Hkv * P rows][128 dims] bf16; one box is
-// one page of one head, 64 dims wide (one 128-byte swizzle span).
-bool make_cache_map(CUtensorMap *map, const void *base, const Geometry &g) {
+// 2-D bf16 tensor map over `rows` rows of 128 dims (256-byte rows), box = 64 dims x box_rows
+// (one 128-byte swizzle span), 128-byte swizzle.
+bool make_map(CUtensorMap *map, const void *base, uint64_t rows, uint32_t box_rows) {
     auto fn = encode_fn();
     if (!fn) return false;
-    const cuuint64_t dims[2] = {(cuuint64_t)kD, (cuuint64_t)g.num_pages * g.Hkv * g.P};
+    const cuuint64_t dims[2] = {(cuuint64_t)kD, (cuuint64_t)rows};
     const cuuint64_t strides[1] = {(cuuint64_t)kD * 2};
-    const cuuint32_t box[2] = {64, (cuuint32_t)g.P};
+    const cuuint32_t box[2] = {64, box_rows};
     const cuuint32_t estr[2] = {1, 1};
     return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides,
               box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -545,12 +605,18 @@ bool make_cache_map(CUtensorMap *map, const void *base, const Geometry &g) {
 template <bool kStandard>
 cudaError_t launch(const DecodeArgs &a) {
     const Geometry &g = a.geo;
-    CUtensorMap vmap, kmap;
-    if (!make_cache_map(&vmap, a.v_cache, g)) return cudaErrorInvalidValue;
-    if (kStandard) {
-        if (!make_cache_map(&kmap, a.k_cache, g)) return cudaErrorInvalidValue;
-    } else {
-        kmap = vmap;
+    // cache viewed as [num_pages * Hkv * P rows][128]; one box = one page of one head
+    const uint64_t cache_rows = (uint64_t)g.num_pages * g.Hkv * g.P;
+    CUtensorMap vmap, kmap, wmap, qmap;
+    if (!make_map(&vmap, a.v_cache, cache_rows, (uint32_t)g.P)) return cudaErrorInvalidValue;
+    kmap = wmap = qmap = vmap;
+    if (kStandard && !make_map(&kmap, a.k_cache, cache_rows, (uint32_t)g.P))
+        return cudaErrorInvalidValue;
+    if (!kStandard && !g.wr_per_qh) {
+        // W^R [Hkv * 128 rows (k)][128 (j)], one box = one 64-column half of one matrix;
+        // q [B * Hq rows][128], one box = the G rows of one value group.
+        if (!make_map(&wmap, a.w_r, (uint64_t)g.Hkv * kD, kD)) return cudaErrorInvalidValue;
+        if (!make_map(&qmap, a.q, (uint64_t)g.B * g.Hq, (uint32_t)g.G)) return cudaErrorInvalidValue;
     }
     const size_t smem = sizeof(Smem<kStandard>) + 1024;
     static bool configured = false;
@@ -560,7 +626,8 @@ cudaError_t launch(const DecodeArgs &a) {
         if (e != cudaSuccess) return e;
         configured = true;
     }
-    decode_tc_kernel<kStandard><<<dim3(g.S, g.Hkv, g.B), kThreads, smem, a.stream>>>(vmap, kmap, a);
+    decode_tc_kernel<kStandard><<<dim3(g.S, g.Hkv, g.B), kThreads, smem, a.stream>>>(vmap, kmap, wmap,
+                                                                                    qmap, a);
     return cudaGetLastError();
 }
 

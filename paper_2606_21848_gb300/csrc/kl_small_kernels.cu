@@ -50,44 +50,77 @@ __global__ void route_kernel(int Hq, int G, int D, int wr_per_qh, const uint16_t
     q_r[row + j] = acc;
 }
 
-// Combine: one CTA per (h, b); thread j merges column j of the S split states.
-__global__ void combine_kernel(int Hq, int D, int S, const float *__restrict__ part_o,
-                               const float2 *__restrict__ part_ml, void *out, int out_fp32) {
-    __shared__ float red[4];
-    const int h = blockIdx.x, b = blockIdx.y, j = threadIdx.x;
+// Combine: one CTA of 4 warps per (h, b). The split weights w_s = l_s exp(m_s - M) are formed
+// once in shared memory; then warp w folds the states s = w, w + 4, ... (each lane 4 dims of
+// one state row, float4 loads), and the four warp sums are added and normalized.
+constexpr int kCombineWarps = 4;
+constexpr int kCombineMaxSplits = 1024;
+
+__global__ void __launch_bounds__(kCombineWarps * 32)
+    combine_kernel(int Hq, int D, int S, const float *__restrict__ part_o,
+                   const float2 *__restrict__ part_ml, void *out, int out_fp32) {
+    __shared__ float w_s[kCombineMaxSplits];
+    __shared__ float red[kCombineWarps];
+    __shared__ float4 acc_s[kCombineWarps][32];
+    const int h = blockIdx.x, b = blockIdx.y;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const size_t bh = (size_t)b * Hq + h;
     const float2 *ml = part_ml + bh * S;
 
     float M = -INFINITY;
-    for (int s = j; s < S; s += blockDim.x) {
+    for (int s = tid; s < S; s += blockDim.x) {
         const float2 v = ml[s];
         if (v.y > 0.f) M = fmaxf(M, v.x);
     }
     for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-    if ((j & 31) == 0) red[j >> 5] = M;
+    if (lane == 0) red[warp] = M;
     __syncthreads();
-    M = red[0];
-    for (int w = 1; w < (int)(blockDim.x >> 5); ++w) M = fmaxf(M, red[w]);
+    M = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
+    __syncthreads();
 
-    float res = 0.f;
-    if (M != -INFINITY) {
-        float z = 0.f, acc = 0.f;
-        const float *po = part_o + bh * S * D + j;
-        for (int s = 0; s < S; ++s) {
-            const float2 v = ml[s];
-            if (v.y > 0.f) {
-                const float w = v.y * expf(v.x - M);
-                z += w;
-                acc = fmaf(w, po[(size_t)s * D], acc);
+    float z = 0.f;
+    for (int s = tid; s < S; s += blockDim.x) {
+        const float2 v = ml[s];
+        const float w = (v.y > 0.f && M != -INFINITY) ? v.y * expf(v.x - M) : 0.f;
+        w_s[s] = w;
+        z += w;
+    }
+    for (int o = 16; o > 0; o >>= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
+    if (lane == 0) red[warp] = z;
+    __syncthreads();
+    z = red[0] + red[1] + red[2] + red[3];
+
+    // D / 4 lanes hold 4 dims each (D = 128: all 32 lanes; D = 64: 16 lanes)
+    const int nl = D / 4;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (lane < nl) {
+        const float4 *po = reinterpret_cast<const float4 *>(part_o + bh * S * D) + lane;
+#pragma unroll 4
+        for (int s = warp; s < S; s += kCombineWarps) {
+            const float w = w_s[s];
+            if (w != 0.f) {
+                const float4 v = po[(size_t)s * nl];
+                acc.x = fmaf(w, v.x, acc.x);
+                acc.y = fmaf(w, v.y, acc.y);
+                acc.z = fmaf(w, v.z, acc.z);
+                acc.w = fmaf(w, v.w, acc.w);
             }
         }
-        res = acc / z;
     }
-    const size_t oi = bh * D + j;
-    if (out_fp32)
-        static_cast<float *>(out)[oi] = res;
-    else
-        static_cast<__nv_bfloat16 *>(out)[oi] = __float2bfloat16_rn(res);
+    acc_s[warp][lane] = acc;
+    __syncthreads();
+    if (tid < D) {
+        const int l = tid >> 2, c = tid & 3;
+        float r = 0.f;
+#pragma unroll
+        for (int w = 0; w < kCombineWarps; ++w) r += reinterpret_cast<const float *>(&acc_s[w][l])[c];
+        r = z > 0.f ? r / z : 0.f;
+        const size_t oi = bh * D + tid;
+        if (out_fp32)
+            static_cast<float *>(out)[oi] = r;
+        else
+            static_cast<__nv_bfloat16 *>(out)[oi] = __float2bfloat16_rn(r);
+    }
 }
 
 }  // namespace
@@ -113,7 +146,8 @@ cudaError_t launch_combine(int B, int Hq, int D, int S, const float *part_o,
                            const float *part_ml, void *out, kl_dtype out_dtype,
                            cudaStream_t stream) {
     if (B == 0) return cudaSuccess;
-    combine_kernel<<<dim3(Hq, B), D, 0, stream>>>(Hq, D, S, part_o,
+    if (S > kCombineMaxSplits) return cudaErrorInvalidValue;
+    combine_kernel<<<dim3(Hq, B), kCombineWarps * 32, 0, stream>>>(Hq, D, S, part_o,
                                                  reinterpret_cast<const float2 *>(part_ml), out,
                                                  out_dtype == KL_FP32);
     return cudaGetLastError();
