@@ -1,8 +1,9 @@
 """Benchmark of one keyless decode step (append + decode attention) on GB300.
 
-A step is one pass of the whole hot path over one batch: kl_append_v writes the current
-token's value rows into the paged Value-Only Cache, then kl_decode_attention runs the routed
-decode (fused routing prologue, split-sequence decode, cross-split combine). Inputs are
+A step is one pass of the whole hot path over one batch: kl_decode_step appends the current
+token's value rows to the paged Value-Only Cache and runs the routed decode (routing prologue,
+split-sequence decode, cross-split merge) -- one kernel when the splits merge inside a
+thread-block cluster, else the decode kernel plus the combine kernel. Inputs are
 seeded synthetic tensors with the shapes of the selected workload, resident in HBM before the
 timed region; L2 is flushed between timed steps (a 512 MiB write, then a read of it, so the
 lines left in L2 are clean).
@@ -160,7 +161,9 @@ def algorithmic_bytes(x, standard: bool) -> dict:
     q = B * Hq * D * 2
     out = B * Hq * D * 2
     bt = sum(math.ceil(int(L) / P) for L in x["seq_lens"].tolist()) * 4 + B * 4
-    return {"cache": cache, "wr": wr, "total": cache + wr + q + out + bt, "tokens": tokens}
+    append = 0 if standard else 2 * B * Hkv * D * 2     # v_new read + cache row written
+    return {"cache": cache, "wr": wr, "total": cache + wr + q + out + bt + append,
+            "tokens": tokens}
 
 
 # ----------------------------------------------------------------------------- CPU arm --
@@ -271,7 +274,7 @@ def run_ours(args):
     out = torch.empty(B, Hq, D, dtype=torch.bfloat16, device=dev)
     part_o = torch.empty(B, Hq, S, D, dtype=torch.float32, device=dev)
     part_ml = torch.empty(B, Hq, S, 2, dtype=torch.float32, device=dev)
-    ws = torch.empty(max(256, kl.kl_decode_workspace_size(sh, splits_req)), dtype=torch.uint8,
+    ws = torch.zeros(max(256, kl.kl_decode_workspace_size(sh, splits_req)), dtype=torch.uint8,
                      device=dev)
     err = torch.zeros(1, dtype=torch.int32, device=dev)
     flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
@@ -285,51 +288,44 @@ def run_ours(args):
 
     stream = torch.cuda.current_stream(dev)
     opts_states = kl.decode_options(S, kernel, part_o, part_ml)
-    opts_full = kl.decode_options(splits_req, kernel)
+    opts_full = kl.decode_options(S, kernel)
 
-    def decode_states():
+    tc = kernel != kl.KL_KERNEL_SIMT and kl.kl_decode_kernel_available(sh, kl.KL_KERNEL_TENSOR,
+                                                                      args.standard)
+    # the merge happens inside the decode kernel when its ring can stage the split states
+    one_kernel = S == 1 or (tc and (Hq // Hkv) * S * (D * 4 + 12) <= 3 * 32768 * (2 if args.standard else 1))
+
+    def decode_call(opts, o, w):
         if args.standard:
             kl.kl_standard_decode(sh, g["q"], k_cache, g["v_cache"], g["block_table"],
-                                  g["seq_lens"], opts_states, None, kl.KL_BF16, None, err, stream)
+                                  g["seq_lens"], opts, o, kl.KL_BF16, w, err, stream)
         else:
-            kl.kl_decode_attention_ex(sh, g["q"], g["w_r"], g["v_cache"], g["block_table"],
-                                      g["seq_lens"], opts_states, None, kl.KL_BF16, None, err,
-                                      stream)
-
-    def decode_direct():
-        # S == 1: the production call writes the output itself (one kernel, no combine)
-        if args.standard:
-            kl.kl_standard_decode(sh, g["q"], k_cache, g["v_cache"], g["block_table"],
-                                  g["seq_lens"], opts_full, out, kl.KL_BF16, ws, err, stream)
-        else:
-            kl.kl_decode_attention(sh, g["q"], g["w_r"], g["v_cache"], g["block_table"],
-                                   g["seq_lens"], splits_req, out, kl.KL_BF16, ws, err, stream)
+            kl.kl_decode_step(sh, g["q"], g["w_r"], g["v_new"], g["positions"], g["v_cache"],
+                              g["block_table"], g["seq_lens"], opts, o, kl.KL_BF16, w, err,
+                              stream)
 
     def step_timed(ev):
-        # append | decode kernel | combine, each bracketed by events on the launching stream;
-        # the kernels are the ones kl_decode_attention launches, called one by one
+        # [append +] decode kernel | combine, bracketed by events on the launching stream; the
+        # kernels are the ones kl_decode_step launches (the K+V comparison appends nothing)
         ev[0].record(stream)
-        kl.kl_append_v(sh, g["v_new"], g["block_table"], g["positions"], g["v_cache"], err,
-                       stream)
-        ev[1].record(stream)
-        if S == 1:
-            decode_direct()
-            ev[2].record(stream)
+        if one_kernel:
+            decode_call(opts_full, out, ws)
+            ev[1].record(stream)
         else:
-            decode_states()
-            ev[2].record(stream)
+            decode_call(opts_states, None, None)
+            ev[1].record(stream)
             kl.kl_combine(sh, part_o, part_ml, S, out, kl.KL_BF16, stream)
-        ev[3].record(stream)
+        ev[2].record(stream)
 
-    launches_per_step = 2 if S == 1 else 3
+    launches_per_step = 1 if one_kernel else 2
     E = lambda: torch.cuda.Event(enable_timing=True)
     for _ in range(args.warmup):
         flush_l2()
-        step_timed([E() for _ in range(4)])
+        step_timed([E() for _ in range(3)])
     torch.cuda.synchronize()
     assert int(err.item()) == 0, f"device error flags {int(err.item())}"
 
-    evs = [[E() for _ in range(4)] for _ in range(args.steps)]
+    evs = [[E() for _ in range(3)] for _ in range(args.steps)]
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
@@ -340,10 +336,9 @@ def run_ours(args):
         torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
-    step_ms = [e[0].elapsed_time(e[3]) for e in evs]
-    dec_ms = [e[1].elapsed_time(e[2]) for e in evs]
-    app_ms = [e[0].elapsed_time(e[1]) for e in evs]
-    comb_ms = [e[2].elapsed_time(e[3]) for e in evs]
+    step_ms = [e[0].elapsed_time(e[2]) for e in evs]
+    dec_ms = [e[0].elapsed_time(e[1]) for e in evs]
+    comb_ms = [e[1].elapsed_time(e[2]) for e in evs]
     mean_step = statistics.mean(step_ms)
     mean_dec = statistics.mean(dec_ms)
     if world > 1:
@@ -371,16 +366,14 @@ def run_ours(args):
         def e2e_step():
             for k in h_in:
                 d_in[k].copy_(h_in[k], non_blocking=True)
-            kl.kl_append_v(sh, d_in["v_new"], d_in["block_table"], d_in["positions"],
-                           g["v_cache"], err, stream)
             if args.standard:
                 kl.kl_standard_decode(sh, d_in["q"], k_cache, g["v_cache"], d_in["block_table"],
                                       d_in["seq_lens"], opts_full, out, kl.KL_BF16, ws, err,
                                       stream)
             else:
-                kl.kl_decode_attention(sh, d_in["q"], g["w_r"], g["v_cache"], d_in["block_table"],
-                                       d_in["seq_lens"], splits_req, out, kl.KL_BF16, ws, err,
-                                       stream)
+                kl.kl_decode_step(sh, d_in["q"], g["w_r"], d_in["v_new"], d_in["positions"],
+                                  g["v_cache"], d_in["block_table"], d_in["seq_lens"], opts_full,
+                                  out, kl.KL_BF16, ws, err, stream)
             h_out.copy_(out, non_blocking=True)
 
         for _ in range(args.warmup):
@@ -415,9 +408,7 @@ def run_ours(args):
                "sample": f"{n} whole sequences of {wl.name} (all {Hq} heads, decode only, "
                          f"fp64) in {el:.1f}s"}
 
-    kname = "tensor" if kernel == kl.KL_KERNEL_TENSOR or (
-        kernel == kl.KL_KERNEL_AUTO and kl.kl_decode_kernel_available(sh, kl.KL_KERNEL_TENSOR,
-                                                                       args.standard)) else "simt"
+    kname = "tensor" if tc else "simt"
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": mean_step,
@@ -432,8 +423,8 @@ def run_ours(args):
                    "parallelism": f"replicas x{world}"},
         "hbm_gbs_step": step_gbs,
         "pct_of_8tbs_step": 100.0 * step_gbs / NOMINAL_HBM_GBS,
-        "ms_breakdown": {"append": statistics.mean(app_ms), "decode": mean_dec,
-                         "combine": statistics.mean(comb_ms)},
+        "ms_breakdown": {"decode": mean_dec, "combine": statistics.mean(comb_ms)},
+        "kernels_per_step": launches_per_step,
         "roofline": {"bound": "hbm", "achieved": dec_gbs, "peak": peak, "unit": "GB/s",
                      "frac": dec_gbs / peak, "peak_kind": peak_kind,
                      "pct_of_8tbs": 100.0 * dec_gbs / NOMINAL_HBM_GBS,

@@ -112,8 +112,14 @@ kl_status kl_append_v(const kl_shape *shape, const void *v_new, const int32_t *b
                       kl_stream_t stream);
 
 /*
- * Bytes of device workspace kl_decode_attention / kl_standard_decode need for `num_splits`
- * (0 = the automatic choice); 0 when no workspace is needed. Returns 0 on invalid shapes.
+ * Bytes of device workspace kl_decode_attention / kl_decode_step / kl_standard_decode need for
+ * `num_splits` (0 = the automatic choice); 0 when no workspace is needed (one split). Returns
+ * 0 on invalid shapes. The workspace holds the split states and, for the tensor-core kernel,
+ * one merge counter per (sequence, value head): it must be zero-filled (cudaMemsetAsync)
+ * before its first use. Every call leaves the counters at zero again, so the workspace can
+ * be reused across calls and shapes -- except after a call that raised KL_FLAG_TIMEOUT,
+ * which may leave counters behind: zero the workspace again then. Calls that share a
+ * workspace must not overlap on the GPU.
  */
 size_t kl_decode_workspace_size(const kl_shape *shape, int32_t num_splits);
 
@@ -130,15 +136,33 @@ int32_t kl_decode_num_splits(const kl_shape *shape, int32_t num_splits);
  * q: [B][Hq][D] bf16; w_r: [Hw][D][D] bf16; v_cache: [num_pages][Hkv][P][D] bf16;
  * block_table: [B][max_pages_per_seq] int32; seq_lens: [B] int32; out: [B][Hq][D] of
  * `out_dtype`. The sequence is cut into `num_splits` chunks processed in parallel and merged
- * as in kl_combine; `workspace` must hold kl_decode_workspace_size(shape, num_splits) bytes
- * (256-byte aligned). A bad page id or length raises its flag and leaves that output
- * unspecified.
+ * as in kl_combine (by the last chunk of each sequence to finish, or by a second kernel);
+ * `workspace` must hold kl_decode_workspace_size(shape, num_splits) bytes (256-byte aligned,
+ * zero-filled before its first use). A bad page id or length raises its flag and leaves that
+ * output unspecified.
  */
 kl_status kl_decode_attention(const kl_shape *shape, const void *q, const void *w_r,
                               const void *v_cache, const int32_t *block_table,
                               const int32_t *seq_lens, int32_t num_splits, void *out,
                               kl_dtype out_dtype, void *workspace, size_t workspace_bytes,
                               int32_t *err, kl_stream_t stream);
+
+/*
+ * One whole decode step in one pass: the Value-Only Cache append of the current token
+ * (Section 3: V holds the rows of the earlier steps and the row obtained at the current step)
+ * followed by the keyless decode over the n+1 rows, i.e. kl_append_v then
+ * kl_decode_attention_ex, fused: the decode CTA whose split holds row positions[b] writes
+ * v_new[b][g] there before reading it, so the new row never makes a separate round trip.
+ * v_new: [B][Hkv][D] bf16; positions: [B] int32 (normally seq_lens[b] - 1); v_cache is
+ * written in place. Other arguments, layouts and flags as in kl_append_v and
+ * kl_decode_attention_ex.
+ */
+kl_status kl_decode_step(const kl_shape *shape, const void *q, const void *w_r,
+                         const void *v_new, const int32_t *positions, void *v_cache,
+                         const int32_t *block_table, const int32_t *seq_lens,
+                         const kl_decode_options *opts, void *out, kl_dtype out_dtype,
+                         void *workspace, size_t workspace_bytes, int32_t *err,
+                         kl_stream_t stream);
 
 /* kl_decode_attention with an explicit kernel choice (opts may be NULL = defaults). */
 kl_status kl_decode_attention_ex(const kl_shape *shape, const void *q, const void *w_r,

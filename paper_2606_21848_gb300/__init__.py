@@ -11,7 +11,7 @@ from ._lib import (  # noqa: F401
     KL_ERR_CUDA, KL_ERR_INVALID_ARG, KL_ERR_UNSUPPORTED, KL_ERR_WORKSPACE,
     KL_FLAG_BAD_LENGTH, KL_FLAG_BAD_PAGE, KL_FLAG_BAD_POSITION, KL_FLAG_TIMEOUT,
     KLError, decode_options, kl_append_v, kl_combine, kl_decode_attention, kl_decode_attention_ex,
-    kl_decode_attention_noalloc, kl_decode_kernel_available, KL_NOALLOC_SCRATCH_BYTES,
+    kl_decode_attention_noalloc, kl_decode_kernel_available, kl_decode_step, KL_NOALLOC_SCRATCH_BYTES,
     kl_decode_num_splits, kl_decode_options, kl_decode_workspace_size, kl_route_query,
     kl_shape, kl_standard_decode, kl_status_string, load, make_shape,
 )

@@ -70,6 +70,7 @@ def load() -> ctypes.CDLL:
         "kl_decode_attention_ex": ([SH, P, P, P, P, P, OP, P, I32, P, SZ, P, P], I32),
         "kl_combine": ([SH, P, P, I32, P, I32, P], I32),
         "kl_standard_decode": ([SH, P, P, P, P, P, OP, P, I32, P, SZ, P, P], I32),
+        "kl_decode_step": ([SH, P, P, P, P, P, P, P, OP, P, I32, P, SZ, P, P], I32),
         "kl_decode_attention_noalloc": ([SH, P, P, P, P, P, I32, P, I32, P, P], I32),
         "kl_decode_kernel_available": ([SH, I32, I32], I32),
         "kl_status_string": ([I32], ctypes.c_char_p),
@@ -160,6 +161,16 @@ def kl_decode_attention_ex(shape, q, w_r, v_cache, block_table, seq_lens, opts, 
                                          None if opts is None else ctypes.byref(opts), _p(out),
                                          out_dtype, _p(workspace), _nbytes(workspace), _p(err),
                                          _stream(stream)), "kl_decode_attention_ex")
+
+
+def kl_decode_step(shape, q, w_r, v_new, positions, v_cache, block_table, seq_lens, opts, out,
+                   out_dtype, workspace, err=None, stream=None):
+    """Append of the current token's rows fused with the keyless decode (one pass)."""
+    _check(load().kl_decode_step(ctypes.byref(shape), _p(q), _p(w_r), _p(v_new), _p(positions),
+                                 _p(v_cache), _p(block_table), _p(seq_lens),
+                                 None if opts is None else ctypes.byref(opts), _p(out),
+                                 out_dtype, _p(workspace), _nbytes(workspace), _p(err),
+                                 _stream(stream)), "kl_decode_step")
 
 
 def kl_combine(shape, partial_o, partial_ml, num_splits, out, out_dtype, stream=None):

@@ -57,10 +57,12 @@ kl_status resolve(const kl_shape *s, int32_t num_splits, Geometry *g) {
     const int64_t Lmax = (int64_t)g->max_pages * g->P;
     int64_t S = num_splits;
     if (S == 0) {
-        // Enough (split, value head, sequence) items to fill every SM about twice, and splits
-        // of at most 8192 tokens so that ragged batches balance; never below 256 tokens.
+        // As many splits as fit one wave of two CTAs per SM over the (value head, sequence)
+        // units, and splits of at most 8192 tokens so that ragged batches balance; never
+        // below 256 tokens per split.
         const int64_t units = (int64_t)(g->B > 0 ? g->B : 1) * g->Hkv;
-        const int64_t fill = (2 * (int64_t)device_sm_count() + units - 1) / units;
+        const int64_t slots = 2 * (int64_t)device_sm_count();
+        const int64_t fill = units < slots ? slots / units : 1;
         const int64_t cap = (Lmax + 8191) / 8192;
         S = fill > cap ? fill : cap;
         const int64_t smax = (Lmax + 255) / 256;
@@ -77,16 +79,18 @@ kl_status resolve(const kl_shape *s, int32_t num_splits, Geometry *g) {
 }
 
 struct WorkspaceLayout {
-    size_t part_o, part_ml, total;
+    size_t part_o, part_ml, counters, total;
 };
 
+// [B][Hq][S][D] fp32 states, [B][Hq][S][2] fp32 {m, l}, [B][Hkv] u32 merge counters.
 WorkspaceLayout layout(const Geometry &g) {
-    WorkspaceLayout w{0, 0, 0};
+    WorkspaceLayout w{0, 0, 0, 0};
     if (g.S <= 1) return w;
     const size_t rows = (size_t)g.B * g.Hq * g.S;
     w.part_o = 0;
     w.part_ml = round_up(rows * g.D * sizeof(float), 256);
-    w.total = w.part_ml + round_up(rows * 2 * sizeof(float), 256);
+    w.counters = w.part_ml + round_up(rows * 2 * sizeof(float), 256);
+    w.total = w.counters + round_up((size_t)g.B * g.Hkv * sizeof(unsigned int), 256);
     return w;
 }
 
@@ -96,7 +100,8 @@ kl_status decode_common(bool standard, const kl_shape *shape, const void *q, con
                         const void *k_cache, const void *v_cache, const int32_t *block_table,
                         const int32_t *seq_lens, const kl_decode_options *opts, void *out,
                         kl_dtype out_dtype, void *workspace, size_t workspace_bytes,
-                        int32_t *err, kl_stream_t stream) {
+                        int32_t *err, kl_stream_t stream, const void *v_new = nullptr,
+                        const int32_t *positions = nullptr) {
     const int32_t ns = opts ? opts->num_splits : 0;
     const int32_t kernel = opts ? opts->kernel : KL_KERNEL_AUTO;
     if (ns < 0 || kernel < KL_KERNEL_AUTO || kernel > KL_KERNEL_SIMT) return KL_ERR_INVALID_ARG;
@@ -129,11 +134,16 @@ kl_status decode_common(bool standard, const kl_shape *shape, const void *q, con
     a.v_cache = static_cast<const uint16_t *>(v_cache);
     a.block_table = block_table;
     a.seq_lens = seq_lens;
+    a.v_new = static_cast<const uint16_t *>(v_new);
+    a.positions = positions;
+    a.cache_rw = static_cast<uint16_t *>(const_cast<void *>(v_cache));
     char *ws = static_cast<char *>(workspace);
     a.part_o = states ? opts->partial_o : wl.total ? reinterpret_cast<float *>(ws + wl.part_o) : nullptr;
     a.part_ml = states ? opts->partial_ml : wl.total ? reinterpret_cast<float *>(ws + wl.part_ml) : nullptr;
     a.out = out;
     a.direct_out = !states && g.S == 1;
+    a.merge_inside = false;
+    a.counters = wl.total ? reinterpret_cast<unsigned int *>(ws + wl.counters) : nullptr;
     a.out_dtype = out_dtype;
     a.err = err;
     a.stream = reinterpret_cast<cudaStream_t>(stream);
@@ -145,6 +155,7 @@ kl_status decode_common(bool standard, const kl_shape *shape, const void *q, con
     } else if (kernel == KL_KERNEL_AUTO) {
         use_tc = tc_supported(g, standard);
     }
+    a.merge_inside = use_tc && !states && tc_merge_inside(g, standard);
     cudaError_t e = use_tc ? launch_decode_tc(a, standard) : launch_decode_simt(a, standard);
     if (e == cudaSuccess) e = finish_decode(a, states);
     return from_cuda(e);
@@ -153,7 +164,7 @@ kl_status decode_common(bool standard, const kl_shape *shape, const void *q, con
 }  // namespace
 
 cudaError_t finish_decode(const DecodeArgs &a, bool states_requested) {
-    if (a.direct_out || states_requested) return cudaSuccess;
+    if (a.direct_out || a.merge_inside || states_requested) return cudaSuccess;
     return launch_combine(a.geo.B, a.geo.Hq, a.geo.D, a.geo.S, a.part_o, a.part_ml, a.out,
                           a.out_dtype, a.stream);
 }
@@ -218,6 +229,19 @@ kl_status kl_decode_attention_ex(const kl_shape *shape, const void *q, const voi
                                  size_t workspace_bytes, int32_t *err, kl_stream_t stream) {
     return decode_common(false, shape, q, w_r, nullptr, v_cache, block_table, seq_lens, opts,
                          out, out_dtype, workspace, workspace_bytes, err, stream);
+}
+
+kl_status kl_decode_step(const kl_shape *shape, const void *q, const void *w_r,
+                         const void *v_new, const int32_t *positions, void *v_cache,
+                         const int32_t *block_table, const int32_t *seq_lens,
+                         const kl_decode_options *opts, void *out, kl_dtype out_dtype,
+                         void *workspace, size_t workspace_bytes, int32_t *err,
+                         kl_stream_t stream) {
+    if (!v_new || !positions) return KL_ERR_INVALID_ARG;
+    if (!aligned(v_new, 16)) return KL_ERR_INVALID_ARG;
+    return decode_common(false, shape, q, w_r, nullptr, v_cache, block_table, seq_lens, opts,
+                         out, out_dtype, workspace, workspace_bytes, err, stream, v_new,
+                         positions);
 }
 
 kl_status kl_standard_decode(const kl_shape *shape, const void *q, const void *k_cache,

@@ -57,6 +57,26 @@ __global__ void __launch_bounds__(kWarps * 32) decode_simt_kernel(DecodeArgs a) 
     const int t0 = split * geo.chunk;
     const int t1 = min(t0 + geo.chunk, L);
 
+    // Fused append (kl_decode_step): the CTA whose split holds row positions[b] writes the
+    // current token's value row there before any row is read.
+    if (a.v_new) {
+        const int pos = a.positions[b];
+        if (pos < 0 || pos >= geo.max_pages * geo.P) {
+            if (tid == 0 && split == 0 && g == 0) raise_flag(a.err, KL_FLAG_BAD_POSITION);
+        } else if (pos / geo.chunk == split) {
+            const int page = a.block_table[(size_t)b * geo.max_pages + pos / geo.P];
+            if (page >= 0 && page < geo.num_pages) {
+                if (tid < D / 8)
+                    reinterpret_cast<uint4 *>(a.cache_rw + (((size_t)page * geo.Hkv + g) * geo.P +
+                                                            pos % geo.P) * D)[tid] =
+                        reinterpret_cast<const uint4 *>(a.v_new + ((size_t)b * geo.Hkv + g) * D)[tid];
+            } else if (tid == 0) {
+                raise_flag(a.err, KL_FLAG_BAD_PAGE);
+            }
+        }
+        __syncthreads();
+    }
+
     // Routed, pre-scaled query of every head of the group.
     for (int i = tid; i < G * D; i += kWarps * 32) {
         const int h = i / D, k = i % D;

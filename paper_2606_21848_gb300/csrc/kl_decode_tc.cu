@@ -64,7 +64,8 @@ struct __align__(1024) Smem {
     float red[2][kComputeWarps][kNG];
     uint64_t full[Cfg<kStandard>::kStages], empty[Cfg<kStandard>::kStages];
     uint64_t s_full[2], s_empty[2], p_full[2], o_full[2], o_empty[2], red_bar[2];
-    uint64_t qr_full, q_ready, r_full, drain;
+    uint64_t qr_full, q_ready, r_full, drain, ep_bar, ep_bar2, ep_bar3, ep_bar4, merge_full;
+    int is_last;
     uint32_t tmem_base;
     int abort;
 };
@@ -111,6 +112,101 @@ __device__ __forceinline__ uint32_t qr_offset(int n, int k) {
            ((kk & 7) << 1);
 }
 
+// Arrival of one split of a (b, g) unit on its counter in the workspace: true for the last of
+// the unit's n splits. The increment wraps the counter back to zero on that arrival, so the
+// workspace is ready for the next call without any reset; one atomic per split, no retry.
+// Acquire-release at GPU scope: it publishes the split state that this CTA's threads wrote
+// before the CTA barrier that precedes it, and, for the last arrival, makes every other
+// split's state visible to the threads that synchronize with this one afterwards.
+__device__ __forceinline__ bool arrive_last(unsigned int *counter, int n) {
+    unsigned int old;
+    asm volatile("atom.acq_rel.gpu.global.inc.u32 %0, [%1], %2;"
+                 : "=r"(old)
+                 : "l"(counter), "r"((unsigned int)(n - 1))
+                 : "memory");
+    return old == (unsigned int)(n - 1);
+}
+
+// Merge of the n_u split states of (b, g) by the compute warps of the CTA that finished last
+// (kl_combine's formula). The cache ring is idle by now: one TMA bulk copy per head brings the
+// n_u normalized state rows into it while the threads gather the {m, l} table; each warp forms
+// the normalized weights of its heads, then thread (head, 4 dims) folds the rows from shared
+// memory.
+template <typename SmemT, typename WaitT>
+__device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int g, int n_u, int t,
+                             int warp, int lane, const WaitT &wait) {
+    const Geometry &geo = a.geo;
+    const int G = geo.G;
+    float *rows = reinterpret_cast<float *>(&sm.tiles[0][0][0]);          // [G][n_u][128]
+    float2 *tab = reinterpret_cast<float2 *>(rows + (size_t)G * n_u * kD);  // [G][n_u] {m, l}
+    float *wt = reinterpret_cast<float *>(tab + G * n_u);                   // [G][n_u] weights
+    const uint32_t row_bytes = (uint32_t)n_u * kD * sizeof(float);
+    if (t == 0) {
+        ptx::fence_proxy_async_global();
+        ptx::mbar_arrive_expect_tx(&sm.merge_full, row_bytes * (uint32_t)G);
+        for (int h = 0; h < G; ++h)
+            ptx::bulk_load(rows + (size_t)h * n_u * kD,
+                           a.part_o + ((size_t)b * geo.Hq + g * G + h) * geo.S * kD, row_bytes,
+                           &sm.merge_full);
+    }
+    const float2 *ml = reinterpret_cast<const float2 *>(a.part_ml);
+    for (int i = t; i < G * n_u; i += kTile) {
+        const int h = i / n_u, j = i - h * n_u;
+        tab[i] = __ldcg(ml + ((size_t)b * geo.Hq + g * G + h) * geo.S + j);
+    }
+    __syncwarp();
+    if (lane == 0) ptx::mbar_arrive(&sm.ep_bar3);
+    if (!wait(&sm.ep_bar3, 0)) return;
+    for (int h = warp; h < G; h += kComputeWarps) {
+        float M = -INFINITY;
+        for (int j = lane; j < n_u; j += 32) {
+            const float2 v = tab[h * n_u + j];
+            if (v.y > 0.f) M = fmaxf(M, v.x);
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+        float z = 0.f;
+        for (int j = lane; j < n_u; j += 32) {
+            const float2 v = tab[h * n_u + j];
+            const float w = (v.y > 0.f && M != -INFINITY) ? v.y * expf(v.x - M) : 0.f;
+            wt[h * n_u + j] = w;
+            z += w;
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) z += __shfl_xor_sync(0xffffffffu, z, off);
+        const float inv = z > 0.f ? 1.f / z : 0.f;
+        for (int j = lane; j < n_u; j += 32) wt[h * n_u + j] *= inv;
+    }
+    __syncwarp();
+    if (lane == 0) ptx::mbar_arrive(&sm.ep_bar4);
+    if (!wait(&sm.ep_bar4, 0)) return;
+    if (!wait(&sm.merge_full, 0)) return;
+    // thread t: head h = t / 32 (+ 4 for the second pass), dims 4 * (t % 32) .. + 3
+    for (int h = warp; h < G; h += kComputeWarps) {
+        const size_t bh = (size_t)b * geo.Hq + g * G + h;
+        const float4 *po = reinterpret_cast<const float4 *>(rows + (size_t)h * n_u * kD) + lane;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+        for (int j = 0; j < n_u; ++j) {
+            const float w = wt[h * n_u + j];
+            if (w != 0.f) {
+                const float4 v = po[(size_t)j * (kD / 4)];
+                acc.x = fmaf(w, v.x, acc.x);
+                acc.y = fmaf(w, v.y, acc.y);
+                acc.z = fmaf(w, v.z, acc.z);
+                acc.w = fmaf(w, v.w, acc.w);
+            }
+        }
+        const size_t oi = bh * kD + 4 * lane;
+        if (a.out_dtype == KL_FP32) {
+            *reinterpret_cast<float4 *>(static_cast<float *>(a.out) + oi) = acc;
+        } else {
+            __nv_bfloat16 *o16 = static_cast<__nv_bfloat16 *>(a.out) + oi;
+            *reinterpret_cast<uint2 *>(o16) = make_uint2(pack_bf16(acc.x, acc.y), pack_bf16(acc.z, acc.w));
+        }
+    }
+}
+
 template <bool kStandard>
 __global__ void __launch_bounds__(kThreads, 1)
     decode_tc_kernel(const __grid_constant__ CUtensorMap vmap,
@@ -141,8 +237,45 @@ __global__ void __launch_bounds__(kThreads, 1)
     const bool tc_route = !kStandard && !geo.wr_per_qh;
     const int ro = tc_route ? 1 : 0;
 
-    // Empty split: a zero output or an empty state, no pipeline.
+    // Fused append: does this CTA own the current token's row of (b, g)?
+    int app_page = -1, app_pos = -1;
+    if (a.v_new) {
+        const int pos = a.positions[b];
+        if (pos < 0 || pos >= geo.max_pages * geo.P) {
+            if (tid == 0 && split == 0 && g == 0) raise_flag(a.err, KL_FLAG_BAD_POSITION);
+        } else if (pos / geo.chunk == split) {
+            const int page = a.block_table[(size_t)b * geo.max_pages + pos / geo.P];
+            if (page >= 0 && page < geo.num_pages) {
+                app_page = page;
+                app_pos = pos;
+            } else if (tid == 0) {
+                raise_flag(a.err, KL_FLAG_BAD_PAGE);
+            }
+        }
+    }
+    const size_t app_off =
+        app_page >= 0 ? (((size_t)app_page * geo.Hkv + g) * geo.P + app_pos % geo.P) * kD : 0;
+
+    // Empty split, no pipeline: in the split-state layout an empty state; otherwise the split
+    // of a zero-length sequence writes the zero output, and the empty splits of a longer
+    // sequence take no part (the merge counts only the splits that hold tokens).
+    if (n_tiles == 0 && a.merge_inside) {
+        if (app_page >= 0 && tid < 32)
+            reinterpret_cast<uint2 *>(a.cache_rw + app_off)[tid] =
+                reinterpret_cast<const uint2 *>(a.v_new + ((size_t)b * geo.Hkv + g) * kD)[tid];
+        if (L == 0 && split == 0 && tid < kD) {
+            for (int h = 0; h < G; ++h) {
+                const size_t oi = ((size_t)b * geo.Hq + g * G + h) * kD + tid;
+                if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[oi] = 0.f;
+                else static_cast<__nv_bfloat16 *>(a.out)[oi] = __float2bfloat16_rn(0.f);
+            }
+        }
+        return;
+    }
     if (n_tiles == 0) {
+        if (app_page >= 0 && tid < 32)
+            reinterpret_cast<uint2 *>(a.cache_rw + app_off)[tid] =
+                reinterpret_cast<const uint2 *>(a.v_new + ((size_t)b * geo.Hkv + g) * kD)[tid];
         if (tid < kD) {
             for (int h = 0; h < G; ++h) {
                 const size_t bh = (size_t)b * geo.Hq + g * G + h;
@@ -178,6 +311,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::mbar_init(&sm.qr_full, kComputeWarps);
         ptx::mbar_init(&sm.q_ready, kComputeWarps);
         ptx::mbar_init(&sm.r_full, 1);
+        ptx::mbar_init(&sm.ep_bar, kComputeWarps);
+        ptx::mbar_init(&sm.ep_bar2, 1);
+        ptx::mbar_init(&sm.ep_bar3, kComputeWarps);
+        ptx::mbar_init(&sm.ep_bar4, kComputeWarps);
+        ptx::mbar_init(&sm.merge_full, 1);
         ptx::mbar_init(&sm.drain, 1);
         sm.abort = 0;
         ptx::fence_mbar_init();
@@ -210,6 +348,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t page_bytes = (uint32_t)P * 128u;   // one half of one page
         bool bad = false;
         int issued = 0;
+        // The new token's row (fused append), 8 bytes per lane, written just before the loads of
+        // the tile that holds it (or first, when it lies past the sequence's end).
+        const int app_tile = app_page < 0 ? -1 : (app_pos < t_end ? (app_pos - t_begin) / kTile : 0);
+        uint2 app_val = make_uint2(0, 0);
+        if (app_page >= 0)
+            app_val = reinterpret_cast<const uint2 *>(a.v_new + ((size_t)b * geo.Hkv + g) * kD)[lane];
         if (tc_route) {
             // ring position 0: W^R[g] as the MN-major A operand [j half][128 k rows][128 B] and
             // the group's query rows as the K-major B operand (rows 0..G-1 of the q_r buffer)
@@ -223,14 +367,30 @@ __global__ void __launch_bounds__(kThreads, 1)
             __syncwarp();
             issued = 1;
         }
+        // Block-table entries of the split, 32 pages per warp load, one batch ahead.
+        const int split_pages = end_page - first_page;
+        int bt_cur = lane < split_pages ? bt[first_page + lane] : -1;
+        int bt_nxt = 32 + lane < split_pages ? bt[first_page + 32 + lane] : -1;
+        int bt_batch = 0;
         for (int i = 0; i < n_tiles; ++i) {
             const int r = i + ro, s = r % NS;
-            const int pidx = first_page + i * ppt + lane;
-            int page = -1;
-            if (lane < ppt && pidx < end_page) page = bt[pidx];
+            const int p0 = i * ppt;                       // first page of the tile in the split
+            if ((p0 >> 5) != bt_batch) {
+                bt_batch = p0 >> 5;
+                bt_cur = bt_nxt;
+                const int q = (bt_batch + 1) * 32 + lane;
+                bt_nxt = q < split_pages ? bt[first_page + q] : -1;
+            }
+            int page = __shfl_sync(0xffffffffu, bt_cur, ((p0 & 31) + lane) & 31);
+            const bool exists = lane < ppt && p0 + lane < split_pages;
             if (r >= NS && !wait(&sm.empty[s], ((r / NS) & 1) ^ 1)) break;
-            const bool in_range = page >= 0 && page < geo.num_pages;
-            if (lane < ppt && pidx < end_page && !in_range) bad = true;
+            const bool in_range = exists && page >= 0 && page < geo.num_pages;
+            if (exists && !in_range) bad = true;
+            if (i == app_tile) {
+                reinterpret_cast<uint2 *>(a.cache_rw + app_off)[lane] = app_val;
+                ptx::fence_proxy_async_global();
+                __syncwarp();
+            }
             const unsigned mask = __ballot_sync(0xffffffffu, in_range);
             if (lane == 0)
                 ptx::mbar_arrive_expect_tx(&sm.full[s], __popc(mask) * page_bytes * 2u *
@@ -541,15 +701,22 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ptx::mbar_arrive(&sm.red_bar[rb]);
             }
             if (wait(&sm.red_bar[rb], (n_tiles >> 1) & 1)) {
+                // splits of this (b, g) that hold tokens; one split writes the output itself
+                const int n_u = (L + geo.chunk - 1) / geo.chunk;
+                const bool write_out = a.direct_out || (a.merge_inside && n_u == 1);
+                float lt[kNG];
+#pragma unroll
+                for (int h = 0; h < kNG; ++h) {
+                    lt[h] = 0.f;
+#pragma unroll
+                    for (int w = 0; w < kComputeWarps; ++w) lt[h] += sm.red[rb][w][h];
+                }
 #pragma unroll
                 for (int h = 0; h < kNG; ++h) {
                     if (h >= G) continue;
-                    float l = 0.f;
-#pragma unroll
-                    for (int w = 0; w < kComputeWarps; ++w) l += sm.red[rb][w][h];
-                    const float val = o[h] / l;
+                    const float val = o[h] / lt[h];
                     const size_t bh = (size_t)b * geo.Hq + g * G + h;
-                    if (a.direct_out) {
+                    if (write_out) {
                         if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * kD + t] = val;
                         else static_cast<__nv_bfloat16 *>(a.out)[bh * kD + t] = __float2bfloat16_rn(val);
                     } else {
@@ -557,8 +724,24 @@ __global__ void __launch_bounds__(kThreads, 1)
                         a.part_o[slot * kD + t] = val;
                         if (t == 0) {
                             a.part_ml[slot * 2] = m[h] * kLn2;
-                            a.part_ml[slot * 2 + 1] = l;
+                            a.part_ml[slot * 2 + 1] = lt[h];
                         }
+                    }
+                }
+                if (a.merge_inside && !write_out) {
+                    // The last split of (b, g) to finish merges the n_u states (as kl_combine).
+                    __syncwarp();
+                    if (lane == 0) ptx::mbar_arrive(&sm.ep_bar);
+                    if (wait(&sm.ep_bar, 0)) {
+                        if (warp == 0) {
+                            if (lane == 0) {
+                                sm.is_last = arrive_last(a.counters + (size_t)b * geo.Hkv + g, n_u) ? 1 : 0;
+                                ptx::mbar_arrive(&sm.ep_bar2);
+                            }
+                            __syncwarp();
+                        }
+                        if (wait(&sm.ep_bar2, 0) && sm.is_last)
+                            merge_states(sm, a, b, g, n_u, t, warp, lane, wait);
                     }
                 }
             }
@@ -626,12 +809,22 @@ cudaError_t launch(const DecodeArgs &a) {
         if (e != cudaSuccess) return e;
         configured = true;
     }
-    decode_tc_kernel<kStandard><<<dim3(g.S, g.Hkv, g.B), kThreads, smem, a.stream>>>(vmap, kmap, wmap,
-                                                                                    qmap, a);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(g.S, g.Hkv, g.B);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = a.stream;
+    return cudaLaunchKernelEx(&cfg, decode_tc_kernel<kStandard>, vmap, kmap, wmap, qmap, a);
 }
 
 }  // namespace
+
+bool tc_merge_inside(const Geometry &g, bool standard) {
+    // the merging CTA stages G * S state rows (512 B), weights and {m, l} (12 B) in its ring
+    const size_t need = (size_t)g.G * g.S * (kD * sizeof(float) + 12);
+    const size_t ring = standard ? sizeof(Smem<true>::tiles) : sizeof(Smem<false>::tiles);
+    return g.S > 1 && need <= ring;
+}
 
 bool tc_supported(const Geometry &g, bool standard) {
     (void)standard;

@@ -29,10 +29,18 @@ struct DecodeArgs {
     const uint16_t *v_cache;  // [num_pages][Hkv][P][D] bf16
     const int32_t *block_table;
     const int32_t *seq_lens;
+    // Fused append (kl_decode_step): when v_new is set, the CTA whose split holds row
+    // positions[b] writes v_new[b][g] there (into cache_rw, the value cache) before it reads it.
+    const uint16_t *v_new;            // [B][Hkv][D] bf16 or nullptr
+    const int32_t *positions;         // [B]
+    uint16_t *cache_rw;
     float *part_o;            // [B][Hq][S][D]   split states (unless direct_out)
     float *part_ml;           // [B][Hq][S][2]
     void *out;                // [B][Hq][D]
     bool direct_out;          // true: S == 1 and the CTA writes `out` itself (no split states)
+    bool merge_inside;        // true: the last split of each (b, g) merges the split states
+                              // into `out` (tensor-core kernel), using the workspace counters
+    unsigned int *counters;   // [B][Hkv] arrivals of the current call (zero between calls)
     kl_dtype out_dtype;
     int32_t *err;
     cudaStream_t stream;
@@ -62,6 +70,8 @@ cudaError_t finish_decode(const DecodeArgs &a, bool states_requested);
 
 // Tensor-core path: whether it supports a geometry, and its launcher.
 bool tc_supported(const Geometry &g, bool standard);
+// Whether the tensor-core kernel can merge this geometry's split states itself.
+bool tc_merge_inside(const Geometry &g, bool standard);
 cudaError_t launch_decode_tc(const DecodeArgs &a, bool standard);
 
 // Number of SMs of the current device (cached per device).

@@ -40,7 +40,7 @@ def decode(g: dict, sh, *, kernel=kl.KL_KERNEL_AUTO, num_splits=0, out_dtype=kl.
     out = torch.full((B, Hq, D), float("nan"), dtype=dt, device=dev())
     err = torch.zeros(1, dtype=torch.int32, device=dev())
     nbytes = kl.kl_decode_workspace_size(sh, num_splits)
-    ws = torch.empty(max(nbytes, 256), dtype=torch.uint8, device=dev())
+    ws = torch.zeros(max(nbytes, 256), dtype=torch.uint8, device=dev())
     opts = kl.decode_options(num_splits, kernel)
     if k_cache is None:
         kl.kl_decode_attention_ex(sh, g["q"], g["w_r"], g["v_cache"], g["block_table"],

@@ -144,13 +144,97 @@ def test_block_table_permutation_is_bit_exact(kname):
     assert torch.equal(out1.cpu(), out2.cpu())
 
 
-def test_kernels_agree_across_split_counts():
+@pytest.mark.parametrize("kname", ["simt", "tensor"])
+def test_split_counts_agree(kname):
+    """S = 1 writes the output directly; 2..8 merge inside a thread-block cluster (tensor-core
+    kernel); larger S go through the combine kernel."""
     x = tiny(B=2, Hq=32, Hkv=8, D=128, P=16, lens=(2000, 4096))
+    k = _kernel_or_skip(kname, x)
     want = oracle_decode(x, _gpu.default_scale(x))
-    for s in (1, 2, 5, 16, 32):
-        out, err = decode(to_dev(x), shape_of(x), kernel=kl.KL_KERNEL_SIMT, num_splits=s)
+    for s in (1, 2, 5, 8, 16, 32):
+        out, err = decode(to_dev(x), shape_of(x), kernel=k, num_splits=s)
         assert err == 0
-        assert_parity(out.cpu().numpy(), want, f"S={s}")
+        assert_parity(out.cpu().numpy(), want, f"{kname} S={s}")
+
+
+@pytest.mark.parametrize("kname", ["simt", "tensor"])
+def test_workspace_reused_across_calls_and_shapes(kname):
+    """One zero-filled workspace serves repeated calls and different shapes (the merge
+    counters are tagged per call), with identical results for identical inputs."""
+    xa = tiny(B=2, Hq=32, Hkv=8, D=128, P=16, lens=(900, 3000), seed=21)
+    xb = tiny(B=3, Hq=16, Hkv=4, D=128, P=16, lens=(129, 2500, 40), seed=22)
+    k = _kernel_or_skip(kname, xa)
+    ws = torch.zeros(1 << 22, dtype=torch.uint8, device=_gpu.dev())
+    outs = []
+    for x, splits in ((xa, 6), (xb, 11), (xa, 6), (xb, 3), (xa, 6)):
+        g = to_dev(x)
+        sh = shape_of(x)
+        assert kl.kl_decode_workspace_size(sh, splits) <= ws.numel()
+        out = torch.full(g["q"].shape, float("nan"), dtype=torch.float32, device=_gpu.dev())
+        err = torch.zeros(1, dtype=torch.int32, device=_gpu.dev())
+        kl.kl_decode_attention_ex(sh, g["q"], g["w_r"], g["v_cache"], g["block_table"],
+                                  g["seq_lens"], kl.decode_options(splits, k), out, kl.KL_FP32,
+                                  ws, err)
+        torch.cuda.synchronize()
+        assert int(err.item()) == 0
+        assert_parity(out.cpu().numpy(), oracle_decode(x, _gpu.default_scale(x)), f"S={splits}")
+        outs.append(out.cpu())
+    assert torch.equal(outs[0], outs[2]) and torch.equal(outs[0], outs[4])
+
+
+def _step(x, kernel, num_splits, out_dtype=kl.KL_FP32):
+    g = to_dev(x)
+    sh = shape_of(x)
+    B, Hq, D = g["q"].shape
+    out = torch.full((B, Hq, D), float("nan"), dtype=torch.float32, device=_gpu.dev())
+    err = torch.zeros(1, dtype=torch.int32, device=_gpu.dev())
+    ws = torch.zeros(max(256, kl.kl_decode_workspace_size(sh, num_splits)), dtype=torch.uint8,
+                     device=_gpu.dev())
+    kl.kl_decode_step(sh, g["q"], g["w_r"], g["v_new"], g["positions"], g["v_cache"],
+                      g["block_table"], g["seq_lens"], kl.decode_options(num_splits, kernel), out,
+                      out_dtype, ws, err)
+    torch.cuda.synchronize()
+    return out.cpu().numpy(), bf16_bits(g["v_cache"].cpu()), int(err.item())
+
+
+@pytest.mark.parametrize("kname", ["simt", "tensor"])
+@pytest.mark.parametrize("splits", [1, 3, 16])
+@pytest.mark.parametrize("where", ["last", "middle", "past_end"])
+def test_fused_decode_step_matches_append_then_decode(kname, splits, where):
+    """kl_decode_step = kl_append_v then decode: cache bit-exact, output at tolerance."""
+    x = tiny(B=3, Hq=32, Hkv=8, D=128, P=16, lens=(1, 700, 2048))
+    k = _kernel_or_skip(kname, x)
+    L = x["seq_lens"]
+    if where == "middle":
+        x["positions"] = (L // 2).to(torch.int32)
+    elif where == "past_end":
+        # past the sequence's end but inside its last allocated page
+        x["positions"] = torch.minimum(L + 5, (L + 15) // 16 * 16 - 1).to(torch.int32)
+    out, cache, err = _step(x, k, splits)
+    assert err == 0
+    want_cache = oracle.append(bf16_bits(x["v_cache"]), bf16_bits(x["v_new"]),
+                               x["block_table"].numpy(), x["positions"].numpy())
+    np.testing.assert_array_equal(cache, want_cache)
+    y = dict(x)
+    y["v_cache"] = torch.from_numpy(want_cache.view(np.int16)).view(torch.bfloat16)
+    assert_parity(out, oracle_decode(y, _gpu.default_scale(x)), f"{kname} {where} S={splits}")
+
+
+@pytest.mark.parametrize("kname", ["simt", "tensor"])
+def test_fused_decode_step_flags_bad_position_and_page(kname):
+    x = tiny(B=3, Hq=16, Hkv=4, D=128, P=16, lens=(40, 90, 130))
+    k = _kernel_or_skip(kname, x)
+    x["positions"] = torch.tensor([39, -3, 129], dtype=torch.int32)
+    x["block_table"][2, 129 // 16] = -1                     # page of sequence 2's new row
+    y = dict(x)
+    y["block_table"] = x["block_table"].clone()
+    before = bf16_bits(x["v_cache"]).copy()
+    _, cache, err = _step(x, k, 1)
+    assert err & kl.KL_FLAG_BAD_POSITION and err & kl.KL_FLAG_BAD_PAGE
+    # only sequence 0's row changed
+    want = oracle.append(before, bf16_bits(x["v_new"])[:1], x["block_table"].numpy()[:1],
+                         x["positions"].numpy()[:1])
+    np.testing.assert_array_equal(cache, want)
 
 
 @pytest.mark.parametrize("kname", ["simt", "tensor"])

@@ -27,7 +27,7 @@ def lib():
 
 def _reference(g, sh, splits):
     out = torch.empty(g["q"].shape, dtype=torch.float32, device="cuda")
-    ws = torch.empty(max(256, kl.kl_decode_workspace_size(sh, splits)), dtype=torch.uint8,
+    ws = torch.zeros(max(256, kl.kl_decode_workspace_size(sh, splits)), dtype=torch.uint8,
                      device="cuda")
     err = torch.zeros(1, dtype=torch.int32, device="cuda")
     kl.kl_decode_attention(sh, g["q"], g["w_r"], g["v_cache"], g["block_table"], g["seq_lens"],
