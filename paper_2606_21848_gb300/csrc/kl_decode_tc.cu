@@ -44,6 +44,38 @@ constexpr uint32_t kTileBytes = kTile * kD * 2;   // 32 KiB per cache tile
 constexpr uint32_t kHalfBytes = kTileBytes / 2;   // one 64-dim half: 128 rows x 128 B
 constexpr uint32_t kTmemCols = 64;                // S: 2 x 16 columns, O: 2 x 16 columns
 constexpr uint64_t kTimeoutNs = 1000000000ull;
+// Named barriers of the 128 compute threads (id 0 is __syncthreads).
+constexpr uint32_t kBarCompute = 1;       // plain sync
+constexpr uint32_t kBarComputeAnd = 2;    // sync + AND of a flag
+
+// Per-head maximum over the 32 lanes of a warp by transposed halving: after the three
+// exchange steps lane l holds one head, h(l) = 4 * bit4 + 2 * bit3 + bit2, reduced over the
+// lanes it shares with 3 others, then two more steps finish it. 9 shuffles instead of 40.
+__device__ __forceinline__ float warp_max8(const float (&x)[8], int lane) {
+    const bool b4 = lane & 16, b3 = lane & 8, b2 = lane & 4;
+    float a4[4], a2[2];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const float send = b4 ? x[j] : x[j + 4];
+        const float keep = b4 ? x[j + 4] : x[j];
+        a4[j] = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, 16));
+    }
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+        const float send = b3 ? a4[j] : a4[j + 2];
+        const float keep = b3 ? a4[j + 2] : a4[j];
+        a2[j] = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, 8));
+    }
+    float a1;
+    {
+        const float send = b2 ? a2[0] : a2[1];
+        const float keep = b2 ? a2[1] : a2[0];
+        a1 = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, 4));
+    }
+    a1 = fmaxf(a1, __shfl_xor_sync(0xffffffffu, a1, 2));
+    a1 = fmaxf(a1, __shfl_xor_sync(0xffffffffu, a1, 1));
+    return a1;
+}
 
 template <bool kStandard>
 struct Cfg {
@@ -63,8 +95,8 @@ struct __align__(1024) Smem {
     uint8_t p[2][kTile * kN * 2];
     float red[2][kComputeWarps][kNG];
     uint64_t full[Cfg<kStandard>::kStages], empty[Cfg<kStandard>::kStages];
-    uint64_t s_full[2], s_empty[2], p_full[2], o_full[2], o_empty[2], red_bar[2];
-    uint64_t qr_full, q_ready, r_full, drain, ep_bar, ep_bar2, ep_bar3, ep_bar4, merge_full;
+    uint64_t s_full[2], s_empty[2], p_full[2], o_full[2], o_empty[2];
+    uint64_t qr_full, q_ready, r_full, drain, merge_full;
     int is_last;
     uint32_t tmem_base;
     int abort;
@@ -154,9 +186,7 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int g, int n
         const int h = i / n_u, j = i - h * n_u;
         tab[i] = __ldcg(ml + ((size_t)b * geo.Hq + g * G + h) * geo.S + j);
     }
-    __syncwarp();
-    if (lane == 0) ptx::mbar_arrive(&sm.ep_bar3);
-    if (!wait(&sm.ep_bar3, 0)) return;
+    ptx::bar_sync(kBarCompute, kTile);
     for (int h = warp; h < G; h += kComputeWarps) {
         float M = -INFINITY;
         for (int j = lane; j < n_u; j += 32) {
@@ -177,10 +207,7 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int g, int n
         const float inv = z > 0.f ? 1.f / z : 0.f;
         for (int j = lane; j < n_u; j += 32) wt[h * n_u + j] *= inv;
     }
-    __syncwarp();
-    if (lane == 0) ptx::mbar_arrive(&sm.ep_bar4);
-    if (!wait(&sm.ep_bar4, 0)) return;
-    if (!wait(&sm.merge_full, 0)) return;
+    if (!ptx::bar_and(kBarComputeAnd, kTile, wait(&sm.merge_full, 0))) return;
     // thread t: head h = t / 32 (+ 4 for the second pass), dims 4 * (t % 32) .. + 3
     for (int h = warp; h < G; h += kComputeWarps) {
         const size_t bh = (size_t)b * geo.Hq + g * G + h;
@@ -306,15 +333,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             ptx::mbar_init(&sm.p_full[i], kComputeWarps);
             ptx::mbar_init(&sm.o_full[i], 1);
             ptx::mbar_init(&sm.o_empty[i], kComputeWarps);
-            ptx::mbar_init(&sm.red_bar[i], kComputeWarps);
         }
         ptx::mbar_init(&sm.qr_full, kComputeWarps);
         ptx::mbar_init(&sm.q_ready, kComputeWarps);
         ptx::mbar_init(&sm.r_full, 1);
-        ptx::mbar_init(&sm.ep_bar, kComputeWarps);
-        ptx::mbar_init(&sm.ep_bar2, 1);
-        ptx::mbar_init(&sm.ep_bar3, kComputeWarps);
-        ptx::mbar_init(&sm.ep_bar4, kComputeWarps);
         ptx::mbar_init(&sm.merge_full, 1);
         ptx::mbar_init(&sm.drain, 1);
         sm.abort = 0;
@@ -583,6 +605,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (lane == 0) ptx::mbar_arrive(&sm.qr_full);
         }
 
+        // every decision below is taken by the four compute warps together
+        ok = ptx::bar_and(kBarComputeAnd, kTile, ok);
+
         float m[kNG], lsum[kNG], o[kNG];
         Heads alpha_prev;
 #pragma unroll
@@ -596,7 +621,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // O accumulation of tile j: o = o * alpha_j + O_j (thread = output dim t).
         auto correct = [&](int j, const Heads alpha) -> bool {
             const int ob = j & 1;
-            if (!wait(&sm.o_full[ob], (j >> 1) & 1)) return false;
+            if (!ptx::bar_and(kBarComputeAnd, kTile, wait(&sm.o_full[ob], (j >> 1) & 1))) return false;
             ptx::tc_fence_after();
             float ov[16];
             ptx::tmem_ld16(tmem + 2 * kN + ob * kN + lane_base, ov);
@@ -610,7 +635,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 
         for (int i = 0; ok && i < n_tiles; ++i) {
             const int sb = i & 1;
-            if (!wait(&sm.s_full[sb], (i >> 1) & 1)) { ok = false; break; }
+            if (!ptx::bar_and(kBarComputeAnd, kTile, wait(&sm.s_full[sb], (i >> 1) & 1))) {
+                ok = false;
+                break;
+            }
             ptx::tc_fence_after();
             float sv[16];
             ptx::tmem_ld16(tmem + sb * kN + lane_base, sv);
@@ -626,18 +654,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 s[h] = (valid && h < G) ? sv[h] + sv[kNG + h] : -INFINITY;
                 mx[h] = s[h];
             }
-            // per-head maximum over the tile's 128 tokens
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1)
-#pragma unroll
-                for (int h = 0; h < kNG; ++h)
-                    mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], off));
-            if (lane == 0) {
-#pragma unroll
-                for (int h = 0; h < kNG; ++h) sm.red[sb][warp][h] = mx[h];
-                ptx::mbar_arrive(&sm.red_bar[sb]);
+            // per-head maximum over the tile's 128 tokens: warp reduce, then across the 4 warps
+            {
+                const float wm = warp_max8(mx, lane);
+                if ((lane & 3) == 0)
+                    sm.red[sb][warp][((lane >> 4) & 1) * 4 + ((lane >> 3) & 1) * 2 + ((lane >> 2) & 1)] = wm;
             }
-            if (!wait(&sm.red_bar[sb], (i >> 1) & 1)) { ok = false; break; }
+            ptx::bar_sync(kBarCompute, kTile);
             Heads alpha;
             float p[kNG];
 #pragma unroll
@@ -669,7 +692,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             // Rows past the end inside the last 16-token MMA step must be finite: zero them.
             if (nvalid < kTile) {
                 const int st = (i + ro) % NS;
-                if (wait(&sm.full[st], ((i + ro) / NS) & 1) && t >= nvalid && t < ((nvalid + 15) & ~15)) {
+                if (ptx::bar_and(kBarComputeAnd, kTile, wait(&sm.full[st], ((i + ro) / NS) & 1)) &&
+                    t >= nvalid && t < ((nvalid + 15) & ~15)) {
                     uint4 *r0 = reinterpret_cast<uint4 *>(sm.tiles[st][0] + t * 128);
                     uint4 *r1 = reinterpret_cast<uint4 *>(sm.tiles[st][0] + kHalfBytes + t * 128);
 #pragma unroll
@@ -694,13 +718,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int off = 16; off > 0; off >>= 1)
 #pragma unroll
                 for (int h = 0; h < kNG; ++h) lsum[h] += __shfl_xor_sync(0xffffffffu, lsum[h], off);
-            const int rb = n_tiles & 1;   // red buffer / phase after the tile loop
+            const int rb = n_tiles & 1;   // red buffer not read by the last tile's exchange
             if (lane == 0) {
 #pragma unroll
                 for (int h = 0; h < kNG; ++h) sm.red[rb][warp][h] = lsum[h];
-                ptx::mbar_arrive(&sm.red_bar[rb]);
             }
-            if (wait(&sm.red_bar[rb], (n_tiles >> 1) & 1)) {
+            ptx::bar_sync(kBarCompute, kTile);
+            {
                 // splits of this (b, g) that hold tokens; one split writes the output itself
                 const int n_u = (L + geo.chunk - 1) / geo.chunk;
                 const bool write_out = a.direct_out || (a.merge_inside && n_u == 1);
@@ -730,19 +754,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 if (a.merge_inside && !write_out) {
                     // The last split of (b, g) to finish merges the n_u states (as kl_combine).
-                    __syncwarp();
-                    if (lane == 0) ptx::mbar_arrive(&sm.ep_bar);
-                    if (wait(&sm.ep_bar, 0)) {
-                        if (warp == 0) {
-                            if (lane == 0) {
-                                sm.is_last = arrive_last(a.counters + (size_t)b * geo.Hkv + g, n_u) ? 1 : 0;
-                                ptx::mbar_arrive(&sm.ep_bar2);
-                            }
-                            __syncwarp();
-                        }
-                        if (wait(&sm.ep_bar2, 0) && sm.is_last)
-                            merge_states(sm, a, b, g, n_u, t, warp, lane, wait);
-                    }
+                    ptx::bar_sync(kBarCompute, kTile);
+                    if (t == 0)
+                        sm.is_last = arrive_last(a.counters + (size_t)b * geo.Hkv + g, n_u) ? 1 : 0;
+                    ptx::bar_sync(kBarCompute, kTile);
+                    if (sm.is_last) merge_states(sm, a, b, g, n_u, t, warp, lane, wait);
                 }
             }
         }
