@@ -14,13 +14,16 @@
 // routed query and of the softmax weights keeps about 16 significant bits where a plain bf16
 // operand would keep 8; the tensor cores have ample headroom for the doubled N.
 //
-// Roles (192 threads):
+// Roles (224 threads, two CTAs per SM):
 //   warps 0-3  compute: routing prologue; per tile read S from TMEM (thread = token), online
 //              softmax in base 2 (per-head running max across the CTA), write P^T to shared
 //              memory; read O from TMEM (thread = output dim) and accumulate with rescaling;
-//              epilogue writes the output or the split state.
+//              epilogue writes the output or the split state, or merges the splits.
 //   warp 4     producer: block-table lookups and TMA loads of (page, head) tiles.
-//   warp 5     MMA issuer (one elected lane) and TMEM owner.
+//   warp 5     score-MMA issuer (one elected lane; also the routing MMA) and TMEM owner.
+//   warp 6     output-MMA issuer. Two issuing threads raise the SM's MMA issue rate (each
+//              small-N tcgen05.mma costs tens of cycles to issue) and keep the output MMA of
+//              one tile from waiting behind the score MMA of the next.
 // Every wait is bounded (about one second); a wait that runs out raises KL_FLAG_TIMEOUT,
 // makes every role leave its loop, drains outstanding copies and MMAs and frees TMEM.
 #include <cudaTypedefs.h>
@@ -38,8 +41,9 @@ constexpr int kNG = 8;                      // query heads per value group (padd
 constexpr int kN = 2 * kNG;                 // MMA N: hi and lo halves
 constexpr int kComputeWarps = 4;
 constexpr int kProducerWarp = 4;
-constexpr int kMmaWarp = 5;
-constexpr int kThreads = 6 * 32;
+constexpr int kMmaWarp = 5;                 // score MMAs (and the routing MMA); owns TMEM
+constexpr int kPvWarp = 6;                  // output MMAs
+constexpr int kThreads = 7 * 32;
 constexpr uint32_t kTileBytes = kTile * kD * 2;   // 32 KiB per cache tile
 constexpr uint32_t kHalfBytes = kTileBytes / 2;   // one 64-dim half: 128 rows x 128 B
 constexpr uint32_t kTmemCols = 64;                // S: 2 x 16 columns, O: 2 x 16 columns
@@ -96,7 +100,7 @@ struct __align__(1024) Smem {
     float red[2][kComputeWarps][kNG];
     uint64_t full[Cfg<kStandard>::kStages], empty[Cfg<kStandard>::kStages];
     uint64_t s_full[2], s_empty[2], p_full[2], o_full[2], o_empty[2];
-    uint64_t qr_full, q_ready, r_full, drain, merge_full;
+    uint64_t qr_full, q_ready, r_full, drain, drain2, merge_full;
     int is_last;
     uint32_t tmem_base;
     int abort;
@@ -235,7 +239,7 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int g, int n
 }
 
 template <bool kStandard>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads, 2)
     decode_tc_kernel(const __grid_constant__ CUtensorMap vmap,
                      const __grid_constant__ CUtensorMap kmap,
                      const __grid_constant__ CUtensorMap wmap,
@@ -339,6 +343,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::mbar_init(&sm.r_full, 1);
         ptx::mbar_init(&sm.merge_full, 1);
         ptx::mbar_init(&sm.drain, 1);
+        ptx::mbar_init(&sm.drain2, 1);
         sm.abort = 0;
         ptx::fence_mbar_init();
     }
@@ -444,26 +449,30 @@ __global__ void __launch_bounds__(kThreads, 1)
             (void)drain_wait;
         }
     } else if (warp == kMmaWarp) {
-        // --------------------------------------------------------------- MMA issuer ----
+        // ------------------------------------------------------- score MMA issuer -------
+        // Descriptors are formed once; a k step or a ring stage only moves the start address
+        // (the low field, in 16-byte units; shared addresses stay below 256 KiB).
         constexpr uint32_t idesc_s = ptx::idesc_bf16(128, kN, false, false);
-        constexpr uint32_t idesc_o = ptx::idesc_bf16(128, kN, true, true);
+        constexpr uint32_t kStageBytes = sizeof(sm.tiles[0]);
         const uint32_t qr_addr = ptx::smem_addr(sm.qr);
+        const uint64_t q_desc = ptx::smem_desc(qr_addr, 16, 1024, ptx::kSwizzle128B);
+        const uint64_t k_desc = ptx::smem_desc(
+            ptx::smem_addr(sm.tiles[0][Cfg<kStandard>::kTilesPerStage - 1]), 16, 1024, ptx::kSwizzle128B);
         bool ok = true;
         if (tc_route) {
             // q_r^T[128 j x 16] = W^R^T (MN-major, from ring slot 0) . q^T (K-major rows of the
             // q_r buffer), into the columns of O buffer 0, which the first output MMA reuses.
             constexpr uint32_t idesc_r = ptx::idesc_bf16(128, kN, true, false);
+            const uint64_t w_desc = ptx::smem_desc(ptx::smem_addr(sm.tiles[0][0]), kHalfBytes, 1024,
+                                                   ptx::kSwizzle128B);
             ok = wait(&sm.full[0], 0);
             if (ok) {
                 ptx::tc_fence_after();
                 if (lane == 0) {
-                    const uint32_t wt = ptx::smem_addr(sm.tiles[0][0]);
 #pragma unroll
                     for (int kk = 0; kk < kD / 16; ++kk) {
                         const uint32_t qoff = (kk >> 2) * (kN * 128) + (kk & 3) * 32;
-                        ptx::mma_bf16(tmem + 2 * kN,
-                                      ptx::smem_desc(wt + kk * 2048, kHalfBytes, 1024, ptx::kSwizzle128B),
-                                      ptx::smem_desc(qr_addr + qoff, 16, 1024, ptx::kSwizzle128B),
+                        ptx::mma_bf16(tmem + 2 * kN, w_desc + ((kk * 2048) >> 4), q_desc + (qoff >> 4),
                                       idesc_r, kk > 0);
                     }
                     ptx::mma_commit(&sm.r_full);
@@ -474,53 +483,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         ok = ok && wait(&sm.qr_full, 0);
         if (ok) ptx::tc_fence_after();
-        for (int i = 0; ok && i <= n_tiles; ++i) {
-            if (i < n_tiles) {
-                const int s = (i + ro) % NS, sb = i & 1;
-                if (!wait(&sm.full[s], ((i + ro) / NS) & 1)) break;
-                if (i >= 2 && !wait(&sm.s_empty[sb], ((i >> 1) - 1) & 1)) break;
-                ptx::tc_fence_after();
-                if (lane == 0) {
-                    const uint32_t score_tile =
-                        ptx::smem_addr(sm.tiles[s][Cfg<kStandard>::kTilesPerStage - 1]);
+        for (int i = 0; ok && i < n_tiles; ++i) {
+            const int s = (i + ro) % NS, sb = i & 1;
+            if (!wait(&sm.full[s], ((i + ro) / NS) & 1)) break;
+            if (i >= 2 && !wait(&sm.s_empty[sb], ((i >> 1) - 1) & 1)) break;
+            ptx::tc_fence_after();
+            if (lane == 0) {
+                const uint64_t a0 = k_desc + ((s * kStageBytes) >> 4);
 #pragma unroll
-                    for (int kk = 0; kk < kD / 16; ++kk) {
-                        const uint32_t koff = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
-                        const uint32_t qoff = (kk >> 2) * (kN * 128) + (kk & 3) * 32;
-                        ptx::mma_bf16(tmem + sb * kN,
-                                      ptx::smem_desc(score_tile + koff, 16, 1024, ptx::kSwizzle128B),
-                                      ptx::smem_desc(qr_addr + qoff, 16, 1024, ptx::kSwizzle128B),
-                                      idesc_s, kk > 0);
-                    }
-                    ptx::mma_commit(&sm.s_full[sb]);
+                for (int kk = 0; kk < kD / 16; ++kk) {
+                    const uint32_t koff = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
+                    const uint32_t qoff = (kk >> 2) * (kN * 128) + (kk & 3) * 32;
+                    ptx::mma_bf16(tmem + sb * kN, a0 + (koff >> 4), q_desc + (qoff >> 4), idesc_s, kk > 0);
                 }
-                __syncwarp();
+                ptx::mma_commit(&sm.s_full[sb]);
             }
-            if (i >= 1) {
-                const int j = i - 1, s = (j + ro) % NS, pb = j & 1;
-                if (!wait(&sm.p_full[pb], (j >> 1) & 1)) break;
-                if (j >= 2 && !wait(&sm.o_empty[pb], ((j >> 1) - 1) & 1)) break;
-                ptx::tc_fence_after();
-                const int nvalid = min(kTile, t_end - (t_begin + j * kTile));
-                const int ksteps = (nvalid + 15) >> 4;
-                if (lane == 0) {
-                    const uint32_t vt = ptx::smem_addr(sm.tiles[s][0]);
-                    const uint32_t pt = ptx::smem_addr(sm.p[pb]);
-                    for (int kk = 0; kk < ksteps; ++kk) {
-                        // A = V^T: MN-major SW128, 64-dim halves kHalfBytes apart (LBO),
-                        //          8-token row groups 1 KiB apart (SBO); 16 tokens per step.
-                        // B = P^T: MN-major, no swizzle; hi/lo blocks 128 B apart (SBO),
-                        //          8-token groups 256 B apart (LBO).
-                        ptx::mma_bf16(tmem + 2 * kN + pb * kN,
-                                      ptx::smem_desc(vt + kk * 2048, kHalfBytes, 1024, ptx::kSwizzle128B),
-                                      ptx::smem_desc(pt + kk * 512, 256, 128, ptx::kSwizzleNone),
-                                      idesc_o, kk > 0);
-                    }
-                    ptx::mma_commit(&sm.o_full[pb]);
-                    ptx::mma_commit(&sm.empty[s]);
-                }
-                __syncwarp();
-            }
+            __syncwarp();
         }
         // Drain: every MMA this warp issued completes before TMEM is freed.
         if (lane == 0) ptx::mma_commit(&sm.drain);
@@ -530,8 +508,46 @@ __global__ void __launch_bounds__(kThreads, 1)
             while (!ptx::mbar_try_wait(&sm.drain, 0) && ptx::globaltimer() - t0 < kTimeoutNs) {
             }
         }
+    } else if (warp == kPvWarp) {
+        // ------------------------------------------------------ output MMA issuer -------
+        // A = V^T: MN-major SW128, 64-dim halves kHalfBytes apart (LBO), 8-token row groups
+        //          1 KiB apart (SBO); 16 tokens per step.
+        // B = P^T: MN-major, no swizzle; hi/lo blocks 128 B apart (SBO), 8-token groups 256 B
+        //          apart (LBO).
+        constexpr uint32_t idesc_o = ptx::idesc_bf16(128, kN, true, true);
+        constexpr uint32_t kStageBytes = sizeof(sm.tiles[0]);
+        const uint64_t v_desc =
+            ptx::smem_desc(ptx::smem_addr(sm.tiles[0][0]), kHalfBytes, 1024, ptx::kSwizzle128B);
+        const uint64_t p_desc = ptx::smem_desc(ptx::smem_addr(sm.p[0]), 256, 128, ptx::kSwizzleNone);
+        constexpr uint32_t kPBytes = sizeof(sm.p[0]);
+        for (int j = 0; j < n_tiles; ++j) {
+            const int s = (j + ro) % NS, pb = j & 1;
+            if (!wait(&sm.p_full[pb], (j >> 1) & 1)) break;
+            if (j >= 2 && !wait(&sm.o_empty[pb], ((j >> 1) - 1) & 1)) break;
+            ptx::tc_fence_after();
+            const int nvalid = min(kTile, t_end - (t_begin + j * kTile));
+            const int ksteps = (nvalid + 15) >> 4;
+            if (lane == 0) {
+                const uint64_t a0 = v_desc + ((s * kStageBytes) >> 4);
+                const uint64_t b0 = p_desc + ((pb * kPBytes) >> 4);
+                for (int kk = 0; kk < ksteps; ++kk)
+                    ptx::mma_bf16(tmem + 2 * kN + pb * kN, a0 + ((kk * 2048) >> 4),
+                                  b0 + ((kk * 512) >> 4), idesc_o, kk > 0);
+                ptx::mma_commit(&sm.o_full[pb]);
+                ptx::mma_commit(&sm.empty[s]);
+            }
+            __syncwarp();
+        }
+        if (lane == 0) ptx::mma_commit(&sm.drain2);
+        __syncwarp();
+        {
+            const uint64_t t0 = ptx::globaltimer();
+            while (!ptx::mbar_try_wait(&sm.drain2, 0) && ptx::globaltimer() - t0 < kTimeoutNs) {
+            }
+        }
     } else {
         // ------------------------------------------------------------------ compute -----
+        // (warps 0-3: the TMEM lane quarters 0-3)
         const int t = tid;                                  // 0..127
         const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
         float *qf = reinterpret_cast<float *>(sm.p[0]);     // [k][8] raw query (prologue only)
