@@ -27,7 +27,10 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-DEFAULT_WORKLOAD = "small_gqa"   # batch 8, 32/8 heads, D 128, 4096 tokens, P 16
+# The large-batch workload: batch 256, 64/8 heads, D 128, 8192 tokens, P 32 (4 GiB of cached
+# values). The metric's ">= 80% of 8 TB/s" target is stated for the long-context and
+# large-batch workloads; this is the larger of the two. Others: --workload NAME.
+DEFAULT_WORKLOAD = "high_concurrency_70b"
 METRIC = "decode attention tokens/s and achieved HBM GB/s (% of 8 TB/s) on 1 GB300"
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0

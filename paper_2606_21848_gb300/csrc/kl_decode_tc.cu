@@ -173,6 +173,51 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int g, int n
                              int warp, int lane, const WaitT &wait) {
     const Geometry &geo = a.geo;
     const int G = geo.G;
+    if (n_u <= 8) {
+        // Few splits: thread (head, 4 dims) loads its n_u {m, l} pairs and state rows at once
+        // (one round trip) and folds them; no staging.
+        const float2 *ml = reinterpret_cast<const float2 *>(a.part_ml);
+        for (int h = warp; h < G; h += kComputeWarps) {
+            const size_t bh = (size_t)b * geo.Hq + g * G + h;
+            const float4 *po = reinterpret_cast<const float4 *>(a.part_o + bh * geo.S * kD) + lane;
+            float2 v[8];
+            float4 r[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                if (j < n_u) {
+                    v[j] = __ldcg(ml + bh * geo.S + j);
+                    r[j] = __ldcg(po + (size_t)j * (kD / 4));
+                }
+            }
+            float M = -INFINITY;
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+                if (j < n_u && v[j].y > 0.f) M = fmaxf(M, v[j].x);
+            float z = 0.f;
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                if (j < n_u && v[j].y > 0.f) {
+                    const float w = v[j].y * expf(v[j].x - M);
+                    z += w;
+                    acc.x = fmaf(w, r[j].x, acc.x);
+                    acc.y = fmaf(w, r[j].y, acc.y);
+                    acc.z = fmaf(w, r[j].z, acc.z);
+                    acc.w = fmaf(w, r[j].w, acc.w);
+                }
+            }
+            const float inv = z > 0.f ? 1.f / z : 0.f;
+            acc.x *= inv; acc.y *= inv; acc.z *= inv; acc.w *= inv;
+            const size_t oi = bh * kD + 4 * lane;
+            if (a.out_dtype == KL_FP32) {
+                *reinterpret_cast<float4 *>(static_cast<float *>(a.out) + oi) = acc;
+            } else {
+                __nv_bfloat16 *o16 = static_cast<__nv_bfloat16 *>(a.out) + oi;
+                *reinterpret_cast<uint2 *>(o16) = make_uint2(pack_bf16(acc.x, acc.y), pack_bf16(acc.z, acc.w));
+            }
+        }
+        return;
+    }
     float *rows = reinterpret_cast<float *>(&sm.tiles[0][0][0]);          // [G][n_u][128]
     float2 *tab = reinterpret_cast<float2 *>(rows + (size_t)G * n_u * kD);  // [G][n_u] {m, l}
     float *wt = reinterpret_cast<float *>(tab + G * n_u);                   // [G][n_u] weights
@@ -255,75 +300,23 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int G = geo.G;
 
-    int L = a.seq_lens[b];
-    if (L < 0 || L > geo.max_pages * geo.P) {
-        if (tid == 0 && split == 0 && g == 0) raise_flag(a.err, KL_FLAG_BAD_LENGTH);
-        L = 0;
-    }
-    const int t_begin = split * geo.chunk;
-    const int t_end = min(t_begin + geo.chunk, L);
-    const int n_tiles = t_end > t_begin ? (t_end - t_begin + kTile - 1) / kTile : 0;
     // With one W^R per value head the routing runs on the tensor cores: W^R[g] and the G query
     // rows arrive by TMA as ring position 0 and the cache tiles follow at positions 1, 2, ...
     const bool tc_route = !kStandard && !geo.wr_per_qh;
     const int ro = tc_route ? 1 : 0;
 
-    // Fused append: does this CTA own the current token's row of (b, g)?
-    int app_page = -1, app_pos = -1;
-    if (a.v_new) {
-        const int pos = a.positions[b];
-        if (pos < 0 || pos >= geo.max_pages * geo.P) {
-            if (tid == 0 && split == 0 && g == 0) raise_flag(a.err, KL_FLAG_BAD_POSITION);
-        } else if (pos / geo.chunk == split) {
-            const int page = a.block_table[(size_t)b * geo.max_pages + pos / geo.P];
-            if (page >= 0 && page < geo.num_pages) {
-                app_page = page;
-                app_pos = pos;
-            } else if (tid == 0) {
-                raise_flag(a.err, KL_FLAG_BAD_PAGE);
-            }
-        }
-    }
-    const size_t app_off =
-        app_page >= 0 ? (((size_t)app_page * geo.Hkv + g) * geo.P + app_pos % geo.P) * kD : 0;
-
-    // Empty split, no pipeline: in the split-state layout an empty state; otherwise the split
-    // of a zero-length sequence writes the zero output, and the empty splits of a longer
-    // sequence take no part (the merge counts only the splits that hold tokens).
-    if (n_tiles == 0 && a.merge_inside) {
-        if (app_page >= 0 && tid < 32)
-            reinterpret_cast<uint2 *>(a.cache_rw + app_off)[tid] =
-                reinterpret_cast<const uint2 *>(a.v_new + ((size_t)b * geo.Hkv + g) * kD)[tid];
-        if (L == 0 && split == 0 && tid < kD) {
-            for (int h = 0; h < G; ++h) {
-                const size_t oi = ((size_t)b * geo.Hq + g * G + h) * kD + tid;
-                if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[oi] = 0.f;
-                else static_cast<__nv_bfloat16 *>(a.out)[oi] = __float2bfloat16_rn(0.f);
-            }
-        }
-        return;
-    }
-    if (n_tiles == 0) {
-        if (app_page >= 0 && tid < 32)
-            reinterpret_cast<uint2 *>(a.cache_rw + app_off)[tid] =
-                reinterpret_cast<const uint2 *>(a.v_new + ((size_t)b * geo.Hkv + g) * kD)[tid];
-        if (tid < kD) {
-            for (int h = 0; h < G; ++h) {
-                const size_t bh = (size_t)b * geo.Hq + g * G + h;
-                if (a.direct_out) {
-                    if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * kD + tid] = 0.f;
-                    else static_cast<__nv_bfloat16 *>(a.out)[bh * kD + tid] = __float2bfloat16_rn(0.f);
-                } else {
-                    const size_t slot = bh * geo.S + split;
-                    a.part_o[slot * kD + tid] = 0.f;
-                    if (tid == 0) {
-                        a.part_ml[slot * 2] = -INFINITY;
-                        a.part_ml[slot * 2 + 1] = 0.f;
-                    }
-                }
-            }
-        }
-        return;
+    // Loads that do not depend on one another go out first, so their latency overlaps the
+    // set-up: the length, the append position and (producer) the split's first block-table
+    // entries, 32 pages per warp load, two batches.
+    const int L_raw = a.seq_lens[b];
+    const int pos_raw = a.v_new ? a.positions[b] : -1;
+    const int t_begin = split * geo.chunk;
+    const int first_page = t_begin / geo.P;
+    const int32_t *bt = a.block_table + (size_t)b * geo.max_pages;
+    int bt_cur = -1, bt_nxt = -1;
+    if (warp == kProducerWarp) {
+        if (first_page + lane < geo.max_pages) bt_cur = bt[first_page + lane];
+        if (first_page + 32 + lane < geo.max_pages) bt_nxt = bt[first_page + 32 + lane];
     }
 
     if (tid == 0) {
@@ -362,6 +355,60 @@ __global__ void __launch_bounds__(kThreads, 2)
     ptx::tc_fence_before();
     __syncthreads();
     ptx::tc_fence_after();
+
+    int L = L_raw;
+    if (L < 0 || L > geo.max_pages * geo.P) {
+        if (tid == 0 && split == 0 && g == 0) raise_flag(a.err, KL_FLAG_BAD_LENGTH);
+        L = 0;
+    }
+    const int t_end = min(t_begin + geo.chunk, L);
+    const int n_tiles = t_end > t_begin ? (t_end - t_begin + kTile - 1) / kTile : 0;
+
+    // Fused append: the CTA whose split holds row positions[b] owns the current token's row.
+    const bool pos_ok = pos_raw >= 0 && pos_raw < geo.max_pages * geo.P;
+    if (a.v_new && !pos_ok && tid == 0 && split == 0 && g == 0)
+        raise_flag(a.err, KL_FLAG_BAD_POSITION);
+    const bool app_owner = a.v_new && pos_ok && pos_raw / geo.chunk == split;
+
+    // Empty split, no pipeline: in the split-state layout an empty state; otherwise the split
+    // of a zero-length sequence writes the zero output, and the empty splits of a longer
+    // sequence take no part (the merge counts only the splits that hold tokens).
+    if (n_tiles == 0) {
+        if (app_owner && warp == 0) {
+            const int page = bt[pos_raw / geo.P];
+            if (page >= 0 && page < geo.num_pages) {
+                const size_t off = (((size_t)page * geo.Hkv + g) * geo.P + pos_raw % geo.P) * kD;
+                reinterpret_cast<uint2 *>(a.cache_rw + off)[lane] =
+                    reinterpret_cast<const uint2 *>(a.v_new + ((size_t)b * geo.Hkv + g) * kD)[lane];
+            } else if (lane == 0) {
+                raise_flag(a.err, KL_FLAG_BAD_PAGE);
+            }
+        }
+        if (tid < kD) {
+            for (int h = 0; h < G; ++h) {
+                const size_t bh = (size_t)b * geo.Hq + g * G + h;
+                if (a.merge_inside) {
+                    if (L == 0 && split == 0) {
+                        if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * kD + tid] = 0.f;
+                        else static_cast<__nv_bfloat16 *>(a.out)[bh * kD + tid] = __float2bfloat16_rn(0.f);
+                    }
+                } else if (a.direct_out) {
+                    if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * kD + tid] = 0.f;
+                    else static_cast<__nv_bfloat16 *>(a.out)[bh * kD + tid] = __float2bfloat16_rn(0.f);
+                } else {
+                    const size_t slot = bh * geo.S + split;
+                    a.part_o[slot * kD + tid] = 0.f;
+                    if (tid == 0) {
+                        a.part_ml[slot * 2] = -INFINITY;
+                        a.part_ml[slot * 2 + 1] = 0.f;
+                    }
+                }
+            }
+        }
+        if (warp == kMmaWarp) ptx::tmem_dealloc(sm.tmem_base, kTmemCols);
+        return;
+    }
+
     const uint32_t tmem = sm.tmem_base;
     const Waiter wait{&sm.abort, a.err};
 
@@ -369,18 +416,25 @@ __global__ void __launch_bounds__(kThreads, 2)
         // ------------------------------------------------------------------ producer ----
         const int P = geo.P;
         const int ppt = kTile / P;                   // pages per tile (<= 8)
-        const int first_page = t_begin / P;
         const int end_page = (t_end + P - 1) / P;
-        const int32_t *bt = a.block_table + (size_t)b * geo.max_pages;
         const uint32_t page_bytes = (uint32_t)P * 128u;   // one half of one page
         bool bad = false;
         int issued = 0;
         // The new token's row (fused append), 8 bytes per lane, written just before the loads of
         // the tile that holds it (or first, when it lies past the sequence's end).
-        const int app_tile = app_page < 0 ? -1 : (app_pos < t_end ? (app_pos - t_begin) / kTile : 0);
+        int app_tile = -1;
+        size_t app_off = 0;
         uint2 app_val = make_uint2(0, 0);
-        if (app_page >= 0)
-            app_val = reinterpret_cast<const uint2 *>(a.v_new + ((size_t)b * geo.Hkv + g) * kD)[lane];
+        if (app_owner) {
+            const int page = bt[pos_raw / P];
+            if (page >= 0 && page < geo.num_pages) {
+                app_tile = pos_raw < t_end ? (pos_raw - t_begin) / kTile : 0;
+                app_off = (((size_t)page * geo.Hkv + g) * P + pos_raw % P) * kD;
+                app_val = reinterpret_cast<const uint2 *>(a.v_new + ((size_t)b * geo.Hkv + g) * kD)[lane];
+            } else if (lane == 0) {
+                raise_flag(a.err, KL_FLAG_BAD_PAGE);
+            }
+        }
         if (tc_route) {
             // ring position 0: W^R[g] as the MN-major A operand [j half][128 k rows][128 B] and
             // the group's query rows as the K-major B operand (rows 0..G-1 of the q_r buffer)
@@ -394,10 +448,9 @@ __global__ void __launch_bounds__(kThreads, 2)
             __syncwarp();
             issued = 1;
         }
-        // Block-table entries of the split, 32 pages per warp load, one batch ahead.
+        // Block-table entries of the split, 32 pages per warp load, one batch ahead (the
+        // first two batches were loaded before the set-up).
         const int split_pages = end_page - first_page;
-        int bt_cur = lane < split_pages ? bt[first_page + lane] : -1;
-        int bt_nxt = 32 + lane < split_pages ? bt[first_page + 32 + lane] : -1;
         int bt_batch = 0;
         for (int i = 0; i < n_tiles; ++i) {
             const int r = i + ro, s = r % NS;
