@@ -47,6 +47,8 @@ def parse_args():
     p.add_argument("--num-splits", type=int, default=-1, help="-1: the workload's setting")
     p.add_argument("--standard", action="store_true",
                    help="time the same-design K+V decode (comparison) instead of keyless")
+    p.add_argument("--wr-per-query-head", action="store_true",
+                   help="one W^R per query head (the paper's GQA models) instead of per value head")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=10.0)
     return p.parse_args()
@@ -255,6 +257,8 @@ def run_ours(args):
     kl.load()
 
     wl = WORKLOADS[args.workload]
+    if args.wr_per_query_head:
+        wl = wl.with_(wr_per_query_head=True)
     x = generate(wl, seed=wl.seed + rank)           # replicas: each rank its own batch
     B, Hq, D = x["q"].shape
     num_pages, Hkv, P, _ = x["v_cache"].shape
@@ -422,6 +426,7 @@ def run_ours(args):
                    "seq_len": wl.seq_len or list(wl.seq_len_range),
                    "context_tokens": ab["tokens"], "num_splits": S, "kernel": kname,
                    "decode": "standard K+V (comparison)" if args.standard else "keyless",
+                   "w_r": "per query head" if wl.wr_per_query_head else "per value head",
                    "l2": "flushed between timed steps (512 MiB write, then read back)",
                    "parallelism": f"replicas x{world}"},
         "hbm_gbs_step": step_gbs,
