@@ -2,8 +2,9 @@
 // tcgen05 MMAs with TMEM accumulators, warp-specialized roles.
 //
 // One CTA per (split, value head g, sequence b); head_dim 128, up to 8 query heads per value
-// group. The value-space routing (Section 2.2: q_r = q W^R) runs first, on CUDA cores, into a
-// split-bf16 operand (q_r * scale * log2 e = hi + lo, both bf16) for the G heads of the group.
+// group. The value-space routing (Section 2.2: q_r = q W^R) runs first, as tensor-core MMAs on
+// W^R tiles that stream through the ring, into a split-bf16 operand (q_r * scale * log2 e =
+// hi + lo, both bf16) for the G heads of the group.
 // Then each 128-token tile of cached value rows V_t [128 x 128] (Section 3) is used twice by
 // the tensor cores, straight from one shared-memory copy:
 //
@@ -47,6 +48,7 @@ constexpr int kThreads = 7 * 32;
 constexpr uint32_t kTileBytes = kTile * kD * 2;   // 32 KiB per cache tile
 constexpr uint32_t kHalfBytes = kTileBytes / 2;   // one 64-dim half: 128 rows x 128 B
 constexpr uint32_t kTmemCols = 64;                // S: 2 x 16 columns, O: 2 x 16 columns
+constexpr uint32_t kTmemColsPq = 256;             // + one 16-column routing result per head
 constexpr uint64_t kTimeoutNs = 1000000000ull;
 // Named barriers of the 128 compute threads (id 0 is __syncthreads).
 constexpr uint32_t kBarCompute = 1;       // plain sync
@@ -300,10 +302,14 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int G = geo.G;
 
-    // With one W^R per value head the routing runs on the tensor cores: W^R[g] and the G query
-    // rows arrive by TMA as ring position 0 and the cache tiles follow at positions 1, 2, ...
-    const bool tc_route = !kStandard && !geo.wr_per_qh;
-    const int ro = tc_route ? 1 : 0;
+    // The routing runs on the tensor cores: W^R[g] (one per value head) or the G matrices
+    // W^R[g G + h] (one per query head) arrive by TMA as ring positions 0 .. route_tiles - 1,
+    // with the group's query rows, and the cache tiles follow.
+    const bool tc_route = !kStandard;
+    const bool route_pq = tc_route && geo.wr_per_qh;
+    const int route_tiles = !tc_route ? 0 : route_pq ? G : 1;
+    const int ro = route_tiles;
+    const uint32_t tmem_cols = route_pq ? kTmemColsPq : kTmemCols;
 
     // Loads that do not depend on one another go out first, so their latency overlaps the
     // set-up: the length, the append position and (producer) the split's first block-table
@@ -341,7 +347,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         ptx::fence_mbar_init();
     }
     if (warp == kMmaWarp) {
-        ptx::tmem_alloc(&sm.tmem_base, kTmemCols);
+        ptx::tmem_alloc(&sm.tmem_base, tmem_cols);
         ptx::tmem_relinquish();
     }
     if (warp == kProducerWarp && lane == 0) {
@@ -405,7 +411,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                 }
             }
         }
-        if (warp == kMmaWarp) ptx::tmem_dealloc(sm.tmem_base, kTmemCols);
+        if (warp == kMmaWarp) ptx::tmem_dealloc(sm.tmem_base, tmem_cols);
         return;
     }
 
@@ -435,18 +441,24 @@ __global__ void __launch_bounds__(kThreads, 2)
                 raise_flag(a.err, KL_FLAG_BAD_PAGE);
             }
         }
-        if (tc_route) {
-            // ring position 0: W^R[g] as the MN-major A operand [j half][128 k rows][128 B] and
-            // the group's query rows as the K-major B operand (rows 0..G-1 of the q_r buffer)
+        // Ring positions 0 .. route_tiles - 1: the W^R matrices as the MN-major A operand
+        // [j half][128 k rows][128 B]; position 0 also brings the group's query rows as the
+        // K-major B operand (rows 0..G-1 of the q_r buffer).
+        for (int r = 0; r < route_tiles; ++r) {
+            const int s = r % NS;
+            if (r >= NS && !wait(&sm.empty[s], ((r / NS) & 1) ^ 1)) break;
             if (lane == 0) {
-                ptx::mbar_arrive_expect_tx(&sm.full[0], kTileBytes + 2u * (uint32_t)G * 128u);
-                ptx::tma_load_2d(sm.tiles[0][0], &wmap, &sm.full[0], 0, g * kD);
-                ptx::tma_load_2d(sm.tiles[0][0] + kHalfBytes, &wmap, &sm.full[0], 64, g * kD);
-                ptx::tma_load_2d(sm.qr, &qmap, &sm.full[0], 0, b * geo.Hq + g * G);
-                ptx::tma_load_2d(sm.qr + kN * 128, &qmap, &sm.full[0], 64, b * geo.Hq + g * G);
+                const int wrow = (route_pq ? g * G + r : g) * kD;
+                ptx::mbar_arrive_expect_tx(&sm.full[s], kTileBytes + (r == 0 ? 2u * (uint32_t)G * 128u : 0u));
+                ptx::tma_load_2d(sm.tiles[s][0], &wmap, &sm.full[s], 0, wrow);
+                ptx::tma_load_2d(sm.tiles[s][0] + kHalfBytes, &wmap, &sm.full[s], 64, wrow);
+                if (r == 0) {
+                    ptx::tma_load_2d(sm.qr, &qmap, &sm.full[s], 0, b * geo.Hq + g * G);
+                    ptx::tma_load_2d(sm.qr + kN * 128, &qmap, &sm.full[s], 64, b * geo.Hq + g * G);
+                }
             }
             __syncwarp();
-            issued = 1;
+            issued = r + 1;
         }
         // Block-table entries of the split, 32 pages per warp load, one batch ahead (the
         // first two batches were loaded before the set-up).
@@ -513,23 +525,28 @@ __global__ void __launch_bounds__(kThreads, 2)
             ptx::smem_addr(sm.tiles[0][Cfg<kStandard>::kTilesPerStage - 1]), 16, 1024, ptx::kSwizzle128B);
         bool ok = true;
         if (tc_route) {
-            // q_r^T[128 j x 16] = W^R^T (MN-major, from ring slot 0) . q^T (K-major rows of the
-            // q_r buffer), into the columns of O buffer 0, which the first output MMA reuses.
+            // q_r^T[128 j x 16] = W^R^T (MN-major, ring slot) . q^T (K-major rows of the q_r
+            // buffer). One W^R per value head: into the columns of O buffer 0, which the first
+            // output MMA reuses. One per query head: matrix h into its own 16 columns
+            // (64 + 16 h), of which column h is q_r of head h.
             constexpr uint32_t idesc_r = ptx::idesc_bf16(128, kN, true, false);
-            const uint64_t w_desc = ptx::smem_desc(ptx::smem_addr(sm.tiles[0][0]), kHalfBytes, 1024,
-                                                   ptx::kSwizzle128B);
-            ok = wait(&sm.full[0], 0);
-            if (ok) {
+            for (int r = 0; ok && r < route_tiles; ++r) {
+                const int s = r % NS;
+                ok = wait(&sm.full[s], (r / NS) & 1);
+                if (!ok) break;
                 ptx::tc_fence_after();
                 if (lane == 0) {
+                    const uint64_t w_desc = ptx::smem_desc(ptx::smem_addr(sm.tiles[s][0]), kHalfBytes,
+                                                           1024, ptx::kSwizzle128B);
+                    const uint32_t dst = route_pq ? tmem + 64 + 16 * r : tmem + 2 * kN;
 #pragma unroll
                     for (int kk = 0; kk < kD / 16; ++kk) {
                         const uint32_t qoff = (kk >> 2) * (kN * 128) + (kk & 3) * 32;
-                        ptx::mma_bf16(tmem + 2 * kN, w_desc + ((kk * 2048) >> 4), q_desc + (qoff >> 4),
-                                      idesc_r, kk > 0);
+                        ptx::mma_bf16(dst, w_desc + ((kk * 2048) >> 4), q_desc + (qoff >> 4), idesc_r,
+                                      kk > 0);
                     }
-                    ptx::mma_commit(&sm.r_full);
-                    ptx::mma_commit(&sm.empty[0]);
+                    ptx::mma_commit(&sm.empty[s]);
+                    if (r == route_tiles - 1) ptx::mma_commit(&sm.r_full);
                 }
                 __syncwarp();
             }
@@ -607,9 +624,8 @@ __global__ void __launch_bounds__(kThreads, 2)
         const float sl2 = geo.scale * kLog2e;
         bool ok = true;
 
-        // Routing prologue: thread j obtains q_r[h][j] for the G heads in fp32 -- from the
-        // routing MMA in TMEM (one W^R per value head), or on CUDA cores (one W^R per query
-        // head), or, for the K+V comparison, the unrouted query itself.
+        // Routing prologue: thread j obtains q_r[h][j] for the G heads in fp32 from the routing
+        // MMAs in TMEM, or, for the K+V comparison, the unrouted query itself.
         float acc[kNG];
 #pragma unroll
         for (int h = 0; h < kNG; ++h) acc[h] = 0.f;
@@ -617,11 +633,17 @@ __global__ void __launch_bounds__(kThreads, 2)
             ok = wait(&sm.r_full, 0);
             if (ok) {
                 ptx::tc_fence_after();
-                float rv[16];
-                ptx::tmem_ld16(tmem + 2 * kN + lane_base, rv);
-                ptx::tc_fence_before();
+                if (route_pq) {
 #pragma unroll
-                for (int h = 0; h < kNG; ++h) acc[h] = h < G ? rv[h] : 0.f;
+                    for (int h = 0; h < kNG; ++h)
+                        acc[h] = h < G ? ptx::tmem_ld1(tmem + 64 + 17 * h + lane_base) : 0.f;
+                } else {
+                    float rv[16];
+                    ptx::tmem_ld16(tmem + 2 * kN + lane_base, rv);
+#pragma unroll
+                    for (int h = 0; h < kNG; ++h) acc[h] = h < G ? rv[h] : 0.f;
+                }
+                ptx::tc_fence_before();
                 // the q rows in the q_r buffer were read by the routing MMA; now overwrite them
                 ptx::fence_proxy_async_smem();
             }
@@ -636,27 +658,8 @@ __global__ void __launch_bounds__(kThreads, 2)
             if (lane == 0) ptx::mbar_arrive(&sm.q_ready);
             ok = wait(&sm.q_ready, 0);
             if (ok) {
-                if constexpr (kStandard) {
 #pragma unroll
-                    for (int h = 0; h < kNG; ++h) acc[h] = qf[t * kNG + h];
-                } else {
-#pragma unroll
-                    for (int h = 0; h < kNG; ++h) {
-                        if (h < G) {
-                            const uint16_t *W = a.w_r + (size_t)(g * G + h) * kD * kD + t;
-                            float sum = 0.f;
-                            for (int k0 = 0; k0 < kD; k0 += 32) {
-                                uint32_t w[32];
-#pragma unroll
-                                for (int u = 0; u < 32; ++u) w[u] = W[(size_t)(k0 + u) * kD];
-#pragma unroll
-                                for (int u = 0; u < 32; ++u)
-                                    sum = fmaf(qf[(k0 + u) * kNG + h], __uint_as_float(w[u] << 16), sum);
-                            }
-                            acc[h] = sum;
-                        }
-                    }
-                }
+                for (int h = 0; h < kNG; ++h) acc[h] = qf[t * kNG + h];
             }
         }
         if (ok) {
@@ -837,7 +840,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     __syncthreads();
     if (warp == kMmaWarp) {
         ptx::tc_fence_after();
-        ptx::tmem_dealloc(tmem, kTmemCols);
+        ptx::tmem_dealloc(tmem, tmem_cols);
     }
 }
 
@@ -880,10 +883,11 @@ cudaError_t launch(const DecodeArgs &a) {
     kmap = wmap = qmap = vmap;
     if (kStandard && !make_map(&kmap, a.k_cache, cache_rows, (uint32_t)g.P))
         return cudaErrorInvalidValue;
-    if (!kStandard && !g.wr_per_qh) {
-        // W^R [Hkv * 128 rows (k)][128 (j)], one box = one 64-column half of one matrix;
-        // q [B * Hq rows][128], one box = the G rows of one value group.
-        if (!make_map(&wmap, a.w_r, (uint64_t)g.Hkv * kD, kD)) return cudaErrorInvalidValue;
+    if (!kStandard) {
+        // W^R [Hw * 128 rows (k)][128 (j)], Hw = Hkv or Hq, one box = one 64-column half of one
+        // matrix; q [B * Hq rows][128], one box = the G rows of one value group.
+        const uint64_t hw = g.wr_per_qh ? (uint64_t)g.Hq : (uint64_t)g.Hkv;
+        if (!make_map(&wmap, a.w_r, hw * kD, kD)) return cudaErrorInvalidValue;
         if (!make_map(&qmap, a.q, (uint64_t)g.B * g.Hq, (uint32_t)g.G)) return cudaErrorInvalidValue;
     }
     const size_t smem = sizeof(Smem<kStandard>) + 1024;

@@ -173,6 +173,14 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&r)[16]) {
     for (int i = 0; i < 16; ++i) r[i] = __uint_as_float(u[i]);
 }
 
+// One 32-bit column of the thread's TMEM lane.
+__device__ __forceinline__ float tmem_ld1(uint32_t taddr) {
+    uint32_t u;
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(u) : "r"(taddr) : "memory");
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+    return __uint_as_float(u);
+}
+
 // Shared-memory matrix descriptor of tcgen05: start address, leading / stride byte offsets
 // (units of 16 bytes), descriptor version 1, swizzle mode in bits 61..63.
 enum : uint32_t { kSwizzleNone = 0, kSwizzle128B = 2 };
