@@ -299,8 +299,9 @@ def run_ours(args):
 
     tc = kernel != kl.KL_KERNEL_SIMT and kl.kl_decode_kernel_available(sh, kl.KL_KERNEL_TENSOR,
                                                                       args.standard)
-    # the merge happens inside the decode kernel when its ring can stage the split states
-    one_kernel = S == 1 or (tc and (Hq // Hkv) * S * (D * 4 + 12) <= 3 * 32768 * (2 if args.standard else 1))
+    # the tensor-core kernel merges the split states itself (ring-staged, any S up to the
+    # library's limit); the CUDA-core kernel leaves them to the combine kernel
+    one_kernel = S == 1 or tc
 
     def decode_call(opts, o, w):
         if args.standard:

@@ -166,10 +166,9 @@ __device__ __forceinline__ bool arrive_last(unsigned int *counter, int n) {
 }
 
 // Merge of the n_u split states of (b, g) by the compute warps of the CTA that finished last
-// (kl_combine's formula). The cache ring is idle by now: one TMA bulk copy per head brings the
-// n_u normalized state rows into it while the threads gather the {m, l} table; each warp forms
-// the normalized weights of its heads, then thread (head, 4 dims) folds the rows from shared
-// memory.
+// (kl_combine's formula). Up to eight splits: direct loads. More: the cache ring is idle by
+// now; the {m, l} table and the normalized weights go to its front, and TMA bulk copies bring
+// the state rows through the rest, folded by thread (head, 4 dims) from shared memory.
 template <typename SmemT, typename WaitT>
 __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int g, int n_u, int t,
                              int warp, int lane, const WaitT &wait) {
@@ -220,18 +219,15 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int g, int n
         }
         return;
     }
-    float *rows = reinterpret_cast<float *>(&sm.tiles[0][0][0]);          // [G][n_u][128]
-    float2 *tab = reinterpret_cast<float2 *>(rows + (size_t)G * n_u * kD);  // [G][n_u] {m, l}
-    float *wt = reinterpret_cast<float *>(tab + G * n_u);                   // [G][n_u] weights
-    const uint32_t row_bytes = (uint32_t)n_u * kD * sizeof(float);
-    if (t == 0) {
-        ptx::fence_proxy_async_global();
-        ptx::mbar_arrive_expect_tx(&sm.merge_full, row_bytes * (uint32_t)G);
-        for (int h = 0; h < G; ++h)
-            ptx::bulk_load(rows + (size_t)h * n_u * kD,
-                           a.part_o + ((size_t)b * geo.Hq + g * G + h) * geo.S * kD, row_bytes,
-                           &sm.merge_full);
-    }
+    // Many splits: the {m, l} table and the weights go to the front of the idle ring, then the
+    // state rows stream through the rest of it, `cap` splits per head per bulk-copy round.
+    uint8_t *ring = &sm.tiles[0][0][0];
+    constexpr uint32_t kRingBytes = sizeof(sm.tiles);
+    float2 *tab = reinterpret_cast<float2 *>(ring);                        // [G][n_u] {m, l}
+    float *wt = reinterpret_cast<float *>(tab + G * n_u);                  // [G][n_u] weights
+    const uint32_t table_bytes = ((uint32_t)G * n_u * 12u + 1023u) & ~1023u;
+    float *rows = reinterpret_cast<float *>(ring + table_bytes);           // [G][cap][128]
+    const int cap = (int)((kRingBytes - table_bytes) / ((uint32_t)G * kD * sizeof(float)));
     const float2 *ml = reinterpret_cast<const float2 *>(a.part_ml);
     for (int i = t; i < G * n_u; i += kTile) {
         const int h = i / n_u, j = i - h * n_u;
@@ -258,29 +254,53 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int g, int n
         const float inv = z > 0.f ? 1.f / z : 0.f;
         for (int j = lane; j < n_u; j += 32) wt[h * n_u + j] *= inv;
     }
-    if (!ptx::bar_and(kBarComputeAnd, kTile, wait(&sm.merge_full, 0))) return;
     // thread t: head h = t / 32 (+ 4 for the second pass), dims 4 * (t % 32) .. + 3
-    for (int h = warp; h < G; h += kComputeWarps) {
-        const size_t bh = (size_t)b * geo.Hq + g * G + h;
-        const float4 *po = reinterpret_cast<const float4 *>(rows + (size_t)h * n_u * kD) + lane;
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    float4 acc[2] = {make_float4(0.f, 0.f, 0.f, 0.f), make_float4(0.f, 0.f, 0.f, 0.f)};
+    int round = 0;
+    for (int c0 = 0; c0 < n_u; c0 += cap, ++round) {
+        const int nrow = min(cap, n_u - c0);
+        // every thread is done with the previous chunk (and the weights are written)
+        ptx::fence_proxy_async_smem();
+        ptx::bar_sync(kBarCompute, kTile);
+        if (t == 0) {
+            ptx::fence_proxy_async_global();
+            ptx::mbar_arrive_expect_tx(&sm.merge_full, (uint32_t)(G * nrow * kD * sizeof(float)));
+            for (int h = 0; h < G; ++h)
+                ptx::bulk_load(rows + (size_t)h * cap * kD,
+                               a.part_o + (((size_t)b * geo.Hq + g * G + h) * geo.S + c0) * kD,
+                               (uint32_t)(nrow * kD * sizeof(float)), &sm.merge_full);
+        }
+        if (!ptx::bar_and(kBarComputeAnd, kTile, wait(&sm.merge_full, round & 1))) return;
+#pragma unroll
+        for (int pass = 0; pass < 2; ++pass) {
+            const int h = warp + pass * kComputeWarps;
+            if (h >= G) continue;
+            const float4 *po = reinterpret_cast<const float4 *>(rows + (size_t)h * cap * kD) + lane;
+            const float *w = wt + h * n_u + c0;
 #pragma unroll 4
-        for (int j = 0; j < n_u; ++j) {
-            const float w = wt[h * n_u + j];
-            if (w != 0.f) {
-                const float4 v = po[(size_t)j * (kD / 4)];
-                acc.x = fmaf(w, v.x, acc.x);
-                acc.y = fmaf(w, v.y, acc.y);
-                acc.z = fmaf(w, v.z, acc.z);
-                acc.w = fmaf(w, v.w, acc.w);
+            for (int j = 0; j < nrow; ++j) {
+                const float wj = w[j];
+                if (wj != 0.f) {
+                    const float4 v = po[(size_t)j * (kD / 4)];
+                    acc[pass].x = fmaf(wj, v.x, acc[pass].x);
+                    acc[pass].y = fmaf(wj, v.y, acc[pass].y);
+                    acc[pass].z = fmaf(wj, v.z, acc[pass].z);
+                    acc[pass].w = fmaf(wj, v.w, acc[pass].w);
+                }
             }
         }
-        const size_t oi = bh * kD + 4 * lane;
+    }
+#pragma unroll
+    for (int pass = 0; pass < 2; ++pass) {
+        const int h = warp + pass * kComputeWarps;
+        if (h >= G) continue;
+        const size_t oi = ((size_t)b * geo.Hq + g * G + h) * kD + 4 * lane;
         if (a.out_dtype == KL_FP32) {
-            *reinterpret_cast<float4 *>(static_cast<float *>(a.out) + oi) = acc;
+            *reinterpret_cast<float4 *>(static_cast<float *>(a.out) + oi) = acc[pass];
         } else {
             __nv_bfloat16 *o16 = static_cast<__nv_bfloat16 *>(a.out) + oi;
-            *reinterpret_cast<uint2 *>(o16) = make_uint2(pack_bf16(acc.x, acc.y), pack_bf16(acc.z, acc.w));
+            *reinterpret_cast<uint2 *>(o16) =
+                make_uint2(pack_bf16(acc[pass].x, acc[pass].y), pack_bf16(acc[pass].z, acc[pass].w));
         }
     }
 }
@@ -909,10 +929,11 @@ cudaError_t launch(const DecodeArgs &a) {
 }  // namespace
 
 bool tc_merge_inside(const Geometry &g, bool standard) {
-    // the merging CTA stages G * S state rows (512 B), weights and {m, l} (12 B) in its ring
-    const size_t need = (size_t)g.G * g.S * (kD * sizeof(float) + 12);
+    // the merging CTA keeps {m, l} and the weights of G * S states (12 B each) in its ring and
+    // streams the state rows (512 B) through the rest, at least one split per round
+    const size_t table = ((size_t)g.G * g.S * 12 + 1023) & ~(size_t)1023;
     const size_t ring = standard ? sizeof(Smem<true>::tiles) : sizeof(Smem<false>::tiles);
-    return g.S > 1 && need <= ring;
+    return g.S > 1 && table + (size_t)g.G * kD * sizeof(float) <= ring;
 }
 
 bool tc_supported(const Geometry &g, bool standard) {

@@ -89,6 +89,8 @@ SHAPES = [
     dict(B=2, Hq=8, Hkv=8, D=128, P=16, lens=(700, 64)),                 # MHA, D 128
     dict(B=2, Hq=16, Hkv=8, D=128, P=16, lens=(333, 1280)),              # GQA 2
     dict(B=2, Hq=8, Hkv=1, D=128, P=16, lens=(1500, 9)),                 # MQA, group 8
+    dict(B=2, Hq=12, Hkv=2, D=128, P=16, lens=(2222, 640)),              # Qwen2-1.5B heads, group 6
+    dict(B=3, Hq=24, Hkv=8, D=128, P=64, lens=(5, 300, 1025)),           # group 3, P 64
 ]
 
 
@@ -151,7 +153,7 @@ def test_split_counts_agree(kname):
     x = tiny(B=2, Hq=32, Hkv=8, D=128, P=16, lens=(2000, 4096))
     k = _kernel_or_skip(kname, x)
     want = oracle_decode(x, _gpu.default_scale(x))
-    for s in (1, 2, 5, 8, 16, 32):
+    for s in (1, 2, 5, 8, 16, 32, 64):
         out, err = decode(to_dev(x), shape_of(x), kernel=k, num_splits=s)
         assert err == 0
         assert_parity(out.cpu().numpy(), want, f"{kname} S={s}")
