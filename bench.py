@@ -73,13 +73,16 @@ def measured_peaks():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def kernel_source_digest() -> str:
+# the sources the decode kernel is compiled from
+DECODE_SOURCES = ("kl_decode_tc.cu", "kl_internal.cuh", "kl_tc_ptx.cuh")
+
+
+def kernel_source_digest(names=DECODE_SOURCES) -> str:
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2606_21848_gb300", "csrc")
-    for name in sorted(os.listdir(csrc)):
-        if name.endswith((".cu", ".cuh")):
-            with open(os.path.join(csrc, name), "rb") as f:
-                h.update(f.read())
+    for name in sorted(names):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(f.read())
     return h.hexdigest()[:16]
 
 
@@ -317,8 +320,8 @@ def run_ours(args):
         # kernels are the ones kl_decode_step launches (the K+V comparison appends nothing)
         ev[0].record(stream)
         if one_kernel:
+            # no middle event: two back-to-back event records alone read about 2 us apart
             decode_call(opts_full, out, ws)
-            ev[1].record(stream)
         else:
             decode_call(opts_states, None, None)
             ev[1].record(stream)
@@ -345,8 +348,8 @@ def run_ours(args):
     if world > 1:
         torch.distributed.barrier()
     step_ms = [e[0].elapsed_time(e[2]) for e in evs]
-    dec_ms = [e[0].elapsed_time(e[1]) for e in evs]
-    comb_ms = [e[1].elapsed_time(e[2]) for e in evs]
+    dec_ms = [e[0].elapsed_time(e[2] if one_kernel else e[1]) for e in evs]
+    comb_ms = [0.0 if one_kernel else e[1].elapsed_time(e[2]) for e in evs]
     mean_step = statistics.mean(step_ms)
     mean_dec = statistics.mean(dec_ms)
     if world > 1:
