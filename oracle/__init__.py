@@ -11,6 +11,8 @@ Two independent formulations live here:
   s_i = scale * <q_r, v_i>, softmax weights alpha_{n+1,i} and output O_{n+1} = sum alpha v_i
   (Section 3), plus the split-state merge, the cache append and, for the K+V comparison,
   standard attention (Eq. 1).
+  The prefill of a chunk of new tokens (Eq. 3 with a causal mask) and the chunk append use
+  the same per-row attention.
 * ``dense.py`` -- a NumPy brute force that first un-pages the cache with its own code and then
   evaluates the same formulas on dense arrays; it is used for tiny inputs only.
 
@@ -63,8 +65,11 @@ def _load():
         _lib.ko_decode_partial.argtypes = [i, i, i, i, i, i, i, i, d, p, p, p, p, p, i, i, p, p]
         _lib.ko_combine.argtypes = [i, i, i, i, p, p, p]
         _lib.ko_append.argtypes = [i, i, i, i, i, i, p, p, p, p]
+        _lib.ko_prefill.argtypes = [i, i, i, i, i, i, i, i, d, p, p, p, p, p, p, i, p, p]
+        _lib.ko_append_chunk.argtypes = [i, i, i, i, i, i, p, p, p, p, p]
         for f in ("ko_route", "ko_decode", "ko_standard_decode", "ko_attention_weights",
-                  "ko_decode_partial", "ko_combine", "ko_append"):
+                  "ko_decode_partial", "ko_combine", "ko_append", "ko_prefill",
+                  "ko_append_chunk"):
             getattr(_lib, f).restype = ctypes.c_int
     return _lib
 
@@ -188,4 +193,39 @@ def append(v_cache, v_new, block_table, positions) -> np.ndarray:
     rc = _load().ko_append(B, Hkv, D, P, num_pages, bt.shape[1], _ptr(v_new), _ptr(bt),
                            _ptr(pos), _ptr(cache))
     _check(rc, "append")
+    return cache
+
+
+def prefill(q, w_r, v_cache, block_table, seq_lens, cu_q, *, scale: float,
+            wr_per_query_head: bool = False, rows=None) -> np.ndarray:
+    """Keyless prefill of chunks under the causal mask: [T, Hq, D] fp64, or [len(rows), D].
+
+    q is [T, Hq, D] (bf16 bits), the rows of sequence b being cu_q[b]..cu_q[b+1]-1; the chunk
+    is the last cu_q[b+1]-cu_q[b] of the seq_lens[b] cached rows. ``rows`` selects (r, h) pairs.
+    """
+    q, w_r, v_cache = _c(q, np.uint16), _c(w_r, np.uint16), _c(v_cache, np.uint16)
+    bt, sl, cu = _c(block_table, np.int32), _c(seq_lens, np.int32), _c(cu_q, np.int32)
+    T, Hq, D = q.shape
+    num_pages, Hkv, P, _ = v_cache.shape
+    B = len(sl)
+    if len(cu) != B + 1 or int(cu[-1]) != T:
+        raise ValueError("cu_q must have B + 1 entries ending at the number of query rows")
+    sel = None if rows is None else _c(np.asarray(rows, np.int32).reshape(-1, 2), np.int32)
+    out = np.zeros(((T * Hq) if sel is None else len(sel), D), np.float64)
+    rc = _load().ko_prefill(B, Hq, Hkv, D, P, num_pages, bt.shape[1], int(wr_per_query_head),
+                            float(scale), _ptr(q), _ptr(w_r), _ptr(v_cache), _ptr(bt), _ptr(sl),
+                            _ptr(cu), 0 if sel is None else len(sel), _ptr(sel), _ptr(out))
+    _check(rc, "prefill")
+    return out.reshape(T, Hq, D) if sel is None else out
+
+
+def append_chunk(v_cache, v_new, block_table, seq_lens, cu_q) -> np.ndarray:
+    """Copy of the cache with the rows of each chunk written at positions L_b - n_b .. L_b - 1."""
+    cache = np.array(_c(v_cache, np.uint16), copy=True)
+    v_new = _c(v_new, np.uint16)
+    bt, sl, cu = _c(block_table, np.int32), _c(seq_lens, np.int32), _c(cu_q, np.int32)
+    num_pages, Hkv, P, D = cache.shape
+    rc = _load().ko_append_chunk(len(sl), Hkv, D, P, num_pages, bt.shape[1], _ptr(v_new),
+                                 _ptr(bt), _ptr(sl), _ptr(cu), _ptr(cache))
+    _check(rc, "append_chunk")
     return cache

@@ -72,3 +72,32 @@ def standard_decode(q_bits, k_seqs, v_seqs, *, scale: float):
             a /= a.sum()
             out[b, h] = a @ V
     return out
+
+
+def keyless_prefill(q_bits, w_r_bits, v_seqs, q_lens, *, scale: float,
+                    wr_per_query_head: bool = False):
+    """Keyless prefill over dense value sequences with an explicit causal mask matrix.
+
+    Sequence b has n_b = q_lens[b] query rows (stacked in q_bits, [T, Hq, D]) for its last n_b
+    positions; row i may see tokens t <= L_b - n_b + i. Returns [T, Hq, D] fp64.
+    """
+    q = bf16_bits_to_f64(q_bits)
+    w = bf16_bits_to_f64(w_r_bits)
+    T, Hq, D = q.shape
+    Hkv = v_seqs[0].shape[0] if v_seqs else 1
+    G = Hq // Hkv
+    out = np.zeros((T, Hq, D))
+    r0 = 0
+    for b, n in enumerate(q_lens):
+        n = int(n)
+        L = v_seqs[b].shape[1]
+        allowed = np.arange(L)[None, :] <= (L - n + np.arange(n))[:, None]   # [n, L]
+        for h in range(Hq):
+            V = v_seqs[b][h // G]                                          # [L, D]
+            Qr = q[r0:r0 + n, h] @ w[h if wr_per_query_head else h // G]   # [n, D]
+            s = np.where(allowed, scale * (Qr @ V.T), -np.inf)
+            a = np.exp(s - s.max(axis=1, keepdims=True))
+            a /= a.sum(axis=1, keepdims=True)
+            out[r0:r0 + n, h] = a @ V
+        r0 += n
+    return out

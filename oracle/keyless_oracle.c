@@ -18,7 +18,8 @@
  *   - the head mapping of Section 3 ("Multi-Head", "Multi-Query", "Grouped Query" paragraphs):
  *     heads that share a value group read the same cached value rows;
  *   - for the comparison only: standard decode softmax(q K^T / sqrt(d_k)) V (Eq. 1) over a
- *     paged K cache and a paged V cache.
+ *     paged K cache and a paged V cache;
+ *   - prefill of a chunk of new tokens (Eq. 3 under a causal mask) and the chunk append.
  *
  * Readings where the paper is silent (each is listed in the design notes):
  *   - lambda / sqrt(d_k) is the caller's `scale`; lambda = 1 gives 1/sqrt(d_k);
@@ -27,7 +28,9 @@
  *   - q_r = q W^R with q a row vector and W^R stored row-major, W^R[k][j] at k*D + j;
  *   - the softmax is evaluated as exp(s_i - max s) / sum exp(s_j - max s): the same number as
  *     the paper's ratio (the factor exp(max s) cancels), without overflow;
- *   - a sequence of length 0 gives a zero output.
+ *   - a sequence of length 0 gives a zero output;
+ *   - in prefill, query i of a chunk of n new tokens of a sequence of length L (after the
+ *     append) sits at position L - n + i and attends tokens 0..L - n + i.
  * Paging follows PagedAttention, which the paper cites for KV-cache management: token t of
  * sequence b is row t % P of physical page block_table[b][t / P]; the cache is laid out as
  * [num_pages][Hkv][P][D].
@@ -379,6 +382,94 @@ int ko_append(int B, int Hkv, int D, int P, int num_pages, int max_pages,
         for (int g = 0; g < Hkv; ++g)
             memcpy(v_cache + (((size_t)page * Hkv + g) * P + (size_t)(pos % P)) * D,
                    v_new + ((size_t)b * Hkv + g) * D, sizeof(uint16_t) * (size_t)D);
+    }
+    return err ? -1 : 0;
+}
+
+/*
+ * Keyless prefill over the Value-Only Cache: the full attention of Eq. 3 for the rows of a
+ * chunk of new tokens, under the causal mask of an autoregressive model (Section 5 builds it
+ * on the fly; a token attends itself and the tokens before it).
+ * Sequence b holds L_b = seq_lens[b] cached rows. Its last n_b = cu_q[b + 1] - cu_q[b] rows are
+ * the chunk, already appended; query row r = cu_q[b] + i (0 <= i < n_b) sits at position
+ * p = L_b - n_b + i and, for query head h,
+ *     q_r = q[r][h] W^R[w(h)],  s_t = scale * <q_r, v_t>  (t = 0..p),  out = sum_t alpha_t v_t.
+ * q and out are [T][Hq][D] with T = cu_q[B]; with sel != NULL only the n_sel pairs (r, h) are
+ * computed and out is [n_sel][D].
+ */
+int ko_prefill(int B, int Hq, int Hkv, int D, int P, int num_pages, int max_pages,
+               int wr_per_query_head, double scale, const uint16_t *q, const uint16_t *w_r,
+               const uint16_t *v_cache, const int32_t *block_table, const int32_t *seq_lens,
+               const int32_t *cu_q, int n_sel, const int32_t *sel, double *out)
+{
+    if (check_dims(B, Hq, Hkv, D) || P <= 0 || max_pages < 0 || cu_q[0] != 0)
+        return -1;
+    for (int b = 0; b < B; ++b) {
+        int n = cu_q[b + 1] - cu_q[b];
+        if (n < 0 || n > seq_lens[b] || seq_lens[b] > max_pages * P)
+            return -1;
+    }
+    int G = Hq / Hkv, T = cu_q[B];
+    long n_items = sel ? n_sel : (long)T * Hq;
+    int err = 0;
+
+#pragma omp parallel for schedule(dynamic, 1) reduction(| : err)
+    for (long it = 0; it < n_items; ++it) {
+        int r = sel ? sel[2 * it] : (int)(it / Hq);
+        int h = sel ? sel[2 * it + 1] : (int)(it % Hq);
+        double *o = out + (size_t)it * D;
+        if (r < 0 || r >= T || h < 0 || h >= Hq) {
+            err |= 1;
+            continue;
+        }
+        int b = 0;
+        while (cu_q[b + 1] <= r)
+            ++b;
+        int n = cu_q[b + 1] - cu_q[b];
+        int p = seq_lens[b] - n + (r - cu_q[b]);
+        int g = h / G, w = wr_per_query_head ? h : g;
+        double *qr = (double *)malloc(sizeof(double) * (size_t)D);
+        double *s = (double *)malloc(sizeof(double) * (size_t)(p + 1));
+        route_row(D, q + ((size_t)r * Hq + h) * D, w_r + (size_t)w * D * D, qr);
+        double m, l;
+        if (attend(D, Hkv, P, num_pages, scale, qr, v_cache, v_cache,
+                   block_table + (size_t)b * max_pages, g, 0, p + 1, s, o, &m, &l))
+            err |= 1;
+        free(s);
+        free(qr);
+    }
+    return err ? -1 : 0;
+}
+
+/*
+ * Append of a chunk: the n_b = cu_q[b + 1] - cu_q[b] value rows of sequence b go to positions
+ * L_b - n_b .. L_b - 1 (L_b = seq_lens[b], the length after the append):
+ *   cache[block_table[b][p / P]][g][p % P][:] = v_new[cu_q[b] + i][g][:],  p = L_b - n_b + i.
+ * v_new is [T][Hkv][D]. Rows whose position or page id is out of range are skipped; -1 then.
+ */
+int ko_append_chunk(int B, int Hkv, int D, int P, int num_pages, int max_pages,
+                    const uint16_t *v_new, const int32_t *block_table, const int32_t *seq_lens,
+                    const int32_t *cu_q, uint16_t *v_cache)
+{
+    int err = 0;
+    for (int b = 0; b < B; ++b) {
+        int n = cu_q[b + 1] - cu_q[b];
+        for (int i = 0; i < n; ++i) {
+            int pos = seq_lens[b] - n + i;
+            if (pos < 0 || pos >= max_pages * P) {
+                err = 1;
+                continue;
+            }
+            int page = block_table[(size_t)b * max_pages + pos / P];
+            if (page < 0 || page >= num_pages) {
+                err = 1;
+                continue;
+            }
+            for (int g = 0; g < Hkv; ++g)
+                memcpy(v_cache + (((size_t)page * Hkv + g) * P + (size_t)(pos % P)) * D,
+                       v_new + ((size_t)(cu_q[b] + i) * Hkv + g) * D,
+                       sizeof(uint16_t) * (size_t)D);
+        }
     }
     return err ? -1 : 0;
 }

@@ -46,3 +46,22 @@ def default_scale(D: int) -> float:
 def to_bf16_bits(a: np.ndarray) -> np.ndarray:
     """Round fp64/fp32 values to bf16 (round-to-nearest-even, via torch) and return the bits."""
     return bf16_bits(torch.from_numpy(np.asarray(a, np.float32)).to(torch.bfloat16))
+
+
+def tiny_prefill(B=3, Hq=8, Hkv=2, D=64, P=16, lens=(5, 37, 100), q_lens=(5, 12, 1), seed=21,
+                 table="permuted", wr_per_query_head=False):
+    """A tiny chunked-prefill input: the cache of ``tiny`` plus a chunk of q_lens[b] query rows
+    for the last q_lens[b] positions of each sequence (q is [T, Hq, D], cu_q its row offsets)."""
+    assert all(0 <= n <= L for n, L in zip(q_lens, lens))
+    x = tiny(B, Hq, Hkv, D, P, lens, seed, table, wr_per_query_head)
+    g = torch.Generator().manual_seed(seed + 7)
+    T = int(sum(q_lens))
+    x["q"] = torch.randn(T, Hq, D, generator=g).to(torch.bfloat16)
+    x["cu_q"] = torch.tensor(np.concatenate([[0], np.cumsum(q_lens)]), dtype=torch.int32)
+    x["q_lens"] = torch.tensor(q_lens, dtype=torch.int32)
+    return x
+
+
+def prefill_bits(x: dict):
+    """NumPy views for the prefill oracle: (q, w_r, v_cache, block_table, seq_lens, cu_q)."""
+    return bits(x) + (x["cu_q"].numpy(),)

@@ -17,6 +17,7 @@ import pytest
 import oracle
 from oracle import dense
 from tests import test_oracle as pins
+from tests import test_oracle_prefill as prefill_pins
 from tests._inputs import bits, default_scale, tiny
 
 SRC = os.path.join(os.path.dirname(oracle.__file__), "keyless_oracle.c")
@@ -32,6 +33,15 @@ MUTATIONS = {
     "flipped_exponent": ("double e = exp(s[t - t0] - m);", "double e = exp(m - s[t - t0]);"),
     "combine_drops_l": ("double w = ml[2 * s + 1] * exp(ml[2 * s] - M);",
                         "double w = exp(ml[2 * s] - M);"),
+    # prefill: the causal limit of a chunk row
+    "prefill_mask_off_by_one": ("int p = seq_lens[b] - n + (r - cu_q[b]);",
+                                "int p = seq_lens[b] - n + (r - cu_q[b]) - 1;"),
+    "prefill_ignores_prefix": ("int p = seq_lens[b] - n + (r - cu_q[b]);",
+                               "int p = r - cu_q[b];"),
+    "prefill_not_causal": ("int p = seq_lens[b] - n + (r - cu_q[b]);",
+                           "int p = seq_lens[b] - 1;"),
+    "prefill_wrong_row_base": ("route_row(D, q + ((size_t)r * Hq + h) * D, w_r + (size_t)w * D * D, qr);",
+                               "route_row(D, q + ((size_t)(r - cu_q[b]) * Hq + h) * D, w_r + (size_t)w * D * D, qr);"),
 }
 
 
@@ -53,6 +63,9 @@ def _pin_results():
     run("dominant", pins.test_dominant_score_selects_that_row)
     run("split_merge", pins.test_split_merge_identity, 33)
     run("route", pins.test_route_matches_row_times_matrix)
+    run("prefill_dense", prefill_pins.test_paged_prefill_equals_dense_causal_bruteforce,
+        dict(B=3, Hq=8, Hkv=2, D=64, P=16, lens=(5, 37, 100), q_lens=(5, 12, 1)))
+    run("prefill_sdpa", prefill_pins.test_full_causal_prefill_equals_sdpa_with_k_equal_v_wr_transposed)
     return res
 
 
@@ -69,7 +82,7 @@ def test_planted_mistake_is_caught(name, tmp_path, monkeypatch):
     lib = ctypes.CDLL(str(so))
     real = oracle._load()
     for f in ("ko_route", "ko_decode", "ko_standard_decode", "ko_attention_weights",
-              "ko_decode_partial", "ko_combine", "ko_append"):
+              "ko_decode_partial", "ko_combine", "ko_append", "ko_prefill", "ko_append_chunk"):
         getattr(lib, f).argtypes = getattr(real, f).argtypes
         getattr(lib, f).restype = ctypes.c_int
     monkeypatch.setattr(oracle, "_lib", lib)
