@@ -197,6 +197,43 @@ kl_status kl_standard_decode(const kl_shape *shape, const void *q, const void *k
                              kl_dtype out_dtype, void *workspace, size_t workspace_bytes,
                              int32_t *err, kl_stream_t stream);
 
+/*
+ * Chunk append, the prefill counterpart of kl_append_v: sequence b's chunk of
+ * n_b = cu_q_lens[b + 1] - cu_q_lens[b] new tokens takes the last n_b of its seq_lens[b] rows,
+ *   v_cache[block_table[b][p / P]][g][p % P][:] = v_new[cu_q_lens[b] + i][g][:],
+ *   p = seq_lens[b] - n_b + i,  0 <= i < n_b,  all g.
+ * v_new: [total_q][Hkv][D] bf16 (total_q = cu_q_lens[B]); cu_q_lens: [B + 1] int32 on the
+ * device, non-decreasing from 0; max_q_len: a host-side bound on every n_b (it sizes the grid;
+ * rows past it are not written). A length that breaks 0 <= n_b <= seq_lens[b] <=
+ * max_pages_per_seq * P raises KL_FLAG_BAD_LENGTH and skips the sequence; a page id outside the
+ * pool raises KL_FLAG_BAD_PAGE and skips that row.
+ */
+kl_status kl_append_v_chunk(const kl_shape *shape, const void *v_new, const int32_t *block_table,
+                            const int32_t *seq_lens, const int32_t *cu_q_lens, int32_t total_q,
+                            int32_t max_q_len, void *v_cache, int32_t *err, kl_stream_t stream);
+
+/*
+ * Chunked keyless prefill: the full attention of Eq. 3 for a chunk of new tokens under the
+ * causal mask of an autoregressive model (Section 5), over the paged Value-Only Cache, with
+ * the routing projection of Section 2.2 fused into the kernel. Sequence b's chunk is its last
+ * n_b = cu_q_lens[b + 1] - cu_q_lens[b] cached rows (append them first, kl_append_v_chunk);
+ * query row r = cu_q_lens[b] + i sits at position p = seq_lens[b] - n_b + i and, per query
+ * head h,
+ *   q_r = q[r][h] W^R[w(h)],  s_t = scale * <q_r, v_t> (t = 0 .. p),
+ *   out[r][h] = sum_t softmax(s)_t v_t.
+ * A whole prompt is the case n_b = seq_lens[b]; a decode step is n_b = 1.
+ * q, out: [total_q][Hq][D] (q bf16, out of out_dtype); w_r, v_cache, block_table as in
+ * kl_decode_attention; cu_q_lens: [B + 1] int32 on the device; max_q_len: a host-side bound on
+ * every n_b (it sizes the grid; rows past it get no output). head_dim 128 only
+ * (KL_ERR_UNSUPPORTED otherwise). Needs no workspace. Flags as in kl_append_v_chunk, and a bad
+ * page id leaves the affected outputs unspecified.
+ */
+kl_status kl_prefill_attention(const kl_shape *shape, const void *q, const void *w_r,
+                               const void *v_cache, const int32_t *block_table,
+                               const int32_t *seq_lens, const int32_t *cu_q_lens,
+                               int32_t total_q, int32_t max_q_len, void *out, kl_dtype out_dtype,
+                               int32_t *err, kl_stream_t stream);
+
 /* Size of the fixed device scratch that kl_decode_attention_noalloc uses (32 MiB). */
 #define KL_NOALLOC_SCRATCH_BYTES (32u * 1024u * 1024u)
 

@@ -1,4 +1,4 @@
-"""GB300-native decode of Keyless Attention over a paged Value-Only Cache.
+"""GB300-native decode (and chunked prefill) of Keyless Attention over a paged Value-Only Cache.
 
 The compute lives in ``libkeyless.so`` (hand-written CUDA for sm_103a behind the C ABI of
 ``include/keyless.h``); this package holds its build script, a ctypes binding with the same
@@ -14,4 +14,5 @@ from ._lib import (  # noqa: F401
     kl_decode_attention_noalloc, kl_decode_kernel_available, kl_decode_step, KL_NOALLOC_SCRATCH_BYTES,
     kl_decode_num_splits, kl_decode_options, kl_decode_workspace_size, kl_route_query,
     kl_shape, kl_standard_decode, kl_status_string, load, make_shape,
+    kl_append_v_chunk, kl_prefill_attention,
 )

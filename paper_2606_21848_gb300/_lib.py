@@ -73,6 +73,8 @@ def load() -> ctypes.CDLL:
         "kl_decode_step": ([SH, P, P, P, P, P, P, P, OP, P, I32, P, SZ, P, P], I32),
         "kl_decode_attention_noalloc": ([SH, P, P, P, P, P, I32, P, I32, P, P], I32),
         "kl_decode_kernel_available": ([SH, I32, I32], I32),
+        "kl_append_v_chunk": ([SH, P, P, P, P, I32, I32, P, P, P], I32),
+        "kl_prefill_attention": ([SH, P, P, P, P, P, P, I32, I32, P, I32, P, P], I32),
         "kl_status_string": ([I32], ctypes.c_char_p),
     }
     for name, (args, res) in sig.items():
@@ -194,6 +196,21 @@ def kl_decode_attention_noalloc(shape, q, w_r, v_cache, block_table, seq_lens, n
                                               _p(block_table), _p(seq_lens), num_splits, _p(out),
                                               out_dtype, _p(err), _stream(stream)),
            "kl_decode_attention_noalloc")
+
+
+def kl_append_v_chunk(shape, v_new, block_table, seq_lens, cu_q_lens, total_q, max_q_len, v_cache,
+                      err=None, stream=None):
+    _check(load().kl_append_v_chunk(ctypes.byref(shape), _p(v_new), _p(block_table), _p(seq_lens),
+                                    _p(cu_q_lens), total_q, max_q_len, _p(v_cache), _p(err),
+                                    _stream(stream)), "kl_append_v_chunk")
+
+
+def kl_prefill_attention(shape, q, w_r, v_cache, block_table, seq_lens, cu_q_lens, total_q,
+                         max_q_len, out, out_dtype, err=None, stream=None):
+    _check(load().kl_prefill_attention(ctypes.byref(shape), _p(q), _p(w_r), _p(v_cache),
+                                       _p(block_table), _p(seq_lens), _p(cu_q_lens), total_q,
+                                       max_q_len, _p(out), out_dtype, _p(err), _stream(stream)),
+           "kl_prefill_attention")
 
 
 def kl_decode_kernel_available(shape, kernel, standard=False) -> bool:

@@ -267,6 +267,56 @@ kl_status kl_combine(const kl_shape *shape, const float *partial_o, const float 
                                     out_dtype, reinterpret_cast<cudaStream_t>(stream)));
 }
 
+kl_status kl_append_v_chunk(const kl_shape *shape, const void *v_new, const int32_t *block_table,
+                            const int32_t *seq_lens, const int32_t *cu_q_lens, int32_t total_q,
+                            int32_t max_q_len, void *v_cache, int32_t *err, kl_stream_t stream) {
+    Geometry g;
+    kl_status st = resolve(shape, -1, &g);
+    if (st != KL_OK) return st;
+    if (total_q < 0 || max_q_len < 0) return KL_ERR_INVALID_ARG;
+    if (g.B == 0 || total_q == 0 || max_q_len == 0) return KL_OK;
+    if (!v_new || !block_table || !seq_lens || !cu_q_lens || !v_cache) return KL_ERR_INVALID_ARG;
+    if (!aligned(v_new, 16) || !aligned(v_cache, 16)) return KL_ERR_INVALID_ARG;
+    return from_cuda(launch_append_chunk(g, total_q, max_q_len, static_cast<const uint16_t *>(v_new),
+                                         block_table, seq_lens, cu_q_lens,
+                                         static_cast<uint16_t *>(v_cache), err,
+                                         reinterpret_cast<cudaStream_t>(stream)));
+}
+
+kl_status kl_prefill_attention(const kl_shape *shape, const void *q, const void *w_r,
+                               const void *v_cache, const int32_t *block_table,
+                               const int32_t *seq_lens, const int32_t *cu_q_lens,
+                               int32_t total_q, int32_t max_q_len, void *out, kl_dtype out_dtype,
+                               int32_t *err, kl_stream_t stream) {
+    Geometry g;
+    kl_status st = resolve(shape, -1, &g);
+    if (st != KL_OK) return st;
+    if (total_q < 0 || max_q_len < 0) return KL_ERR_INVALID_ARG;
+    if (out_dtype != KL_BF16 && out_dtype != KL_FP32) return KL_ERR_INVALID_ARG;
+    if (!prefill_tc_supported(g)) return KL_ERR_UNSUPPORTED;
+    if (g.B == 0 || total_q == 0 || max_q_len == 0) return KL_OK;
+    if (!q || !w_r || !v_cache || !block_table || !seq_lens || !cu_q_lens || !out)
+        return KL_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(w_r, 16) || !aligned(v_cache, 16) || !aligned(out, 16))
+        return KL_ERR_INVALID_ARG;
+    if ((int64_t)max_q_len > (int64_t)65535 * 128) return KL_ERR_UNSUPPORTED;
+    PrefillArgs a;
+    a.geo = g;
+    a.total_q = total_q;
+    a.max_q = max_q_len;
+    a.q = static_cast<const uint16_t *>(q);
+    a.w_r = static_cast<const uint16_t *>(w_r);
+    a.v_cache = static_cast<const uint16_t *>(v_cache);
+    a.block_table = block_table;
+    a.seq_lens = seq_lens;
+    a.cu_q = cu_q_lens;
+    a.out = out;
+    a.out_dtype = out_dtype;
+    a.err = err;
+    a.stream = reinterpret_cast<cudaStream_t>(stream);
+    return from_cuda(launch_prefill_tc(a));
+}
+
 int32_t kl_decode_kernel_available(const kl_shape *shape, int32_t kernel, int32_t standard) {
     Geometry g;
     if (resolve(shape, 1, &g) != KL_OK || g.G > 8) return 0;

@@ -46,6 +46,25 @@ struct DecodeArgs {
     cudaStream_t stream;
 };
 
+// Arguments of a chunked-prefill launch (kl_prefill_attention). Sequence b's query rows are
+// cu_q[b] .. cu_q[b + 1] - 1 of q / out ([total_q][Hq][D]); they are the last n_b rows of its
+// seq_lens[b] cached rows, so query row i sits at position seq_lens[b] - n_b + i.
+struct PrefillArgs {
+    Geometry geo;             // S and chunk unused
+    int total_q;              // rows of q and out
+    int max_q;                // host bound on n_b (grid sizing)
+    const uint16_t *q;        // [total_q][Hq][D] bf16
+    const uint16_t *w_r;      // [Hw][D][D] bf16
+    const uint16_t *v_cache;  // [num_pages][Hkv][P][D] bf16
+    const int32_t *block_table;
+    const int32_t *seq_lens;
+    const int32_t *cu_q;      // [B + 1]
+    void *out;                // [total_q][Hq][D]
+    kl_dtype out_dtype;
+    int32_t *err;
+    cudaStream_t stream;
+};
+
 // bf16 bit helpers (a bf16 value is the upper half of a binary32 value).
 __device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
@@ -73,6 +92,15 @@ bool tc_supported(const Geometry &g, bool standard);
 // Whether the tensor-core kernel can merge this geometry's split states itself.
 bool tc_merge_inside(const Geometry &g, bool standard);
 cudaError_t launch_decode_tc(const DecodeArgs &a, bool standard);
+
+// Chunked prefill on the tensor cores (head_dim 128, compute capability 10.3) and the
+// chunk append.
+bool prefill_tc_supported(const Geometry &g);
+cudaError_t launch_prefill_tc(const PrefillArgs &a);
+cudaError_t launch_append_chunk(const Geometry &g, int total_q, int max_q, const uint16_t *v_new,
+                                const int32_t *block_table, const int32_t *seq_lens,
+                                const int32_t *cu_q, uint16_t *v_cache, int32_t *err,
+                                cudaStream_t stream);
 
 // Number of SMs of the current device (cached per device).
 int device_sm_count();

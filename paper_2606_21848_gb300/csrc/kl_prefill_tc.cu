@@ -1,0 +1,615 @@
+// Tensor-core chunked prefill for sm_103a: the full attention of Eq. 3 for the query rows of a
+// chunk of new tokens, over the paged Value-Only Cache, under the causal mask.
+//
+// One CTA per (query head h, sequence b, block of 128 query rows); head_dim 128. The rows of the
+// block sit at consecutive positions p0 .. p0 + 127 of the sequence (the chunk is the tail of the
+// cached rows), so the CTA walks the cache tiles 0 .. p_last / 128 and masks only the last ones.
+//
+//   routing  Q_r = Q . W^R[w(h)]                      M = 128 rows, N = 128, K = 128 (Section 2.2)
+//   scores   S   = Q_hi . V_t^T + Q_lo . V_t^T        M = 128 rows, N = 128 tokens, K = 2 x 128
+//   output   O  += P_hi . V_t + P_lo . V_t            M = 128 rows, N = 128 dims,  K = 2 x 128
+//
+// Each cached tile V_t [128 tokens x 128 dims] arrives once by TMA (one box per page) and feeds
+// both products from the same shared-memory copy: as the K-major B operand of the score MMAs and
+// as the MN-major B operand of the output MMAs. Accumulators live in TMEM: S in two 128-column
+// buffers (the score MMAs of tile t + 1 run while tile t is in the softmax), O in a third.
+//
+// Precision: the routed query (times scale * log2 e) and the softmax weights are each carried as
+// a pair of bf16 operands, x = hi + lo, which keeps about 16 significant bits where one bf16
+// operand keeps 8. With one bf16 operand each, rows whose softmax mass sits on a few tokens (the
+// first positions of a prompt, peaked scores) miss |err| <= 2e-3 + 1e-2 |ref| by up to 7e-3; the
+// pair costs twice the tensor-core work of a plain bf16 attention.
+//
+// Softmax (thread = query row = TMEM lane): scores arrive already scaled by scale * log2 e (the
+// routed query is scaled before its bf16 rounding), so p = 2^(s - m). The reference maximum m of
+// a row only moves when the tile maximum exceeds it by more than 8 (a factor 256): then the row's
+// O in TMEM and its running sum l are rescaled; otherwise p may reach 2^8, well inside bf16 and
+// fp32 range, and the final O / l is unchanged because O and l share the same reference.
+//
+// Roles (192 threads, one CTA per SM):
+//   warps 0-3  softmax and epilogue (TMEM lane quarters 0-3)
+//   warp 4     producer: TMA of W^R and the query block (ring position 0), then cache tiles
+//   warp 5     MMA issuer (one elected lane) and TMEM owner
+// Every wait is bounded (about one second); a wait that runs out raises KL_FLAG_TIMEOUT, makes
+// every role leave its loop, drains outstanding copies and MMAs and frees TMEM.
+#include <cudaTypedefs.h>
+#include <math.h>
+
+#include "kl_internal.cuh"
+#include "kl_tc_ptx.cuh"
+
+namespace kl {
+namespace {
+
+constexpr int kD = 128;
+constexpr int kBM = 128;                          // query rows per CTA
+constexpr int kBN = 128;                          // cache rows per tile
+constexpr int kStages = 3;
+constexpr int kComputeWarps = 4;
+constexpr int kProducerWarp = 4;
+constexpr int kMmaWarp = 5;
+constexpr int kThreads = 6 * 32;
+constexpr uint32_t kTileBytes = kBN * kD * 2;     // 32 KiB
+constexpr uint32_t kHalfBytes = kTileBytes / 2;   // one 64-column half: 128 rows x 128 B
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kColS = 0;                     // S buffers: columns 0 and 128
+constexpr uint32_t kColO = 256;                   // O: columns 256 .. 383
+constexpr float kRescaleLog2 = 8.f;
+constexpr uint64_t kTimeoutNs = 1000000000ull;
+
+struct __align__(1024) PrefillSmem {
+    // q[0]: the query block, then hi of the routed, scaled query Q_r; q[1]: its lo. K-major,
+    // 128B-swizzled: [64-dim half][128 rows][128 B].
+    uint8_t q[2][kBM * kD * 2];
+    // Ring of 32 KiB slots: W^R[w(h)] at position 0 ([64-column half][128 k rows][128 B]), then
+    // the cache tiles ([64-dim half][128 tokens][128 B]); all 128B-swizzled.
+    uint8_t tiles[kStages][kTileBytes];
+    // Softmax weights of one tile, hi (p[0]) and lo (p[1]), the A operands of the output MMAs;
+    // K-major, 128B-swizzled: [64-token half][128 rows][128 B].
+    uint8_t p[2][kBM * kBN * 2];
+    uint64_t full[kStages], empty[kStages];
+    uint64_t s_full[2], s_empty[2], p_full, pv_done;
+    uint64_t r_full, qr_ready, drain;
+    uint32_t tmem_base;
+    int abort;
+};
+
+// Warp-collective bounded wait (every lane calls it in uniform control flow and gets the same
+// answer). False when the CTA is aborting or the wait ran out (about 1 s).
+struct Waiter {
+    volatile int *abort;
+    int32_t *err;
+    __device__ bool operator()(uint64_t *bar, uint32_t parity) const {
+        bool ok = ptx::mbar_try_wait(bar, parity);
+        if (!ok) {
+            const uint64_t t0 = ptx::globaltimer();
+            while (true) {
+                if (ptx::mbar_try_wait(bar, parity)) { ok = true; break; }
+                if (*abort) break;
+                if (ptx::globaltimer() - t0 > kTimeoutNs) {
+                    *abort = 1;
+                    raise_flag(err, KL_FLAG_TIMEOUT);
+                    break;
+                }
+            }
+        }
+        return __all_sync(0xffffffffu, ok);
+    }
+};
+
+// Byte offset of the 16-byte chunk that holds columns c .. c + 7 (c a multiple of 8) of row r
+// in a K-major, 128B-swizzled operand of 128 rows and 128 columns laid out as
+// [64-column half][128 rows][128 B]: the chunk index inside the row is XORed with r mod 8.
+__device__ __forceinline__ uint32_t sw128_chunk(int r, int c) {
+    return (uint32_t)((c >> 6) * kHalfBytes + r * 128 + ((((c >> 3) & 7) ^ (r & 7)) << 4));
+}
+
+__device__ __forceinline__ uint32_t pack2(float a, float b) {
+    const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<const uint32_t *>(&v);
+}
+
+// x = hi + lo with hi = bf16(x), lo = bf16(x - hi), for two values packed as bf16 pairs.
+__device__ __forceinline__ void split2(float x0, float x1, uint32_t &hi, uint32_t &lo) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(x0, x1);
+    const float2 hf = __bfloat1622float2(h);
+    const __nv_bfloat162 l = __floats2bfloat162_rn(x0 - hf.x, x1 - hf.y);
+    hi = *reinterpret_cast<const uint32_t *>(&h);
+    lo = *reinterpret_cast<const uint32_t *>(&l);
+}
+
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
+                                             uint32_t d) {
+    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c),
+                 "r"(d)
+                 : "memory");
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    prefill_tc_kernel(const __grid_constant__ CUtensorMap vmap,
+                      const __grid_constant__ CUtensorMap wmap,
+                      const __grid_constant__ CUtensorMap qmap, const PrefillArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    PrefillSmem &sm = *reinterpret_cast<PrefillSmem *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const Geometry &geo = a.geo;
+    const int h = blockIdx.x, b = blockIdx.y;
+    const int mblk = (int)gridDim.z - 1 - (int)blockIdx.z;   // the longest blocks start first
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+    const int q0 = a.cu_q[b], q1 = a.cu_q[b + 1];
+    const int L = a.seq_lens[b];
+    const int n = q1 - q0;
+    if (q0 < 0 || n < 0 || q1 > a.total_q || L < n || L > geo.max_pages * geo.P) {
+        if (tid == 0 && h == 0 && mblk == 0) raise_flag(a.err, KL_FLAG_BAD_LENGTH);
+        return;
+    }
+    const int m0 = mblk * kBM;
+    if (m0 >= n) return;
+    const int rows = min(kBM, n - m0);           // query rows of this block
+    const int pos0 = L - n + m0;                 // position of row 0
+    const int pos_last = pos0 + rows - 1;        // <= L - 1
+    const int n_tiles = pos_last / kBN + 1;      // cache tiles 0 .. n_tiles - 1
+    const int g = h / geo.G;
+    const int wsel = geo.wr_per_qh ? h : g;
+
+    if (tid == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            ptx::mbar_init(&sm.full[s], 1);
+            ptx::mbar_init(&sm.empty[s], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            ptx::mbar_init(&sm.s_full[i], 1);
+            ptx::mbar_init(&sm.s_empty[i], kComputeWarps);
+        }
+        ptx::mbar_init(&sm.p_full, kComputeWarps);
+        ptx::mbar_init(&sm.pv_done, 1);
+        ptx::mbar_init(&sm.r_full, 1);
+        ptx::mbar_init(&sm.qr_ready, kComputeWarps);
+        ptx::mbar_init(&sm.drain, 1);
+        sm.abort = 0;
+        ptx::fence_mbar_init();
+    }
+    if (warp == kMmaWarp) {
+        ptx::tmem_alloc(&sm.tmem_base, kTmemCols);
+        ptx::tmem_relinquish();
+    }
+    if (warp == kProducerWarp && lane == 0) {
+        ptx::prefetch_tensormap(&vmap);
+        ptx::prefetch_tensormap(&wmap);
+        ptx::prefetch_tensormap(&qmap);
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+
+    const uint32_t tmem = sm.tmem_base;
+    const Waiter wait{&sm.abort, a.err};
+
+    if (warp == kProducerWarp) {
+        // ------------------------------------------------------------------ producer ----
+        const int P = geo.P;
+        const int ppt = kBN / P;                          // pages per tile (<= 8)
+        const int seq_pages = (L + P - 1) / P;
+        const uint32_t page_bytes = (uint32_t)P * 128u;  // one half of one page
+        const int32_t *bt = a.block_table + (size_t)b * geo.max_pages;
+        int issued = 0;
+        bool bad = false;
+        // position 0: W^R[w(h)] (B operand of the routing MMA) and the query block
+        if (lane == 0) {
+            ptx::mbar_arrive_expect_tx(&sm.full[0], kTileBytes + kBM * kD * 2);
+            ptx::tma_load_2d(sm.tiles[0], &wmap, &sm.full[0], 0, wsel * kD);
+            ptx::tma_load_2d(sm.tiles[0] + kHalfBytes, &wmap, &sm.full[0], 64, wsel * kD);
+            ptx::tma_load_3d(sm.q[0], &qmap, &sm.full[0], 0, h, q0 + m0);
+            ptx::tma_load_3d(sm.q[0] + kHalfBytes, &qmap, &sm.full[0], 64, h, q0 + m0);
+        }
+        __syncwarp();
+        issued = 1;
+        for (int i = 0; i < n_tiles; ++i) {
+            const int r = i + 1, s = r % kStages;
+            const int pg = i * ppt + lane;                // page index within the sequence
+            const bool exists = lane < ppt && pg < seq_pages;
+            const int page = exists ? bt[pg] : -1;
+            if (r >= kStages && !wait(&sm.empty[s], ((r / kStages) & 1) ^ 1)) break;
+            const bool in_range = exists && page >= 0 && page < geo.num_pages;
+            if (exists && !in_range) bad = true;
+            const unsigned mask = __ballot_sync(0xffffffffu, in_range);
+            if (lane == 0) ptx::mbar_arrive_expect_tx(&sm.full[s], __popc(mask) * page_bytes * 2u);
+            __syncwarp();
+            if (in_range) {
+                const int row = (page * geo.Hkv + g) * P;
+                uint8_t *dst = sm.tiles[s] + lane * page_bytes;
+                ptx::tma_load_2d(dst, &vmap, &sm.full[s], 0, row);
+                ptx::tma_load_2d(dst + kHalfBytes, &vmap, &sm.full[s], 64, row);
+            }
+            issued = r + 1;
+        }
+        if (__any_sync(0xffffffffu, bad) && lane == 0) raise_flag(a.err, KL_FLAG_BAD_PAGE);
+        if (sm.abort) {
+            // copies still in flight land before the CTA's shared memory goes away
+            for (int i = max(0, issued - kStages); i < issued; ++i) {
+                const uint64_t t0 = ptx::globaltimer();
+                while (!ptx::mbar_try_wait(&sm.full[i % kStages], (i / kStages) & 1) &&
+                       ptx::globaltimer() - t0 < kTimeoutNs) {
+                }
+            }
+        }
+    } else if (warp == kMmaWarp) {
+        // ------------------------------------------------------------- MMA issuer -------
+        // K-major SW128 operands step 32 B per 16 columns inside a 64-column half and jump a
+        // half (kHalfBytes) every 4 steps; MN-major SW128 operands step 16 rows = 2 KiB.
+        constexpr uint32_t idesc_qk = ptx::idesc_bf16(128, 128, false, false);
+        constexpr uint32_t idesc_pv = ptx::idesc_bf16(128, 128, false, true);
+        const uint64_t q_desc = ptx::smem_desc(ptx::smem_addr(sm.q[0]), 16, 1024, ptx::kSwizzle128B);
+        constexpr uint32_t kOpUnits = (kBM * kD * 2) >> 4;   // hi -> lo operand, 16-byte units
+        const uint64_t k_desc = ptx::smem_desc(ptx::smem_addr(sm.tiles[0]), 16, 1024, ptx::kSwizzle128B);
+        const uint64_t mn_desc =
+            ptx::smem_desc(ptx::smem_addr(sm.tiles[0]), kHalfBytes, 1024, ptx::kSwizzle128B);
+        const uint64_t p_desc = ptx::smem_desc(ptx::smem_addr(sm.p[0]), 16, 1024, ptx::kSwizzle128B);
+        auto kstep = [](int kk) -> uint32_t { return ((kk >> 2) * kHalfBytes + (kk & 3) * 32) >> 4; };
+
+        bool ok = wait(&sm.full[0], 0);
+        if (ok) {
+            ptx::tc_fence_after();
+            if (lane == 0) {
+                // Q_r = Q . W^R: A = query block (K-major), B = W^R (N = output dim j, MN-major)
+#pragma unroll
+                for (int kk = 0; kk < kD / 16; ++kk)
+                    ptx::mma_bf16(tmem + kColS, q_desc + kstep(kk), mn_desc + ((kk * 2048) >> 4),
+                                  idesc_pv, kk > 0);
+                ptx::mma_commit(&sm.empty[0]);
+                ptx::mma_commit(&sm.r_full);
+            }
+            __syncwarp();
+        }
+        ok = ok && wait(&sm.qr_ready, 0);
+        if (ok) ptx::tc_fence_after();
+        // output MMAs of tile j: O += P_hi . V_j + P_lo . V_j (B = the tile, N = dims, MN-major)
+        auto issue_pv = [&](int j) -> bool {
+            const int s = (j + 1) % kStages;
+            if (!wait(&sm.p_full, j & 1)) return false;
+            ptx::tc_fence_after();
+            if (lane == 0) {
+                const uint64_t b0 = mn_desc + ((s * kTileBytes) >> 4);
+#pragma unroll
+                for (int kk = 0; kk < 2 * kBN / 16; ++kk)
+                    ptx::mma_bf16(tmem + kColO, p_desc + (kk >= 8 ? kOpUnits : 0u) + kstep(kk & 7),
+                                  b0 + (((kk & 7) * 2048) >> 4), idesc_pv, (j > 0 || kk > 0) ? 1u : 0u);
+                ptx::mma_commit(&sm.empty[s]);
+                ptx::mma_commit(&sm.pv_done);
+            }
+            __syncwarp();
+            return true;
+        };
+        for (int i = 0; ok && i < n_tiles; ++i) {
+            const int r = i + 1, s = r % kStages, sb = i & 1;
+            if (!wait(&sm.full[s], (r / kStages) & 1)) { ok = false; break; }
+            if (i >= 2 && !wait(&sm.s_empty[sb], ((i >> 1) - 1) & 1)) { ok = false; break; }
+            ptx::tc_fence_after();
+            if (lane == 0) {
+                // S = Q_hi . V_i^T + Q_lo . V_i^T: A = Q_r (K-major), B = the tile (N = tokens,
+                // K-major)
+                const uint64_t b0 = k_desc + ((s * kTileBytes) >> 4);
+#pragma unroll
+                for (int kk = 0; kk < 2 * kD / 16; ++kk)
+                    ptx::mma_bf16(tmem + kColS + sb * kBN, q_desc + (kk >= 8 ? kOpUnits : 0u) + kstep(kk & 7),
+                                  b0 + kstep(kk & 7), idesc_qk, kk > 0);
+                ptx::mma_commit(&sm.s_full[sb]);
+            }
+            __syncwarp();
+            // the output MMA of the previous tile goes after this tile's score MMA, so the
+            // softmax of this tile overlaps it
+            if (i >= 1 && !issue_pv(i - 1)) { ok = false; break; }
+        }
+        if (ok) ok = issue_pv(n_tiles - 1);
+        // every MMA issued completes before TMEM is freed
+        if (lane == 0) ptx::mma_commit(&sm.drain);
+        __syncwarp();
+        const uint64_t t0 = ptx::globaltimer();
+        while (!ptx::mbar_try_wait(&sm.drain, 0) && ptx::globaltimer() - t0 < kTimeoutNs) {
+        }
+    } else {
+        // --------------------------------------------------------- softmax, epilogue ----
+        const int r = tid;                                   // query row = TMEM lane
+        const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+        const uint32_t q_s = ptx::smem_addr(sm.q[0]), q_lo = ptx::smem_addr(sm.q[1]);
+        // rows past the block's end take the last valid position: finite, never stored
+        const int pos_r = min(pos0 + r, pos_last);
+        const float sl2 = geo.scale * kLog2e;
+        bool ok = wait(&sm.r_full, 0);
+
+        // Routed query row: Q_r * scale * log2 e as hi + lo bf16, hi over the raw query rows
+        // (the routing MMA has read them).
+        if (ok) {
+            ptx::tc_fence_after();
+#pragma unroll
+            for (int c4 = 0; c4 < 4; ++c4) {
+                uint32_t u[32];
+                ptx::tmem_ld32(tmem + kColS + c4 * 32 + lane_base, u);
+                ptx::tmem_wait_ld();
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    uint32_t hi[4], lo[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e)
+                        split2(__uint_as_float(u[c * 8 + 2 * e]) * sl2,
+                               __uint_as_float(u[c * 8 + 2 * e + 1]) * sl2, hi[e], lo[e]);
+                    const uint32_t off = sw128_chunk(r, c4 * 32 + c * 8);
+                    st_shared_v4(q_s + off, hi[0], hi[1], hi[2], hi[3]);
+                    st_shared_v4(q_lo + off, lo[0], lo[1], lo[2], lo[3]);
+                }
+            }
+            ptx::tc_fence_before();
+            ptx::fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&sm.qr_ready);
+        }
+
+        float m_ref = -INFINITY;   // reference maximum of the row (base 2)
+        float l = 0.f;             // sum of 2^(s - m_ref) over the tokens seen
+        for (int i = 0; ok && i < n_tiles; ++i) {
+            const int sb = i & 1, t0 = i * kBN;
+            if (!wait(&sm.s_full[sb], (i >> 1) & 1)) { ok = false; break; }
+            ptx::tc_fence_after();
+            float sv[kBN];
+#pragma unroll
+            for (int c4 = 0; c4 < 4; ++c4) {
+                uint32_t u[32];
+                ptx::tmem_ld32(tmem + kColS + sb * kBN + c4 * 32 + lane_base, u);
+                ptx::tmem_wait_ld();
+#pragma unroll
+                for (int c = 0; c < 32; ++c) sv[c4 * 32 + c] = __uint_as_float(u[c]);
+            }
+            ptx::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&sm.s_empty[sb]);
+
+            // causal mask: token t0 + c is visible to the row when t0 + c <= pos_r
+            if (t0 + kBN - 1 > pos0) {
+                const int lim = pos_r - t0;
+#pragma unroll
+                for (int c = 0; c < kBN; ++c)
+                    if (c > lim) sv[c] = -INFINITY;
+            }
+            float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+            for (int c = 0; c < kBN; c += 4) {
+                mx[0] = fmaxf(mx[0], sv[c]);
+                mx[1] = fmaxf(mx[1], sv[c + 1]);
+                mx[2] = fmaxf(mx[2], sv[c + 2]);
+                mx[3] = fmaxf(mx[3], sv[c + 3]);
+            }
+            const float m_tile = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+            const float m_new = fmaxf(m_ref, m_tile);
+            // a new reference when the maximum grew by more than 2^8 (or is the first finite)
+            const bool grow = m_new > m_ref + kRescaleLog2;
+            // O holds tiles 0 .. i - 1 and the P buffers are free once the output MMAs of tile
+            // i - 1 are done
+            if (i > 0 && !wait(&sm.pv_done, (i - 1) & 1)) { ok = false; break; }
+            if (__any_sync(0xffffffffu, grow)) {
+                const float f = (m_new == -INFINITY || m_ref == -INFINITY) ? 0.f : ptx::ex2(m_ref - m_new);
+                if (i > 0) {
+                    ptx::tc_fence_after();
+#pragma unroll
+                    for (int c4 = 0; c4 < 4; ++c4) {
+                        uint32_t u[32];
+                        ptx::tmem_ld32(tmem + kColO + c4 * 32 + lane_base, u);
+                        ptx::tmem_wait_ld();
+#pragma unroll
+                        for (int c = 0; c < 32; ++c) u[c] = __float_as_uint(__uint_as_float(u[c]) * f);
+                        ptx::tmem_st32(tmem + kColO + c4 * 32 + lane_base, u);
+                    }
+                    ptx::tmem_wait_st();
+                }
+                l *= f;
+                m_ref = m_new;
+            }
+            const float mr = m_ref == -INFINITY ? 0.f : m_ref;
+
+            const uint32_t p_hi = ptx::smem_addr(sm.p[0]), p_lo = ptx::smem_addr(sm.p[1]);
+            float ls[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int c = 0; c < kBN; c += 8) {
+                float e[8];
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    e[k] = ptx::ex2(sv[c + k] - mr);
+                    ls[k & 3] += e[k];
+                }
+                uint32_t hi[4], lo[4];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) split2(e[2 * k], e[2 * k + 1], hi[k], lo[k]);
+                const uint32_t off = sw128_chunk(r, c);
+                st_shared_v4(p_hi + off, hi[0], hi[1], hi[2], hi[3]);
+                st_shared_v4(p_lo + off, lo[0], lo[1], lo[2], lo[3]);
+            }
+            l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+            // cache rows at or past the sequence's end (an unwritten page tail, or a page slot
+            // no TMA filled) become zeros, so that 0-weights never meet a non-finite value
+            if (t0 + kBN > L && t0 + r >= L) {
+                const uint32_t v_s = ptx::smem_addr(sm.tiles[(i + 1) % kStages]) + r * 128;
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    st_shared_v4(v_s + c * 16, 0u, 0u, 0u, 0u);
+                    st_shared_v4(v_s + kHalfBytes + c * 16, 0u, 0u, 0u, 0u);
+                }
+            }
+            ptx::tc_fence_before();
+            ptx::fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&sm.p_full);
+        }
+
+        // Epilogue: out = O / l for the block's rows.
+        if (ok && wait(&sm.pv_done, (n_tiles - 1) & 1)) {
+            ptx::tc_fence_after();
+            const float inv = l > 0.f ? 1.f / l : 0.f;
+            const size_t orow = ((size_t)(q0 + m0 + r) * geo.Hq + h) * kD;
+#pragma unroll
+            for (int c4 = 0; c4 < 4; ++c4) {
+                uint32_t u[32];
+                ptx::tmem_ld32(tmem + kColO + c4 * 32 + lane_base, u);
+                ptx::tmem_wait_ld();
+                if (r < rows) {
+                    if (a.out_dtype == KL_FP32) {
+                        float4 *o = reinterpret_cast<float4 *>(static_cast<float *>(a.out) + orow + c4 * 32);
+#pragma unroll
+                        for (int c = 0; c < 8; ++c)
+                            o[c] = make_float4(__uint_as_float(u[4 * c]) * inv, __uint_as_float(u[4 * c + 1]) * inv,
+                                               __uint_as_float(u[4 * c + 2]) * inv, __uint_as_float(u[4 * c + 3]) * inv);
+                    } else {
+                        uint4 *o = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(a.out) + orow + c4 * 32);
+#pragma unroll
+                        for (int c = 0; c < 4; ++c) {
+                            uint32_t w[4];
+#pragma unroll
+                            for (int e = 0; e < 4; ++e)
+                                w[e] = pack2(__uint_as_float(u[8 * c + 2 * e]) * inv,
+                                             __uint_as_float(u[8 * c + 2 * e + 1]) * inv);
+                            o[c] = make_uint4(w[0], w[1], w[2], w[3]);
+                        }
+                    }
+                }
+            }
+        }
+    }
+
+    ptx::tc_fence_before();
+    __syncthreads();
+    if (warp == kMmaWarp) {
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tmem, kTmemCols);
+    }
+}
+
+// Chunk append: row i of sequence b's chunk goes to position seq_lens[b] - n_b + i. One CTA per
+// (16 chunk rows, sequence); 16-byte copies.
+constexpr int kAppendRows = 16;
+
+__global__ void __launch_bounds__(128) append_chunk_kernel(int Hkv, int D, int P, int num_pages,
+                                                           int max_pages, int total_q,
+                                                           const uint4 *__restrict__ v_new,
+                                                           const int32_t *__restrict__ block_table,
+                                                           const int32_t *__restrict__ seq_lens,
+                                                           const int32_t *__restrict__ cu_q,
+                                                           uint4 *__restrict__ v_cache, int32_t *err) {
+    const int b = blockIdx.y;
+    const int q0 = cu_q[b], n = cu_q[b + 1] - q0, L = seq_lens[b];
+    if (q0 < 0 || n < 0 || q0 + n > total_q || L < n || L > max_pages * P) {
+        if (threadIdx.x == 0 && blockIdx.x == 0) raise_flag(err, KL_FLAG_BAD_LENGTH);
+        return;
+    }
+    const int i0 = blockIdx.x * kAppendRows;
+    const int cpr = D / 8;   // 16-byte chunks per row
+    const int per_row = Hkv * cpr;
+    for (int k = threadIdx.x; k < kAppendRows * per_row; k += blockDim.x) {
+        const int i = i0 + k / per_row;
+        if (i >= n) break;
+        const int gc = k % per_row, g = gc / cpr, c = gc % cpr;
+        const int pos = L - n + i;
+        const int page = block_table[(size_t)b * max_pages + pos / P];
+        if (page < 0 || page >= num_pages) {
+            raise_flag(err, KL_FLAG_BAD_PAGE);
+            continue;
+        }
+        v_cache[(((size_t)page * Hkv + g) * P + pos % P) * cpr + c] =
+            v_new[((size_t)(q0 + i) * Hkv + g) * cpr + c];
+    }
+}
+
+// ------------------------------------------------------------------------ host side ------
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (!fn) {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    }
+    return fn;
+}
+
+// bf16 tensor map of `rank` dimensions, innermost 128 elements (256-byte rows), box 64 x ...,
+// 128-byte swizzle.
+bool encode(CUtensorMap *map, const void *base, int rank, const cuuint64_t *dims,
+            const cuuint64_t *strides, const cuuint32_t *box) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    const cuuint32_t estr[3] = {1, 1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void *>(base), dims, strides,
+              box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+bool prefill_tc_supported(const Geometry &g) {
+    if (g.D != kD) return false;
+    if (g.P != 16 && g.P != 32 && g.P != 64 && g.P != 128) return false;
+    if ((int64_t)g.num_pages * g.Hkv * g.P >= ((int64_t)1 << 31)) return false;
+    int dev = 0, major = 0, minor = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return false;
+    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+    return major == 10 && minor == 3;
+}
+
+cudaError_t launch_prefill_tc(const PrefillArgs &a) {
+    const Geometry &g = a.geo;
+    if (g.B == 0 || a.total_q == 0 || a.max_q == 0) return cudaSuccess;
+    CUtensorMap vmap, wmap, qmap;
+    {
+        // cache as [num_pages * Hkv * P rows][128], one box = one page of one head (64 dims)
+        const cuuint64_t dims[2] = {kD, (cuuint64_t)g.num_pages * g.Hkv * g.P};
+        const cuuint64_t strides[1] = {kD * 2};
+        const cuuint32_t box[2] = {64, (cuuint32_t)g.P};
+        if (!encode(&vmap, a.v_cache, 2, dims, strides, box)) return cudaErrorInvalidValue;
+    }
+    {
+        // W^R as [Hw * 128 k rows][128 j], one box = a 64-column half of one matrix
+        const cuuint64_t hw = g.wr_per_qh ? (cuuint64_t)g.Hq : (cuuint64_t)g.Hkv;
+        const cuuint64_t dims[2] = {kD, hw * kD};
+        const cuuint64_t strides[1] = {kD * 2};
+        const cuuint32_t box[2] = {64, kD};
+        if (!encode(&wmap, a.w_r, 2, dims, strides, box)) return cudaErrorInvalidValue;
+    }
+    {
+        // q as [total_q][Hq][128], one box = 128 consecutive rows of one head (64 dims); rows
+        // past total_q read as zeros
+        const cuuint64_t dims[3] = {kD, (cuuint64_t)g.Hq, (cuuint64_t)a.total_q};
+        const cuuint64_t strides[2] = {kD * 2, (cuuint64_t)g.Hq * kD * 2};
+        const cuuint32_t box[3] = {64, 1, kBM};
+        if (!encode(&qmap, a.q, 3, dims, strides, box)) return cudaErrorInvalidValue;
+    }
+    const size_t smem = sizeof(PrefillSmem) + 1024;
+    static bool configured = false;
+    if (!configured) {
+        cudaError_t e = cudaFuncSetAttribute(prefill_tc_kernel,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(g.Hq, g.B, (a.max_q + kBM - 1) / kBM);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = a.stream;
+    return cudaLaunchKernelEx(&cfg, prefill_tc_kernel, vmap, wmap, qmap, a);
+}
+
+cudaError_t launch_append_chunk(const Geometry &g, int total_q, int max_q, const uint16_t *v_new,
+                                const int32_t *block_table, const int32_t *seq_lens,
+                                const int32_t *cu_q, uint16_t *v_cache, int32_t *err,
+                                cudaStream_t stream) {
+    if (g.B == 0 || total_q == 0 || max_q == 0) return cudaSuccess;
+    const dim3 grid((max_q + kAppendRows - 1) / kAppendRows, g.B);
+    append_chunk_kernel<<<grid, 128, 0, stream>>>(g.Hkv, g.D, g.P, g.num_pages, g.max_pages, total_q,
+                                                  reinterpret_cast<const uint4 *>(v_new), block_table,
+                                                  seq_lens, cu_q, reinterpret_cast<uint4 *>(v_cache), err);
+    return cudaGetLastError();
+}
+
+}  // namespace kl
