@@ -10,6 +10,8 @@ lines left in L2 are clean).
 
 Prints ONE JSON line (rank 0). `--impl reference` times the fp64 CPU oracle instead (the
 reference arm: a slow CPU program, timed on a bounded sample of the same workload).
+`--workload prefill_*` times the chunked prefill instead: one step = the chunk append plus the
+prefill attention, reported as query tokens/s against the bf16 tensor roofline.
 """
 from __future__ import annotations
 
@@ -214,6 +216,8 @@ def run_reference(args):
     import oracle
     wl = WORKLOADS[args.workload]
     x = generate(wl)
+    if wl.q_len > 0:
+        return run_reference_prefill(args, wl, x)
     per_step = max(1.0, args.cpu_seconds / max(1, args.steps))
     rates = []
     total_seqs = 0
@@ -263,6 +267,8 @@ def run_ours(args):
     if args.wr_per_query_head:
         wl = wl.with_(wr_per_query_head=True)
     x = generate(wl, seed=wl.seed + rank)           # replicas: each rank its own batch
+    if wl.q_len > 0:
+        return run_prefill(args, wl, x, dev, rank, world)
     B, Hq, D = x["q"].shape
     num_pages, Hkv, P, _ = x["v_cache"].shape
     max_pages = x["block_table"].shape[1]
@@ -443,6 +449,226 @@ def run_ours(args):
                      "algorithmic_bytes": ab["total"],
                      "traffic": recorded_traffic(wl.name, kname)},
         "gpu_launches": launches_per_step * args.steps,
+        "clocks": clk.summary(),
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+# --------------------------------------------------------------------------- prefill ----
+
+PREFILL_METRIC = "prefill attention query tokens/s and TFLOP/s on 1 GB300"
+
+
+def prefill_flops(x) -> dict:
+    """Useful FLOPs of a chunked prefill: 4 D per (query row, head, visible token) -- the score
+    and the output accumulation, 2 FLOPs each per dimension -- plus the routing projection,
+    2 D^2 per (query row, head). The kernel issues twice the attention MMA work (hi/lo pairs)."""
+    D = x["q_chunk"].shape[2]
+    Hq = x["q_chunk"].shape[1]
+    pairs = 0
+    for L, n in zip(x["seq_lens"].tolist(), x["q_lens"].tolist()):
+        # row i at position L - n + i sees L - n + i + 1 tokens
+        pairs += n * (L - n) + n * (n + 1) // 2
+    T = int(x["cu_q"][-1])
+    attn = 4.0 * D * Hq * pairs
+    route = 2.0 * T * Hq * D * D
+    return {"attention": attn, "routing": route, "total": attn + route, "pairs": pairs, "rows": T}
+
+
+def cpu_oracle_prefill_rate(x, seconds: float):
+    """Time the fp64 oracle (as it stands) on query rows (all heads) spread over the chunk."""
+    import numpy as np
+
+    import oracle
+    from paper_2606_21848_gb300.workloads import bf16_bits
+
+    q, w, v = bf16_bits(x["q_chunk"]), bf16_bits(x["w_r"]), bf16_bits(x["v_cache"])
+    bt, sl, cu = x["block_table"].numpy(), x["seq_lens"].numpy(), x["cu_q"].numpy()
+    T, Hq, D = x["q_chunk"].shape
+    wr_pq = bool(x["workload"].wr_per_query_head)
+    oracle.build()
+    stride = 7919                       # a fixed walk over the rows, early and late positions
+    rows, r = 0, 0
+    t0 = time.perf_counter()
+    while True:
+        sel = np.array([(r, h) for h in range(Hq)], np.int32)
+        oracle.prefill(q, w, v, bt, sl, cu, scale=1.0 / math.sqrt(D), wr_per_query_head=wr_pq,
+                       rows=sel)
+        rows += 1
+        r = (r + stride) % T
+        el = time.perf_counter() - t0
+        if el >= seconds:
+            break
+    return rows / el, rows, el
+
+
+def run_reference_prefill(args, wl, x):
+    import oracle
+    per_step = max(1.0, args.cpu_seconds / max(1, args.steps))
+    rates, total = [], 0
+    for i in range(args.warmup + args.steps):
+        rt, n, _ = cpu_oracle_prefill_rate(x, per_step if i >= args.warmup else 0.0)
+        if i >= args.warmup:
+            rates.append(rt)
+            total += n
+    value = statistics.mean(rates)
+    T = int(x["cu_q"][-1])
+    line = {
+        "impl": "reference", "metric": PREFILL_METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1000.0 * T / value, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": wl.name, "num_seqs": wl.num_seqs, "q_heads": wl.num_q_heads,
+                   "kv_heads": wl.num_kv_heads, "head_dim": wl.head_dim,
+                   "page_size": wl.page_size, "seq_len": wl.seq_len, "chunk": wl.q_len},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": oracle.threads(),
+                         "kind": "oracle",
+                         "sample": f"{total} query rows (all heads) of {wl.name} on a fixed "
+                                   f"stride over the chunk, ~{per_step:.1f}s per step"},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_prefill(args, wl, x, dev, rank, world):
+    """One prefill step = the chunk append (kl_append_v_chunk) + the chunked prefill
+    (kl_prefill_attention), inputs resident in HBM, L2 flushed between steps."""
+    import torch
+
+    import paper_2606_21848_gb300 as kl
+
+    T, Hq, D = x["q_chunk"].shape
+    B = x["seq_lens"].shape[0]
+    num_pages, Hkv, P, _ = x["v_cache"].shape
+    sh = kl.make_shape(B, Hq, Hkv, D, P, num_pages, x["block_table"].shape[1],
+                       wl.wr_per_query_head)
+    max_q = int(x["q_lens"].max())
+    g = {k: x[k].to(dev) for k in ("q_chunk", "v_chunk", "w_r", "v_cache", "block_table",
+                                    "seq_lens", "cu_q")}
+    out = torch.empty(T, Hq, D, dtype=torch.bfloat16, device=dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    flush_sink = torch.empty((), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def flush_l2():
+        flush.zero_()
+        torch.sum(flush, dim=0, out=flush_sink)
+
+    def step(d, ev=None):
+        if ev: ev[0].record(stream)
+        kl.kl_append_v_chunk(sh, d["v_chunk"], d["block_table"], d["seq_lens"], d["cu_q"], T,
+                             max_q, g["v_cache"], err, stream)
+        if ev: ev[1].record(stream)
+        kl.kl_prefill_attention(sh, d["q_chunk"], g["w_r"], g["v_cache"], d["block_table"],
+                                d["seq_lens"], d["cu_q"], T, max_q, out, kl.KL_BF16, err, stream)
+        if ev: ev[2].record(stream)
+
+    E = lambda: torch.cuda.Event(enable_timing=True)
+    for _ in range(args.warmup):
+        flush_l2()
+        step(g, [E(), E(), E()])
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0, f"device error flags {int(err.item())}"
+    evs = [[E(), E(), E()] for _ in range(args.steps)]
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(dev.index) as clk:
+        for i in range(args.steps):
+            flush_l2()
+            step(g, evs[i])
+        torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    step_ms = statistics.mean(e[0].elapsed_time(e[2]) for e in evs)
+    app_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+    pre_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+    if world > 1:
+        t = torch.tensor([step_ms, app_ms, pre_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        step_ms, app_ms, pre_ms = (float(v) for v in t)
+    assert int(err.item()) == 0, f"device error flags {int(err.item())}"
+
+    fl = prefill_flops(x)
+    tflops = fl["total"] / (pre_ms / 1e3) / 1e12
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            peak, peak_kind = float(json.load(f)["bf16_tflops"]), "measured (cuBLAS bf16 burst)"
+    except Exception:
+        peak, peak_kind = 1900.0, "fallback"
+
+    e2e = None
+    if not args.no_e2e:
+        h_in = {k: x[k].pin_memory() for k in ("q_chunk", "v_chunk", "block_table", "seq_lens",
+                                               "cu_q")}
+        h_out = torch.empty(T, Hq, D, dtype=torch.bfloat16).pin_memory()
+        d_in = {k: torch.empty_like(g[k]) for k in h_in}
+        h2d = sum(t.numel() * t.element_size() for t in h_in.values())
+        d2h = h_out.numel() * h_out.element_size()
+
+        def e2e_step():
+            for k in h_in:
+                d_in[k].copy_(h_in[k], non_blocking=True)
+            step(d_in)
+            h_out.copy_(out, non_blocking=True)
+
+        for _ in range(args.warmup):
+            flush_l2()
+            e2e_step()
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(args.steps):
+            flush_l2()
+            a, b = E(), E()
+            a.record(stream)
+            e2e_step()
+            b.record(stream)
+            ts.append((a, b))
+        torch.cuda.synchronize()
+        e2e_ms = statistics.mean(a.elapsed_time(b) for a, b in ts)
+        if world > 1:
+            t = torch.tensor([e2e_ms], device=dev)
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+            e2e_ms = float(t[0])
+        e2e = {"value": T * world / (e2e_ms / 1e3), "unit": "tokens/s",
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms}
+
+    if rank != 0:
+        return 0
+    cpu = None
+    if world == 1:
+        import oracle
+        rate, n, el = cpu_oracle_prefill_rate(x, args.cpu_seconds)
+        cpu = {"value": rate, "unit": "tokens/s", "cores": oracle.threads(), "kind": "oracle",
+               "sample": f"{n} query rows (all {Hq} heads) of {wl.name} on a fixed stride over "
+                         f"the chunk, fp64, in {el:.1f}s"}
+    line = {
+        "metric": PREFILL_METRIC, "value": T * world / (step_ms / 1e3), "unit": "tokens/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded; inputs resident in HBM)",
+        "config": {"workload": wl.name, "num_seqs": B, "q_heads": Hq, "kv_heads": Hkv,
+                   "head_dim": D, "page_size": P, "seq_len": wl.seq_len, "chunk": wl.q_len,
+                   "query_rows": T, "visible_pairs": fl["pairs"],
+                   "w_r": "per query head" if wl.wr_per_query_head else "per value head",
+                   "operands": "hi + lo bf16 pairs (2x the attention MMA work)",
+                   "l2": "flushed between timed steps (512 MiB write, then read back)",
+                   "parallelism": f"replicas x{world}"},
+        "ms_breakdown": {"append": app_ms, "prefill": pre_ms},
+        "tflops": tflops,
+        "kernels_per_step": 2,
+        "roofline": {"bound": "tensor", "achieved": tflops, "peak": peak, "unit": "TFLOP/s",
+                     "frac": tflops / peak, "peak_kind": peak_kind,
+                     "algorithmic_flops": fl["total"], "traffic": None},
+        "gpu_launches": 2 * args.steps,
         "clocks": clk.summary(),
         "e2e": e2e,
         "cpu_baseline": cpu,

@@ -18,7 +18,11 @@ Recipe (fixed, so that a seed names one input set):
    offset_b + j; ``permuted`` applies one ``randperm(num_pages)`` to that list, which scatters
    every sequence over one shared pool. The pool holds exactly the pages the sequences use;
    block-table entries past a sequence's last page are -1;
-6. the current token: ``positions = seq_lens - 1`` and v_new ~ N(0, 1) of shape [B, Hkv, D].
+6. the current token: ``positions = seq_lens - 1`` and v_new ~ N(0, 1) of shape [B, Hkv, D];
+7. prefill workloads only (q_len > 0): the chunk of each sequence is its last
+   n_b = min(q_len, L_b) rows; its queries q_chunk ~ N(0, 1) [T, Hq, D] (T = sum n_b, rows of
+   sequence b at cu_q[b] ..) and its value rows v_chunk ~ N(0, 1) [T, Hkv, D] (for the chunk
+   append; the pool already holds values at those rows).
 """
 from __future__ import annotations
 
@@ -49,6 +53,7 @@ class Workload:
     wr_per_query_head: bool = False
     num_splits: int = 0                   # 0: the library chooses
     seed: int = 0
+    q_len: int = 0                        # prefill: query rows per sequence (its last rows)
 
     @property
     def group(self) -> int:
@@ -83,6 +88,18 @@ WORKLOADS: dict[str, Workload] = {
 }
 
 ORDER = ["tiny_mha", "small_gqa", "long_context", "ragged_serving", "high_concurrency_70b"]
+
+# Prefill workloads (chunked prefill, the step before decode): a whole 32K-token prompt with
+# the paper's Qwen2-1.5B attention (12 query heads, 2 value heads, head dim 128, W^R per query
+# head, trained at 32,768 tokens), and a serving-style chunk of 512 new tokens on an
+# 8192-token sequence (7680 cached) for a batch of 8, GQA 32 / 8.
+WORKLOADS.update({
+    "prefill_qwen2_32k": Workload("prefill_qwen2_32k", 1, 12, 2, 128, 16, seq_len=32768,
+                                  wr_std=math.sqrt(1 / 128), wr_per_query_head=True, seed=5,
+                                  q_len=32768),
+    "prefill_chunked_gqa": Workload("prefill_chunked_gqa", 8, 32, 8, 128, 16, seq_len=8192,
+                                    wr_std=math.sqrt(1 / 128), seed=6, q_len=512),
+})
 
 
 def _pool_chunk(args):
@@ -148,8 +165,17 @@ def generate(wl: Workload, seed: int | None = None) -> dict:
 
     positions = (seq_lens - 1).clamp_min(0).to(torch.int32)
     v_new = torch.randn(B, Hkv, D, generator=g).to(torch.bfloat16)
-    return dict(q=q, w_r=w_r, v_cache=v_cache, block_table=block_table, seq_lens=seq_lens,
-                positions=positions, v_new=v_new, num_pages=num_pages, workload=wl)
+    out = dict(q=q, w_r=w_r, v_cache=v_cache, block_table=block_table, seq_lens=seq_lens,
+               positions=positions, v_new=v_new, num_pages=num_pages, workload=wl)
+    if wl.q_len > 0:
+        q_lens = torch.clamp(seq_lens, max=wl.q_len).to(torch.int32)
+        cu_q = torch.zeros(B + 1, dtype=torch.int32)
+        cu_q[1:] = torch.cumsum(q_lens, 0).to(torch.int32)
+        T = int(cu_q[-1])
+        out.update(q_chunk=torch.randn(T, Hq, D, generator=g).to(torch.bfloat16),
+                   v_chunk=torch.randn(T, Hkv, D, generator=g).to(torch.bfloat16),
+                   q_lens=q_lens, cu_q=cu_q)
+    return out
 
 
 def bf16_bits(t: torch.Tensor):
