@@ -11,8 +11,12 @@
 //
 // Each cached tile V_t [128 tokens x 128 dims] arrives once by TMA (one box per page) and feeds
 // both products from the same shared-memory copy: as the K-major B operand of the score MMAs and
-// as the MN-major B operand of the output MMAs. Accumulators live in TMEM: S in two 128-column
-// buffers (the score MMAs of tile t + 1 run while tile t is in the softmax), O in a third.
+// as the MN-major B operand of the output MMAs. Everything else lives in TMEM (512 columns, 128
+// each): S, the softmax weights P_hi | P_lo, O, and the routed query Q_hi | Q_lo. Q and P enter
+// the MMAs as A operands straight from TMEM, so the only operand the tensor cores read from
+// shared memory is the cache tile. The softmax copies S of tile t into registers and releases
+// it at once, so the score MMAs of tile t + 1 run during the softmax of tile t, and the output
+// MMAs of tile t during the softmax of tile t + 1 (P is rewritten only after they finish).
 //
 // Precision: the routed query (times scale * log2 e) and the softmax weights are each carried as
 // a pair of bf16 operands, x = hi + lo, which keeps about 16 significant bits where one bf16
@@ -26,10 +30,13 @@
 // O in TMEM and its running sum l are rescaled; otherwise p may reach 2^8, well inside bf16 and
 // fp32 range, and the final O / l is unchanged because O and l share the same reference.
 //
-// Roles (192 threads, one CTA per SM):
+// Roles (224 threads, one CTA per SM):
 //   warps 0-3  softmax and epilogue (TMEM lane quarters 0-3)
 //   warp 4     producer: TMA of W^R and the query block (ring position 0), then cache tiles
-//   warp 5     MMA issuer (one elected lane) and TMEM owner
+//   warp 5     routing and score MMA issuer (one elected lane) and TMEM owner
+//   warp 6     output MMA issuer. One thread issuing tcgen05.mma back to back reaches about
+//              88 cycles per 128 x 128 x 16 MMA; two issuing threads together reach the
+//              tensor cores' 64.
 // Every wait is bounded (about one second); a wait that runs out raises KL_FLAG_TIMEOUT, makes
 // every role leave its loop, drains outstanding copies and MMAs and frees TMEM.
 #include <cudaTypedefs.h>
@@ -44,32 +51,33 @@ namespace {
 constexpr int kD = 128;
 constexpr int kBM = 128;                          // query rows per CTA
 constexpr int kBN = 128;                          // cache rows per tile
-constexpr int kStages = 3;
+constexpr int kStages = 4;
 constexpr int kComputeWarps = 4;
 constexpr int kProducerWarp = 4;
-constexpr int kMmaWarp = 5;
-constexpr int kThreads = 6 * 32;
+constexpr int kMmaWarp = 5;                       // routing and score MMAs; TMEM owner
+constexpr int kPvWarp = 6;                        // output MMAs
+constexpr int kThreads = 7 * 32;
 constexpr uint32_t kTileBytes = kBN * kD * 2;     // 32 KiB
 constexpr uint32_t kHalfBytes = kTileBytes / 2;   // one 64-column half: 128 rows x 128 B
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColS = 0;                     // S buffers: columns 0 and 128
+constexpr uint32_t kColS = 0;                     // S: columns 0 .. 127
+constexpr uint32_t kColP = 128;                   // P_hi: 128 .. 191, P_lo: 192 .. 255
 constexpr uint32_t kColO = 256;                   // O: columns 256 .. 383
+constexpr uint32_t kColQ = 384;                   // Q_hi: 384 .. 447, Q_lo: 448 .. 511
+constexpr uint32_t kLoCols = 64;                  // hi -> lo of a packed bf16 operand
 constexpr float kRescaleLog2 = 8.f;
 constexpr uint64_t kTimeoutNs = 1000000000ull;
 
 struct __align__(1024) PrefillSmem {
-    // q[0]: the query block, then hi of the routed, scaled query Q_r; q[1]: its lo. K-major,
-    // 128B-swizzled: [64-dim half][128 rows][128 B].
-    uint8_t q[2][kBM * kD * 2];
+    // The query block (A operand of the routing MMA); K-major, 128B-swizzled:
+    // [64-dim half][128 rows][128 B].
+    uint8_t q[kBM * kD * 2];
     // Ring of 32 KiB slots: W^R[w(h)] at position 0 ([64-column half][128 k rows][128 B]), then
     // the cache tiles ([64-dim half][128 tokens][128 B]); all 128B-swizzled.
     uint8_t tiles[kStages][kTileBytes];
-    // Softmax weights of one tile, hi (p[0]) and lo (p[1]), the A operands of the output MMAs;
-    // K-major, 128B-swizzled: [64-token half][128 rows][128 B].
-    uint8_t p[2][kBM * kBN * 2];
     uint64_t full[kStages], empty[kStages];
-    uint64_t s_full[2], s_empty[2], p_full, pv_done;
-    uint64_t r_full, qr_ready, drain;
+    uint64_t s_full, s_free, p_full, pv_done;
+    uint64_t r_full, qr_ready, drain, drain2;
     uint32_t tmem_base;
     int abort;
 };
@@ -96,13 +104,6 @@ struct Waiter {
         return __all_sync(0xffffffffu, ok);
     }
 };
-
-// Byte offset of the 16-byte chunk that holds columns c .. c + 7 (c a multiple of 8) of row r
-// in a K-major, 128B-swizzled operand of 128 rows and 128 columns laid out as
-// [64-column half][128 rows][128 B]: the chunk index inside the row is XORed with r mod 8.
-__device__ __forceinline__ uint32_t sw128_chunk(int r, int c) {
-    return (uint32_t)((c >> 6) * kHalfBytes + r * 128 + ((((c >> 3) & 7) ^ (r & 7)) << 4));
-}
 
 __device__ __forceinline__ uint32_t pack2(float a, float b) {
     const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
@@ -158,15 +159,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             ptx::mbar_init(&sm.full[s], 1);
             ptx::mbar_init(&sm.empty[s], 1);
         }
-        for (int i = 0; i < 2; ++i) {
-            ptx::mbar_init(&sm.s_full[i], 1);
-            ptx::mbar_init(&sm.s_empty[i], kComputeWarps);
-        }
+        // One completion per tile on each. Every wait names the completion it needs: MMAs
+        // that write different TMEM ranges are not assumed to complete in issue order.
+        ptx::mbar_init(&sm.s_full, 1);
+        ptx::mbar_init(&sm.s_free, kComputeWarps);
         ptx::mbar_init(&sm.p_full, kComputeWarps);
         ptx::mbar_init(&sm.pv_done, 1);
         ptx::mbar_init(&sm.r_full, 1);
         ptx::mbar_init(&sm.qr_ready, kComputeWarps);
         ptx::mbar_init(&sm.drain, 1);
+        ptx::mbar_init(&sm.drain2, 1);
         sm.abort = 0;
         ptx::fence_mbar_init();
     }
@@ -200,8 +202,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             ptx::mbar_arrive_expect_tx(&sm.full[0], kTileBytes + kBM * kD * 2);
             ptx::tma_load_2d(sm.tiles[0], &wmap, &sm.full[0], 0, wsel * kD);
             ptx::tma_load_2d(sm.tiles[0] + kHalfBytes, &wmap, &sm.full[0], 64, wsel * kD);
-            ptx::tma_load_3d(sm.q[0], &qmap, &sm.full[0], 0, h, q0 + m0);
-            ptx::tma_load_3d(sm.q[0] + kHalfBytes, &qmap, &sm.full[0], 64, h, q0 + m0);
+            ptx::tma_load_3d(sm.q, &qmap, &sm.full[0], 0, h, q0 + m0);
+            ptx::tma_load_3d(sm.q + kHalfBytes, &qmap, &sm.full[0], 64, h, q0 + m0);
         }
         __syncwarp();
         issued = 1;
@@ -234,113 +236,119 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
         }
-    } else if (warp == kMmaWarp) {
-        // ------------------------------------------------------------- MMA issuer -------
+    } else if (warp == kMmaWarp || warp == kPvWarp) {
+        // ---------------------------------------------------------------- MMA issuers ----
         // K-major SW128 operands step 32 B per 16 columns inside a 64-column half and jump a
-        // half (kHalfBytes) every 4 steps; MN-major SW128 operands step 16 rows = 2 KiB.
+        // half (kHalfBytes) every 4 steps; MN-major SW128 operands step 16 rows = 2 KiB; TMEM
+        // A operands step 8 columns (16 packed bf16).
         constexpr uint32_t idesc_qk = ptx::idesc_bf16(128, 128, false, false);
         constexpr uint32_t idesc_pv = ptx::idesc_bf16(128, 128, false, true);
-        const uint64_t q_desc = ptx::smem_desc(ptx::smem_addr(sm.q[0]), 16, 1024, ptx::kSwizzle128B);
-        constexpr uint32_t kOpUnits = (kBM * kD * 2) >> 4;   // hi -> lo operand, 16-byte units
+        const uint64_t q_desc = ptx::smem_desc(ptx::smem_addr(sm.q), 16, 1024, ptx::kSwizzle128B);
         const uint64_t k_desc = ptx::smem_desc(ptx::smem_addr(sm.tiles[0]), 16, 1024, ptx::kSwizzle128B);
         const uint64_t mn_desc =
             ptx::smem_desc(ptx::smem_addr(sm.tiles[0]), kHalfBytes, 1024, ptx::kSwizzle128B);
-        const uint64_t p_desc = ptx::smem_desc(ptx::smem_addr(sm.p[0]), 16, 1024, ptx::kSwizzle128B);
         auto kstep = [](int kk) -> uint32_t { return ((kk >> 2) * kHalfBytes + (kk & 3) * 32) >> 4; };
-
-        bool ok = wait(&sm.full[0], 0);
-        if (ok) {
-            ptx::tc_fence_after();
-            if (lane == 0) {
-                // Q_r = Q . W^R: A = query block (K-major), B = W^R (N = output dim j, MN-major)
+        bool ok = true;
+        if (warp == kMmaWarp) {
+            // routing, then the score MMAs of every tile
+            ok = wait(&sm.full[0], 0);
+            if (ok) {
+                ptx::tc_fence_after();
+                if (lane == 0) {
+                    // Q_r = Q . W^R: A = query block (K-major), B = W^R (N = output dim j,
+                    // MN-major)
 #pragma unroll
-                for (int kk = 0; kk < kD / 16; ++kk)
-                    ptx::mma_bf16(tmem + kColS, q_desc + kstep(kk), mn_desc + ((kk * 2048) >> 4),
-                                  idesc_pv, kk > 0);
-                ptx::mma_commit(&sm.empty[0]);
-                ptx::mma_commit(&sm.r_full);
+                    for (int kk = 0; kk < kD / 16; ++kk)
+                        ptx::mma_bf16(tmem + kColS, q_desc + kstep(kk), mn_desc + ((kk * 2048) >> 4),
+                                      idesc_pv, kk > 0);
+                    ptx::mma_commit(&sm.empty[0]);
+                    ptx::mma_commit(&sm.r_full);
+                }
+                __syncwarp();
             }
-            __syncwarp();
+            ok = ok && wait(&sm.qr_ready, 0);
+            for (int i = 0; ok && i < n_tiles; ++i) {
+                const int r = i + 1, s = r % kStages;
+                if (!wait(&sm.full[s], (r / kStages) & 1)) { ok = false; break; }
+                // the softmax has copied S of tile i - 1 out of TMEM
+                if (i >= 1 && !wait(&sm.s_free, (i - 1) & 1)) { ok = false; break; }
+                ptx::tc_fence_after();
+                if (lane == 0) {
+                    // S = Q_hi . V_i^T + Q_lo . V_i^T: A = Q_r in TMEM, B = the tile
+                    // (N = tokens, K-major)
+                    const uint64_t b0 = k_desc + ((s * kTileBytes) >> 4);
+#pragma unroll
+                    for (int kk = 0; kk < 2 * kD / 16; ++kk)
+                        ptx::mma_bf16_ts(tmem + kColS,
+                                         tmem + kColQ + (kk >= 8 ? kLoCols : 0u) + (kk & 7) * 8,
+                                         b0 + kstep(kk & 7), idesc_qk, kk > 0);
+                    ptx::mma_commit(&sm.s_full);
+                }
+                __syncwarp();
+            }
+        } else {
+            // the output MMAs of every tile: O += P_hi . V_j + P_lo . V_j; A = P in TMEM,
+            // B = the tile (N = dims, MN-major)
+            for (int j = 0; j < n_tiles; ++j) {
+                const int s = (j + 1) % kStages;
+                if (!wait(&sm.p_full, j & 1)) { ok = false; break; }
+                ptx::tc_fence_after();
+                if (lane == 0) {
+                    const uint64_t b0 = mn_desc + ((s * kTileBytes) >> 4);
+                    const uint32_t pa = tmem + kColP;
+#pragma unroll
+                    for (int kk = 0; kk < 2 * kBN / 16; ++kk)
+                        ptx::mma_bf16_ts(tmem + kColO, pa + (kk >= 8 ? kLoCols : 0u) + (kk & 7) * 8,
+                                         b0 + (((kk & 7) * 2048) >> 4), idesc_pv,
+                                         (j > 0 || kk > 0) ? 1u : 0u);
+                    ptx::mma_commit(&sm.empty[s]);
+                    ptx::mma_commit(&sm.pv_done);
+                }
+                __syncwarp();
+            }
         }
-        ok = ok && wait(&sm.qr_ready, 0);
-        if (ok) ptx::tc_fence_after();
-        // output MMAs of tile j: O += P_hi . V_j + P_lo . V_j (B = the tile, N = dims, MN-major)
-        auto issue_pv = [&](int j) -> bool {
-            const int s = (j + 1) % kStages;
-            if (!wait(&sm.p_full, j & 1)) return false;
-            ptx::tc_fence_after();
-            if (lane == 0) {
-                const uint64_t b0 = mn_desc + ((s * kTileBytes) >> 4);
-#pragma unroll
-                for (int kk = 0; kk < 2 * kBN / 16; ++kk)
-                    ptx::mma_bf16(tmem + kColO, p_desc + (kk >= 8 ? kOpUnits : 0u) + kstep(kk & 7),
-                                  b0 + (((kk & 7) * 2048) >> 4), idesc_pv, (j > 0 || kk > 0) ? 1u : 0u);
-                ptx::mma_commit(&sm.empty[s]);
-                ptx::mma_commit(&sm.pv_done);
-            }
-            __syncwarp();
-            return true;
-        };
-        for (int i = 0; ok && i < n_tiles; ++i) {
-            const int r = i + 1, s = r % kStages, sb = i & 1;
-            if (!wait(&sm.full[s], (r / kStages) & 1)) { ok = false; break; }
-            if (i >= 2 && !wait(&sm.s_empty[sb], ((i >> 1) - 1) & 1)) { ok = false; break; }
-            ptx::tc_fence_after();
-            if (lane == 0) {
-                // S = Q_hi . V_i^T + Q_lo . V_i^T: A = Q_r (K-major), B = the tile (N = tokens,
-                // K-major)
-                const uint64_t b0 = k_desc + ((s * kTileBytes) >> 4);
-#pragma unroll
-                for (int kk = 0; kk < 2 * kD / 16; ++kk)
-                    ptx::mma_bf16(tmem + kColS + sb * kBN, q_desc + (kk >= 8 ? kOpUnits : 0u) + kstep(kk & 7),
-                                  b0 + kstep(kk & 7), idesc_qk, kk > 0);
-                ptx::mma_commit(&sm.s_full[sb]);
-            }
-            __syncwarp();
-            // the output MMA of the previous tile goes after this tile's score MMA, so the
-            // softmax of this tile overlaps it
-            if (i >= 1 && !issue_pv(i - 1)) { ok = false; break; }
-        }
-        if (ok) ok = issue_pv(n_tiles - 1);
-        // every MMA issued completes before TMEM is freed
-        if (lane == 0) ptx::mma_commit(&sm.drain);
+        (void)ok;
+        // every MMA this warp issued completes before TMEM is freed
+        uint64_t *drain = warp == kMmaWarp ? &sm.drain : &sm.drain2;
+        if (lane == 0) ptx::mma_commit(drain);
         __syncwarp();
         const uint64_t t0 = ptx::globaltimer();
-        while (!ptx::mbar_try_wait(&sm.drain, 0) && ptx::globaltimer() - t0 < kTimeoutNs) {
+        while (!ptx::mbar_try_wait(drain, 0) && ptx::globaltimer() - t0 < kTimeoutNs) {
         }
     } else {
         // --------------------------------------------------------- softmax, epilogue ----
         const int r = tid;                                   // query row = TMEM lane
         const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-        const uint32_t q_s = ptx::smem_addr(sm.q[0]), q_lo = ptx::smem_addr(sm.q[1]);
         // rows past the block's end take the last valid position: finite, never stored
         const int pos_r = min(pos0 + r, pos_last);
         const float sl2 = geo.scale * kLog2e;
         bool ok = wait(&sm.r_full, 0);
 
-        // Routed query row: Q_r * scale * log2 e as hi + lo bf16, hi over the raw query rows
-        // (the routing MMA has read them).
+        // Routed query row: Q_r * scale * log2 e as hi + lo bf16 pairs into the Q columns.
         if (ok) {
             ptx::tc_fence_after();
 #pragma unroll
-            for (int c4 = 0; c4 < 4; ++c4) {
-                uint32_t u[32];
-                ptx::tmem_ld32(tmem + kColS + c4 * 32 + lane_base, u);
+            for (int c4 = 0; c4 < 4; c4 += 2) {
+                uint32_t u0[32], u1[32];
+                ptx::tmem_ld32(tmem + kColS + c4 * 32 + lane_base, u0);
+                ptx::tmem_ld32(tmem + kColS + c4 * 32 + 32 + lane_base, u1);
                 ptx::tmem_wait_ld();
+                ptx::reg_fence(u0);
+                ptx::reg_fence(u1);
+                uint32_t hi[32], lo[32];
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    uint32_t hi[4], lo[4];
-#pragma unroll
-                    for (int e = 0; e < 4; ++e)
-                        split2(__uint_as_float(u[c * 8 + 2 * e]) * sl2,
-                               __uint_as_float(u[c * 8 + 2 * e + 1]) * sl2, hi[e], lo[e]);
-                    const uint32_t off = sw128_chunk(r, c4 * 32 + c * 8);
-                    st_shared_v4(q_s + off, hi[0], hi[1], hi[2], hi[3]);
-                    st_shared_v4(q_lo + off, lo[0], lo[1], lo[2], lo[3]);
+                for (int e = 0; e < 16; ++e) {
+                    split2(__uint_as_float(u0[2 * e]) * sl2, __uint_as_float(u0[2 * e + 1]) * sl2,
+                           hi[e], lo[e]);
+                    split2(__uint_as_float(u1[2 * e]) * sl2, __uint_as_float(u1[2 * e + 1]) * sl2,
+                           hi[16 + e], lo[16 + e]);
                 }
+                // 64 values -> 32 packed columns
+                ptx::tmem_st32(tmem + kColQ + c4 * 16 + lane_base, hi);
+                ptx::tmem_st32(tmem + kColQ + kLoCols + c4 * 16 + lane_base, lo);
             }
+            ptx::tmem_wait_st();
             ptx::tc_fence_before();
-            ptx::fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&sm.qr_ready);
         }
@@ -348,21 +356,35 @@ __global__ void __launch_bounds__(kThreads, 1)
         float m_ref = -INFINITY;   // reference maximum of the row (base 2)
         float l = 0.f;             // sum of 2^(s - m_ref) over the tokens seen
         for (int i = 0; ok && i < n_tiles; ++i) {
-            const int sb = i & 1, t0 = i * kBN;
-            if (!wait(&sm.s_full[sb], (i >> 1) & 1)) { ok = false; break; }
+            const int t0 = i * kBN;
+            if (!wait(&sm.s_full, i & 1)) { ok = false; break; }
             ptx::tc_fence_after();
             float sv[kBN];
-#pragma unroll
-            for (int c4 = 0; c4 < 4; ++c4) {
-                uint32_t u[32];
-                ptx::tmem_ld32(tmem + kColS + sb * kBN + c4 * 32 + lane_base, u);
+            {
+                // the four loads in flight together, one wait
+                uint32_t u0[32], u1[32], u2[32], u3[32];
+                const uint32_t sa = tmem + kColS + lane_base;
+                ptx::tmem_ld32(sa, u0);
+                ptx::tmem_ld32(sa + 32, u1);
+                ptx::tmem_ld32(sa + 64, u2);
+                ptx::tmem_ld32(sa + 96, u3);
                 ptx::tmem_wait_ld();
+                ptx::reg_fence(u0);
+                ptx::reg_fence(u1);
+                ptx::reg_fence(u2);
+                ptx::reg_fence(u3);
 #pragma unroll
-                for (int c = 0; c < 32; ++c) sv[c4 * 32 + c] = __uint_as_float(u[c]);
+                for (int c = 0; c < 32; ++c) {
+                    sv[c] = __uint_as_float(u0[c]);
+                    sv[32 + c] = __uint_as_float(u1[c]);
+                    sv[64 + c] = __uint_as_float(u2[c]);
+                    sv[96 + c] = __uint_as_float(u3[c]);
+                }
             }
+            // S is in registers: the score MMAs of the next tile may overwrite it
             ptx::tc_fence_before();
             __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(&sm.s_empty[sb]);
+            if (lane == 0) ptx::mbar_arrive(&sm.s_free);
 
             // causal mask: token t0 + c is visible to the row when t0 + c <= pos_r
             if (t0 + kBN - 1 > pos0) {
@@ -383,18 +405,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float m_new = fmaxf(m_ref, m_tile);
             // a new reference when the maximum grew by more than 2^8 (or is the first finite)
             const bool grow = m_new > m_ref + kRescaleLog2;
-            // O holds tiles 0 .. i - 1 and the P buffers are free once the output MMAs of tile
-            // i - 1 are done
-            if (i > 0 && !wait(&sm.pv_done, (i - 1) & 1)) { ok = false; break; }
             if (__any_sync(0xffffffffu, grow)) {
                 const float f = (m_new == -INFINITY || m_ref == -INFINITY) ? 0.f : ptx::ex2(m_ref - m_new);
                 if (i > 0) {
+                    // O holds tiles 0 .. i - 1 once the output MMAs of tile i - 1 are done
+                    if (!wait(&sm.pv_done, (i - 1) & 1)) { ok = false; break; }
                     ptx::tc_fence_after();
 #pragma unroll
                     for (int c4 = 0; c4 < 4; ++c4) {
                         uint32_t u[32];
                         ptx::tmem_ld32(tmem + kColO + c4 * 32 + lane_base, u);
                         ptx::tmem_wait_ld();
+                        ptx::reg_fence(u);
 #pragma unroll
                         for (int c = 0; c < 32; ++c) u[c] = __float_as_uint(__uint_as_float(u[c]) * f);
                         ptx::tmem_st32(tmem + kColO + c4 * 32 + lane_base, u);
@@ -406,24 +428,30 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             const float mr = m_ref == -INFINITY ? 0.f : m_ref;
 
-            const uint32_t p_hi = ptx::smem_addr(sm.p[0]), p_lo = ptx::smem_addr(sm.p[1]);
+            // P_hi | P_lo, 128 weights -> 64 packed columns each: computed in registers first
+            // (this overlaps the output MMAs of tile i - 1), stored once those MMAs have read
+            // the previous P
+            uint32_t ph0[32], ph1[32], pl0[32], pl1[32];
             float ls[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-            for (int c = 0; c < kBN; c += 8) {
-                float e[8];
-#pragma unroll
-                for (int k = 0; k < 8; ++k) {
-                    e[k] = ptx::ex2(sv[c + k] - mr);
-                    ls[k & 3] += e[k];
-                }
-                uint32_t hi[4], lo[4];
-#pragma unroll
-                for (int k = 0; k < 4; ++k) split2(e[2 * k], e[2 * k + 1], hi[k], lo[k]);
-                const uint32_t off = sw128_chunk(r, c);
-                st_shared_v4(p_hi + off, hi[0], hi[1], hi[2], hi[3]);
-                st_shared_v4(p_lo + off, lo[0], lo[1], lo[2], lo[3]);
+            for (int e = 0; e < 32; ++e) {
+                const float a0 = ptx::ex2(sv[2 * e] - mr), a1 = ptx::ex2(sv[2 * e + 1] - mr);
+                const float b0 = ptx::ex2(sv[64 + 2 * e] - mr), b1 = ptx::ex2(sv[64 + 2 * e + 1] - mr);
+                ls[0] += a0;
+                ls[1] += a1;
+                ls[2] += b0;
+                ls[3] += b1;
+                split2(a0, a1, ph0[e], pl0[e]);
+                split2(b0, b1, ph1[e], pl1[e]);
             }
             l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+            if (i >= 1 && !wait(&sm.pv_done, (i - 1) & 1)) { ok = false; break; }
+            const uint32_t pa = tmem + kColP + lane_base;
+            ptx::tmem_st32(pa, ph0);
+            ptx::tmem_st32(pa + 32, ph1);
+            ptx::tmem_st32(pa + kLoCols, pl0);
+            ptx::tmem_st32(pa + kLoCols + 32, pl1);
+            ptx::tmem_wait_st();
             // cache rows at or past the sequence's end (an unwritten page tail, or a page slot
             // no TMA filled) become zeros, so that 0-weights never meet a non-finite value
             if (t0 + kBN > L && t0 + r >= L) {
@@ -450,6 +478,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 uint32_t u[32];
                 ptx::tmem_ld32(tmem + kColO + c4 * 32 + lane_base, u);
                 ptx::tmem_wait_ld();
+                ptx::reg_fence(u);
                 if (r < rows) {
                     if (a.out_dtype == KL_FP32) {
                         float4 *o = reinterpret_cast<float4 *>(static_cast<float *>(a.out) + orow + c4 * 32);

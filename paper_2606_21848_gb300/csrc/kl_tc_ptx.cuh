@@ -159,6 +159,18 @@ __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint6
         : "memory");
 }
 
+// D[tmem] (+)= A[tmem] x B[smem desc], kind::f16: A is read from tensor memory, row i of A in
+// lane i, 16-bit elements packed two per 32-bit column (element 2c in the low half of column c).
+__device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                            uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
 // Arrive once on `bar` when every tcgen05 operation this thread issued so far has completed.
 __device__ __forceinline__ void mma_commit(uint64_t *bar) {
     asm volatile(
@@ -211,6 +223,16 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&u)[32]) {
 
 __device__ __forceinline__ void tmem_wait_ld() {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// After tmem_wait_ld(): tie the loaded registers to that point. tcgen05.ld writes its
+// destination registers asynchronously, and nothing else tells the compiler that their values
+// only become valid at the wait; each empty volatile asm below redefines one register after
+// the wait (volatile asm statements keep their order), so every use follows the wait.
+template <int N>
+__device__ __forceinline__ void reg_fence(uint32_t (&u)[N]) {
+#pragma unroll
+    for (int i = 0; i < N; ++i) asm volatile("" : "+r"(u[i]));
 }
 
 // Store 32 consecutive 32-bit columns of the thread's TMEM lane (complete with tmem_wait_st()).
