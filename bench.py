@@ -2,8 +2,9 @@
 
 A step is one pass of the whole hot path over one batch: kl_decode_step appends the current
 token's value rows to the paged Value-Only Cache and runs the routed decode (routing prologue,
-split-sequence decode, cross-split merge) -- one kernel when the splits merge inside a
-thread-block cluster, else the decode kernel plus the combine kernel. Inputs are
+split-sequence decode, cross-split merge) -- one kernel on the tensor-core path (the last split
+of each sequence and value head merges the split states), the decode kernel plus the combine
+kernel on the CUDA-core path. Inputs are
 seeded synthetic tensors with the shapes of the selected workload, resident in HBM before the
 timed region; L2 is flushed between timed steps (a 512 MiB write, then a read of it, so the
 lines left in L2 are clean).

@@ -180,27 +180,32 @@ __device__ __forceinline__ void mma_commit(uint64_t *bar) {
 }
 
 // Each thread of the warp reads 16 consecutive 32-bit columns of its own TMEM lane
-// (lanes 32 * (warp % 4) .. +31 for the warp's quarter).
+// (lanes 32 * (warp % 4) .. +31 for the warp's quarter). The wait is part of the same asm
+// statement, so the compiler sees the registers defined only once the load has landed.
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&r)[16]) {
     uint32_t u[16];
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];\n\t"
+        "tcgen05.wait::ld.sync.aligned;"
         : "=r"(u[0]), "=r"(u[1]), "=r"(u[2]), "=r"(u[3]), "=r"(u[4]), "=r"(u[5]), "=r"(u[6]),
           "=r"(u[7]), "=r"(u[8]), "=r"(u[9]), "=r"(u[10]), "=r"(u[11]), "=r"(u[12]),
           "=r"(u[13]), "=r"(u[14]), "=r"(u[15])
         : "r"(taddr)
         : "memory");
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
     for (int i = 0; i < 16; ++i) r[i] = __uint_as_float(u[i]);
 }
 
-// One 32-bit column of the thread's TMEM lane.
+// One 32-bit column of the thread's TMEM lane (load and wait in one statement).
 __device__ __forceinline__ float tmem_ld1(uint32_t taddr) {
     uint32_t u;
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(u) : "r"(taddr) : "memory");
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];\n\t"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(u)
+        : "r"(taddr)
+        : "memory");
     return __uint_as_float(u);
 }
 

@@ -148,8 +148,9 @@ def test_block_table_permutation_is_bit_exact(kname):
 
 @pytest.mark.parametrize("kname", ["simt", "tensor"])
 def test_split_counts_agree(kname):
-    """S = 1 writes the output directly; 2..8 merge inside a thread-block cluster (tensor-core
-    kernel); larger S go through the combine kernel."""
+    """S = 1 writes the output directly; larger S are merged by the last split of each
+    (sequence, value head) to finish (tensor-core kernel: direct loads up to 8 splits, staged
+    through the ring beyond) or by the combine kernel (CUDA-core kernel)."""
     x = tiny(B=2, Hq=32, Hkv=8, D=128, P=16, lens=(2000, 4096))
     k = _kernel_or_skip(kname, x)
     want = oracle_decode(x, _gpu.default_scale(x))
