@@ -11,8 +11,8 @@ Two independent formulations live here:
   s_i = scale * <q_r, v_i>, softmax weights alpha_{n+1,i} and output O_{n+1} = sum alpha v_i
   (Section 3), plus the split-state merge, the cache append and, for the K+V comparison,
   standard attention (Eq. 1).
-  The prefill of a chunk of new tokens (Eq. 3 with a causal mask) and the chunk append use
-  the same per-row attention.
+  The prefill of a chunk of new tokens (Eq. 3 with a causal mask), the chunk append and the
+  decode over a latent value-only cache (Section 3) use the same per-row attention.
 * ``dense.py`` -- a NumPy brute force that first un-pages the cache with its own code and then
   evaluates the same formulas on dense arrays; it is used for tiny inputs only.
 
@@ -67,9 +67,10 @@ def _load():
         _lib.ko_append.argtypes = [i, i, i, i, i, i, p, p, p, p]
         _lib.ko_prefill.argtypes = [i, i, i, i, i, i, i, i, d, p, p, p, p, p, p, i, p, p]
         _lib.ko_append_chunk.argtypes = [i, i, i, i, i, i, p, p, p, p, p]
+        _lib.ko_latent_decode.argtypes = [i, i, i, i, i, i, i, i, i, d, p, p, p, p, p, p, i, p, p]
         for f in ("ko_route", "ko_decode", "ko_standard_decode", "ko_attention_weights",
                   "ko_decode_partial", "ko_combine", "ko_append", "ko_prefill",
-                  "ko_append_chunk"):
+                  "ko_append_chunk", "ko_latent_decode"):
             getattr(_lib, f).restype = ctypes.c_int
     return _lib
 
@@ -229,3 +230,25 @@ def append_chunk(v_cache, v_new, block_table, seq_lens, cu_q) -> np.ndarray:
                                  _ptr(bt), _ptr(sl), _ptr(cu), _ptr(cache))
     _check(rc, "append_chunk")
     return cache
+
+
+def latent_decode(q, w_r, w_post, v_lat, block_table, seq_lens, *, scale: float,
+                  wr_per_query_head: bool = False, heads=None) -> np.ndarray:
+    """Decode over a latent value-only cache (Section 3): absorbed query q* = (q W^R) W_post^T,
+    softmax(scale q* V*^T) V* W_post. q [B, Hq, D], w_post [Hq, r, D], v_lat [pages, Hl, P, r]
+    (bf16 bits). Returns [B, Hq, D] fp64, or [len(heads), D] for (b, h) pairs."""
+    q, w_r, w_post = _c(q, np.uint16), _c(w_r, np.uint16), _c(w_post, np.uint16)
+    v_lat = _c(v_lat, np.uint16)
+    bt, sl = _c(block_table, np.int32), _c(seq_lens, np.int32)
+    B, Hq, D = q.shape
+    num_pages, Hl, P, r = v_lat.shape
+    if w_post.shape != (Hq, r, D):
+        raise ValueError("w_post must be [Hq, r, D]")
+    sel = None if heads is None else _c(np.asarray(heads, np.int32).reshape(-1, 2), np.int32)
+    out = np.zeros(((B * Hq) if sel is None else len(sel), D), np.float64)
+    rc = _load().ko_latent_decode(B, Hq, Hl, D, r, P, num_pages, bt.shape[1],
+                                  int(wr_per_query_head), float(scale), _ptr(q), _ptr(w_r),
+                                  _ptr(w_post), _ptr(v_lat), _ptr(bt), _ptr(sl),
+                                  0 if sel is None else len(sel), _ptr(sel), _ptr(out))
+    _check(rc, "latent_decode")
+    return out.reshape(B, Hq, D) if sel is None else out

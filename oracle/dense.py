@@ -101,3 +101,30 @@ def keyless_prefill(q_bits, w_r_bits, v_seqs, q_lens, *, scale: float,
             out[r0:r0 + n, h] = a @ V
         r0 += n
     return out
+
+
+def keyless_latent_decode(q_bits, w_r_bits, w_post_bits, lat_seqs, *, scale: float,
+                          wr_per_query_head: bool = False):
+    """Latent value-only cache decode by expanding the values: head h attends the rows
+    V_h = V* W_post[h] (L x D) with its routed query q_r = q W^R, i.e.
+    softmax(scale V_h q_r) V_h. (The oracle instead absorbs W_post into the query and expands
+    only the output; the two agree by associativity.) lat_seqs from ``unpage``; [B, Hq, D]."""
+    q = bf16_bits_to_f64(q_bits)
+    w = bf16_bits_to_f64(w_r_bits)
+    wp = bf16_bits_to_f64(w_post_bits)              # [Hq, r, D]
+    B, Hq, D = q.shape
+    Hl = lat_seqs[0].shape[0] if lat_seqs else 1
+    G = Hq // Hl
+    out = np.zeros((B, Hq, D))
+    for b in range(B):
+        for h in range(Hq):
+            Vs = lat_seqs[b][h // G]                # [L, r]
+            if Vs.shape[0] == 0:
+                continue
+            Vh = Vs @ wp[h]                         # [L, D]
+            qr = q[b, h] @ w[h if wr_per_query_head else h // G]
+            s = scale * (Vh @ qr)
+            a = np.exp(s - s.max())
+            a /= a.sum()
+            out[b, h] = a @ Vh
+    return out

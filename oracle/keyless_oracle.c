@@ -19,7 +19,8 @@
  *     heads that share a value group read the same cached value rows;
  *   - for the comparison only: standard decode softmax(q K^T / sqrt(d_k)) V (Eq. 1) over a
  *     paged K cache and a paged V cache;
- *   - prefill of a chunk of new tokens (Eq. 3 under a causal mask) and the chunk append.
+ *   - prefill of a chunk of new tokens (Eq. 3 under a causal mask) and the chunk append;
+ *   - decode over a latent value-only cache (Section 3, latent value-only cache paragraph).
  *
  * Readings where the paper is silent (each is listed in the design notes):
  *   - lambda / sqrt(d_k) is the caller's `scale`; lambda = 1 gives 1/sqrt(d_k);
@@ -470,6 +471,74 @@ int ko_append_chunk(int B, int Hkv, int D, int P, int num_pages, int max_pages,
                        v_new + ((size_t)(cu_q[b] + i) * Hkv + g) * D,
                        sizeof(uint16_t) * (size_t)D);
         }
+    }
+    return err ? -1 : 0;
+}
+
+/*
+ * Multi-head attention over a latent value-only cache (Section 3, "Multihead with Latent
+ * Value-only Cache"): the cache holds V* = X W^V_pre (width r) and head h expands it with
+ * W^V_{h,post} (r x d_k). For query head h of latent group g = h / (Hq / Hl):
+ *   q_r = q W^R[w(h)]                                (Section 2.2)
+ *   q*[k] = sum_j q_r[j] W_post[h][k][j]              (absorbed query Q* = Q (W_post)^T)
+ *   s_t = scale * <q*, v*_t>,  alpha = softmax(s),  o*[k] = sum_t alpha_t v*_t[k]
+ *   out[j] = sum_k o*[k] W_post[h][k][j]              (output V* W_post)
+ * with scale = 1 / sqrt(r) in the paper (the caller's `scale`). W_post is [Hq][r][D] row-major
+ * (row k = latent dimension); the latent cache is [num_pages][Hl][P][r]; out is [B][Hq][D], or
+ * [n_sel][D] for the selected (b, h) pairs.
+ */
+int ko_latent_decode(int B, int Hq, int Hl, int D, int r, int P, int num_pages, int max_pages,
+                     int wr_per_query_head, double scale, const uint16_t *q, const uint16_t *w_r,
+                     const uint16_t *w_post, const uint16_t *v_lat, const int32_t *block_table,
+                     const int32_t *seq_lens, int n_sel, const int32_t *sel, double *out)
+{
+    if (check_dims(B, Hq, Hl, D) || r <= 0 || P <= 0 || max_pages < 0)
+        return -1;
+    int G = Hq / Hl;
+    long n_items = sel ? n_sel : (long)B * Hq;
+    int err = 0;
+
+#pragma omp parallel for schedule(dynamic, 1) reduction(| : err)
+    for (long it = 0; it < n_items; ++it) {
+        int b = sel ? sel[2 * it] : (int)(it / Hq);
+        int h = sel ? sel[2 * it + 1] : (int)(it % Hq);
+        double *o = out + (size_t)it * D;
+        if (b < 0 || b >= B || h < 0 || h >= Hq) {
+            err |= 1;
+            continue;
+        }
+        int L = seq_lens[b];
+        if (L < 0 || L > max_pages * P) {
+            err |= 1;
+            continue;
+        }
+        int g = h / G, w = wr_per_query_head ? h : g;
+        const uint16_t *Wp = w_post + (size_t)h * r * D;
+        double *qr = (double *)malloc(sizeof(double) * (size_t)D);
+        double *qs = (double *)malloc(sizeof(double) * (size_t)r);
+        double *os = (double *)malloc(sizeof(double) * (size_t)r);
+        double *s = (double *)malloc(sizeof(double) * (size_t)(L > 0 ? L : 1));
+        route_row(D, q + ((size_t)b * Hq + h) * D, w_r + (size_t)w * D * D, qr);
+        for (int k = 0; k < r; ++k) {
+            double acc = 0.0;
+            for (int j = 0; j < D; ++j)
+                acc += qr[j] * bf16_to_f64(Wp[(size_t)k * D + j]);
+            qs[k] = acc;
+        }
+        double m, l;
+        if (attend(r, Hl, P, num_pages, scale, qs, v_lat, v_lat,
+                   block_table + (size_t)b * max_pages, g, 0, L, s, os, &m, &l))
+            err |= 1;
+        for (int j = 0; j < D; ++j) {
+            double acc = 0.0;
+            for (int k = 0; k < r; ++k)
+                acc += os[k] * bf16_to_f64(Wp[(size_t)k * D + j]);
+            o[j] = acc;
+        }
+        free(s);
+        free(os);
+        free(qs);
+        free(qr);
     }
     return err ? -1 : 0;
 }

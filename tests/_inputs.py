@@ -65,3 +65,17 @@ def tiny_prefill(B=3, Hq=8, Hkv=2, D=64, P=16, lens=(5, 37, 100), q_lens=(5, 12,
 def prefill_bits(x: dict):
     """NumPy views for the prefill oracle: (q, w_r, v_cache, block_table, seq_lens, cu_q)."""
     return bits(x) + (x["cu_q"].numpy(),)
+
+
+def tiny_latent(B=3, Hq=8, Hl=2, D=128, r=64, P=16, lens=(1, 37, 100), seed=51,
+                table="permuted", wr_per_query_head=False):
+    """A tiny decode over a latent value-only cache: latent rows [pages][Hl][P][r] ~ N(0, 1),
+    W_post [Hq][r][D] ~ N(0, 1/r) (so that the expanded values are ~ N(0, 1)), q and W^R as in
+    ``tiny``."""
+    x = tiny(B, Hq, Hl, D, P, lens, seed, table, wr_per_query_head)
+    g = torch.Generator().manual_seed(seed + 13)
+    num_pages = x["num_pages"]
+    x["v_lat"] = torch.randn(num_pages, Hl, P, r, generator=g).to(torch.bfloat16)
+    x["w_post"] = (torch.randn(Hq, r, D, generator=g) * math.sqrt(1.0 / r)).to(torch.bfloat16)
+    x["r"] = r
+    return x

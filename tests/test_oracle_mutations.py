@@ -17,6 +17,7 @@ import pytest
 import oracle
 from oracle import dense
 from tests import test_oracle as pins
+from tests import test_oracle_latent as latent_pins
 from tests import test_oracle_prefill as prefill_pins
 from tests._inputs import bits, default_scale, tiny
 
@@ -40,6 +41,12 @@ MUTATIONS = {
                                "int p = r - cu_q[b];"),
     "prefill_not_causal": ("int p = seq_lens[b] - n + (r - cu_q[b]);",
                            "int p = seq_lens[b] - 1;"),
+    # latent cache: the absorbed query, the output expansion, the latent group
+    "latent_no_absorb": ("            qs[k] = acc;\n", "            qs[k] = qr[k];\n"),
+    "latent_no_up_projection": ("            o[j] = acc;\n        }\n        free(s);\n        free(os);",
+                                "            o[j] = j < r ? os[j] : 0.0;\n        }\n        free(s);\n        free(os);"),
+    "latent_wrong_group": ("        int g = h / G, w = wr_per_query_head ? h : g;\n        const uint16_t *Wp",
+                           "        int g = h % Hl, w = wr_per_query_head ? h : g;\n        const uint16_t *Wp"),
     "prefill_wrong_row_base": ("route_row(D, q + ((size_t)r * Hq + h) * D, w_r + (size_t)w * D * D, qr);",
                                "route_row(D, q + ((size_t)(r - cu_q[b]) * Hq + h) * D, w_r + (size_t)w * D * D, qr);"),
 }
@@ -66,6 +73,9 @@ def _pin_results():
     run("prefill_dense", prefill_pins.test_paged_prefill_equals_dense_causal_bruteforce,
         dict(B=3, Hq=8, Hkv=2, D=64, P=16, lens=(5, 37, 100), q_lens=(5, 12, 1)))
     run("prefill_sdpa", prefill_pins.test_full_causal_prefill_equals_sdpa_with_k_equal_v_wr_transposed)
+    run("latent_expand", latent_pins.test_absorbed_query_equals_expanded_values,
+        dict(B=3, Hq=8, Hl=2, D=128, r=64, P=16, lens=(1, 37, 100)))
+    run("latent_identity", latent_pins.test_identity_expansion_is_the_plain_keyless_decode)
     return res
 
 
@@ -82,7 +92,8 @@ def test_planted_mistake_is_caught(name, tmp_path, monkeypatch):
     lib = ctypes.CDLL(str(so))
     real = oracle._load()
     for f in ("ko_route", "ko_decode", "ko_standard_decode", "ko_attention_weights",
-              "ko_decode_partial", "ko_combine", "ko_append", "ko_prefill", "ko_append_chunk"):
+              "ko_decode_partial", "ko_combine", "ko_append", "ko_prefill", "ko_append_chunk",
+              "ko_latent_decode"):
         getattr(lib, f).argtypes = getattr(real, f).argtypes
         getattr(lib, f).restype = ctypes.c_int
     monkeypatch.setattr(oracle, "_lib", lib)
