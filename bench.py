@@ -60,10 +60,8 @@ def parse_args():
 # ------------------------------------------------------------------------------ helpers --
 
 def dist_env():
-    rank = int(os.environ.get("RANK", "0"))
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    return rank, world, local
+    from paper_2606_21848_gb300.multi import dist_env as env
+    return env()
 
 
 def measured_peaks():
@@ -219,6 +217,8 @@ def run_reference(args):
     x = generate(wl)
     if wl.q_len > 0:
         return run_reference_prefill(args, wl, x)
+    if wl.latent_dim > 0:
+        return run_reference_latent(args, wl, x)
     per_step = max(1.0, args.cpu_seconds / max(1, args.steps))
     rates = []
     total_seqs = 0
@@ -267,9 +267,12 @@ def run_ours(args):
     wl = WORKLOADS[args.workload]
     if args.wr_per_query_head:
         wl = wl.with_(wr_per_query_head=True)
-    x = generate(wl, seed=wl.seed + rank)           # replicas: each rank its own batch
+    from paper_2606_21848_gb300.multi import job_throughput, max_over_ranks, replica_seed
+    x = generate(wl, seed=replica_seed(wl.seed, rank))   # replicas: each rank its own batch
     if wl.q_len > 0:
         return run_prefill(args, wl, x, dev, rank, world)
+    if wl.latent_dim > 0:
+        return run_latent(args, wl, x, dev, rank, world)
     B, Hq, D = x["q"].shape
     num_pages, Hkv, P, _ = x["v_cache"].shape
     max_pages = x["block_table"].shape[1]
@@ -359,14 +362,11 @@ def run_ours(args):
     comb_ms = [0.0 if one_kernel else e[1].elapsed_time(e[2]) for e in evs]
     mean_step = statistics.mean(step_ms)
     mean_dec = statistics.mean(dec_ms)
-    if world > 1:
-        t = torch.tensor([mean_step, mean_dec], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        mean_step, mean_dec = float(t[0]), float(t[1])
+    mean_step, mean_dec = max_over_ranks([mean_step, mean_dec], device=dev)
     assert int(err.item()) == 0, f"device error flags {int(err.item())}"
 
     ab = algorithmic_bytes(x, args.standard)
-    value = B * world / (mean_step / 1e3)
+    value = job_throughput(B, world, mean_step / 1e3)
     peak, peak_kind = measured_peaks()
     dec_gbs = ab["total"] / (mean_dec / 1e3) / 1e9
     step_gbs = ab["total"] / (mean_step / 1e3) / 1e9
@@ -408,10 +408,7 @@ def run_ours(args):
             ts.append((a, b))
         torch.cuda.synchronize()
         e2e_ms = statistics.mean(a.elapsed_time(b) for a, b in ts)
-        if world > 1:
-            t = torch.tensor([e2e_ms], device=dev)
-            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-            e2e_ms = float(t[0])
+        e2e_ms, = max_over_ranks([e2e_ms], device=dev)
         e2e = {"value": B * world / (e2e_ms / 1e3), "unit": "tokens/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms}
 
@@ -544,6 +541,7 @@ def run_prefill(args, wl, x, dev, rank, world):
     import torch
 
     import paper_2606_21848_gb300 as kl
+    from paper_2606_21848_gb300.multi import job_throughput, max_over_ranks
 
     T, Hq, D = x["q_chunk"].shape
     B = x["seq_lens"].shape[0]
@@ -592,10 +590,7 @@ def run_prefill(args, wl, x, dev, rank, world):
     step_ms = statistics.mean(e[0].elapsed_time(e[2]) for e in evs)
     app_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
     pre_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
-    if world > 1:
-        t = torch.tensor([step_ms, app_ms, pre_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        step_ms, app_ms, pre_ms = (float(v) for v in t)
+    step_ms, app_ms, pre_ms = max_over_ranks([step_ms, app_ms, pre_ms], device=dev)
     assert int(err.item()) == 0, f"device error flags {int(err.item())}"
 
     fl = prefill_flops(x)
@@ -635,10 +630,7 @@ def run_prefill(args, wl, x, dev, rank, world):
             ts.append((a, b))
         torch.cuda.synchronize()
         e2e_ms = statistics.mean(a.elapsed_time(b) for a, b in ts)
-        if world > 1:
-            t = torch.tensor([e2e_ms], device=dev)
-            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-            e2e_ms = float(t[0])
+        e2e_ms, = max_over_ranks([e2e_ms], device=dev)
         e2e = {"value": T * world / (e2e_ms / 1e3), "unit": "tokens/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms}
 
@@ -652,7 +644,7 @@ def run_prefill(args, wl, x, dev, rank, world):
                "sample": f"{n} query rows (all {Hq} heads) of {wl.name} on a fixed stride over "
                          f"the chunk, fp64, in {el:.1f}s"}
     line = {
-        "metric": PREFILL_METRIC, "value": T * world / (step_ms / 1e3), "unit": "tokens/s",
+        "metric": PREFILL_METRIC, "value": job_throughput(T, world, step_ms / 1e3), "unit": "tokens/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded; inputs resident in HBM)",
@@ -670,6 +662,213 @@ def run_prefill(args, wl, x, dev, rank, world):
                      "frac": tflops / peak, "peak_kind": peak_kind,
                      "algorithmic_flops": fl["total"], "traffic": None},
         "gpu_launches": 2 * args.steps,
+        "clocks": clk.summary(),
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+# ---------------------------------------------------------------------------- latent ----
+
+LATENT_METRIC = ("latent value-only cache decode tokens/s and achieved HBM GB/s "
+                 "(% of 8 TB/s) on 1 GB300")
+
+
+def latent_bytes(x) -> dict:
+    """Bytes a latent decode step must move once: the latent rows, W^R, W_post, q, out, the
+    block table, and the appended latent row (read and written)."""
+    B, Hq, D = x["q"].shape
+    num_pages, Hl, P, r = x["v_lat"].shape
+    tokens = int(x["seq_lens"].sum())
+    lat = tokens * Hl * r * 2
+    w = x["w_r"].numel() * 2 + x["w_post"].numel() * 2
+    io = 2 * B * Hq * D * 2
+    bt = sum(math.ceil(int(L) / P) for L in x["seq_lens"].tolist()) * 4 + B * 4
+    append = 2 * B * Hl * r * 2
+    return {"latent": lat, "total": lat + w + io + bt + append, "tokens": tokens}
+
+
+def cpu_oracle_latent_rate(x, seconds: float):
+    import numpy as np
+
+    import oracle
+    from paper_2606_21848_gb300.workloads import bf16_bits
+    q, w, wp, v = (bf16_bits(x[k]) for k in ("q", "w_r", "w_post", "v_lat"))
+    bt, sl = x["block_table"].numpy(), x["seq_lens"].numpy()
+    B, Hq, D = x["q"].shape
+    r = x["v_lat"].shape[3]
+    oracle.build()
+    seqs, b = 0, 0
+    t0 = time.perf_counter()
+    while True:
+        heads = np.array([(b, h) for h in range(Hq)], np.int32)
+        oracle.latent_decode(q, w, wp, v, bt, sl, scale=1.0 / math.sqrt(r), heads=heads)
+        seqs += 1
+        b = (b + 1) % B
+        el = time.perf_counter() - t0
+        if el >= seconds:
+            break
+    return seqs / el, seqs, el
+
+
+def run_reference_latent(args, wl, x):
+    import oracle
+    per_step = max(1.0, args.cpu_seconds / max(1, args.steps))
+    rates, total = [], 0
+    for i in range(args.warmup + args.steps):
+        rt, n, _ = cpu_oracle_latent_rate(x, per_step if i >= args.warmup else 0.0)
+        if i >= args.warmup:
+            rates.append(rt)
+            total += n
+    value = statistics.mean(rates)
+    line = {
+        "impl": "reference", "metric": LATENT_METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1000.0 * wl.num_seqs / value, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": wl.name, "num_seqs": wl.num_seqs, "q_heads": wl.num_q_heads,
+                   "latent_heads": wl.num_kv_heads, "head_dim": wl.head_dim,
+                   "latent_dim": wl.latent_dim, "page_size": wl.page_size,
+                   "seq_len": wl.seq_len},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": oracle.threads(),
+                         "kind": "oracle",
+                         "sample": f"{total} whole sequences (all heads) of {wl.name}, "
+                                   f"~{per_step:.1f}s per step"},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_latent(args, wl, x, dev, rank, world):
+    """One latent decode step = kl_append_v of the current token's latent rows +
+    kl_latent_decode (absorbed query, tensor-core decode over the latent rows, expansion)."""
+    import torch
+
+    import paper_2606_21848_gb300 as kl
+    from paper_2606_21848_gb300.multi import job_throughput, max_over_ranks
+
+    B, Hq, D = x["q"].shape
+    num_pages, Hl, P, r = x["v_lat"].shape
+    max_pages = x["block_table"].shape[1]
+    lsh = kl.make_latent_shape(B, Hq, Hl, D, r, P, num_pages, max_pages, wl.wr_per_query_head)
+    ash = kl.make_shape(B, Hq, Hl, r, P, num_pages, max_pages)      # the append over latent rows
+    splits_req = wl.num_splits if args.num_splits < 0 else args.num_splits
+    S = kl.kl_decode_num_splits(ash, splits_req)
+    g = {k: x[k].to(dev) for k in ("q", "w_r", "w_post", "v_lat", "block_table", "seq_lens",
+                                    "positions", "v_new")}
+    out = torch.empty(B, Hq, D, dtype=torch.bfloat16, device=dev)
+    ws = torch.zeros(kl.kl_latent_workspace_size(lsh, splits_req), dtype=torch.uint8, device=dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    flush_sink = torch.empty((), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def flush_l2():
+        flush.zero_()
+        torch.sum(flush, dim=0, out=flush_sink)
+
+    def step(d, ev=None):
+        if ev: ev[0].record(stream)
+        kl.kl_append_v(ash, d["v_new"], d["block_table"], d["positions"], g["v_lat"], err, stream)
+        if ev: ev[1].record(stream)
+        kl.kl_latent_decode(lsh, d["q"], g["w_r"], g["w_post"], g["v_lat"], d["block_table"],
+                            d["seq_lens"], splits_req, out, kl.KL_BF16, ws, err, stream)
+        if ev: ev[2].record(stream)
+
+    E = lambda: torch.cuda.Event(enable_timing=True)
+    for _ in range(args.warmup):
+        flush_l2()
+        step(g, [E(), E(), E()])
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0, f"device error flags {int(err.item())}"
+    evs = [[E(), E(), E()] for _ in range(args.steps)]
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(dev.index) as clk:
+        for i in range(args.steps):
+            flush_l2()
+            step(g, evs[i])
+        torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    step_ms = statistics.mean(e[0].elapsed_time(e[2]) for e in evs)
+    app_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+    dec_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+    step_ms, app_ms, dec_ms = max_over_ranks([step_ms, app_ms, dec_ms], device=dev)
+    assert int(err.item()) == 0, f"device error flags {int(err.item())}"
+    ab = latent_bytes(x)
+    peak, peak_kind = measured_peaks()
+    dec_gbs = ab["total"] / (dec_ms / 1e3) / 1e9
+
+    e2e = None
+    if not args.no_e2e:
+        h_in = {k: x[k].pin_memory() for k in ("q", "v_new", "positions", "seq_lens",
+                                               "block_table")}
+        h_out = torch.empty(B, Hq, D, dtype=torch.bfloat16).pin_memory()
+        d_in = {k: torch.empty_like(g[k]) for k in h_in}
+        h2d = sum(t.numel() * t.element_size() for t in h_in.values())
+        d2h = h_out.numel() * h_out.element_size()
+
+        def e2e_step():
+            for k in h_in:
+                d_in[k].copy_(h_in[k], non_blocking=True)
+            step(d_in)
+            h_out.copy_(out, non_blocking=True)
+
+        for _ in range(args.warmup):
+            flush_l2()
+            e2e_step()
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(args.steps):
+            flush_l2()
+            a, b = E(), E()
+            a.record(stream)
+            e2e_step()
+            b.record(stream)
+            ts.append((a, b))
+        torch.cuda.synchronize()
+        e2e_ms = statistics.mean(a.elapsed_time(b) for a, b in ts)
+        e2e_ms, = max_over_ranks([e2e_ms], device=dev)
+        e2e = {"value": B * world / (e2e_ms / 1e3), "unit": "tokens/s",
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms}
+
+    if rank != 0:
+        return 0
+    cpu = None
+    if world == 1:
+        import oracle
+        rate, n, el = cpu_oracle_latent_rate(x, args.cpu_seconds)
+        cpu = {"value": rate, "unit": "tokens/s", "cores": oracle.threads(), "kind": "oracle",
+               "sample": f"{n} whole sequences of {wl.name} (all {Hq} heads, fp64) in {el:.1f}s"}
+    line = {
+        "metric": LATENT_METRIC, "value": job_throughput(B, world, step_ms / 1e3), "unit": "tokens/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded; inputs resident in HBM)",
+        "config": {"workload": wl.name, "num_seqs": B, "q_heads": Hq, "latent_heads": Hl,
+                   "head_dim": D, "latent_dim": r, "page_size": P, "seq_len": wl.seq_len,
+                   "context_tokens": ab["tokens"], "num_splits": S,
+                   "w_r": "per query head" if wl.wr_per_query_head else "per latent group",
+                   "w_post": "per query head",
+                   "l2": "flushed between timed steps (512 MiB write, then read back)",
+                   "parallelism": f"replicas x{world}"},
+        "ms_breakdown": {"append": app_ms, "latent_decode": dec_ms},
+        "kernels_per_step": 4,
+        "roofline": {"bound": "hbm", "achieved": dec_gbs, "peak": peak, "unit": "GB/s",
+                     "frac": dec_gbs / peak, "peak_kind": peak_kind,
+                     "pct_of_8tbs": 100.0 * dec_gbs / NOMINAL_HBM_GBS,
+                     "algorithmic_bytes": ab["total"],
+                     "timed": "the kl_latent_decode call (absorbed query, decode, expansion)",
+                     "traffic": None},
+        "gpu_launches": 4 * args.steps,
         "clocks": clk.summary(),
         "e2e": e2e,
         "cpu_baseline": cpu,

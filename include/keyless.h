@@ -234,6 +234,48 @@ kl_status kl_prefill_attention(const kl_shape *shape, const void *q, const void 
                                int32_t total_q, int32_t max_q_len, void *out, kl_dtype out_dtype,
                                int32_t *err, kl_stream_t stream);
 
+/*
+ * Shape of a decode over a latent value-only cache (Section 3, "Multihead with Latent Value-only
+ * Cache"): the cache holds V* = X W^V_pre, latent_dim (r) wide, one latent row per token and
+ * latent group; query head h reads latent group h / (num_q_heads / num_latent_heads) and
+ * expands it with its own W^V_{h,post} (r x head_dim).
+ */
+typedef struct {
+    int32_t num_seqs;            /* B */
+    int32_t num_q_heads;         /* Hq */
+    int32_t num_latent_heads;    /* Hl: latent groups (1 = one latent shared by every head) */
+    int32_t head_dim;            /* D: width of q, W^R and the output (64 or 128) */
+    int32_t latent_dim;          /* r: width of the cached latent rows (128) */
+    int32_t page_size;           /* P */
+    int32_t num_pages;           /* latent pool size */
+    int32_t max_pages_per_seq;   /* block_table row stride */
+    int32_t wr_per_query_head;   /* W^R: Hq matrices (1) or Hl matrices (0) */
+    float scale;                 /* <= 0: 1 / sqrt(latent_dim), the paper's 1/sqrt(r) */
+} kl_latent_shape;
+
+/* Bytes of device workspace kl_latent_decode needs for `num_splits` (0 = automatic); 0 on an
+ * invalid or unsupported shape. Same zero-fill contract as kl_decode_workspace_size. */
+size_t kl_latent_workspace_size(const kl_latent_shape *shape, int32_t num_splits);
+
+/*
+ * Keyless decode over a latent value-only cache (Section 3): for every sequence b and query
+ * head h of latent group g,
+ *   q*  = (q[b][h] W^R[w(h)]) W_post[h]^T          (the absorbed query, width r)
+ *   o*  = sum_t softmax(scale <q*, v*_t>)_t v*_t    (over the L_b cached latent rows)
+ *   out[b][h] = o* W_post[h]                         (width D)
+ * q: [B][Hq][D] bf16; w_r: [Hw][D][D] bf16; w_post: [Hq][r][D] bf16 row-major (row k = latent
+ * dimension); v_lat: [num_pages][Hl][P][r] bf16 (append with kl_append_v and a kl_shape whose
+ * num_kv_heads = Hl and head_dim = r); block_table, seq_lens, num_splits, out, workspace and
+ * flags as in kl_decode_attention. Three launches on `stream`: the absorbed queries, the
+ * tensor-core decode over the latent rows, the expansion. latent_dim 128 and compute
+ * capability 10.3 only (KL_ERR_UNSUPPORTED otherwise); at most 8 query heads per latent group.
+ */
+kl_status kl_latent_decode(const kl_latent_shape *shape, const void *q, const void *w_r,
+                           const void *w_post, const void *v_lat, const int32_t *block_table,
+                           const int32_t *seq_lens, int32_t num_splits, void *out,
+                           kl_dtype out_dtype, void *workspace, size_t workspace_bytes,
+                           int32_t *err, kl_stream_t stream);
+
 /* Size of the fixed device scratch that kl_decode_attention_noalloc uses (32 MiB). */
 #define KL_NOALLOC_SCRATCH_BYTES (32u * 1024u * 1024u)
 

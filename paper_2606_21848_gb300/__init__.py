@@ -15,4 +15,5 @@ from ._lib import (  # noqa: F401
     kl_decode_num_splits, kl_decode_options, kl_decode_workspace_size, kl_route_query,
     kl_shape, kl_standard_decode, kl_status_string, load, make_shape,
     kl_append_v_chunk, kl_prefill_attention,
+    kl_latent_shape, make_latent_shape, kl_latent_workspace_size, kl_latent_decode,
 )

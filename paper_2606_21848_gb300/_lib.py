@@ -36,6 +36,14 @@ class kl_shape(ctypes.Structure):
                 ("scale", ctypes.c_float)]
 
 
+class kl_latent_shape(ctypes.Structure):
+    _fields_ = [("num_seqs", ctypes.c_int32), ("num_q_heads", ctypes.c_int32),
+                ("num_latent_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("latent_dim", ctypes.c_int32), ("page_size", ctypes.c_int32),
+                ("num_pages", ctypes.c_int32), ("max_pages_per_seq", ctypes.c_int32),
+                ("wr_per_query_head", ctypes.c_int32), ("scale", ctypes.c_float)]
+
+
 class kl_decode_options(ctypes.Structure):
     _fields_ = [("num_splits", ctypes.c_int32), ("kernel", ctypes.c_int32),
                 ("partial_o", ctypes.c_void_p), ("partial_ml", ctypes.c_void_p)]
@@ -61,6 +69,7 @@ def load() -> ctypes.CDLL:
     P, I32, SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_size_t
     SH = ctypes.POINTER(kl_shape)
     OP = ctypes.POINTER(kl_decode_options)
+    LS = ctypes.POINTER(kl_latent_shape)
     sig = {
         "kl_route_query": ([SH, P, P, P, P], I32),
         "kl_append_v": ([SH, P, P, P, P, P, P], I32),
@@ -74,6 +83,8 @@ def load() -> ctypes.CDLL:
         "kl_decode_attention_noalloc": ([SH, P, P, P, P, P, I32, P, I32, P, P], I32),
         "kl_decode_kernel_available": ([SH, I32, I32], I32),
         "kl_append_v_chunk": ([SH, P, P, P, P, I32, I32, P, P, P], I32),
+        "kl_latent_workspace_size": ([LS, I32], SZ),
+        "kl_latent_decode": ([LS, P, P, P, P, P, P, I32, P, I32, P, SZ, P, P], I32),
         "kl_prefill_attention": ([SH, P, P, P, P, P, P, I32, I32, P, I32, P, P], I32),
         "kl_status_string": ([I32], ctypes.c_char_p),
     }
@@ -211,6 +222,25 @@ def kl_prefill_attention(shape, q, w_r, v_cache, block_table, seq_lens, cu_q_len
                                        _p(block_table), _p(seq_lens), _p(cu_q_lens), total_q,
                                        max_q_len, _p(out), out_dtype, _p(err), _stream(stream)),
            "kl_prefill_attention")
+
+
+def make_latent_shape(num_seqs, num_q_heads, num_latent_heads, head_dim, latent_dim, page_size,
+                      num_pages, max_pages_per_seq, wr_per_query_head=False, scale=0.0):
+    return kl_latent_shape(num_seqs, num_q_heads, num_latent_heads, head_dim, latent_dim,
+                           page_size, num_pages, max_pages_per_seq, int(bool(wr_per_query_head)),
+                           float(scale))
+
+
+def kl_latent_workspace_size(shape, num_splits=0) -> int:
+    return int(load().kl_latent_workspace_size(ctypes.byref(shape), num_splits))
+
+
+def kl_latent_decode(shape, q, w_r, w_post, v_lat, block_table, seq_lens, num_splits, out,
+                     out_dtype, workspace, err=None, stream=None):
+    _check(load().kl_latent_decode(ctypes.byref(shape), _p(q), _p(w_r), _p(w_post), _p(v_lat),
+                                   _p(block_table), _p(seq_lens), num_splits, _p(out), out_dtype,
+                                   _p(workspace), _nbytes(workspace), _p(err), _stream(stream)),
+           "kl_latent_decode")
 
 
 def kl_decode_kernel_available(shape, kernel, standard=False) -> bool:

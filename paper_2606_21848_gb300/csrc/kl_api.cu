@@ -101,7 +101,7 @@ kl_status decode_common(bool standard, const kl_shape *shape, const void *q, con
                         const int32_t *seq_lens, const kl_decode_options *opts, void *out,
                         kl_dtype out_dtype, void *workspace, size_t workspace_bytes,
                         int32_t *err, kl_stream_t stream, const void *v_new = nullptr,
-                        const int32_t *positions = nullptr) {
+                        const int32_t *positions = nullptr, const float *q_routed = nullptr) {
     const int32_t ns = opts ? opts->num_splits : 0;
     const int32_t kernel = opts ? opts->kernel : KL_KERNEL_AUTO;
     if (ns < 0 || kernel < KL_KERNEL_AUTO || kernel > KL_KERNEL_SIMT) return KL_ERR_INVALID_ARG;
@@ -111,9 +111,9 @@ kl_status decode_common(bool standard, const kl_shape *shape, const void *q, con
     if (st != KL_OK) return st;
     if (g.G > 8) return KL_ERR_UNSUPPORTED;
     if (g.B == 0) return KL_OK;
-    if (!q || !v_cache || !block_table || !seq_lens) return KL_ERR_INVALID_ARG;
-    if (standard ? !k_cache : !w_r) return KL_ERR_INVALID_ARG;
-    if (!aligned(q, 16) || !aligned(v_cache, 16) || (w_r && !aligned(w_r, 16)) ||
+    if ((!q && !q_routed) || !v_cache || !block_table || !seq_lens) return KL_ERR_INVALID_ARG;
+    if (!q_routed && (standard ? !k_cache : !w_r)) return KL_ERR_INVALID_ARG;
+    if ((q && !aligned(q, 16)) || !aligned(v_cache, 16) || (w_r && !aligned(w_r, 16)) ||
         (k_cache && !aligned(k_cache, 16)) || (out && !aligned(out, 16)))
         return KL_ERR_INVALID_ARG;
 
@@ -130,6 +130,7 @@ kl_status decode_common(bool standard, const kl_shape *shape, const void *q, con
     a.geo = g;
     a.q = static_cast<const uint16_t *>(q);
     a.w_r = static_cast<const uint16_t *>(w_r);
+    a.q_routed = q_routed;
     a.k_cache = static_cast<const uint16_t *>(k_cache);
     a.v_cache = static_cast<const uint16_t *>(v_cache);
     a.block_table = block_table;
@@ -149,7 +150,9 @@ kl_status decode_common(bool standard, const kl_shape *shape, const void *q, con
     a.stream = reinterpret_cast<cudaStream_t>(stream);
 
     bool use_tc = false;
-    if (kernel == KL_KERNEL_TENSOR) {
+    if (q_routed && !tc_supported(g, standard)) return KL_ERR_UNSUPPORTED;
+    if (q_routed && kernel == KL_KERNEL_SIMT) return KL_ERR_UNSUPPORTED;
+    if (kernel == KL_KERNEL_TENSOR || q_routed) {
         if (!tc_supported(g, standard)) return KL_ERR_UNSUPPORTED;
         use_tc = true;
     } else if (kernel == KL_KERNEL_AUTO) {
@@ -315,6 +318,89 @@ kl_status kl_prefill_attention(const kl_shape *shape, const void *q, const void 
     a.err = err;
     a.stream = reinterpret_cast<cudaStream_t>(stream);
     return from_cuda(launch_prefill_tc(a));
+}
+
+}  // extern "C"
+
+namespace {
+
+// The decode geometry over the latent rows (value heads = latent groups, head_dim = r) and the
+// workspace carve: q* and o* ([B][Hq][r] fp32 each), then the decode's own workspace.
+struct LatentPlan {
+    kl_shape dec;
+    size_t q_lat, o_lat, dec_ws, total;
+};
+
+kl_status latent_plan(const kl_latent_shape *s, int32_t num_splits, LatentPlan *p) {
+    if (!s) return KL_ERR_INVALID_ARG;
+    if (s->num_seqs < 0 || s->num_q_heads <= 0 || s->num_latent_heads <= 0 || s->head_dim <= 0 ||
+        s->latent_dim <= 0)
+        return KL_ERR_INVALID_ARG;
+    if (s->num_q_heads % s->num_latent_heads != 0) return KL_ERR_INVALID_ARG;
+    if (s->latent_dim != 128 || (s->head_dim != 64 && s->head_dim != 128)) return KL_ERR_UNSUPPORTED;
+    if (num_splits < 0) return KL_ERR_INVALID_ARG;
+    p->dec = kl_shape{s->num_seqs, s->num_q_heads, s->num_latent_heads, s->latent_dim, s->page_size,
+                      s->num_pages, s->max_pages_per_seq, 0,
+                      s->scale > 0.f ? s->scale : 1.0f / sqrtf((float)s->latent_dim)};
+    Geometry g;
+    kl_status st = resolve(&p->dec, num_splits, &g);
+    if (st != KL_OK) return st;
+    if (g.G > 8) return KL_ERR_UNSUPPORTED;
+    const size_t rows = (size_t)s->num_seqs * s->num_q_heads * s->latent_dim * sizeof(float);
+    p->q_lat = 0;
+    p->o_lat = round_up(rows, 256);
+    p->dec_ws = p->o_lat + round_up(rows, 256);
+    p->total = p->dec_ws + layout(g).total;
+    return KL_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t kl_latent_workspace_size(const kl_latent_shape *shape, int32_t num_splits) {
+    LatentPlan p;
+    return latent_plan(shape, num_splits, &p) == KL_OK ? p.total : 0;
+}
+
+kl_status kl_latent_decode(const kl_latent_shape *shape, const void *q, const void *w_r,
+                           const void *w_post, const void *v_lat, const int32_t *block_table,
+                           const int32_t *seq_lens, int32_t num_splits, void *out,
+                           kl_dtype out_dtype, void *workspace, size_t workspace_bytes,
+                           int32_t *err, kl_stream_t stream) {
+    LatentPlan p;
+    kl_status st = latent_plan(shape, num_splits, &p);
+    if (st != KL_OK) return st;
+    if (out_dtype != KL_BF16 && out_dtype != KL_FP32) return KL_ERR_INVALID_ARG;
+    if (shape->num_seqs == 0) return KL_OK;
+    if (!q || !w_r || !w_post || !v_lat || !block_table || !seq_lens || !out)
+        return KL_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(w_r, 16) || !aligned(w_post, 16) || !aligned(v_lat, 16) ||
+        !aligned(out, 16))
+        return KL_ERR_INVALID_ARG;
+    if (!workspace || workspace_bytes < p.total || !aligned(workspace, 256)) return KL_ERR_WORKSPACE;
+    Geometry g;
+    resolve(&p.dec, num_splits, &g);
+    if (!tc_supported(g, false)) return KL_ERR_UNSUPPORTED;
+    char *ws = static_cast<char *>(workspace);
+    float *q_lat = reinterpret_cast<float *>(ws + p.q_lat);
+    float *o_lat = reinterpret_cast<float *>(ws + p.o_lat);
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    const int B = shape->num_seqs, Hq = shape->num_q_heads, D = shape->head_dim,
+              r = shape->latent_dim;
+    cudaError_t e = launch_latent_query(B, Hq, Hq / shape->num_latent_heads, D, r,
+                                        shape->wr_per_query_head ? 1 : 0,
+                                        static_cast<const uint16_t *>(q),
+                                        static_cast<const uint16_t *>(w_r),
+                                        static_cast<const uint16_t *>(w_post), q_lat, s);
+    if (e != cudaSuccess) return KL_ERR_CUDA;
+    kl_decode_options o{num_splits, KL_KERNEL_TENSOR, nullptr, nullptr};
+    st = decode_common(false, &p.dec, nullptr, nullptr, nullptr, v_lat, block_table, seq_lens, &o,
+                       o_lat, KL_FP32, ws + p.dec_ws, workspace_bytes - p.dec_ws, err, stream,
+                       nullptr, nullptr, q_lat);
+    if (st != KL_OK) return st;
+    return from_cuda(launch_latent_expand(B, Hq, D, r, o_lat, static_cast<const uint16_t *>(w_post),
+                                          out, out_dtype, s));
 }
 
 int32_t kl_decode_kernel_available(const kl_shape *shape, int32_t kernel, int32_t standard) {

@@ -325,7 +325,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     // The routing runs on the tensor cores: W^R[g] (one per value head) or the G matrices
     // W^R[g G + h] (one per query head) arrive by TMA as ring positions 0 .. route_tiles - 1,
     // with the group's query rows, and the cache tiles follow.
-    const bool tc_route = !kStandard;
+    const bool tc_route = !kStandard && a.q_routed == nullptr;
     const bool route_pq = tc_route && geo.wr_per_qh;
     const int route_tiles = !tc_route ? 0 : route_pq ? G : 1;
     const int ro = route_tiles;
@@ -645,7 +645,8 @@ __global__ void __launch_bounds__(kThreads, 2)
         bool ok = true;
 
         // Routing prologue: thread j obtains q_r[h][j] for the G heads in fp32 from the routing
-        // MMAs in TMEM, or, for the K+V comparison, the unrouted query itself.
+        // MMAs in TMEM, from the caller's pre-routed queries, or, for the K+V comparison, the
+        // unrouted query itself.
         float acc[kNG];
 #pragma unroll
         for (int h = 0; h < kNG; ++h) acc[h] = 0.f;
@@ -667,6 +668,10 @@ __global__ void __launch_bounds__(kThreads, 2)
                 // the q rows in the q_r buffer were read by the routing MMA; now overwrite them
                 ptx::fence_proxy_async_smem();
             }
+        } else if (a.q_routed) {
+#pragma unroll
+            for (int h = 0; h < kNG; ++h)
+                acc[h] = h < G ? a.q_routed[((size_t)b * geo.Hq + g * G + h) * kD + t] : 0.f;
         } else {
             for (int i = t; i < kD * kNG; i += kTile) {
                 const int k = i >> 3, h = i & 7;
@@ -903,7 +908,7 @@ cudaError_t launch(const DecodeArgs &a) {
     kmap = wmap = qmap = vmap;
     if (kStandard && !make_map(&kmap, a.k_cache, cache_rows, (uint32_t)g.P))
         return cudaErrorInvalidValue;
-    if (!kStandard) {
+    if (!kStandard && !a.q_routed) {
         // W^R [Hw * 128 rows (k)][128 (j)], Hw = Hkv or Hq, one box = one 64-column half of one
         // matrix; q [B * Hq rows][128], one box = the G rows of one value group.
         const uint64_t hw = g.wr_per_qh ? (uint64_t)g.Hq : (uint64_t)g.Hkv;

@@ -25,6 +25,10 @@ struct DecodeArgs {
     Geometry geo;
     const uint16_t *q;        // [B][Hq][D] bf16
     const uint16_t *w_r;      // [Hw][D][D] bf16 (keyless only)
+    // Pre-routed queries (tensor-core kernel only): when set, q and w_r are unused and the
+    // kernel scores with q_routed[b][h][:] (fp32, [B][Hq][D]) as the routed query, e.g. the
+    // absorbed query of a latent value-only cache.
+    const float *q_routed;
     const uint16_t *k_cache;  // [num_pages][Hkv][P][D] bf16 (standard only)
     const uint16_t *v_cache;  // [num_pages][Hkv][P][D] bf16
     const int32_t *block_table;
@@ -101,6 +105,15 @@ cudaError_t launch_append_chunk(const Geometry &g, int total_q, int max_q, const
                                 const int32_t *block_table, const int32_t *seq_lens,
                                 const int32_t *cu_q, uint16_t *v_cache, int32_t *err,
                                 cudaStream_t stream);
+
+// Latent value-only cache (head_dim D of queries and outputs, latent width r):
+// q_lat[b][h] = (q[b][h] W^R[w(h)]) W_post[h]^T and out[b][h] = o_lat[b][h] W_post[h].
+cudaError_t launch_latent_query(int B, int Hq, int G, int D, int r, int wr_per_qh,
+                                const uint16_t *q, const uint16_t *w_r, const uint16_t *w_post,
+                                float *q_lat, cudaStream_t stream);
+cudaError_t launch_latent_expand(int B, int Hq, int D, int r, const float *o_lat,
+                                 const uint16_t *w_post, void *out, kl_dtype out_dtype,
+                                 cudaStream_t stream);
 
 // Number of SMs of the current device (cached per device).
 int device_sm_count();

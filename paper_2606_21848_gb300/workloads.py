@@ -22,7 +22,10 @@ Recipe (fixed, so that a seed names one input set):
 7. prefill workloads only (q_len > 0): the chunk of each sequence is its last
    n_b = min(q_len, L_b) rows; its queries q_chunk ~ N(0, 1) [T, Hq, D] (T = sum n_b, rows of
    sequence b at cu_q[b] ..) and its value rows v_chunk ~ N(0, 1) [T, Hkv, D] (for the chunk
-   append; the pool already holds values at those rows).
+   append; the pool already holds values at those rows);
+8. latent workloads only (latent_dim > 0): the value pool is the latent cache (num_kv_heads =
+   latent groups, head_dim = latent width = 128), and W_post ~ N(0, 1/r) of shape [Hq, r, D]
+   is drawn last.
 """
 from __future__ import annotations
 
@@ -54,6 +57,7 @@ class Workload:
     num_splits: int = 0                   # 0: the library chooses
     seed: int = 0
     q_len: int = 0                        # prefill: query rows per sequence (its last rows)
+    latent_dim: int = 0                   # latent cache: r (the pool holds the latent rows)
 
     @property
     def group(self) -> int:
@@ -99,6 +103,14 @@ WORKLOADS.update({
                                   q_len=32768),
     "prefill_chunked_gqa": Workload("prefill_chunked_gqa", 8, 32, 8, 128, 16, seq_len=8192,
                                     wr_std=math.sqrt(1 / 128), seed=6, q_len=512),
+})
+
+# Latent value-only cache workload (Section 3): 32 query heads reading 4 latent groups of width
+# 128 (8 heads per group), batch 64 at 8192 tokens, W_post per query head: 1 KiB of cache per
+# token, half of a 8-value-head value-only cache and a quarter of its K+V cache.
+WORKLOADS.update({
+    "latent_serving": Workload("latent_serving", 64, 32, 4, 128, 16, seq_len=8192,
+                               wr_std=math.sqrt(1 / 128), seed=7, latent_dim=128),
 })
 
 
@@ -175,6 +187,11 @@ def generate(wl: Workload, seed: int | None = None) -> dict:
         out.update(q_chunk=torch.randn(T, Hq, D, generator=g).to(torch.bfloat16),
                    v_chunk=torch.randn(T, Hkv, D, generator=g).to(torch.bfloat16),
                    q_lens=q_lens, cu_q=cu_q)
+    if wl.latent_dim > 0:
+        r = wl.latent_dim
+        assert r == D, "the value pool doubles as the latent cache"
+        out["w_post"] = (torch.randn(Hq, r, D, generator=g) * math.sqrt(1.0 / r)).to(torch.bfloat16)
+        out["v_lat"] = v_cache
     return out
 
 
