@@ -867,7 +867,8 @@ def run_latent(args, wl, x, dev, rank, world):
                      "pct_of_8tbs": 100.0 * dec_gbs / NOMINAL_HBM_GBS,
                      "algorithmic_bytes": ab["total"],
                      "timed": "the kl_latent_decode call (absorbed query, decode, expansion)",
-                     "traffic": None},
+                     "traffic": recorded_traffic(wl.name, "tensor"),
+                     "traffic_of": "the decode kernel over the latent rows (ncu)"},
         "gpu_launches": 4 * args.steps,
         "clocks": clk.summary(),
         "e2e": e2e,

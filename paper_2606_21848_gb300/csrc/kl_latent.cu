@@ -55,8 +55,9 @@ __global__ void __launch_bounds__(kMaxDim)
     const int ps = D + 8;                   // padded row stride of W_post (values)
     uint16_t *wr = reinterpret_cast<uint16_t *>(smem_raw);             // [D][D]
     uint16_t *wp = wr + D * D;                                         // [r][ps]
-    float *qv = reinterpret_cast<float *>(wp + r * ps);                // [kSeqPass][D]
-    float *qr = qv + kSeqPass * D;                                     // [kSeqPass][D]
+    // per-sequence vectors as [dim][sequence]: one 16-byte load feeds four FMAs
+    float4 *qv = reinterpret_cast<float4 *>(wp + r * ps);              // [D] x 4 sequences
+    float4 *qr = qv + D;                                               // [D] x 4 sequences
     const int h = blockIdx.x, b0 = blockIdx.y * kSeqBlock, t = threadIdx.x;
     stage_rows(wr, w_r + (size_t)(wr_per_qh ? h : h / G) * D * D, D, D, D);
     stage_rows(wp, w_post + (size_t)h * r * D, r, D, ps);
@@ -64,21 +65,26 @@ __global__ void __launch_bounds__(kMaxDim)
     const int b_end = min(B, b0 + kSeqBlock);
     for (int b = b0; b < b_end; b += kSeqPass) {
         const int nb = min(kSeqPass, b_end - b);
-        for (int i = t; i < kSeqPass * D; i += blockDim.x) {
-            const int s = i / D, k = i % D;
-            qv[i] = s < nb ? bf(q[((size_t)(b + s) * Hq + h) * D + k]) : 0.f;
+        if (t < D) {
+            float v[kSeqPass];
+#pragma unroll
+            for (int s = 0; s < kSeqPass; ++s)
+                v[s] = s < nb ? bf(q[((size_t)(b + s) * Hq + h) * D + t]) : 0.f;
+            qv[t] = make_float4(v[0], v[1], v[2], v[3]);
         }
         __syncthreads();
         if (t < D) {
-            float acc[kSeqPass] = {0.f, 0.f, 0.f, 0.f};
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll 8
             for (int k = 0; k < D; ++k) {
                 const float w = bf(wr[k * D + t]);
-#pragma unroll
-                for (int s = 0; s < kSeqPass; ++s) acc[s] = fmaf(qv[s * D + k], w, acc[s]);
+                const float4 x = qv[k];
+                acc.x = fmaf(x.x, w, acc.x);
+                acc.y = fmaf(x.y, w, acc.y);
+                acc.z = fmaf(x.z, w, acc.z);
+                acc.w = fmaf(x.w, w, acc.w);
             }
-#pragma unroll
-            for (int s = 0; s < kSeqPass; ++s) qr[s * D + t] = acc[s];
+            qr[t] = acc;
         }
         __syncthreads();
         if (t < r) {
@@ -91,9 +97,11 @@ __global__ void __launch_bounds__(kMaxDim)
                 for (int e = 0; e < 4; ++e) {
                     const int j = 8 * c + 2 * e;
                     const float w0 = bf16lo(u[e]), w1 = bf16hi(u[e]);
-#pragma unroll
-                    for (int s = 0; s < kSeqPass; ++s)
-                        acc[s] = fmaf(qr[s * D + j + 1], w1, fmaf(qr[s * D + j], w0, acc[s]));
+                    const float4 x0 = qr[j], x1 = qr[j + 1];
+                    acc[0] = fmaf(x1.x, w1, fmaf(x0.x, w0, acc[0]));
+                    acc[1] = fmaf(x1.y, w1, fmaf(x0.y, w0, acc[1]));
+                    acc[2] = fmaf(x1.z, w1, fmaf(x0.z, w0, acc[2]));
+                    acc[3] = fmaf(x1.w, w1, fmaf(x0.w, w0, acc[3]));
                 }
             }
 #pragma unroll
@@ -111,16 +119,19 @@ __global__ void __launch_bounds__(kMaxDim)
                          const uint16_t *__restrict__ w_post, void *out, int out_fp32) {
     extern __shared__ __align__(16) unsigned char smem_raw[];
     uint16_t *wp = reinterpret_cast<uint16_t *>(smem_raw);             // [r][D]
-    float *ov = reinterpret_cast<float *>(wp + r * D);                 // [kSeqPass][r]
+    float4 *ov = reinterpret_cast<float4 *>(wp + r * D);               // [r] x 4 sequences
     const int h = blockIdx.x, b0 = blockIdx.y * kSeqBlock, t = threadIdx.x;
     stage_rows(wp, w_post + (size_t)h * r * D, r, D, D);
     __syncthreads();
     const int b_end = min(B, b0 + kSeqBlock);
     for (int b = b0; b < b_end; b += kSeqPass) {
         const int nb = min(kSeqPass, b_end - b);
-        for (int i = t; i < kSeqPass * r; i += blockDim.x) {
-            const int s = i / r, k = i % r;
-            ov[i] = s < nb ? o_lat[((size_t)(b + s) * Hq + h) * r + k] : 0.f;
+        if (t < r) {
+            float v[kSeqPass];
+#pragma unroll
+            for (int s = 0; s < kSeqPass; ++s)
+                v[s] = s < nb ? o_lat[((size_t)(b + s) * Hq + h) * r + t] : 0.f;
+            ov[t] = make_float4(v[0], v[1], v[2], v[3]);
         }
         __syncthreads();
         if (t < D) {
@@ -128,8 +139,11 @@ __global__ void __launch_bounds__(kMaxDim)
 #pragma unroll 8
             for (int k = 0; k < r; ++k) {
                 const float w = bf(wp[k * D + t]);
-#pragma unroll
-                for (int s = 0; s < kSeqPass; ++s) acc[s] = fmaf(ov[s * r + k], w, acc[s]);
+                const float4 x = ov[k];
+                acc[0] = fmaf(x.x, w, acc[0]);
+                acc[1] = fmaf(x.y, w, acc[1]);
+                acc[2] = fmaf(x.z, w, acc[2]);
+                acc[3] = fmaf(x.w, w, acc[3]);
             }
 #pragma unroll
             for (int s = 0; s < kSeqPass; ++s) {
@@ -152,7 +166,7 @@ cudaError_t launch_latent_query(int B, int Hq, int G, int D, int r, int wr_per_q
                                 float *q_lat, cudaStream_t stream) {
     if (B == 0) return cudaSuccess;
     if (D > kMaxDim || r > kMaxDim || D % 8 || r % 8) return cudaErrorInvalidValue;
-    const size_t smem = (size_t)(D * D + r * (D + 8)) * 2 + 2 * kSeqPass * D * sizeof(float);
+    const size_t smem = (size_t)(D * D + r * (D + 8)) * 2 + 2 * D * sizeof(float4);
     static bool configured = false;
     if (!configured) {
         cudaError_t e = cudaFuncSetAttribute(
@@ -173,7 +187,7 @@ cudaError_t launch_latent_expand(int B, int Hq, int D, int r, const float *o_lat
                                  cudaStream_t stream) {
     if (B == 0) return cudaSuccess;
     if (D > kMaxDim || r > kMaxDim || D % 8 || r % 8) return cudaErrorInvalidValue;
-    const size_t smem = (size_t)r * D * 2 + kSeqPass * r * sizeof(float);
+    const size_t smem = (size_t)r * D * 2 + r * sizeof(float4);
     static bool configured = false;
     if (!configured) {
         cudaError_t e = cudaFuncSetAttribute(
