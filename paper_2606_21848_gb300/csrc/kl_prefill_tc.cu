@@ -30,11 +30,12 @@
 // O in TMEM and its running sum l are rescaled; otherwise p may reach 2^8, well inside bf16 and
 // fp32 range, and the final O / l is unchanged because O and l share the same reference.
 //
-// Roles (224 threads, one CTA per SM):
-//   warps 0-3  softmax and epilogue (TMEM lane quarters 0-3)
-//   warp 4     producer: TMA of W^R and the query block (ring position 0), then cache tiles
-//   warp 5     routing and score MMA issuer (one elected lane) and TMEM owner
-//   warp 6     output MMA issuer. One thread issuing tcgen05.mma back to back reaches about
+// Roles (352 threads, one CTA per SM):
+//   warps 0-7  softmax and epilogue: warps w and w + 4 share TMEM lane quarter w % 4 (its 32
+//              query rows) and split the 128 columns of S, P and O between them
+//   warp 8     producer: TMA of W^R and the query block (ring position 0), then cache tiles
+//   warp 9     routing and score MMA issuer (one elected lane) and TMEM owner
+//   warp 10    output MMA issuer. One thread issuing tcgen05.mma back to back reaches about
 //              88 cycles per 128 x 128 x 16 MMA; two issuing threads together reach the
 //              tensor cores' 64.
 // Every wait is bounded (about one second); a wait that runs out raises KL_FLAG_TIMEOUT, makes
@@ -52,11 +53,11 @@ constexpr int kD = 128;
 constexpr int kBM = 128;                          // query rows per CTA
 constexpr int kBN = 128;                          // cache rows per tile
 constexpr int kStages = 4;
-constexpr int kComputeWarps = 4;
-constexpr int kProducerWarp = 4;
-constexpr int kMmaWarp = 5;                       // routing and score MMAs; TMEM owner
-constexpr int kPvWarp = 6;                        // output MMAs
-constexpr int kThreads = 7 * 32;
+constexpr int kComputeWarps = 8;                  // two per TMEM lane quarter
+constexpr int kProducerWarp = 8;
+constexpr int kMmaWarp = 9;                       // routing and score MMAs; TMEM owner
+constexpr int kPvWarp = 10;                       // output MMAs
+constexpr int kThreads = 11 * 32;
 constexpr uint32_t kTileBytes = kBN * kD * 2;     // 32 KiB
 constexpr uint32_t kHalfBytes = kTileBytes / 2;   // one 64-column half: 128 rows x 128 B
 constexpr uint32_t kTmemCols = 512;
@@ -78,6 +79,8 @@ struct __align__(1024) PrefillSmem {
     uint64_t full[kStages], empty[kStages];
     uint64_t s_full, s_free, p_full, pv_done;
     uint64_t r_full, qr_ready, drain, drain2;
+    float red[2][2][kBM];      // per-tile half-row maxima of the two warps of a pair (2 tiles)
+    float lsum[2][kBM];        // the two warps' shares of the row sums, for the epilogue
     uint32_t tmem_base;
     int abort;
 };
@@ -317,166 +320,173 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else {
         // --------------------------------------------------------- softmax, epilogue ----
-        const int r = tid;                                   // query row = TMEM lane
-        const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+        // Two warps per TMEM lane quarter: warp w serves rows 32 (w % 4) .. + 31 and columns
+        // 64 hf .. + 63 (hf = w / 4) of S, P and O. The pair meets once per tile on a named
+        // barrier (id 1 + w % 4) that also ANDs their progress, so both leave a loop together.
+        const int qd = warp & 3, hf = warp >> 2;
+        const int r = qd * 32 + lane;                        // query row = TMEM lane
+        const int c0 = hf * 64;                              // this warp's columns
+        const uint32_t lane_base = (uint32_t)(qd * 32) << 16;
+        const uint32_t pair_bar = 1 + qd;
         // rows past the block's end take the last valid position: finite, never stored
         const int pos_r = min(pos0 + r, pos_last);
         const float sl2 = geo.scale * kLog2e;
         bool ok = wait(&sm.r_full, 0);
 
-        // Routed query row: Q_r * scale * log2 e as hi + lo bf16 pairs into the Q columns.
+        // Routed query row, this warp's 64 columns: Q_r * scale * log2 e as hi + lo bf16 pairs
+        // into the Q columns (32 packed columns each).
         if (ok) {
             ptx::tc_fence_after();
+            uint32_t u0[32], u1[32];
+            ptx::tmem_ld32(tmem + kColS + c0 + lane_base, u0);
+            ptx::tmem_ld32(tmem + kColS + c0 + 32 + lane_base, u1);
+            ptx::tmem_wait_ld();
+            ptx::reg_fence(u0);
+            ptx::reg_fence(u1);
+            uint32_t hi[32], lo[32];
 #pragma unroll
-            for (int c4 = 0; c4 < 4; c4 += 2) {
-                uint32_t u0[32], u1[32];
-                ptx::tmem_ld32(tmem + kColS + c4 * 32 + lane_base, u0);
-                ptx::tmem_ld32(tmem + kColS + c4 * 32 + 32 + lane_base, u1);
-                ptx::tmem_wait_ld();
-                ptx::reg_fence(u0);
-                ptx::reg_fence(u1);
-                uint32_t hi[32], lo[32];
-#pragma unroll
-                for (int e = 0; e < 16; ++e) {
-                    split2(__uint_as_float(u0[2 * e]) * sl2, __uint_as_float(u0[2 * e + 1]) * sl2,
-                           hi[e], lo[e]);
-                    split2(__uint_as_float(u1[2 * e]) * sl2, __uint_as_float(u1[2 * e + 1]) * sl2,
-                           hi[16 + e], lo[16 + e]);
-                }
-                // 64 values -> 32 packed columns
-                ptx::tmem_st32(tmem + kColQ + c4 * 16 + lane_base, hi);
-                ptx::tmem_st32(tmem + kColQ + kLoCols + c4 * 16 + lane_base, lo);
+            for (int e = 0; e < 16; ++e) {
+                split2(__uint_as_float(u0[2 * e]) * sl2, __uint_as_float(u0[2 * e + 1]) * sl2,
+                       hi[e], lo[e]);
+                split2(__uint_as_float(u1[2 * e]) * sl2, __uint_as_float(u1[2 * e + 1]) * sl2,
+                       hi[16 + e], lo[16 + e]);
             }
+            ptx::tmem_st32(tmem + kColQ + c0 / 2 + lane_base, hi);
+            ptx::tmem_st32(tmem + kColQ + kLoCols + c0 / 2 + lane_base, lo);
             ptx::tmem_wait_st();
             ptx::tc_fence_before();
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&sm.qr_ready);
         }
 
-        float m_ref = -INFINITY;   // reference maximum of the row (base 2)
-        float l = 0.f;             // sum of 2^(s - m_ref) over the tokens seen
-        for (int i = 0; ok && i < n_tiles; ++i) {
-            const int t0 = i * kBN;
-            if (!wait(&sm.s_full, i & 1)) { ok = false; break; }
-            ptx::tc_fence_after();
-            float sv[kBN];
-            {
-                // the four loads in flight together, one wait
-                uint32_t u0[32], u1[32], u2[32], u3[32];
-                const uint32_t sa = tmem + kColS + lane_base;
-                ptx::tmem_ld32(sa, u0);
-                ptx::tmem_ld32(sa + 32, u1);
-                ptx::tmem_ld32(sa + 64, u2);
-                ptx::tmem_ld32(sa + 96, u3);
+        float m_ref = -INFINITY;   // reference maximum of the row (base 2), shared by the pair
+        float l = 0.f;             // this warp's share of sum 2^(s - m_ref)
+        // Both warps of a pair run the same tiles and meet on exactly one pair barrier per
+        // tile and one in the epilogue; a wait that fails only turns this warp's vote false, and
+        // the pair leaves together at the next barrier.
+        bool okl = ok;
+        for (int i = 0; i < n_tiles; ++i) {
+            const int t0 = i * kBN, rb = i & 1;
+            if (okl) okl = wait(&sm.s_full, i & 1);
+            float sv[64];
+            float mp = -INFINITY;
+            if (okl) {
+                ptx::tc_fence_after();
+                uint32_t u0[32], u1[32];
+                ptx::tmem_ld32(tmem + kColS + c0 + lane_base, u0);
+                ptx::tmem_ld32(tmem + kColS + c0 + 32 + lane_base, u1);
                 ptx::tmem_wait_ld();
                 ptx::reg_fence(u0);
                 ptx::reg_fence(u1);
-                ptx::reg_fence(u2);
-                ptx::reg_fence(u3);
 #pragma unroll
                 for (int c = 0; c < 32; ++c) {
                     sv[c] = __uint_as_float(u0[c]);
                     sv[32 + c] = __uint_as_float(u1[c]);
-                    sv[64 + c] = __uint_as_float(u2[c]);
-                    sv[96 + c] = __uint_as_float(u3[c]);
                 }
-            }
-            // S is in registers: the score MMAs of the next tile may overwrite it
-            ptx::tc_fence_before();
-            __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(&sm.s_free);
-
-            // causal mask: token t0 + c is visible to the row when t0 + c <= pos_r
-            if (t0 + kBN - 1 > pos0) {
-                const int lim = pos_r - t0;
+                // S is in registers: the score MMAs of the next tile may overwrite it
+                ptx::tc_fence_before();
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(&sm.s_free);
+                // causal mask: token t0 + c0 + c is visible to the row when it is <= pos_r
+                if (t0 + c0 + 63 > pos0) {
+                    const int lim = pos_r - t0 - c0;
 #pragma unroll
-                for (int c = 0; c < kBN; ++c)
-                    if (c > lim) sv[c] = -INFINITY;
-            }
-            float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                    for (int c = 0; c < 64; ++c)
+                        if (c > lim) sv[c] = -INFINITY;
+                }
+                float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-            for (int c = 0; c < kBN; c += 4) {
-                mx[0] = fmaxf(mx[0], sv[c]);
-                mx[1] = fmaxf(mx[1], sv[c + 1]);
-                mx[2] = fmaxf(mx[2], sv[c + 2]);
-                mx[3] = fmaxf(mx[3], sv[c + 3]);
+                for (int c = 0; c < 64; c += 4) {
+                    mx[0] = fmaxf(mx[0], sv[c]);
+                    mx[1] = fmaxf(mx[1], sv[c + 1]);
+                    mx[2] = fmaxf(mx[2], sv[c + 2]);
+                    mx[3] = fmaxf(mx[3], sv[c + 3]);
+                }
+                mp = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+                sm.red[rb][hf][r] = mp;
             }
-            const float m_tile = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+            // the pair exchanges its half maxima (and leaves together on any failed wait)
+            if (!ptx::bar_and(pair_bar, 64, okl)) {
+                okl = false;
+                break;
+            }
+            const float m_tile = fmaxf(mp, sm.red[rb][hf ^ 1][r]);
             const float m_new = fmaxf(m_ref, m_tile);
-            // a new reference when the maximum grew by more than 2^8 (or is the first finite)
+            // a new reference when the maximum grew by more than 2^8 (or is the first finite);
+            // both warps of the pair take the same decision from the same numbers
             const bool grow = m_new > m_ref + kRescaleLog2;
             if (__any_sync(0xffffffffu, grow)) {
                 const float f = (m_new == -INFINITY || m_ref == -INFINITY) ? 0.f : ptx::ex2(m_ref - m_new);
                 if (i > 0) {
                     // O holds tiles 0 .. i - 1 once the output MMAs of tile i - 1 are done
-                    if (!wait(&sm.pv_done, (i - 1) & 1)) { ok = false; break; }
-                    ptx::tc_fence_after();
+                    okl = okl && wait(&sm.pv_done, (i - 1) & 1);
+                    if (okl) {
+                        ptx::tc_fence_after();
 #pragma unroll
-                    for (int c4 = 0; c4 < 4; ++c4) {
-                        uint32_t u[32];
-                        ptx::tmem_ld32(tmem + kColO + c4 * 32 + lane_base, u);
-                        ptx::tmem_wait_ld();
-                        ptx::reg_fence(u);
+                        for (int c = 0; c < 64; c += 32) {
+                            uint32_t u[32];
+                            ptx::tmem_ld32(tmem + kColO + c0 + c + lane_base, u);
+                            ptx::tmem_wait_ld();
+                            ptx::reg_fence(u);
 #pragma unroll
-                        for (int c = 0; c < 32; ++c) u[c] = __float_as_uint(__uint_as_float(u[c]) * f);
-                        ptx::tmem_st32(tmem + kColO + c4 * 32 + lane_base, u);
+                            for (int e = 0; e < 32; ++e) u[e] = __float_as_uint(__uint_as_float(u[e]) * f);
+                            ptx::tmem_st32(tmem + kColO + c0 + c + lane_base, u);
+                        }
+                        ptx::tmem_wait_st();
                     }
-                    ptx::tmem_wait_st();
                 }
                 l *= f;
                 m_ref = m_new;
             }
             const float mr = m_ref == -INFINITY ? 0.f : m_ref;
 
-            // P_hi | P_lo, 128 weights -> 64 packed columns each: computed in registers first
-            // (this overlaps the output MMAs of tile i - 1), stored once those MMAs have read
-            // the previous P
-            uint32_t ph0[32], ph1[32], pl0[32], pl1[32];
+            // this warp's 64 weights -> 32 packed columns of P_hi and of P_lo: computed in
+            // registers first, stored once the output MMAs of tile i - 1 have read the previous P
+            uint32_t ph[32], pl[32];
             float ls[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
             for (int e = 0; e < 32; ++e) {
                 const float a0 = ptx::ex2(sv[2 * e] - mr), a1 = ptx::ex2(sv[2 * e + 1] - mr);
-                const float b0 = ptx::ex2(sv[64 + 2 * e] - mr), b1 = ptx::ex2(sv[64 + 2 * e + 1] - mr);
-                ls[0] += a0;
-                ls[1] += a1;
-                ls[2] += b0;
-                ls[3] += b1;
-                split2(a0, a1, ph0[e], pl0[e]);
-                split2(b0, b1, ph1[e], pl1[e]);
+                ls[(2 * e) & 3] += a0;
+                ls[(2 * e + 1) & 3] += a1;
+                split2(a0, a1, ph[e], pl[e]);
             }
             l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
-            if (i >= 1 && !wait(&sm.pv_done, (i - 1) & 1)) { ok = false; break; }
-            const uint32_t pa = tmem + kColP + lane_base;
-            ptx::tmem_st32(pa, ph0);
-            ptx::tmem_st32(pa + 32, ph1);
-            ptx::tmem_st32(pa + kLoCols, pl0);
-            ptx::tmem_st32(pa + kLoCols + 32, pl1);
-            ptx::tmem_wait_st();
-            // cache rows at or past the sequence's end (an unwritten page tail, or a page slot
-            // no TMA filled) become zeros, so that 0-weights never meet a non-finite value
-            if (t0 + kBN > L && t0 + r >= L) {
-                const uint32_t v_s = ptx::smem_addr(sm.tiles[(i + 1) % kStages]) + r * 128;
+            if (okl && i >= 1) okl = wait(&sm.pv_done, (i - 1) & 1);
+            if (okl) {
+                ptx::tmem_st32(tmem + kColP + c0 / 2 + lane_base, ph);
+                ptx::tmem_st32(tmem + kColP + kLoCols + c0 / 2 + lane_base, pl);
+                ptx::tmem_wait_st();
+                // cache rows at or past the sequence's end (an unwritten page tail, or a page
+                // slot no TMA filled) become zeros, so that 0-weights never meet a non-finite
+                // value; each warp of the pair clears its own 64-dim half of the row
+                if (t0 + kBN > L && t0 + r >= L) {
+                    const uint32_t v_s = ptx::smem_addr(sm.tiles[(i + 1) % kStages]) +
+                                         hf * kHalfBytes + r * 128;
 #pragma unroll
-                for (int c = 0; c < 8; ++c) {
-                    st_shared_v4(v_s + c * 16, 0u, 0u, 0u, 0u);
-                    st_shared_v4(v_s + kHalfBytes + c * 16, 0u, 0u, 0u, 0u);
+                    for (int c = 0; c < 8; ++c) st_shared_v4(v_s + c * 16, 0u, 0u, 0u, 0u);
                 }
+                ptx::tc_fence_before();
+                ptx::fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(&sm.p_full);
             }
-            ptx::tc_fence_before();
-            ptx::fence_proxy_async_smem();
-            __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(&sm.p_full);
+            // a wait that failed above leaves okl false: this warp skips its work and votes
+            // false at the next pair barrier (or the epilogue's), where the pair leaves together
         }
 
-        // Epilogue: out = O / l for the block's rows.
-        if (ok && wait(&sm.pv_done, (n_tiles - 1) & 1)) {
+        // Epilogue: out = O / l, this warp's 64 output dims; l is the pair's two shares.
+        const bool oke = okl && wait(&sm.pv_done, (n_tiles - 1) & 1);
+        sm.lsum[hf][r] = l;
+        if (ptx::bar_and(pair_bar, 64, oke)) {
             ptx::tc_fence_after();
-            const float inv = l > 0.f ? 1.f / l : 0.f;
-            const size_t orow = ((size_t)(q0 + m0 + r) * geo.Hq + h) * kD;
+            const float lt = l + sm.lsum[hf ^ 1][r];
+            const float inv = lt > 0.f ? 1.f / lt : 0.f;
+            const size_t orow = ((size_t)(q0 + m0 + r) * geo.Hq + h) * kD + c0;
 #pragma unroll
-            for (int c4 = 0; c4 < 4; ++c4) {
+            for (int c4 = 0; c4 < 2; ++c4) {
                 uint32_t u[32];
-                ptx::tmem_ld32(tmem + kColO + c4 * 32 + lane_base, u);
+                ptx::tmem_ld32(tmem + kColO + c0 + c4 * 32 + lane_base, u);
                 ptx::tmem_wait_ld();
                 ptx::reg_fence(u);
                 if (r < rows) {
