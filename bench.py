@@ -52,6 +52,8 @@ def parse_args():
                    help="time the same-design K+V decode (comparison) instead of keyless")
     p.add_argument("--wr-per-query-head", action="store_true",
                    help="one W^R per query head (the paper's GQA models) instead of per value head")
+    p.add_argument("--fused-query", action="store_true",
+                   help="decode with the composed query q = x W^Q W^R (no W^R in the kernel)")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=10.0)
     return p.parse_args()
@@ -156,7 +158,7 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def algorithmic_bytes(x, standard: bool) -> dict:
+def algorithmic_bytes(x, standard: bool, with_wr: bool = True) -> dict:
     """Bytes the decode must move once: cached rows (V, plus K for the comparison), W^R,
     q, out (fp32 read by nobody: bf16 written), block table and lengths."""
     wl = x["workload"]
@@ -166,7 +168,7 @@ def algorithmic_bytes(x, standard: bool) -> dict:
     tokens = int(x["seq_lens"].sum())
     v = tokens * Hkv * D * 2
     cache = 2 * v if standard else v
-    wr = 0 if standard else x["w_r"].numel() * 2
+    wr = 0 if standard or not with_wr else x["w_r"].numel() * 2
     q = B * Hq * D * 2
     out = B * Hq * D * 2
     bt = sum(math.ceil(int(L) / P) for L in x["seq_lens"].tolist()) * 4 + B * 4
@@ -321,9 +323,9 @@ def run_ours(args):
             kl.kl_standard_decode(sh, g["q"], k_cache, g["v_cache"], g["block_table"],
                                   g["seq_lens"], opts, o, kl.KL_BF16, w, err, stream)
         else:
-            kl.kl_decode_step(sh, g["q"], g["w_r"], g["v_new"], g["positions"], g["v_cache"],
-                              g["block_table"], g["seq_lens"], opts, o, kl.KL_BF16, w, err,
-                              stream)
+            kl.kl_decode_step(sh, g["q"], None if args.fused_query else g["w_r"], g["v_new"],
+                              g["positions"], g["v_cache"], g["block_table"], g["seq_lens"], opts,
+                              o, kl.KL_BF16, w, err, stream)
 
     def step_timed(ev):
         # [append +] decode kernel | combine, bracketed by events on the launching stream; the
@@ -365,7 +367,7 @@ def run_ours(args):
     mean_step, mean_dec = max_over_ranks([mean_step, mean_dec], device=dev)
     assert int(err.item()) == 0, f"device error flags {int(err.item())}"
 
-    ab = algorithmic_bytes(x, args.standard)
+    ab = algorithmic_bytes(x, args.standard, with_wr=not args.fused_query)
     value = job_throughput(B, world, mean_step / 1e3)
     peak, peak_kind = measured_peaks()
     dec_gbs = ab["total"] / (mean_dec / 1e3) / 1e9
@@ -389,7 +391,8 @@ def run_ours(args):
                                       d_in["seq_lens"], opts_full, out, kl.KL_BF16, ws, err,
                                       stream)
             else:
-                kl.kl_decode_step(sh, d_in["q"], g["w_r"], d_in["v_new"], d_in["positions"],
+                kl.kl_decode_step(sh, d_in["q"], None if args.fused_query else g["w_r"],
+                                  d_in["v_new"], d_in["positions"],
                                   g["v_cache"], d_in["block_table"], d_in["seq_lens"], opts_full,
                                   out, kl.KL_BF16, ws, err, stream)
             h_out.copy_(out, non_blocking=True)
@@ -433,7 +436,9 @@ def run_ours(args):
                    "head_dim": D, "page_size": P,
                    "seq_len": wl.seq_len or list(wl.seq_len_range),
                    "context_tokens": ab["tokens"], "num_splits": S, "kernel": kname,
-                   "decode": "standard K+V (comparison)" if args.standard else "keyless",
+                   "decode": "standard K+V (comparison)" if args.standard else
+                             "keyless, composed query (x W^Q W^R)" if args.fused_query else
+                             "keyless",
                    "w_r": "per query head" if wl.wr_per_query_head else "per value head",
                    "l2": "flushed between timed steps (512 MiB write, then read back)",
                    "parallelism": f"replicas x{world}"},

@@ -140,6 +140,9 @@ int32_t kl_decode_num_splits(const kl_shape *shape, int32_t num_splits);
  * `workspace` must hold kl_decode_workspace_size(shape, num_splits) bytes (256-byte aligned,
  * zero-filled before its first use). A bad page id or length raises its flag and leaves that
  * output unspecified.
+ * w_r == NULL selects the composed-query form of Section 2.1: at inference W^Q W^R is one
+ * precomputed projection, so q already is the routed query (q = x W^Q W^R) and is used as q_r
+ * directly (no routing in the kernel). The same holds for every decode entry point below.
  */
 kl_status kl_decode_attention(const kl_shape *shape, const void *q, const void *w_r,
                               const void *v_cache, const int32_t *block_table,

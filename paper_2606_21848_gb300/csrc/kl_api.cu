@@ -112,7 +112,7 @@ kl_status decode_common(bool standard, const kl_shape *shape, const void *q, con
     if (g.G > 8) return KL_ERR_UNSUPPORTED;
     if (g.B == 0) return KL_OK;
     if ((!q && !q_routed) || !v_cache || !block_table || !seq_lens) return KL_ERR_INVALID_ARG;
-    if (!q_routed && (standard ? !k_cache : !w_r)) return KL_ERR_INVALID_ARG;
+    if (standard && !k_cache) return KL_ERR_INVALID_ARG;   // keyless: w_r == NULL = composed q
     if ((q && !aligned(q, 16)) || !aligned(v_cache, 16) || (w_r && !aligned(w_r, 16)) ||
         (k_cache && !aligned(k_cache, 16)) || (out && !aligned(out, 16)))
         return KL_ERR_INVALID_ARG;

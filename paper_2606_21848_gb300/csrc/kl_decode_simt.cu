@@ -88,8 +88,8 @@ __global__ void __launch_bounds__(kWarps * 32) decode_simt_kernel(DecodeArgs a) 
         for (int i = tid; i < G * D; i += kWarps * 32) {
             const int h = i / D, j = i % D;
             float acc;
-            if constexpr (kStandard) {
-                acc = q_in[h][j];
+            if (kStandard || a.w_r == nullptr) {
+                acc = q_in[h][j];      // unrouted (K+V) or already composed (q = x W^Q W^R)
             } else {
                 const uint16_t *W = a.w_r + (size_t)(geo.wr_per_qh ? g * G + h : g) * D * D;
                 acc = 0.f;

@@ -325,7 +325,9 @@ __global__ void __launch_bounds__(kThreads, 2)
     // The routing runs on the tensor cores: W^R[g] (one per value head) or the G matrices
     // W^R[g G + h] (one per query head) arrive by TMA as ring positions 0 .. route_tiles - 1,
     // with the group's query rows, and the cache tiles follow.
-    const bool tc_route = !kStandard && a.q_routed == nullptr;
+    // routing on the tensor cores unless the query arrives routed: pre-routed fp32 queries, or
+    // the composed query q = x W^Q W^R of Section 2.1 (no W^R given)
+    const bool tc_route = !kStandard && a.q_routed == nullptr && a.w_r != nullptr;
     const bool route_pq = tc_route && geo.wr_per_qh;
     const int route_tiles = !tc_route ? 0 : route_pq ? G : 1;
     const int ro = route_tiles;
@@ -645,8 +647,8 @@ __global__ void __launch_bounds__(kThreads, 2)
         bool ok = true;
 
         // Routing prologue: thread j obtains q_r[h][j] for the G heads in fp32 from the routing
-        // MMAs in TMEM, from the caller's pre-routed queries, or, for the K+V comparison, the
-        // unrouted query itself.
+        // MMAs in TMEM, from the caller's pre-routed queries, or the query itself (already
+        // composed with W^R, or unrouted for the K+V comparison).
         float acc[kNG];
 #pragma unroll
         for (int h = 0; h < kNG; ++h) acc[h] = 0.f;
@@ -908,7 +910,7 @@ cudaError_t launch(const DecodeArgs &a) {
     kmap = wmap = qmap = vmap;
     if (kStandard && !make_map(&kmap, a.k_cache, cache_rows, (uint32_t)g.P))
         return cudaErrorInvalidValue;
-    if (!kStandard && !a.q_routed) {
+    if (!kStandard && !a.q_routed && a.w_r) {
         // W^R [Hw * 128 rows (k)][128 (j)], Hw = Hkv or Hq, one box = one 64-column half of one
         // matrix; q [B * Hq rows][128], one box = the G rows of one value group.
         const uint64_t hw = g.wr_per_qh ? (uint64_t)g.Hq : (uint64_t)g.Hkv;

@@ -344,3 +344,54 @@ def test_workload_sampled_parity(name, kname):
     got = np.stack([out[b, h].cpu().numpy() for b, h in heads])
     assert_parity(got, want, f"{name} {kname}")
     assert np.isfinite(out.cpu().numpy()).all()
+
+
+# ------------------------------------------------- composed query (fused W^Q W^R) -----------
+
+@pytest.mark.parametrize("kname", ["simt", "tensor"])
+@pytest.mark.parametrize("num_splits", [1, 3, 0])
+def test_composed_query_mode_matches_oracle_with_identity_routing(kname, num_splits):
+    """w_r = NULL: the query already is x W^Q W^R (Section 2.1's precomputed projection), so the
+    decode equals the oracle's decode with W^R = I."""
+    x = tiny(B=3, Hq=16, Hkv=4, D=128, P=16, lens=(1, 300, 1000))
+    k = _kernel_or_skip(kname, x)
+    g = to_dev(x)
+    sh = shape_of(x)
+    out = torch.full((3, 16, 128), float("nan"), dtype=torch.float32, device=_gpu.dev())
+    err = torch.zeros(1, dtype=torch.int32, device=_gpu.dev())
+    ws = torch.zeros(max(256, kl.kl_decode_workspace_size(sh, num_splits)), dtype=torch.uint8,
+                     device=_gpu.dev())
+    kl.kl_decode_attention_ex(sh, g["q"], None, g["v_cache"], g["block_table"], g["seq_lens"],
+                              kl.decode_options(num_splits, k), out, kl.KL_FP32, ws, err)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    eye = np.broadcast_to(np.eye(128, dtype=np.float32)[None], (4, 128, 128))
+    w_eye = bf16_bits(torch.from_numpy(eye.copy()).to(torch.bfloat16))
+    want = oracle.decode(bf16_bits(x["q"]), w_eye, bf16_bits(x["v_cache"]),
+                         x["block_table"].numpy(), x["seq_lens"].numpy(),
+                         scale=_gpu.default_scale(x))
+    assert_parity(out.cpu().numpy(), want, f"composed query {kname} S={num_splits}")
+
+
+def test_composed_query_fused_step_appends_and_decodes():
+    x = tiny(B=2, Hq=32, Hkv=8, D=128, P=32, lens=(700, 64))
+    if not _tc_available(x):
+        pytest.skip("tensor-core kernel does not support this geometry")
+    g = to_dev(x)
+    sh = shape_of(x)
+    out = torch.empty(2, 32, 128, dtype=torch.float32, device=_gpu.dev())
+    err = torch.zeros(1, dtype=torch.int32, device=_gpu.dev())
+    ws = torch.zeros(max(256, kl.kl_decode_workspace_size(sh, 2)), dtype=torch.uint8,
+                     device=_gpu.dev())
+    kl.kl_decode_step(sh, g["q"], None, g["v_new"], g["positions"], g["v_cache"],
+                      g["block_table"], g["seq_lens"], kl.decode_options(2), out, kl.KL_FP32, ws,
+                      err)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    cache = oracle.append(bf16_bits(x["v_cache"]), bf16_bits(x["v_new"]),
+                          x["block_table"].numpy(), x["positions"].numpy())
+    eye = np.broadcast_to(np.eye(128, dtype=np.float32)[None], (8, 128, 128))
+    w_eye = bf16_bits(torch.from_numpy(eye.copy()).to(torch.bfloat16))
+    want = oracle.decode(bf16_bits(x["q"]), w_eye, cache, x["block_table"].numpy(),
+                         x["seq_lens"].numpy(), scale=_gpu.default_scale(x))
+    assert_parity(out.cpu().numpy(), want, "composed query, fused step")
