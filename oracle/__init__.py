@@ -11,8 +11,9 @@ Two independent formulations live here:
   s_i = scale * <q_r, v_i>, softmax weights alpha_{n+1,i} and output O_{n+1} = sum alpha v_i
   (Section 3), plus the split-state merge, the cache append and, for the K+V comparison,
   standard attention (Eq. 1).
-  The prefill of a chunk of new tokens (Eq. 3 with a causal mask), the chunk append and the
-  decode over a latent value-only cache (Section 3) use the same per-row attention.
+  The prefill of a chunk of new tokens (Eq. 3 with a causal mask), the chunk append, the
+  decode over a latent value-only cache (Section 3) and over an FP8 (E4M3, per-row scale) value
+  cache use the same per-row attention.
 * ``dense.py`` -- a NumPy brute force that first un-pages the cache with its own code and then
   evaluates the same formulas on dense arrays; it is used for tiny inputs only.
 
@@ -68,10 +69,18 @@ def _load():
         _lib.ko_prefill.argtypes = [i, i, i, i, i, i, i, i, d, p, p, p, p, p, p, i, p, p]
         _lib.ko_append_chunk.argtypes = [i, i, i, i, i, i, p, p, p, p, p]
         _lib.ko_latent_decode.argtypes = [i, i, i, i, i, i, i, i, i, d, p, p, p, p, p, p, i, p, p]
+        _lib.ko_quantize_rows.argtypes = [i, i, p, p, p]
+        _lib.ko_append_fp8.argtypes = [i, i, i, i, i, i, p, p, p, p, p]
+        _lib.ko_decode_fp8.argtypes = [i, i, i, i, i, i, i, i, d, p, p, p, p, p, p, i, p, p]
         for f in ("ko_route", "ko_decode", "ko_standard_decode", "ko_attention_weights",
                   "ko_decode_partial", "ko_combine", "ko_append", "ko_prefill",
-                  "ko_append_chunk", "ko_latent_decode"):
+                  "ko_append_chunk", "ko_latent_decode", "ko_quantize_rows", "ko_append_fp8",
+                  "ko_decode_fp8"):
             getattr(_lib, f).restype = ctypes.c_int
+        _lib.ko_e4m3_from_f32.argtypes = [ctypes.c_float]
+        _lib.ko_e4m3_from_f32.restype = ctypes.c_uint8
+        _lib.ko_e4m3_value.argtypes = [ctypes.c_uint8]
+        _lib.ko_e4m3_value.restype = ctypes.c_double
     return _lib
 
 
@@ -251,4 +260,63 @@ def latent_decode(q, w_r, w_post, v_lat, block_table, seq_lens, *, scale: float,
                                   _ptr(w_post), _ptr(v_lat), _ptr(bt), _ptr(sl),
                                   0 if sel is None else len(sel), _ptr(sel), _ptr(out))
     _check(rc, "latent_decode")
+    return out.reshape(B, Hq, D) if sel is None else out
+
+
+# ----------------------------------------------------------------- FP8 value cache ----------
+
+def e4m3_value(codes) -> np.ndarray:
+    """Values of OCP FP8 E4M3 codes (uint8) as float64 (NaN for the NaN codes)."""
+    lib = _load()
+    c = np.asarray(codes, np.uint8)
+    return np.array([lib.ko_e4m3_value(int(x)) for x in c.ravel()], np.float64).reshape(c.shape)
+
+
+def e4m3_from_f32(x) -> np.ndarray:
+    """Nearest E4M3 codes of float32 values (ties to even mantissa, saturating at 448)."""
+    lib = _load()
+    a = np.asarray(x, np.float32)
+    return np.array([lib.ko_e4m3_from_f32(float(v)) for v in a.ravel()], np.uint8).reshape(a.shape)
+
+
+def quantize_rows(v_bits) -> tuple[np.ndarray, np.ndarray]:
+    """Per-row FP8 quantization of bf16 rows [..., D]: codes uint8 [..., D], scales float32 [...]."""
+    v = _c(v_bits, np.uint16)
+    D = v.shape[-1]
+    n = v.size // D
+    codes = np.zeros(v.shape, np.uint8)
+    scales = np.zeros(v.shape[:-1], np.float32)
+    _load().ko_quantize_rows(n, D, _ptr(v), _ptr(codes), _ptr(scales))
+    return codes, scales
+
+
+def append_fp8(codes, scales, v_new, block_table, positions):
+    """Copies of the FP8 cache (codes [pages, Hkv, P, D], scales [pages, Hkv, P]) with v_new[b]
+    quantized into row positions[b]."""
+    codes = np.array(_c(codes, np.uint8), copy=True)
+    scales = np.array(_c(scales, np.float32), copy=True)
+    v_new = _c(v_new, np.uint16)
+    bt, pos = _c(block_table, np.int32), _c(positions, np.int32)
+    num_pages, Hkv, P, D = codes.shape
+    rc = _load().ko_append_fp8(v_new.shape[0], Hkv, D, P, num_pages, bt.shape[1], _ptr(v_new),
+                               _ptr(bt), _ptr(pos), _ptr(codes), _ptr(scales))
+    _check(rc, "append_fp8")
+    return codes, scales
+
+
+def decode_fp8(q, w_r, codes, scales, block_table, seq_lens, *, scale: float,
+               wr_per_query_head: bool = False, heads=None) -> np.ndarray:
+    """Keyless decode over the FP8 cache (values scale * e4m3(code)); [B, Hq, D] fp64."""
+    q, w_r = _c(q, np.uint16), _c(w_r, np.uint16)
+    codes, scales = _c(codes, np.uint8), _c(scales, np.float32)
+    bt, sl = _c(block_table, np.int32), _c(seq_lens, np.int32)
+    B, Hq, D = q.shape
+    num_pages, Hkv, P, _ = codes.shape
+    sel = None if heads is None else _c(np.asarray(heads, np.int32).reshape(-1, 2), np.int32)
+    out = np.zeros(((B * Hq) if sel is None else len(sel), D), np.float64)
+    rc = _load().ko_decode_fp8(B, Hq, Hkv, D, P, num_pages, bt.shape[1], int(wr_per_query_head),
+                               float(scale), _ptr(q), _ptr(w_r), _ptr(codes), _ptr(scales),
+                               _ptr(bt), _ptr(sl), 0 if sel is None else len(sel), _ptr(sel),
+                               _ptr(out))
+    _check(rc, "decode_fp8")
     return out.reshape(B, Hq, D) if sel is None else out

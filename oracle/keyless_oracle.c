@@ -20,7 +20,8 @@
  *   - for the comparison only: standard decode softmax(q K^T / sqrt(d_k)) V (Eq. 1) over a
  *     paged K cache and a paged V cache;
  *   - prefill of a chunk of new tokens (Eq. 3 under a causal mask) and the chunk append;
- *   - decode over a latent value-only cache (Section 3, latent value-only cache paragraph).
+ *   - decode over a latent value-only cache (Section 3, latent value-only cache paragraph);
+ *   - the FP8 (E4M3, one fp32 scale per cached row) value cache: encoding, append, decode.
  *
  * Readings where the paper is silent (each is listed in the design notes):
  *   - lambda / sqrt(d_k) is the caller's `scale`; lambda = 1 gives 1/sqrt(d_k);
@@ -538,6 +539,187 @@ int ko_latent_decode(int B, int Hq, int Hl, int D, int r, int P, int num_pages, 
         free(s);
         free(os);
         free(qs);
+        free(qr);
+    }
+    return err ? -1 : 0;
+}
+
+/*
+ * FP8 value cache (the low-precision value cache of the scope table: orthogonal to the method,
+ * compatible with it). Values are stored as OCP FP8 E4M3 codes (1 sign bit, 4 exponent bits
+ * with bias 7, 3 mantissa bits; exponent field 0 encodes subnormals m/8 * 2^-6; the all-ones
+ * exponent with all-ones mantissa is NaN; no infinities; largest finite value 448) with one
+ * fp32 scale per cached row: v = scale * value(code).
+ */
+static double e4m3_value(uint8_t c)
+{
+    int sign = c >> 7, e = (c >> 3) & 15, m = c & 7;
+    double v;
+    if (e == 15 && m == 7)
+        return NAN;
+    if (e == 0)
+        v = (double)m / 8.0 * ldexp(1.0, -6);
+    else
+        v = (1.0 + (double)m / 8.0) * ldexp(1.0, e - 7);
+    return sign ? -v : v;
+}
+
+/* Nearest E4M3 code of x, ties to the code with an even mantissa, magnitudes above 448 clamped
+ * to 448 (saturating conversion). The grid values are exact in double, so the comparisons are
+ * exact. */
+uint8_t ko_e4m3_from_f32(float x)
+{
+    uint8_t sign = (x < 0.0f || (x == 0.0f && signbit(x))) ? 0x80 : 0;
+    double a = fabs((double)x);
+    if (a >= 448.0)
+        return sign | 0x7E;
+    int lo = 0;                       /* largest code with value <= a (codes 0..126 ascend) */
+    for (int c = 1; c <= 126; ++c)
+        if (e4m3_value((uint8_t)c) <= a)
+            lo = c;
+    if (lo == 126)
+        return sign | 126;
+    double vl = e4m3_value((uint8_t)lo), vh = e4m3_value((uint8_t)(lo + 1));
+    int pick;
+    if (a - vl < vh - a)
+        pick = lo;
+    else if (a - vl > vh - a)
+        pick = lo + 1;
+    else
+        pick = (lo & 1) ? lo + 1 : lo;    /* tie: even mantissa */
+    return sign | (uint8_t)pick;
+}
+
+double ko_e4m3_value(uint8_t c) { return e4m3_value(c); }
+
+/* Quantize one row of D bf16 values: scale = max |v| / 448 (fp32), code_j = e4m3(v_j / scale)
+ * with the division in fp32; an all-zero row gets scale 0 and zero codes. */
+static void quantize_row(int D, const uint16_t *v, uint8_t *codes, float *scale)
+{
+    float amax = 0.0f;
+    for (int j = 0; j < D; ++j) {
+        uint32_t u = ((uint32_t)v[j]) << 16;
+        float f;
+        memcpy(&f, &u, sizeof f);
+        if (fabsf(f) > amax)
+            amax = fabsf(f);
+    }
+    float s = amax / 448.0f;
+    *scale = s;
+    for (int j = 0; j < D; ++j) {
+        uint32_t u = ((uint32_t)v[j]) << 16;
+        float f;
+        memcpy(&f, &u, sizeof f);
+        codes[j] = s > 0.0f ? ko_e4m3_from_f32(f / s) : 0;
+    }
+}
+
+int ko_quantize_rows(int n, int D, const uint16_t *v, uint8_t *codes, float *scales)
+{
+    for (int i = 0; i < n; ++i)
+        quantize_row(D, v + (size_t)i * D, codes + (size_t)i * D, scales + i);
+    return 0;
+}
+
+/* Append to the FP8 cache: row pos_b of sequence b, every value head, quantized as above.
+ * Codes are [num_pages][Hkv][P][D], scales [num_pages][Hkv][P]. */
+int ko_append_fp8(int B, int Hkv, int D, int P, int num_pages, int max_pages,
+                  const uint16_t *v_new, const int32_t *block_table, const int32_t *positions,
+                  uint8_t *codes, float *scales)
+{
+    int err = 0;
+    for (int b = 0; b < B; ++b) {
+        int pos = positions[b];
+        if (pos < 0 || pos >= max_pages * P) {
+            err = 1;
+            continue;
+        }
+        int page = block_table[(size_t)b * max_pages + pos / P];
+        if (page < 0 || page >= num_pages) {
+            err = 1;
+            continue;
+        }
+        for (int g = 0; g < Hkv; ++g) {
+            size_t row = ((size_t)page * Hkv + g) * P + (size_t)(pos % P);
+            quantize_row(D, v_new + ((size_t)b * Hkv + g) * D, codes + row * D, scales + row);
+        }
+    }
+    return err ? -1 : 0;
+}
+
+/*
+ * Keyless decode (Section 3) over the FP8 cache: every cached value is scale * value(code),
+ * widened exactly to double; otherwise as ko_decode (routing, GQA mapping, softmax, output).
+ */
+int ko_decode_fp8(int B, int Hq, int Hkv, int D, int P, int num_pages, int max_pages,
+                  int wr_per_query_head, double scale, const uint16_t *q, const uint16_t *w_r,
+                  const uint8_t *codes, const float *scales, const int32_t *block_table,
+                  const int32_t *seq_lens, int n_sel, const int32_t *sel, double *out)
+{
+    if (check_dims(B, Hq, Hkv, D) || P <= 0 || max_pages < 0)
+        return -1;
+    int G = Hq / Hkv;
+    long n_items = sel ? n_sel : (long)B * Hq;
+    int err = 0;
+
+#pragma omp parallel for schedule(dynamic, 1) reduction(| : err)
+    for (long it = 0; it < n_items; ++it) {
+        int b = sel ? sel[2 * it] : (int)(it / Hq);
+        int h = sel ? sel[2 * it + 1] : (int)(it % Hq);
+        double *o = out + (size_t)it * D;
+        for (int j = 0; j < D; ++j)
+            o[j] = 0.0;
+        if (b < 0 || b >= B || h < 0 || h >= Hq) {
+            err |= 1;
+            continue;
+        }
+        int L = seq_lens[b];
+        if (L < 0 || L > max_pages * P) {
+            err |= 1;
+            continue;
+        }
+        if (L == 0)
+            continue;
+        int g = h / G, w = wr_per_query_head ? h : g;
+        const int32_t *bt_row = block_table + (size_t)b * max_pages;
+        double *qr = (double *)malloc(sizeof(double) * (size_t)D);
+        double *rows = (double *)malloc(sizeof(double) * (size_t)L * D);
+        double *s = (double *)malloc(sizeof(double) * (size_t)L);
+        route_row(D, q + ((size_t)b * Hq + h) * D, w_r + (size_t)w * D * D, qr);
+        int bad = 0;
+        for (int t = 0; t < L && !bad; ++t) {
+            int page = bt_row[t / P];
+            if (page < 0 || page >= num_pages) {
+                bad = 1;
+                break;
+            }
+            size_t row = ((size_t)page * Hkv + g) * P + (size_t)(t % P);
+            for (int j = 0; j < D; ++j)
+                rows[(size_t)t * D + j] = (double)scales[row] * e4m3_value(codes[row * D + j]);
+        }
+        if (!bad) {
+            double m = -INFINITY;
+            for (int t = 0; t < L; ++t) {
+                double dot = 0.0;
+                for (int j = 0; j < D; ++j)
+                    dot += qr[j] * rows[(size_t)t * D + j];
+                s[t] = scale * dot;
+                if (s[t] > m)
+                    m = s[t];
+            }
+            double l = 0.0;
+            for (int t = 0; t < L; ++t) {
+                s[t] = exp(s[t] - m);
+                l += s[t];
+            }
+            for (int t = 0; t < L; ++t)
+                for (int j = 0; j < D; ++j)
+                    o[j] += s[t] / l * rows[(size_t)t * D + j];
+        } else {
+            err |= 1;
+        }
+        free(s);
+        free(rows);
         free(qr);
     }
     return err ? -1 : 0;

@@ -17,6 +17,7 @@ import pytest
 import oracle
 from oracle import dense
 from tests import test_oracle as pins
+from tests import test_oracle_fp8 as fp8_pins
 from tests import test_oracle_latent as latent_pins
 from tests import test_oracle_prefill as prefill_pins
 from tests._inputs import bits, default_scale, tiny
@@ -47,6 +48,13 @@ MUTATIONS = {
                                 "            o[j] = j < r ? os[j] : 0.0;\n        }\n        free(s);\n        free(os);"),
     "latent_wrong_group": ("        int g = h / G, w = wr_per_query_head ? h : g;\n        const uint16_t *Wp",
                            "        int g = h % Hl, w = wr_per_query_head ? h : g;\n        const uint16_t *Wp"),
+    # FP8 cache: the exponent bias, the tie rule, the per-row scale
+    "e4m3_wrong_bias": ("v = (1.0 + (double)m / 8.0) * ldexp(1.0, e - 7);",
+                        "v = (1.0 + (double)m / 8.0) * ldexp(1.0, e - 8);"),
+    "e4m3_ties_away": ("pick = (lo & 1) ? lo + 1 : lo;    /* tie: even mantissa */",
+                       "pick = lo + 1;"),
+    "fp8_drops_scale": ("rows[(size_t)t * D + j] = (double)scales[row] * e4m3_value(codes[row * D + j]);",
+                        "rows[(size_t)t * D + j] = e4m3_value(codes[row * D + j]);"),
     "prefill_wrong_row_base": ("route_row(D, q + ((size_t)r * Hq + h) * D, w_r + (size_t)w * D * D, qr);",
                                "route_row(D, q + ((size_t)(r - cu_q[b]) * Hq + h) * D, w_r + (size_t)w * D * D, qr);"),
 }
@@ -76,6 +84,9 @@ def _pin_results():
     run("latent_expand", latent_pins.test_absorbed_query_equals_expanded_values,
         dict(B=3, Hq=8, Hl=2, D=128, r=64, P=16, lens=(1, 37, 100)))
     run("latent_identity", latent_pins.test_identity_expansion_is_the_plain_keyless_decode)
+    run("e4m3_torch", fp8_pins.test_every_code_decodes_like_torch_float8_e4m3fn)
+    run("e4m3_encode", fp8_pins.test_encoding_matches_torch_rounding_in_range)
+    run("fp8_dense", fp8_pins.test_fp8_decode_equals_dense_over_dequantized_rows)
     return res
 
 
@@ -93,9 +104,10 @@ def test_planted_mistake_is_caught(name, tmp_path, monkeypatch):
     real = oracle._load()
     for f in ("ko_route", "ko_decode", "ko_standard_decode", "ko_attention_weights",
               "ko_decode_partial", "ko_combine", "ko_append", "ko_prefill", "ko_append_chunk",
-              "ko_latent_decode"):
+              "ko_latent_decode", "ko_quantize_rows", "ko_append_fp8", "ko_decode_fp8",
+              "ko_e4m3_from_f32", "ko_e4m3_value"):
         getattr(lib, f).argtypes = getattr(real, f).argtypes
-        getattr(lib, f).restype = ctypes.c_int
+        getattr(lib, f).restype = getattr(real, f).restype
     monkeypatch.setattr(oracle, "_lib", lib)
     res = _pin_results()
     assert not all(res.values()), f"mutation {name} survived every pin: {res}"
