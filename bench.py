@@ -54,6 +54,8 @@ def parse_args():
                    help="one W^R per query head (the paper's GQA models) instead of per value head")
     p.add_argument("--fused-query", action="store_true",
                    help="decode with the composed query q = x W^Q W^R (no W^R in the kernel)")
+    p.add_argument("--fp8-cache", action="store_true",
+                   help="FP8 (E4M3, per-row scale) value cache: quantizing append + FP8 decode")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=10.0)
     return p.parse_args()
@@ -158,7 +160,7 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def algorithmic_bytes(x, standard: bool, with_wr: bool = True) -> dict:
+def algorithmic_bytes(x, standard: bool, with_wr: bool = True, fp8: bool = False) -> dict:
     """Bytes the decode must move once: cached rows (V, plus K for the comparison), W^R,
     q, out (fp32 read by nobody: bf16 written), block table and lengths."""
     wl = x["workload"]
@@ -166,13 +168,14 @@ def algorithmic_bytes(x, standard: bool, with_wr: bool = True) -> dict:
     Hkv = x["v_cache"].shape[1]
     P = x["v_cache"].shape[2]
     tokens = int(x["seq_lens"].sum())
-    v = tokens * Hkv * D * 2
+    v = tokens * Hkv * (D + 4) if fp8 else tokens * Hkv * D * 2     # codes + row scale
     cache = 2 * v if standard else v
     wr = 0 if standard or not with_wr else x["w_r"].numel() * 2
     q = B * Hq * D * 2
     out = B * Hq * D * 2
     bt = sum(math.ceil(int(L) / P) for L in x["seq_lens"].tolist()) * 4 + B * 4
-    append = 0 if standard else 2 * B * Hkv * D * 2     # v_new read + cache row written
+    # v_new read + the cache row written (bf16, or codes and scale)
+    append = 0 if standard else B * Hkv * (D * 2 + (D + 4 if fp8 else D * 2))
     return {"cache": cache, "wr": wr, "total": cache + wr + q + out + bt + append,
             "tokens": tokens}
 
@@ -316,10 +319,24 @@ def run_ours(args):
                                                                       args.standard)
     # the tensor-core kernel merges the split states itself (ring-staged, any S up to the
     # library's limit); the CUDA-core kernel leaves them to the combine kernel
-    one_kernel = S == 1 or tc
+    one_kernel = S == 1 or tc or args.fp8_cache
 
-    def decode_call(opts, o, w):
-        if args.standard:
+    if args.fp8_cache:
+        codes = torch.empty(g["v_cache"].shape, dtype=torch.uint8, device=dev)
+        scales = torch.empty(g["v_cache"].shape[:-1], dtype=torch.float32, device=dev)
+        kl.kl_quantize_cache_fp8(sh, g["v_cache"], codes, scales, stream)
+        del g["v_cache"]
+        torch.cuda.synchronize()
+
+    def decode_call(opts, o, w, d=None):
+        d = d or g
+        if args.fp8_cache:
+            kl.kl_append_v_fp8(sh, d["v_new"], d["block_table"], d["positions"], codes, scales,
+                               err, stream)
+            kl.kl_decode_attention_fp8(sh, d["q"], None if args.fused_query else g["w_r"], codes,
+                                       scales, d["block_table"], d["seq_lens"], S, o, kl.KL_BF16,
+                                       w, err, stream)
+        elif args.standard:
             kl.kl_standard_decode(sh, g["q"], k_cache, g["v_cache"], g["block_table"],
                                   g["seq_lens"], opts, o, kl.KL_BF16, w, err, stream)
         else:
@@ -340,7 +357,7 @@ def run_ours(args):
             kl.kl_combine(sh, part_o, part_ml, S, out, kl.KL_BF16, stream)
         ev[2].record(stream)
 
-    launches_per_step = 1 if one_kernel else 2
+    launches_per_step = (2 + (S > 1)) if args.fp8_cache else 1 if one_kernel else 2
     E = lambda: torch.cuda.Event(enable_timing=True)
     for _ in range(args.warmup):
         flush_l2()
@@ -367,7 +384,7 @@ def run_ours(args):
     mean_step, mean_dec = max_over_ranks([mean_step, mean_dec], device=dev)
     assert int(err.item()) == 0, f"device error flags {int(err.item())}"
 
-    ab = algorithmic_bytes(x, args.standard, with_wr=not args.fused_query)
+    ab = algorithmic_bytes(x, args.standard, with_wr=not args.fused_query, fp8=args.fp8_cache)
     value = job_throughput(B, world, mean_step / 1e3)
     peak, peak_kind = measured_peaks()
     dec_gbs = ab["total"] / (mean_dec / 1e3) / 1e9
@@ -386,7 +403,9 @@ def run_ours(args):
         def e2e_step():
             for k in h_in:
                 d_in[k].copy_(h_in[k], non_blocking=True)
-            if args.standard:
+            if args.fp8_cache:
+                decode_call(opts_full, out, ws, d_in)
+            elif args.standard:
                 kl.kl_standard_decode(sh, d_in["q"], k_cache, g["v_cache"], d_in["block_table"],
                                       d_in["seq_lens"], opts_full, out, kl.KL_BF16, ws, err,
                                       stream)
@@ -426,7 +445,7 @@ def run_ours(args):
                "sample": f"{n} whole sequences of {wl.name} (all {Hq} heads, decode only, "
                          f"fp64) in {el:.1f}s"}
 
-    kname = "tensor" if tc else "simt"
+    kname = "tensor-fp8" if args.fp8_cache else "tensor" if tc else "simt"
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": mean_step,
@@ -436,6 +455,7 @@ def run_ours(args):
                    "head_dim": D, "page_size": P,
                    "seq_len": wl.seq_len or list(wl.seq_len_range),
                    "context_tokens": ab["tokens"], "num_splits": S, "kernel": kname,
+                   "cache": "fp8 e4m3 + fp32 row scale" if args.fp8_cache else "bf16",
                    "decode": "standard K+V (comparison)" if args.standard else
                              "keyless, composed query (x W^Q W^R)" if args.fused_query else
                              "keyless",

@@ -83,6 +83,9 @@ def load() -> ctypes.CDLL:
         "kl_decode_attention_noalloc": ([SH, P, P, P, P, P, I32, P, I32, P, P], I32),
         "kl_decode_kernel_available": ([SH, I32, I32], I32),
         "kl_append_v_chunk": ([SH, P, P, P, P, I32, I32, P, P, P], I32),
+        "kl_append_v_fp8": ([SH, P, P, P, P, P, P, P], I32),
+        "kl_quantize_cache_fp8": ([SH, P, P, P, P], I32),
+        "kl_decode_attention_fp8": ([SH, P, P, P, P, P, P, I32, P, I32, P, SZ, P, P], I32),
         "kl_latent_workspace_size": ([LS, I32], SZ),
         "kl_latent_decode": ([LS, P, P, P, P, P, P, I32, P, I32, P, SZ, P, P], I32),
         "kl_prefill_attention": ([SH, P, P, P, P, P, P, I32, I32, P, I32, P, P], I32),
@@ -222,6 +225,26 @@ def kl_prefill_attention(shape, q, w_r, v_cache, block_table, seq_lens, cu_q_len
                                        _p(block_table), _p(seq_lens), _p(cu_q_lens), total_q,
                                        max_q_len, _p(out), out_dtype, _p(err), _stream(stream)),
            "kl_prefill_attention")
+
+
+def kl_append_v_fp8(shape, v_new, block_table, positions, v_codes, v_scales, err=None,
+                    stream=None):
+    _check(load().kl_append_v_fp8(ctypes.byref(shape), _p(v_new), _p(block_table), _p(positions),
+                                  _p(v_codes), _p(v_scales), _p(err), _stream(stream)),
+           "kl_append_v_fp8")
+
+
+def kl_quantize_cache_fp8(shape, v_cache, v_codes, v_scales, stream=None):
+    _check(load().kl_quantize_cache_fp8(ctypes.byref(shape), _p(v_cache), _p(v_codes),
+                                        _p(v_scales), _stream(stream)), "kl_quantize_cache_fp8")
+
+
+def kl_decode_attention_fp8(shape, q, w_r, v_codes, v_scales, block_table, seq_lens, num_splits,
+                            out, out_dtype, workspace, err=None, stream=None):
+    _check(load().kl_decode_attention_fp8(ctypes.byref(shape), _p(q), _p(w_r), _p(v_codes),
+                                          _p(v_scales), _p(block_table), _p(seq_lens), num_splits,
+                                          _p(out), out_dtype, _p(workspace), _nbytes(workspace),
+                                          _p(err), _stream(stream)), "kl_decode_attention_fp8")
 
 
 def make_latent_shape(num_seqs, num_q_heads, num_latent_heads, head_dim, latent_dim, page_size,

@@ -358,6 +358,85 @@ kl_status latent_plan(const kl_latent_shape *s, int32_t num_splits, LatentPlan *
 
 extern "C" {
 
+kl_status kl_append_v_fp8(const kl_shape *shape, const void *v_new, const int32_t *block_table,
+                          const int32_t *positions, void *v_codes, float *v_scales, int32_t *err,
+                          kl_stream_t stream) {
+    Geometry g;
+    kl_status st = resolve(shape, -1, &g);
+    if (st != KL_OK) return st;
+    if (g.D != 128) return KL_ERR_UNSUPPORTED;
+    if (g.B == 0) return KL_OK;
+    if (!v_new || !block_table || !positions || !v_codes || !v_scales) return KL_ERR_INVALID_ARG;
+    if (!aligned(v_new, 16) || !aligned(v_codes, 16) || !aligned(v_scales, 16))
+        return KL_ERR_INVALID_ARG;
+    return from_cuda(launch_append_fp8(g, static_cast<const uint16_t *>(v_new), block_table,
+                                       positions, static_cast<uint8_t *>(v_codes), v_scales, err,
+                                       reinterpret_cast<cudaStream_t>(stream)));
+}
+
+kl_status kl_quantize_cache_fp8(const kl_shape *shape, const void *v_cache, void *v_codes,
+                                float *v_scales, kl_stream_t stream) {
+    Geometry g;
+    kl_status st = resolve(shape, -1, &g);
+    if (st != KL_OK) return st;
+    if (g.D != 128) return KL_ERR_UNSUPPORTED;
+    if (!v_cache || !v_codes || !v_scales) return KL_ERR_INVALID_ARG;
+    if (!aligned(v_cache, 16) || !aligned(v_codes, 16) || !aligned(v_scales, 16))
+        return KL_ERR_INVALID_ARG;
+    const size_t rows = (size_t)g.num_pages * g.Hkv * g.P;
+    return from_cuda(launch_quantize_fp8(rows, static_cast<const uint16_t *>(v_cache),
+                                         static_cast<uint8_t *>(v_codes), v_scales,
+                                         reinterpret_cast<cudaStream_t>(stream)));
+}
+
+kl_status kl_decode_attention_fp8(const kl_shape *shape, const void *q, const void *w_r,
+                                  const void *v_codes, const float *v_scales,
+                                  const int32_t *block_table, const int32_t *seq_lens,
+                                  int32_t num_splits, void *out, kl_dtype out_dtype,
+                                  void *workspace, size_t workspace_bytes, int32_t *err,
+                                  kl_stream_t stream) {
+    if (num_splits < 0) return KL_ERR_INVALID_ARG;
+    if (out_dtype != KL_BF16 && out_dtype != KL_FP32) return KL_ERR_INVALID_ARG;
+    Geometry g;
+    kl_status st = resolve(shape, num_splits, &g);
+    if (st != KL_OK) return st;
+    if (g.G > 8 || g.wr_per_qh || !tc_supported(g, false)) return KL_ERR_UNSUPPORTED;
+    if (g.P < 4) return KL_ERR_UNSUPPORTED;
+    if (g.B == 0) return KL_OK;
+    if (!q || !v_codes || !v_scales || !block_table || !seq_lens || !out) return KL_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(v_codes, 16) || !aligned(v_scales, 16) || !aligned(out, 16) ||
+        (w_r && !aligned(w_r, 16)))
+        return KL_ERR_INVALID_ARG;
+    const WorkspaceLayout wl = layout(g);
+    if (wl.total > 0 && (!workspace || workspace_bytes < wl.total || !aligned(workspace, 256)))
+        return KL_ERR_WORKSPACE;
+    DecodeArgs a{};
+    a.geo = g;
+    a.q = static_cast<const uint16_t *>(q);
+    a.w_r = static_cast<const uint16_t *>(w_r);
+    a.q_routed = nullptr;
+    a.k_cache = nullptr;
+    a.v_cache = static_cast<const uint16_t *>(v_codes);
+    a.block_table = block_table;
+    a.seq_lens = seq_lens;
+    a.v_new = nullptr;
+    a.positions = nullptr;
+    a.cache_rw = nullptr;
+    char *ws = static_cast<char *>(workspace);
+    a.part_o = wl.total ? reinterpret_cast<float *>(ws + wl.part_o) : nullptr;
+    a.part_ml = wl.total ? reinterpret_cast<float *>(ws + wl.part_ml) : nullptr;
+    a.out = out;
+    a.direct_out = g.S == 1;
+    a.merge_inside = false;
+    a.counters = nullptr;
+    a.out_dtype = out_dtype;
+    a.err = err;
+    a.stream = reinterpret_cast<cudaStream_t>(stream);
+    cudaError_t e = launch_decode_fp8(a, v_scales);
+    if (e == cudaSuccess) e = finish_decode(a, false);
+    return from_cuda(e);
+}
+
 size_t kl_latent_workspace_size(const kl_latent_shape *shape, int32_t num_splits) {
     LatentPlan p;
     return latent_plan(shape, num_splits, &p) == KL_OK ? p.total : 0;

@@ -106,6 +106,16 @@ cudaError_t launch_append_chunk(const Geometry &g, int total_q, int max_q, const
                                 const int32_t *cu_q, uint16_t *v_cache, int32_t *err,
                                 cudaStream_t stream);
 
+// FP8 value cache (E4M3 codes [num_pages][Hkv][P][D] with fp32 row scales [num_pages][Hkv][P]):
+// the decode on the tensor cores (a.v_cache holds the codes; states or direct output, merged by
+// the combine kernel) and the quantizing append.
+cudaError_t launch_decode_fp8(const DecodeArgs &a, const float *v_scales);
+cudaError_t launch_append_fp8(const Geometry &g, const uint16_t *v_new, const int32_t *block_table,
+                              const int32_t *positions, uint8_t *codes, float *scales, int32_t *err,
+                              cudaStream_t stream);
+cudaError_t launch_quantize_fp8(size_t rows, const uint16_t *v, uint8_t *codes, float *scales,
+                                cudaStream_t stream);
+
 // Latent value-only cache (head_dim D of queries and outputs, latent width r):
 // q_lat[b][h] = (q[b][h] W^R[w(h)]) W_post[h]^T and out[b][h] = o_lat[b][h] W_post[h].
 cudaError_t launch_latent_query(int B, int Hq, int G, int D, int r, int wr_per_qh,

@@ -9,7 +9,9 @@ from __future__ import annotations
 
 import math
 import os
+import queue
 import socket
+import time
 
 import numpy as np
 import pytest
@@ -78,9 +80,18 @@ def _run(worker):
     procs = [ctx.Process(target=worker, args=(r, port, q)) for r in range(WORLD)]
     for p in procs:
         p.start()
-    out = [q.get(timeout=240) for _ in range(WORLD)]
+    # A spawned rank imports torch afresh; in a cold container that alone can take minutes, so
+    # the wait is long but ends early when a rank dies without reporting.
+    out, deadline = [], time.monotonic() + 900
+    while len(out) < WORLD:
+        try:
+            out.append(q.get(timeout=5))
+        except queue.Empty:
+            dead = [p.exitcode for p in procs if p.exitcode not in (None, 0)]
+            assert not dead, f"a rank exited with {dead} before reporting"
+            assert time.monotonic() < deadline, "ranks did not report within 900 s"
     for p in procs:
-        p.join(timeout=60)
+        p.join(timeout=120)
         assert p.exitcode == 0
     return sorted(out)
 
