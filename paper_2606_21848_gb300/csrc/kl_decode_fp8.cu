@@ -2,27 +2,40 @@
 // tensor cores for sm_103a; and the quantizing append.
 //
 // Same method and split plan as the bf16 decode (routing q_r = q W^R, Section 2.2; one softmax
-// over the cached value rows, each row used for the score and for the output, Section 3), but
-// the cache moves half the bytes: a 128-token tile is 16 KiB of codes plus 512 B of scales.
-// Every code is an exact half-precision value, so two warps widen each landed tile into a
-// half-precision copy in shared memory, and the tensor cores run kind::f16 MMAs on it (the
-// routed query and the softmax weights as hi + lo half pairs):
+// over the cached value rows, each row used for the score and for the output, Section 3). The
+// tensor cores read the codes as TMA lands them: both products are kind::f8f6f4 MMAs (E4M3 x
+// E4M3, fp32 accumulation), so a 128-token tile moves 16 KiB of codes plus 512 B of row scales
+// and is never widened:
 //
-//   scores   S^T = C_t . [q_hi | q_lo]^T        (C_t the codes of tile t, as halves)
-//   output   O^T = C_t^T . [p_hi | p_lo]
+//   scores   S^T = C_t . Q^T     M = 128 tokens, N = 32, K = 128 dims    (C_t K-major)
+//   output   O^T = C_t^T . W     M = 128 dims,   N = 32, K = 128 tokens  (C_t MN-major)
 //
-// A row's scale multiplies its score column (s_t = scale_t <q_r, c_t>) and its softmax weight
-// (p_t scale_t feeds the output MMA), so the codes never need rescaling.
+// The other operands keep more precision than one E4M3 value by being sums of E4M3 terms in
+// separate columns: each term is the rounding residual of the previous one times 16, so each
+// adds four significant bits. Q holds the routed query (times scale * log2 e) of the 8 heads as
+// 4 terms, W the softmax weights times the row scales as 3 terms; head h = 4 hh + k, term j sits
+// in score column 16 hh + 4 j + k and output column 16 hh + 4 j + k (output columns 12..15 of
+// each half zero). Before the split a power of two brings the operand's largest value below
+// 256 (E4M3 reaches 448); it is divided out again after the terms are summed.
 //
-// One CTA per (split, value head g, sequence b); 288 threads, two CTAs per SM:
-//   warps 0-3  softmax (thread = token), O accumulation (thread = output dim), epilogue
-//              (output row, or split state for the combine kernel)
-//   warp 4     producer: W^R[g] and the group's query rows (routing operands), then TMA loads
-//              of code pages and scale rows into a 2-stage ring
-//   warp 5     routing and score MMA issuer, TMEM owner
-//   warp 6     output MMA issuer
-//   warps 7-8  widen each landed code tile into the half tile that the output MMAs two tiles
-//              back have released, so the softmax warps never wait on the widening
+// The softmax keeps a lazy reference maximum per head: a tile's weights are 2^(s - m) with the
+// current reference m, and m moves (rescaling the running sums) only when a score passes it by
+// more than 2, so the weights stay at most 4. Most tiles thus need one vote among the compute
+// warps instead of an exchange of maxima, and one power of two, 2^(6 - e) with the tile's row
+// scales below 2^e, serves the weights of all heads.
+// A row's scale multiplies its score column (s_t = scale_t <q_r, c_t>) and its weight
+// (p_t scale_t), so the codes are used as stored.
+//
+// One CTA per (split, value head g, sequence b); 352 threads, two CTAs per SM:
+//   warps 0-7  compute. Warp w reads TMEM lane quarter w % 4 and takes heads 4 (w / 4) .. + 3:
+//              routing result and query split (thread = dim); per tile the online softmax in
+//              base 2 and the weight split (thread = token), O accumulation (thread = output
+//              dim); epilogue (output row or split state). Two warps per lane quarter halve
+//              the per-thread work of a tile, which bounds the tile rate.
+//   warp 8     producer: W^R[g] (ring stages 0-1) and the group's query rows, then per tile the
+//              TMA loads of code pages and bulk copies of their scale rows
+//   warp 9     routing and score MMA issuer, TMEM owner
+//   warp 10    output MMA issuer; completion of a tile's output MMAs frees its ring stage
 // Every wait is bounded (about one second); a wait that runs out raises KL_FLAG_TIMEOUT and
 // every role leaves its loop, drains its copies and MMAs, and TMEM is freed.
 #include <cuda_fp16.h>
@@ -38,44 +51,64 @@ namespace {
 
 constexpr int kD = 128;
 constexpr int kTile = 128;
-constexpr int kNG = 8;                      // query heads per value group (padded)
-constexpr int kN = 2 * kNG;                 // MMA N: hi and lo halves
-constexpr int kComputeWarps = 4;
-constexpr int kProducerWarp = 4;
-constexpr int kMmaWarp = 5;
-constexpr int kPvWarp = 6;
-constexpr int kConvWarp0 = 7;               // warps 7-8 widen code tiles
-constexpr int kConvWarps = 2;
-constexpr int kThreads = 9 * 32;
-constexpr int kStages = 2;                  // code tiles in flight
+constexpr int kHH = 4;                      // heads per compute warp
+constexpr int kJq = 4;                      // E4M3 terms of the routed query
+constexpr int kJp = 3;                      // E4M3 terms of the weights
+constexpr int kNS = 32;                     // score MMA N: 2 x 16 columns
+constexpr int kNP = 32;                     // output MMA N: 2 x 16 columns (12 used each)
+constexpr int kNR = 16;                     // routing MMA N (query rows, padded)
+constexpr int kComputeWarps = 8;
+constexpr int kComputeThreads = kComputeWarps * 32;
+constexpr int kProducerWarp = 8;
+constexpr int kMmaWarp = 9;
+constexpr int kPvWarp = 10;
+constexpr int kThreads = 11 * 32;
+constexpr int kStages = 5;
 constexpr uint32_t kCodeBytes = kTile * kD;          // 16 KiB of codes per tile
-constexpr uint32_t kTileBytes = kTile * kD * 2;      // 32 KiB half tile (MMA operand)
-constexpr uint32_t kHalfBytes = kTileBytes / 2;      // one 64-dim half: 128 rows x 128 B
-constexpr uint32_t kTmemCols = 64;                   // S: 2 x 16 columns, O: 2 x 16 columns
-constexpr int kScaleFloats = 256;                    // (128 / P) slots of max(32, P) floats
+constexpr uint32_t kHalfBytes = 16384;               // one 64-column half of W^R (bf16)
+constexpr uint32_t kPBytes = kTile * kNP;            // weight operand: 4 KiB
+constexpr uint32_t kTmemCols = 256;
+constexpr uint32_t kColS = 0;                        // S[b]: columns 32 b .. 32 b + 31
+constexpr uint32_t kColO = 64;                       // O[b]: columns 64 + 32 b .. + 31
+constexpr uint32_t kColR = 128;                      // routing result: 128 .. 143
+constexpr float kLazy = 2.f;                         // reference slack (base 2): weights <= 4
 constexpr uint64_t kTimeoutNs = 1000000000ull;
 constexpr uint32_t kBarCompute = 1;
 constexpr uint32_t kBarComputeAnd = 2;
 
 struct __align__(1024) Smem8 {
-    // Half-precision tiles, the MMA operands: [64-dim half][128 rows][128 B], 128B-swizzled.
-    // cvt[1] first holds W^R[g] (bf16) for the routing MMA.
-    uint8_t cvt[2][kTileBytes];
-    // Code tiles as TMA writes them: [128 rows][128 B], 128B-swizzled. Row scales: one slot of
-    // max(32, P) floats per page, so that every TMA destination is 128-byte aligned.
+    // Ring of code tiles as TMA lands them: [128 token rows][128 B], 128B-swizzled. Stages 0
+    // and 1 first hold the two 64-column halves of W^R[g] (bf16) for the routing MMA.
     uint8_t codes[kStages][kCodeBytes];
-    float scl[kStages][kScaleFloats];
-    float cscl[2][kTile];              // row scales of the tile in cvt[b], token order
-    uint8_t qr[2 * kN * 128];          // routed query operand [half][16 rows][128 B], K-major
-    uint8_t p[2][kTile * kN * 2];      // P^T operands, no swizzle, MN-major
-    float red[2][kComputeWarps][kNG];
+    // Query terms, B operand of the score MMAs: [32 rows n][128 dims], K-major, 128B-swizzled.
+    uint8_t qt[kNS * 128];
+    // Weight terms, B operand of the output MMAs: [16 groups of 8 tokens][2 blocks of 16
+    // columns][8 tokens][16 B], MN-major, no swizzle. During the routing prologue the first one
+    // holds the query rows: [64-dim half][16 rows][128 B], K-major, 128B-swizzled.
+    uint8_t p[2][kPBytes];
+    float scl[kStages][kTile];         // row scales of each stage's tile, token order
+    float red[2][kComputeWarps][8];    // per warp: 4 head maxima (or row sums), the scale max
     uint64_t full[kStages], empty[kStages];
-    uint64_t c_full[2];
     uint64_t s_full[2], s_empty[2], p_full[2], o_full[2], o_empty[2];
-    uint64_t r_load, r_full, qr_full, drain, drain2;
+    uint64_t r_full, qt_full, drain, drain2;
     uint32_t tmem_base;
     int abort;
 };
+
+// mbarrier.try_wait with a suspend-time hint: a thread whose phase is not complete sleeps in
+// the instruction (it wakes when the phase completes or the hint runs out) instead of spinning
+// and taking issue slots from the warps that share its scheduler.
+__device__ __forceinline__ bool mbar_wait_sleep(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}\n"
+        : "=r"(ok)
+        : "r"(ptx::smem_addr(bar)), "r"(parity), "r"(20000u)
+        : "memory");
+    return ok != 0;
+}
 
 struct Waiter {
     volatile int *abort;
@@ -85,7 +118,7 @@ struct Waiter {
         if (!ok) {
             const uint64_t t0 = ptx::globaltimer();
             while (true) {
-                if (ptx::mbar_try_wait(bar, parity)) { ok = true; break; }
+                if (mbar_wait_sleep(bar, parity)) { ok = true; break; }
                 if (*abort) break;
                 if (ptx::globaltimer() - t0 > kTimeoutNs) {
                     *abort = 1;
@@ -98,71 +131,99 @@ struct Waiter {
     }
 };
 
-// Per-head maximum over the 32 lanes of a warp by transposed halving (see the bf16 decode).
-__device__ __forceinline__ float warp_max8(const float (&x)[8], int lane) {
-    const bool b4 = lane & 16, b3 = lane & 8, b2 = lane & 4;
-    float a4[4], a2[2];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        const float send = b4 ? x[j] : x[j + 4];
-        const float keep = b4 ? x[j + 4] : x[j];
-        a4[j] = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, 16));
-    }
-#pragma unroll
-    for (int j = 0; j < 2; ++j) {
-        const float send = b3 ? a4[j] : a4[j + 2];
-        const float keep = b3 ? a4[j + 2] : a4[j];
-        a2[j] = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, 8));
-    }
-    float a1;
-    {
-        const float send = b2 ? a2[0] : a2[1];
-        const float keep = b2 ? a2[1] : a2[0];
-        a1 = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, 4));
-    }
-    a1 = fmaxf(a1, __shfl_xor_sync(0xffffffffu, a1, 2));
-    a1 = fmaxf(a1, __shfl_xor_sync(0xffffffffu, a1, 1));
-    return a1;
+// Warp maximum of a float through the integer reduction unit: the key of a float orders as the
+// float does (non-negative floats keep their bits, negative ones flip all but the sign).
+__device__ __forceinline__ int order_key(float f) {
+    const int i = __float_as_int(f);
+    return i >= 0 ? i : i ^ 0x7FFFFFFF;
+}
+__device__ __forceinline__ float warp_max(float f) {
+    const int k = __reduce_max_sync(0xffffffffu, order_key(f));
+    return __int_as_float(k >= 0 ? k : k ^ 0x7FFFFFFF);
 }
 
-// Two E4M3 codes (low byte first) to two halves (low half first): the PTX conversion
-// instruction, exact since every E4M3 value is a half-precision value.
-__device__ __forceinline__ uint32_t e4m3x2_to_f16x2(uint32_t two_codes) {
+// Two E4M3 codes (low byte first) to two halves (low half first), exact: every E4M3 value is a
+// half-precision value.
+__device__ __forceinline__ float2 e4m3x2_to_float2(uint32_t two_codes) {
     uint32_t r;
     const uint16_t v = (uint16_t)two_codes;
     asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(r) : "h"(v));
-    return r;
+    return __half22float2(*reinterpret_cast<const __half2 *>(&r));
 }
 
-// x = hi + lo in half precision for two values.
-__device__ __forceinline__ void split_h2(float x0, float x1, uint32_t &hi, uint32_t &lo) {
-    const __half2 h = __floats2half2_rn(x0, x1);
-    const float2 hf = __half22float2(h);
-    const __half2 l = __floats2half2_rn(x0 - hf.x, x1 - hf.y);
-    hi = *reinterpret_cast<const uint32_t *>(&h);
-    lo = *reinterpret_cast<const uint32_t *>(&l);
+// A power of two 2^(8 - e) with amax < 2^e (so amax * 2^(8 - e) < 256) and its inverse; 1 and 1
+// for amax = 0. e is clamped so that both stay normal floats.
+__device__ __forceinline__ void pow2_scale(float amax, float &sc, float &inv) {
+    int e = (int)((__float_as_uint(amax) >> 23) & 0xFFu) - 126;
+    e = max(-100, min(100, e));
+    if (!(amax > 0.f)) e = 8;
+    sc = __uint_as_float((uint32_t)(127 + 8 - e) << 23);
+    inv = __uint_as_float((uint32_t)(127 - 8 + e) << 23);
 }
 
-// Byte offset of element (row n, column k) in the K-major, 128B-swizzled query operand of 16
-// rows and 128 columns laid out as [half][16 rows][128 B].
-__device__ __forceinline__ uint32_t qr_offset(int n, int k) {
-    const int half = k >> 6, kk = k & 63;
-    return half * (kN * 128) + (n >> 3) * 1024 + (n & 7) * 128 + (((kk >> 3) ^ (n & 7)) << 4) +
-           ((kk & 7) << 1);
+// 2^(8 - e) and 2^(e - 8), e clamped so that both stay normal floats.
+__device__ __forceinline__ void pow2_from_exp(int e, float &sc, float &inv) {
+    e = max(-100, min(100, e));
+    sc = __uint_as_float((uint32_t)(127 + 8 - e) << 23);
+    inv = __uint_as_float((uint32_t)(127 - 8 + e) << 23);
 }
 
-// Instruction descriptor of kind::f16 with half-precision A and B, fp32 accumulator.
-__host__ __device__ constexpr uint32_t idesc_f16(uint32_t M, uint32_t N, bool a_mn, bool b_mn) {
+// x (0 <= x < 448) rounded to an E4M3 value on the FMA pipe: to 4 significant bits by a
+// Veltkamp split (c = x (2^20 + 1), hi = c - (c - x)), and below 2^-6, where the E4M3 values
+// are the multiples of 2^-9, by adding and subtracting 1.5 * 2^14 (whose spacing is 2^-9). The
+// result is an E4M3 value, so its code conversion is exact and x - hi is the exact residual.
+// (The small values matter: with a few large row scales in a tile, most weights sit far below
+// the tile's largest and would lose their residual without the second rounding.)
+__device__ __forceinline__ float e4m3_round(float x) {
+    // explicit roundings: the compiler must not fuse these into FMAs
+    const float c = __fmul_rn(x, 1048577.f);
+    const float hv = __fsub_rn(c, __fsub_rn(c, x));
+    const float hs = __fsub_rn(__fadd_rn(x, 24576.f), 24576.f);
+    return x < 0.015625f ? hs : hv;
+}
+
+// Byte offset of element (row n, column k) of the query-term operand: [48 rows][128 B],
+// K-major, 128B-swizzled (8-row atoms of 1 KiB, 16-byte chunk index XOR row % 8).
+__device__ __forceinline__ uint32_t qt_offset(int n, int k) {
+    return (n >> 3) * 1024 + (n & 7) * 128 + ((((k >> 4) ^ (n & 7))) << 4) + (k & 15);
+}
+
+// D[tmem] (+)= A[smem desc] x B[smem desc], kind::f8f6f4 with E4M3 A and B, fp32 accumulation.
+__device__ __forceinline__ void mma_f8(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                       uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// Instruction descriptor of kind::f8f6f4: fp32 accumulator, E4M3 A and B (format 0), operand
+// majorness (0 = K-major, 1 = MN-major), N and M.
+__host__ __device__ constexpr uint32_t idesc_f8(uint32_t M, uint32_t N, bool a_mn, bool b_mn) {
     return (1u << 4) | ((a_mn ? 1u : 0u) << 15) | ((b_mn ? 1u : 0u) << 16) | ((N >> 3) << 17) |
            ((M >> 4) << 24);
 }
 
+// Barrier `id` over `count` threads that also returns how many of them passed v = true.
+__device__ __forceinline__ uint32_t bar_popc(uint32_t id, uint32_t count, bool v) {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "bar.red.popc.u32 %0, %2, %3, p;\n\t}\n"
+        : "=r"(r)
+        : "r"((uint32_t)v), "r"(id), "r"(count)
+        : "memory");
+    return r;
+}
+
 __global__ void __launch_bounds__(kThreads, 2)
     decode_fp8_kernel(const __grid_constant__ CUtensorMap cmap,
-                      const __grid_constant__ CUtensorMap smap,
                       const __grid_constant__ CUtensorMap wmap,
-                      const __grid_constant__ CUtensorMap qmap, const DecodeArgs a) {
-    constexpr int NS = kStages;
+                      const __grid_constant__ CUtensorMap qmap, const DecodeArgs a,
+                      const float *__restrict__ v_scales) {
     extern __shared__ uint8_t smem_raw[];
     Smem8 &sm = *reinterpret_cast<Smem8 *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                            ~uintptr_t(1023));
@@ -171,27 +232,27 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int G = geo.G;
     const bool route = a.w_r != nullptr;      // W^R given; else q is the composed query
+    // Ring uses: with routing, uses 0 and 1 are the W^R halves and tile i is use i + 2.
+    const int base = route ? 2 : 0;
 
     const int L_raw = a.seq_lens[b];
     const int t_begin = split * geo.chunk;
     const int32_t *bt = a.block_table + (size_t)b * geo.max_pages;
 
     if (tid == 0) {
-        for (int s = 0; s < NS; ++s) {
+        for (int s = 0; s < kStages; ++s) {
             ptx::mbar_init(&sm.full[s], 1);
-            ptx::mbar_init(&sm.empty[s], kConvWarps);
+            ptx::mbar_init(&sm.empty[s], 1);
         }
         for (int i = 0; i < 2; ++i) {
-            ptx::mbar_init(&sm.c_full[i], kConvWarps);
             ptx::mbar_init(&sm.s_full[i], 1);
             ptx::mbar_init(&sm.s_empty[i], kComputeWarps);
             ptx::mbar_init(&sm.p_full[i], kComputeWarps);
             ptx::mbar_init(&sm.o_full[i], 1);
             ptx::mbar_init(&sm.o_empty[i], kComputeWarps);
         }
-        ptx::mbar_init(&sm.r_load, 1);
         ptx::mbar_init(&sm.r_full, 1);
-        ptx::mbar_init(&sm.qr_full, kComputeWarps);
+        ptx::mbar_init(&sm.qt_full, kComputeWarps);
         ptx::mbar_init(&sm.drain, 1);
         ptx::mbar_init(&sm.drain2, 1);
         sm.abort = 0;
@@ -203,7 +264,6 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
     if (warp == kProducerWarp && lane == 0) {
         ptx::prefetch_tensormap(&cmap);
-        ptx::prefetch_tensormap(&smap);
         if (route) {
             ptx::prefetch_tensormap(&wmap);
             ptx::prefetch_tensormap(&qmap);
@@ -253,25 +313,28 @@ __global__ void __launch_bounds__(kThreads, 2)
         const int first_page = t_begin / P;
         const int end_page = (t_end + P - 1) / P;
         const uint32_t page_bytes = (uint32_t)P * 128u + (uint32_t)P * 4u;
-        const int scale_slot = max(32, P);                   // floats per page slot
         bool bad = false;
-        int issued = 0;
-        if (route && lane == 0) {
-            // routing operands: W^R[g] (MN-major A of the routing MMA) into cvt[1], the group's
-            // query rows (K-major B) into the query operand buffer
-            ptx::mbar_arrive_expect_tx(&sm.r_load, kTileBytes + 2u * (uint32_t)G * 128u);
-            ptx::tma_load_2d(sm.cvt[1], &wmap, &sm.r_load, 0, g * kD);
-            ptx::tma_load_2d(sm.cvt[1] + kHalfBytes, &wmap, &sm.r_load, 64, g * kD);
-            ptx::tma_load_2d(sm.qr, &qmap, &sm.r_load, 0, b * geo.Hq + g * G);
-            ptx::tma_load_2d(sm.qr + kN * 128, &qmap, &sm.r_load, 64, b * geo.Hq + g * G);
+        int issued = 0;                                      // ring uses issued
+        if (route) {
+            if (lane == 0) {
+                // W^R[g] halves into stages 0 and 1 (MN-major A of the routing MMA); the
+                // group's query rows into the first weight buffer (K-major B)
+                ptx::mbar_arrive_expect_tx(&sm.full[0], kHalfBytes + 2u * (uint32_t)G * 128u);
+                ptx::tma_load_2d(sm.codes[0], &wmap, &sm.full[0], 0, g * kD);
+                ptx::tma_load_2d(sm.p[0], &qmap, &sm.full[0], 0, b * geo.Hq + g * G);
+                ptx::tma_load_2d(sm.p[0] + kNR * 128, &qmap, &sm.full[0], 64, b * geo.Hq + g * G);
+                ptx::mbar_arrive_expect_tx(&sm.full[1], kHalfBytes);
+                ptx::tma_load_2d(sm.codes[1], &wmap, &sm.full[1], 64, g * kD);
+            }
+            issued = 2;
+            __syncwarp();
         }
-        __syncwarp();
         for (int i = 0; i < n_tiles; ++i) {
-            const int s = i % NS;
+            const int u = i + base, s = u % kStages, round = u / kStages;
             const int p0 = first_page + i * ppt;
             const bool exists = lane < ppt && p0 + lane < end_page;
             const int page = exists ? bt[p0 + lane] : -1;
-            if (i >= NS && !wait(&sm.empty[s], ((i / NS) & 1) ^ 1)) break;
+            if (round >= 1 && !wait(&sm.empty[s], (round - 1) & 1)) break;
             const bool in_range = exists && page >= 0 && page < geo.num_pages;
             if (exists && !in_range) bad = true;
             const unsigned mask = __ballot_sync(0xffffffffu, in_range);
@@ -280,66 +343,66 @@ __global__ void __launch_bounds__(kThreads, 2)
             if (in_range) {
                 const int row = (page * geo.Hkv + g) * P;
                 ptx::tma_load_2d(sm.codes[s] + lane * P * 128, &cmap, &sm.full[s], 0, row);
-                ptx::tma_load_2d(&sm.scl[s][lane * scale_slot], &smap, &sm.full[s], 0,
-                                 page * geo.Hkv + g);
+                ptx::bulk_load(&sm.scl[s][lane * P], v_scales + (size_t)row, (uint32_t)P * 4u,
+                               &sm.full[s]);
             }
-            issued = i + 1;
+            issued = u + 1;
         }
         if (__any_sync(0xffffffffu, bad) && lane == 0) raise_flag(a.err, KL_FLAG_BAD_PAGE);
         if (sm.abort) {
-            for (int i = max(0, issued - NS); i < issued; ++i) {
+            // the most recent use of every stage may still have copies in flight
+            for (int v = max(0, issued - kStages); v < issued; ++v) {
                 const uint64_t t0 = ptx::globaltimer();
-                while (!ptx::mbar_try_wait(&sm.full[i % NS], (i / NS) & 1) &&
+                while (!ptx::mbar_try_wait(&sm.full[v % kStages], (v / kStages) & 1) &&
                        ptx::globaltimer() - t0 < kTimeoutNs) {
-                }
-            }
-            if (route) {
-                const uint64_t t0 = ptx::globaltimer();
-                while (!ptx::mbar_try_wait(&sm.r_load, 0) && ptx::globaltimer() - t0 < kTimeoutNs) {
                 }
             }
         }
     } else if (warp == kMmaWarp) {
-        // ------------------------------------------------------- score MMA issuer -------
-        constexpr uint32_t idesc_s = idesc_f16(128, kN, false, false);
-        const uint64_t q_desc = ptx::smem_desc(ptx::smem_addr(sm.qr), 16, 1024, ptx::kSwizzle128B);
-        const uint64_t c_desc = ptx::smem_desc(ptx::smem_addr(sm.cvt[0]), 16, 1024, ptx::kSwizzle128B);
+        // ------------------------------------------------- routing and score MMA issuer ----
         bool ok = true;
         if (route) {
             // q_r^T[128 j x 16] = W^R^T (MN-major, bf16) . q^T (K-major rows of the query buffer)
-            constexpr uint32_t idesc_r = ptx::idesc_bf16(128, kN, true, false);
-            ok = wait(&sm.r_load, 0);
+            constexpr uint32_t idesc_r = ptx::idesc_bf16(128, kNR, true, false);
+            ok = wait(&sm.full[0], 0);
+            ok = ok && wait(&sm.full[1], 0);
             if (ok) {
                 ptx::tc_fence_after();
                 if (lane == 0) {
-                    const uint64_t w_desc = ptx::smem_desc(ptx::smem_addr(sm.cvt[1]), kHalfBytes,
+                    const uint64_t w_desc = ptx::smem_desc(ptx::smem_addr(sm.codes[0]), kHalfBytes,
                                                            1024, ptx::kSwizzle128B);
+                    const uint64_t q_desc =
+                        ptx::smem_desc(ptx::smem_addr(sm.p[0]), 16, 1024, ptx::kSwizzle128B);
 #pragma unroll
                     for (int kk = 0; kk < kD / 16; ++kk) {
-                        const uint32_t qoff = (kk >> 2) * (kN * 128) + (kk & 3) * 32;
-                        ptx::mma_bf16(tmem + 2 * kN, w_desc + ((kk * 2048) >> 4), q_desc + (qoff >> 4),
-                                      idesc_r, kk > 0);
+                        const uint32_t qoff = (kk >> 2) * (kNR * 128) + (kk & 3) * 32;
+                        ptx::mma_bf16(tmem + kColR, w_desc + ((kk * 2048) >> 4),
+                                      q_desc + (qoff >> 4), idesc_r, kk > 0);
                     }
                     ptx::mma_commit(&sm.r_full);
+                    ptx::mma_commit(&sm.empty[0]);      // stages 0 and 1 are free again
+                    ptx::mma_commit(&sm.empty[1]);
                 }
                 __syncwarp();
             }
         }
-        ok = ok && wait(&sm.qr_full, 0);
+        ok = ok && wait(&sm.qt_full, 0);
         if (ok) ptx::tc_fence_after();
+        constexpr uint32_t idesc_s = idesc_f8(128, kNS, false, false);
+        const uint64_t c_desc =
+            ptx::smem_desc(ptx::smem_addr(sm.codes[0]), 16, 1024, ptx::kSwizzle128B);
+        const uint64_t q_desc = ptx::smem_desc(ptx::smem_addr(sm.qt), 16, 1024, ptx::kSwizzle128B);
         for (int i = 0; ok && i < n_tiles; ++i) {
-            const int cb = i & 1, sb = i & 1;
-            if (!wait(&sm.c_full[cb], (i >> 1) & 1)) break;
+            const int u = i + base, s = u % kStages, sb = i & 1;
+            if (!wait(&sm.full[s], (u / kStages) & 1)) break;
             if (i >= 2 && !wait(&sm.s_empty[sb], ((i >> 1) - 1) & 1)) break;
             ptx::tc_fence_after();
             if (lane == 0) {
-                const uint64_t a0 = c_desc + ((cb * kTileBytes) >> 4);
+                const uint64_t a0 = c_desc + ((s * kCodeBytes) >> 4);
 #pragma unroll
-                for (int kk = 0; kk < kD / 16; ++kk) {
-                    const uint32_t koff = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
-                    const uint32_t qoff = (kk >> 2) * (kN * 128) + (kk & 3) * 32;
-                    ptx::mma_bf16(tmem + sb * kN, a0 + (koff >> 4), q_desc + (qoff >> 4), idesc_s, kk > 0);
-                }
+                for (int kk = 0; kk < kD / 32; ++kk)
+                    mma_f8(tmem + kColS + sb * 32, a0 + ((kk * 32) >> 4), q_desc + ((kk * 32) >> 4),
+                           idesc_s, kk > 0);
                 ptx::mma_commit(&sm.s_full[sb]);
             }
             __syncwarp();
@@ -351,27 +414,27 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
     } else if (warp == kPvWarp) {
         // ------------------------------------------------------ output MMA issuer -------
-        // A = C^T: MN-major SW128 (64-dim halves kHalfBytes apart, 8-token groups 1 KiB apart);
-        // B = P^T: MN-major, no swizzle (hi/lo blocks 128 B apart, 8-token groups 256 B apart)
-        constexpr uint32_t idesc_o = idesc_f16(128, kN, true, true);
+        // A = C^T: the code tile read MN-major (8-token row groups 1 KiB apart); B = W:
+        // MN-major, no swizzle (16-column blocks 128 B apart, 8-token groups 256 B apart)
+        constexpr uint32_t idesc_o = idesc_f8(128, kNP, true, true);
         const uint64_t c_desc =
-            ptx::smem_desc(ptx::smem_addr(sm.cvt[0]), kHalfBytes, 1024, ptx::kSwizzle128B);
+            ptx::smem_desc(ptx::smem_addr(sm.codes[0]), 8192, 1024, ptx::kSwizzle128B);
         const uint64_t p_desc = ptx::smem_desc(ptx::smem_addr(sm.p[0]), 256, 128, ptx::kSwizzleNone);
-        constexpr uint32_t kPBytes = sizeof(sm.p[0]);
         for (int j = 0; j < n_tiles; ++j) {
-            const int cb = j & 1, pb = j & 1;
+            const int u = j + base, s = u % kStages, pb = j & 1;
             if (!wait(&sm.p_full[pb], (j >> 1) & 1)) break;
             if (j >= 2 && !wait(&sm.o_empty[pb], ((j >> 1) - 1) & 1)) break;
             ptx::tc_fence_after();
             const int nvalid = min(kTile, t_end - (t_begin + j * kTile));
-            const int ksteps = (nvalid + 15) >> 4;
+            const int ksteps = (nvalid + 31) >> 5;
             if (lane == 0) {
-                const uint64_t a0 = c_desc + ((cb * kTileBytes) >> 4);
+                const uint64_t a0 = c_desc + ((s * kCodeBytes) >> 4);
                 const uint64_t b0 = p_desc + ((pb * kPBytes) >> 4);
                 for (int kk = 0; kk < ksteps; ++kk)
-                    ptx::mma_bf16(tmem + 2 * kN + pb * kN, a0 + ((kk * 2048) >> 4), b0 + ((kk * 512) >> 4),
-                                  idesc_o, kk > 0);
+                    mma_f8(tmem + kColO + pb * 32, a0 + ((kk * 4096) >> 4), b0 + ((kk * 1024) >> 4),
+                           idesc_o, kk > 0);
                 ptx::mma_commit(&sm.o_full[pb]);
+                ptx::mma_commit(&sm.empty[s]);     // the tile's last reader is done
             }
             __syncwarp();
         }
@@ -380,209 +443,254 @@ __global__ void __launch_bounds__(kThreads, 2)
         const uint64_t t0 = ptx::globaltimer();
         while (!ptx::mbar_try_wait(&sm.drain2, 0) && ptx::globaltimer() - t0 < kTimeoutNs) {
         }
-    } else if (warp >= kConvWarp0) {
-        // ------------------------------------------------------------------ widening ----
-        // Thread u takes rows u and u + 64 of each tile. Tile j goes into cvt[j & 1] once the
-        // output MMAs of tile j - 2 (the last reader of that buffer) are done.
-        const int u = tid - kConvWarp0 * 32;
-        for (int j = 0; j < n_tiles; ++j) {
-            const int s = j % NS, cb = j & 1;
-            if (!wait(&sm.full[s], (j / NS) & 1)) break;
-            if (j >= 2 && !wait(&sm.o_full[cb], ((j - 2) >> 1) & 1)) break;
-            const int nvalid = min(kTile, t_end - (t_begin + j * kTile));
+    } else {
+        // ------------------------------------------------------------------ compute -----
+        // Warp w: TMEM lane quarter q4 = w % 4 (dims / tokens 32 q4 .. 32 q4 + 31) and heads
+        // h = 4 hh + k (k = 0..3) with hh = w / 4.
+        const int q4 = warp & 3, hh = warp >> 2;
+        const int t = q4 * 32 + lane;                       // dim / token / output dim
+        const uint32_t lane_base = (uint32_t)(q4 * 32) << 16;
+        const float sl2 = geo.scale * kLog2e;
+        bool ok = true;
+
+        // Routed query: from the routing MMA (TMEM), or the composed query itself.
+        float acc[kHH];
 #pragma unroll
-            for (int rr = 0; rr < 2; ++rr) {
-                const int t = u + 64 * rr;
-                const bool valid = t < nvalid;
-                sm.cscl[cb][t] = valid ? sm.scl[s][(t / geo.P) * max(32, geo.P) + t % geo.P] : 0.f;
-                const uint32_t src = ptx::smem_addr(sm.codes[s]) + t * 128;
-                const uint32_t dst = ptx::smem_addr(sm.cvt[cb]) + t * 128;
+        for (int k = 0; k < kHH; ++k) acc[k] = 0.f;
+        if (route) {
+            ok = ptx::bar_and(kBarComputeAnd, kComputeThreads, wait(&sm.r_full, 0));
+            if (ok) {
+                ptx::tc_fence_after();
+                float rv[16];
+                ptx::tmem_ld16(tmem + kColR + lane_base, rv);
 #pragma unroll
-                for (int c = 0; c < 8; ++c) {
-                    uint4 v = make_uint4(0, 0, 0, 0);
-                    if (valid)
-                        asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
-                                     : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-                                     : "r"(src + (((c ^ (t & 7))) << 4)));
-                    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-                    uint32_t hv[8];
+                for (int k = 0; k < kHH; ++k)
+                    acc[k] = kHH * hh + k < G ? (hh ? rv[kHH + k] : rv[k]) : 0.f;
+                ptx::tc_fence_before();
+            }
+        } else {
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        hv[2 * e] = e4m3x2_to_f16x2(w[e]);
-                        hv[2 * e + 1] = e4m3x2_to_f16x2(w[e] >> 16);
-                    }
-                    // codes 16c .. 16c + 15: dims of half c / 4, chunks 2 (c % 4) and + 1 there
-                    const int half = c >> 2, ch = 2 * (c & 3);
-                    const uint32_t d0 = dst + half * kHalfBytes + ((ch ^ (t & 7)) << 4);
-                    const uint32_t d1 = dst + half * kHalfBytes + (((ch + 1) ^ (t & 7)) << 4);
-                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(d0), "r"(hv[0]),
-                                 "r"(hv[1]), "r"(hv[2]), "r"(hv[3])
-                                 : "memory");
-                    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(d1), "r"(hv[4]),
-                                 "r"(hv[5]), "r"(hv[6]), "r"(hv[7])
-                                 : "memory");
+            for (int k = 0; k < kHH; ++k) {
+                const int h = kHH * hh + k;
+                acc[k] = h < G ? __uint_as_float((uint32_t)a.q[((size_t)b * geo.Hq + g * G + h) * kD + t] << 16)
+                               : 0.f;
+            }
+        }
+        // Query terms: per head, 2^(8 - e) over its largest |value|, then 6 E4M3 terms.
+        float invq[kHH];
+        if (ok) {
+            float v[kHH], av[kHH];
+#pragma unroll
+            for (int k = 0; k < kHH; ++k) {
+                v[k] = acc[k] * sl2;
+                av[k] = fabsf(v[k]);
+            }
+            float wm[kHH];
+#pragma unroll
+            for (int k = 0; k < kHH; ++k) wm[k] = warp_max(av[k]);
+            if (lane == 0) {
+#pragma unroll
+                for (int k = 0; k < kHH; ++k) sm.red[1][warp][k] = wm[k];
+            }
+            ptx::bar_sync(kBarCompute, kComputeThreads);
+#pragma unroll
+            for (int k = 0; k < kHH; ++k) {
+                float amax = sm.red[1][kHH * hh][k];
+#pragma unroll
+                for (int w = 1; w < 4; ++w) amax = fmaxf(amax, sm.red[1][kHH * hh + w][k]);
+                float sc;
+                pow2_scale(amax, sc, invq[k]);
+                float x = v[k] * sc;
+#pragma unroll
+                for (int j = 0; j < kJq; ++j) {
+                    const __nv_fp8_storage_t c = __nv_cvt_float_to_fp8(x, __NV_SATFINITE, __NV_E4M3);
+                    sm.qt[qt_offset(16 * hh + 4 * j + k, t)] = c;
+                    x = (x - e4m3x2_to_float2((uint32_t)c).x) * 16.f;
                 }
             }
             ptx::fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) {
-                ptx::mbar_arrive(&sm.empty[s]);   // the code stage is free again
-                ptx::mbar_arrive(&sm.c_full[cb]);
-            }
-        }
-    } else {
-        // ------------------------------------------------------------------ compute -----
-        const int t = tid;                                  // 0..127: token / output dim
-        const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-        const float sl2 = geo.scale * kLog2e;
-        bool ok = true;
-
-
-        // Routed query: from the routing MMA (TMEM), or the composed query itself.
-        float acc[kNG];
-#pragma unroll
-        for (int h = 0; h < kNG; ++h) acc[h] = 0.f;
-        if (ok && route) {
-            ok = ptx::bar_and(kBarComputeAnd, kTile, wait(&sm.r_full, 0));
-            if (ok) {
-                ptx::tc_fence_after();
-                float rv[16];
-                ptx::tmem_ld16(tmem + 2 * kN + lane_base, rv);
-#pragma unroll
-                for (int h = 0; h < kNG; ++h) acc[h] = h < G ? rv[h] : 0.f;
-                ptx::tc_fence_before();
-            }
-        } else if (ok) {
-#pragma unroll
-            for (int h = 0; h < kNG; ++h)
-                acc[h] = h < G ? __uint_as_float((uint32_t)a.q[((size_t)b * geo.Hq + g * G + h) * kD + t] << 16)
-                               : 0.f;
-        }
-        ok = ptx::bar_and(kBarComputeAnd, kTile, ok);
-        if (ok) {
-            // half-precision hi/lo operand rows: n = h (hi), n = 8 + h (lo); column k = t
-#pragma unroll
-            for (int h = 0; h < kNG; ++h) {
-                const float v = acc[h] * sl2;
-                const __half hi = __float2half_rn(v);
-                const __half lo = __float2half_rn(v - __half2float(hi));
-                *reinterpret_cast<__half *>(sm.qr + qr_offset(h, t)) = hi;
-                *reinterpret_cast<__half *>(sm.qr + qr_offset(kNG + h, t)) = lo;
-            }
-            ptx::fence_proxy_async_smem();
-            __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(&sm.qr_full);
+            if (lane == 0) ptx::mbar_arrive(&sm.qt_full);
         }
 
-        float m[kNG], lsum[kNG], o[kNG], alpha_prev[kNG];
+        float m[kHH], lsum[kHH], o[kHH], alpha_prev[kHH];
+        float inv_prev = 0.f;
 #pragma unroll
-        for (int h = 0; h < kNG; ++h) {
-            m[h] = -INFINITY;
-            lsum[h] = 0.f;
-            o[h] = 0.f;
-            alpha_prev[h] = 0.f;
+        for (int k = 0; k < kHH; ++k) {
+            m[k] = -INFINITY;
+            lsum[k] = 0.f;
+            o[k] = 0.f;
+            alpha_prev[k] = 0.f;
         }
-        // O accumulation of tile j: o = o * alpha_j + O_j (thread = output dim t)
-        auto correct = [&](int j, const float (&alpha)[kNG]) -> bool {
+        // O accumulation of tile j: o = o * alpha_j + inv_j * (O_0 + O_1 / 16 + O_2 / 256)
+        // (thread = output dim t; O_j the term columns of the output MMA). The wait is the
+        // warp's own; a failure travels to the next barrier of all compute warps.
+        auto correct = [&](int j, const float (&alpha)[kHH], float inv) -> bool {
             const int ob = j & 1;
-            if (!ptx::bar_and(kBarComputeAnd, kTile, wait(&sm.o_full[ob], (j >> 1) & 1))) return false;
+            if (!wait(&sm.o_full[ob], (j >> 1) & 1)) return false;
             ptx::tc_fence_after();
             float ov[16];
-            ptx::tmem_ld16(tmem + 2 * kN + ob * kN + lane_base, ov);
+            ptx::tmem_ld16(tmem + kColO + ob * 32 + 16 * hh + lane_base, ov);
             ptx::tc_fence_before();
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&sm.o_empty[ob]);
 #pragma unroll
-            for (int h = 0; h < kNG; ++h) o[h] = fmaf(o[h], alpha[h], ov[h] + ov[kNG + h]);
+            for (int k = 0; k < kHH; ++k) {
+                const float d = fmaf(ov[8 + k], 1.f / 256.f, fmaf(ov[4 + k], 1.f / 16.f, ov[k]));
+                o[k] = fmaf(o[k], alpha[k], d * inv);
+            }
             return true;
         };
 
+        // One barrier per tile for all compute warps: it publishes the tile's row-scale maximum,
+        // counts the warps whose scores passed a reference (or whose waits failed since the last
+        // barrier). Only then a second one exchanges the head maxima (or lets all of them leave
+        // the loop together after a failed wait).
+        bool carried = true;
         for (int i = 0; ok && i < n_tiles; ++i) {
-            const int sb = i & 1;
-            if (!ptx::bar_and(kBarComputeAnd, kTile, wait(&sm.s_full[sb], (i >> 1) & 1))) {
-                ok = false;
-                break;
-            }
-            ptx::tc_fence_after();
+            const int u = i + base, s = u % kStages, sb = i & 1;
+            // the stage's loads have landed (its scale row is read below) and S is ready
+            bool ready = wait(&sm.full[s], (u / kStages) & 1);
+            ready = ready && wait(&sm.s_full[sb], (i >> 1) & 1);
             float sv[16];
-            ptx::tmem_ld16(tmem + sb * kN + lane_base, sv);
-            ptx::tc_fence_before();
-            __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(&sm.s_empty[sb]);
+            if (ready) {
+                ptx::tc_fence_after();
+                ptx::tmem_ld16(tmem + kColS + sb * 32 + 16 * hh + lane_base, sv);
+                ptx::tc_fence_before();
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(&sm.s_empty[sb]);
+            } else {
+#pragma unroll
+                for (int c = 0; c < 16; ++c) sv[c] = 0.f;
+            }
 
             const int nvalid = min(kTile, t_end - (t_begin + i * kTile));
             const bool valid = t < nvalid;
-            // the row scale of token t: written by the widening warps before c_full[i & 1],
-            // which completed before this tile's score MMAs
-            if (!ptx::bar_and(kBarComputeAnd, kTile, wait(&sm.c_full[sb], (i >> 1) & 1))) {
-                ok = false;
-                break;
-            }
-            const float scale_cur = sm.cscl[sb][t];
-            float s[kNG], mx[kNG];
+            const float st = valid ? sm.scl[s][t] : 0.f;     // the row scale of token t
+            float s_k[kHH];
+            bool grow = false;
 #pragma unroll
-            for (int h = 0; h < kNG; ++h) {
-                // the row scale multiplies the score column of token t
-                s[h] = (valid && h < G) ? (sv[h] + sv[kNG + h]) * scale_cur : -INFINITY;
-                mx[h] = s[h];
+            for (int k = 0; k < kHH; ++k) {
+                // sum of the term columns, 16^-j D_j, from the last term
+                const float d = fmaf(fmaf(fmaf(sv[12 + k], 1.f / 16.f, sv[8 + k]), 1.f / 16.f, sv[4 + k]),
+                                     1.f / 16.f, sv[k]);
+                s_k[k] = (valid && kHH * hh + k < G) ? d * (invq[k] * st) : -INFINITY;
+                grow = grow || s_k[k] > m[k] + kLazy;
             }
-            {
-                const float wm = warp_max8(mx, lane);
-                if ((lane & 3) == 0)
-                    sm.red[sb][warp][((lane >> 4) & 1) * 4 + ((lane >> 3) & 1) * 2 + ((lane >> 2) & 1)] = wm;
+            if (hh == 0) {
+                // row scales are non-negative: their bits order as the values do
+                const float smx = __uint_as_float(__reduce_max_sync(0xffffffffu, __float_as_uint(st)));
+                if (lane == 0) sm.red[sb][warp][kHH] = smx;
             }
-            ptx::bar_sync(kBarCompute, kTile);
-            float alpha[kNG], p[kNG];
+            const bool fine = ready && carried;
+            float alpha[kHH];
 #pragma unroll
-            for (int h = 0; h < kNG; ++h) {
-                float tmax = sm.red[sb][0][h];
+            for (int k = 0; k < kHH; ++k) alpha[k] = 1.f;
+            if (bar_popc(kBarComputeAnd, kComputeThreads, grow || !fine) != 0) {
+                // move the references to the heads' running maxima
+                float wm[kHH];
 #pragma unroll
-                for (int w = 1; w < kComputeWarps; ++w) tmax = fmaxf(tmax, sm.red[sb][w][h]);
-                const float mn = fmaxf(m[h], tmax);
-                const bool live = h < G;
-                alpha[h] = live ? exp2f(m[h] - mn) : 0.f;
-                p[h] = live ? exp2f(s[h] - mn) : 0.f;
-                lsum[h] = fmaf(lsum[h], alpha[h], p[h]);
-                m[h] = live ? mn : m[h];
+                for (int k = 0; k < kHH; ++k) wm[k] = warp_max(s_k[k]);
+                if (lane == 0) {
+#pragma unroll
+                    for (int k = 0; k < kHH; ++k) sm.red[sb][warp][k] = wm[k];
+                }
+                if (!ptx::bar_and(kBarComputeAnd, kComputeThreads, fine)) {
+                    ok = false;
+                    break;
+                }
+                float4 r = *reinterpret_cast<const float4 *>(&sm.red[sb][kHH * hh][0]);
+                float tmax[kHH] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+                for (int w = 1; w < 4; ++w) {
+                    r = *reinterpret_cast<const float4 *>(&sm.red[sb][kHH * hh + w][0]);
+                    tmax[0] = fmaxf(tmax[0], r.x);
+                    tmax[1] = fmaxf(tmax[1], r.y);
+                    tmax[2] = fmaxf(tmax[2], r.z);
+                    tmax[3] = fmaxf(tmax[3], r.w);
+                }
+#pragma unroll
+                for (int k = 0; k < kHH; ++k) {
+                    const bool live = kHH * hh + k < G;
+                    const float mn = fmaxf(m[k], tmax[k]);
+                    alpha[k] = live ? ptx::ex2(m[k] - mn) : 0.f;
+                    m[k] = live ? mn : m[k];
+                }
             }
-            // P^T row of token t, weights times the row scale: hi and lo halves
-            {
-                uint32_t hi[4], lo[4];
+            float smax = sm.red[sb][0][kHH];
 #pragma unroll
-                for (int e = 0; e < 4; ++e)
-                    split_h2(p[2 * e] * scale_cur, p[2 * e + 1] * scale_cur, hi[e], lo[e]);
-                uint8_t *row = sm.p[sb] + (t >> 3) * 256 + (t & 7) * 16;
-                *reinterpret_cast<uint4 *>(row) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-                *reinterpret_cast<uint4 *>(row + 128) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+            for (int w = 1; w < 4; ++w) smax = fmaxf(smax, sm.red[sb][w][kHH]);
+            // weights <= 4 and row scales < 2^es: 2^(6 - es) keeps every weight term below 256
+            const int es = (int)((__float_as_uint(smax) >> 23) & 0xFFu) - 126;
+            float sc, inv;
+            pow2_from_exp(es + 2, sc, inv);
+            const float sts = st * sc;
+            float x[kHH];
+#pragma unroll
+            for (int k = 0; k < kHH; ++k) {
+                const float p = kHH * hh + k < G ? ptx::ex2(s_k[k] - m[k]) : 0.f;
+                lsum[k] = fmaf(lsum[k], alpha[k], p);
+                x[k] = p * sts;
+            }
+            // W row of token t: 3 E4M3 terms of this warp's 4 heads, one 16-byte block. Each
+            // term but the last is the value rounded to E4M3; the residual times 16 goes on.
+            uint32_t w[kJp];
+#pragma unroll
+            for (int j = 0; j < kJp; ++j) {
+                uint32_t c2[2];
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    float v0 = x[2 * e], v1 = x[2 * e + 1];
+                    if (j + 1 < kJp) {
+                        v0 = e4m3_round(v0);
+                        v1 = e4m3_round(v1);
+                        x[2 * e] = (x[2 * e] - v0) * 16.f;
+                        x[2 * e + 1] = (x[2 * e + 1] - v1) * 16.f;
+                    }
+                    c2[e] = (uint32_t)__nv_cvt_float2_to_fp8x2(make_float2(v0, v1), __NV_SATFINITE,
+                                                                __NV_E4M3);
+                }
+                w[j] = c2[0] | (c2[1] << 16);
+            }
+            *reinterpret_cast<uint4 *>(sm.p[sb] + (t >> 3) * 256 + hh * 128 + (t & 7) * 16) =
+                make_uint4(w[0], w[1], w[2], 0u);
+            // The output MMAs read whole 32-token steps of the tile: rows past the end of the
+            // sequence hold stale bytes (possibly NaN codes), so zero them.
+            if (hh == 0 && !valid && t < ((nvalid + 31) & ~31)) {
+                uint4 *cr = reinterpret_cast<uint4 *>(sm.codes[s] + t * 128);
+#pragma unroll
+                for (int c = 0; c < 8; ++c) cr[c] = make_uint4(0u, 0u, 0u, 0u);
             }
             ptx::fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&sm.p_full[sb]);
 
-            if (i >= 1 && !correct(i - 1, alpha_prev)) { ok = false; break; }
+            if (i >= 1) carried = correct(i - 1, alpha_prev, inv_prev);
 #pragma unroll
-            for (int h = 0; h < kNG; ++h) alpha_prev[h] = alpha[h];
+            for (int k = 0; k < kHH; ++k) alpha_prev[k] = alpha[k];
+            inv_prev = inv;
         }
-        if (ok) ok = correct(n_tiles - 1, alpha_prev);
+        if (ok) carried = correct(n_tiles - 1, alpha_prev, inv_prev);
 
-        if (ok) {
+        // the epilogue's barrier (the row sums) settles the last waits
 #pragma unroll
-            for (int off = 16; off > 0; off >>= 1)
+        for (int off = 16; off > 0; off >>= 1)
 #pragma unroll
-                for (int h = 0; h < kNG; ++h) lsum[h] += __shfl_xor_sync(0xffffffffu, lsum[h], off);
-            const int rb = n_tiles & 1;
-            if (lane == 0) {
+            for (int k = 0; k < kHH; ++k) lsum[k] += __shfl_xor_sync(0xffffffffu, lsum[k], off);
+        const int rb = n_tiles & 1;
+        if (lane == 0) {
 #pragma unroll
-                for (int h = 0; h < kNG; ++h) sm.red[rb][warp][h] = lsum[h];
-            }
-            ptx::bar_sync(kBarCompute, kTile);
+            for (int k = 0; k < kHH; ++k) sm.red[rb][warp][k] = lsum[k];
+        }
+        if (ptx::bar_and(kBarComputeAnd, kComputeThreads, ok && carried)) {
 #pragma unroll
-            for (int h = 0; h < kNG; ++h) {
+            for (int k = 0; k < kHH; ++k) {
+                const int h = kHH * hh + k;
                 if (h >= G) continue;
                 float lt = 0.f;
 #pragma unroll
-                for (int w = 0; w < kComputeWarps; ++w) lt += sm.red[rb][w][h];
-                const float val = o[h] / lt;
+                for (int w = 0; w < 4; ++w) lt += sm.red[rb][kHH * hh + w][k];
+                const float val = o[k] / lt;
                 const size_t bh = (size_t)b * geo.Hq + g * G + h;
                 if (a.direct_out) {
                     if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * kD + t] = val;
@@ -591,7 +699,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                     const size_t slot = bh * geo.S + split;
                     a.part_o[slot * kD + t] = val;
                     if (t == 0) {
-                        a.part_ml[slot * 2] = m[h] * kLn2;
+                        a.part_ml[slot * 2] = m[k] * kLn2;
                         a.part_ml[slot * 2 + 1] = lt;
                     }
                 }
@@ -709,14 +817,10 @@ cudaError_t launch_decode_fp8(const DecodeArgs &a, const float *v_scales) {
     const Geometry &g = a.geo;
     if (g.B == 0) return cudaSuccess;
     const uint64_t rows = (uint64_t)g.num_pages * g.Hkv * g.P;
-    CUtensorMap cmap, smap, wmap, qmap;
-    // codes [rows][128] u8, one box = one page of one head; scales [pages * Hkv][P] fp32
+    CUtensorMap cmap, wmap, qmap;
+    // codes [rows][128] u8, one box = one page of one head (scale rows go by bulk copy)
     if (!encode2d(&cmap, CU_TENSOR_MAP_DATA_TYPE_UINT8, a.v_cache, kD, rows, kD, kD, (uint32_t)g.P,
                   CU_TENSOR_MAP_SWIZZLE_128B))
-        return cudaErrorInvalidValue;
-    if (!encode2d(&smap, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, v_scales, (uint64_t)g.P,
-                  (uint64_t)g.num_pages * g.Hkv, (uint64_t)g.P * 4, (uint32_t)g.P, 1,
-                  CU_TENSOR_MAP_SWIZZLE_NONE))
         return cudaErrorInvalidValue;
     wmap = qmap = cmap;
     if (a.w_r) {
@@ -740,7 +844,7 @@ cudaError_t launch_decode_fp8(const DecodeArgs &a, const float *v_scales) {
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = a.stream;
-    return cudaLaunchKernelEx(&cfg, decode_fp8_kernel, cmap, smap, wmap, qmap, a);
+    return cudaLaunchKernelEx(&cfg, decode_fp8_kernel, cmap, wmap, qmap, a, v_scales);
 }
 
 cudaError_t launch_append_fp8(const Geometry &g, const uint16_t *v_new, const int32_t *block_table,
