@@ -21,8 +21,9 @@
 // The softmax keeps a lazy reference maximum per head: a tile's weights are 2^(s - m) with the
 // current reference m, and m moves (rescaling the running sums) only when a score passes it by
 // more than 2, so the weights stay at most 4. Most tiles thus need one vote among the compute
-// warps instead of an exchange of maxima, and one power of two, 2^(6 - e) with the tile's row
-// scales below 2^e, serves the weights of all heads.
+// warps instead of an exchange of maxima. The weights' power of two, 2^(6 - e) with every row
+// scale so far below 2^e, is lazy the same way, so the output MMAs of all tiles accumulate into
+// one O in TMEM; the rare tile that moves a reference or e rescales O there first.
 // A row's scale multiplies its score column (s_t = scale_t <q_r, c_t>) and its weight
 // (p_t scale_t), so the codes are used as stored.
 //
@@ -67,10 +68,10 @@ constexpr int kStages = 5;
 constexpr uint32_t kCodeBytes = kTile * kD;          // 16 KiB of codes per tile
 constexpr uint32_t kHalfBytes = 16384;               // one 64-column half of W^R (bf16)
 constexpr uint32_t kPBytes = kTile * kNP;            // weight operand: 4 KiB
-constexpr uint32_t kTmemCols = 256;
+constexpr uint32_t kTmemCols = 128;
 constexpr uint32_t kColS = 0;                        // S[b]: columns 32 b .. 32 b + 31
-constexpr uint32_t kColO = 64;                       // O[b]: columns 64 + 32 b .. + 31
-constexpr uint32_t kColR = 128;                      // routing result: 128 .. 143
+constexpr uint32_t kColO = 64;                       // O: columns 64 .. 95, summed over tiles
+constexpr uint32_t kColR = 96;                       // routing result: 96 .. 111
 constexpr float kLazy = 2.f;                         // reference slack (base 2): weights <= 4
 constexpr uint64_t kTimeoutNs = 1000000000ull;
 constexpr uint32_t kBarCompute = 1;
@@ -89,7 +90,7 @@ struct __align__(1024) Smem8 {
     float scl[kStages][kTile];         // row scales of each stage's tile, token order
     float red[2][kComputeWarps][8];    // per warp: 4 head maxima (or row sums), the scale max
     uint64_t full[kStages], empty[kStages];
-    uint64_t s_full[2], s_empty[2], p_full[2], o_full[2], o_empty[2];
+    uint64_t s_full[2], s_empty[2], p_full[2], o_full[2];
     uint64_t r_full, qt_full, drain, drain2;
     uint32_t tmem_base;
     int abort;
@@ -206,6 +207,17 @@ __host__ __device__ constexpr uint32_t idesc_f8(uint32_t M, uint32_t N, bool a_m
            ((M >> 4) << 24);
 }
 
+// Store 16 consecutive 32-bit columns of the thread's TMEM lane (complete with tmem_wait_st()).
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&u)[16]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+        "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+        "r"(u[0]), "r"(u[1]), "r"(u[2]), "r"(u[3]), "r"(u[4]), "r"(u[5]), "r"(u[6]), "r"(u[7]),
+        "r"(u[8]), "r"(u[9]), "r"(u[10]), "r"(u[11]), "r"(u[12]), "r"(u[13]), "r"(u[14]),
+        "r"(u[15])
+        : "memory");
+}
+
 // Barrier `id` over `count` threads that also returns how many of them passed v = true.
 __device__ __forceinline__ uint32_t bar_popc(uint32_t id, uint32_t count, bool v) {
     uint32_t r;
@@ -248,9 +260,9 @@ __global__ void __launch_bounds__(kThreads, 2)
             ptx::mbar_init(&sm.s_full[i], 1);
             ptx::mbar_init(&sm.s_empty[i], kComputeWarps);
             ptx::mbar_init(&sm.p_full[i], kComputeWarps);
-            ptx::mbar_init(&sm.o_full[i], 1);
-            ptx::mbar_init(&sm.o_empty[i], kComputeWarps);
         }
+        ptx::mbar_init(&sm.o_full[0], 1);
+        ptx::mbar_init(&sm.o_full[1], 1);
         ptx::mbar_init(&sm.r_full, 1);
         ptx::mbar_init(&sm.qt_full, kComputeWarps);
         ptx::mbar_init(&sm.drain, 1);
@@ -423,7 +435,6 @@ __global__ void __launch_bounds__(kThreads, 2)
         for (int j = 0; j < n_tiles; ++j) {
             const int u = j + base, s = u % kStages, pb = j & 1;
             if (!wait(&sm.p_full[pb], (j >> 1) & 1)) break;
-            if (j >= 2 && !wait(&sm.o_empty[pb], ((j >> 1) - 1) & 1)) break;
             ptx::tc_fence_after();
             const int nvalid = min(kTile, t_end - (t_begin + j * kTile));
             const int ksteps = (nvalid + 31) >> 5;
@@ -431,9 +442,9 @@ __global__ void __launch_bounds__(kThreads, 2)
                 const uint64_t a0 = c_desc + ((s * kCodeBytes) >> 4);
                 const uint64_t b0 = p_desc + ((pb * kPBytes) >> 4);
                 for (int kk = 0; kk < ksteps; ++kk)
-                    mma_f8(tmem + kColO + pb * 32, a0 + ((kk * 4096) >> 4), b0 + ((kk * 1024) >> 4),
-                           idesc_o, kk > 0);
-                ptx::mma_commit(&sm.o_full[pb]);
+                    mma_f8(tmem + kColO, a0 + ((kk * 4096) >> 4), b0 + ((kk * 1024) >> 4), idesc_o,
+                           (j > 0 || kk > 0) ? 1u : 0u);
+                ptx::mma_commit(&sm.o_full[pb]);   // one phase per tile of this parity
                 ptx::mma_commit(&sm.empty[s]);     // the tile's last reader is done
             }
             __syncwarp();
@@ -513,45 +524,43 @@ __global__ void __launch_bounds__(kThreads, 2)
             if (lane == 0) ptx::mbar_arrive(&sm.qt_full);
         }
 
-        float m[kHH], lsum[kHH], o[kHH], alpha_prev[kHH];
-        float inv_prev = 0.f;
+        float m[kHH], lsum[kHH];
 #pragma unroll
         for (int k = 0; k < kHH; ++k) {
             m[k] = -INFINITY;
             lsum[k] = 0.f;
-            o[k] = 0.f;
-            alpha_prev[k] = 0.f;
         }
-        // O accumulation of tile j: o = o * alpha_j + inv_j * (O_0 + O_1 / 16 + O_2 / 256)
-        // (thread = output dim t; O_j the term columns of the output MMA). The wait is the
-        // warp's own; a failure travels to the next barrier of all compute warps.
-        auto correct = [&](int j, const float (&alpha)[kHH], float inv) -> bool {
-            const int ob = j & 1;
-            if (!wait(&sm.o_full[ob], (j >> 1) & 1)) return false;
-            ptx::tc_fence_after();
-            float ov[16];
-            ptx::tmem_ld16(tmem + kColO + ob * 32 + 16 * hh + lane_base, ov);
-            ptx::tc_fence_before();
-            __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(&sm.o_empty[ob]);
-#pragma unroll
-            for (int k = 0; k < kHH; ++k) {
-                const float d = fmaf(ov[8 + k], 1.f / 256.f, fmaf(ov[4 + k], 1.f / 16.f, ov[k]));
-                o[k] = fmaf(o[k], alpha[k], d * inv);
+        // Lazy weight scale: every row scale so far is below lim = 2^es; weights are taken
+        // times sc = 2^(6 - es) and O times inv = 2^(es - 6) at the end.
+        int es = -1000;
+        float lim = 0.f, sc = 1.f, inv = 1.f;
+        // Completions of the output MMAs: tile j is phase j / 2 of o_full[j % 2]. Each barrier's
+        // phases are observed in order, and a warp observes tile i - 2 before it releases the
+        // weights of tile i, so no barrier runs more than one phase ahead of its observer and
+        // no phase is mistaken for a later one of the same parity.
+        int o_seen0 = 0, o_seen1 = 0;                  // phases observed on o_full[0], [1]
+        auto observe = [&](int j) -> bool {            // the output MMAs of tile j are done
+            if (j < 0) return true;
+            int &seen = (j & 1) ? o_seen1 : o_seen0;
+            while (seen <= (j >> 1)) {
+                if (!wait(&sm.o_full[j & 1], seen & 1)) return false;
+                ++seen;
             }
             return true;
         };
 
-        // One barrier per tile for all compute warps: it publishes the tile's row-scale maximum,
-        // counts the warps whose scores passed a reference (or whose waits failed since the last
-        // barrier). Only then a second one exchanges the head maxima (or lets all of them leave
-        // the loop together after a failed wait).
+        // One barrier per tile for all compute warps: it counts the warps with a score past its
+        // reference, a row scale past lim, or a failed wait since the last barrier. Only then a
+        // second one exchanges the tile maxima (or lets all of them leave the loop together
+        // after a failed wait).
         bool carried = true;
         for (int i = 0; ok && i < n_tiles; ++i) {
             const int u = i + base, s = u % kStages, sb = i & 1;
-            // the stage's loads have landed (its scale row is read below) and S is ready
+            // the stage's loads have landed (its scale row is read below), S is ready, and the
+            // output MMAs of tile i - 2 (the last reader of this weight buffer) are done
             bool ready = wait(&sm.full[s], (u / kStages) & 1);
             ready = ready && wait(&sm.s_full[sb], (i >> 1) & 1);
+            ready = ready && observe(i - 2);
             float sv[16];
             if (ready) {
                 ptx::tc_fence_after();
@@ -577,17 +586,16 @@ __global__ void __launch_bounds__(kThreads, 2)
                 s_k[k] = (valid && kHH * hh + k < G) ? d * (invq[k] * st) : -INFINITY;
                 grow = grow || s_k[k] > m[k] + kLazy;
             }
-            if (hh == 0) {
-                // row scales are non-negative: their bits order as the values do
-                const float smx = __uint_as_float(__reduce_max_sync(0xffffffffu, __float_as_uint(st)));
-                if (lane == 0) sm.red[sb][warp][kHH] = smx;
-            }
+            // row scales are non-negative: their bits order as the values do
+            const float smx = __uint_as_float(__reduce_max_sync(0xffffffffu, __float_as_uint(st)));
+            grow = grow || smx >= lim;
+            if (lane == 0) sm.red[sb][warp][kHH] = smx;
             const bool fine = ready && carried;
             float alpha[kHH];
 #pragma unroll
             for (int k = 0; k < kHH; ++k) alpha[k] = 1.f;
             if (bar_popc(kBarComputeAnd, kComputeThreads, grow || !fine) != 0) {
-                // move the references to the heads' running maxima
+                // move the references to the heads' running maxima and lim past the row scales
                 float wm[kHH];
 #pragma unroll
                 for (int k = 0; k < kHH; ++k) wm[k] = warp_max(s_k[k]);
@@ -609,27 +617,53 @@ __global__ void __launch_bounds__(kThreads, 2)
                     tmax[2] = fmaxf(tmax[2], r.z);
                     tmax[3] = fmaxf(tmax[3], r.w);
                 }
+                float smax = sm.red[sb][0][kHH];
+#pragma unroll
+                for (int w = 1; w < 4; ++w) smax = fmaxf(smax, sm.red[sb][w][kHH]);
+                const int es_new =
+                    smax > 0.f ? max(es, (int)((__float_as_uint(smax) >> 23) & 0xFFu) - 126) : es;
+                // O so far was taken with 2^(6 - es): bring it to 2^(6 - es_new)
+                const float shift = es_new > es && es > -1000 ? __uint_as_float((uint32_t)max(1, 127 + es - es_new) << 23)
+                                                               : 1.f;
+                bool rescale = shift != 1.f;
 #pragma unroll
                 for (int k = 0; k < kHH; ++k) {
                     const bool live = kHH * hh + k < G;
                     const float mn = fmaxf(m[k], tmax[k]);
-                    alpha[k] = live ? ptx::ex2(m[k] - mn) : 0.f;
+                    alpha[k] = live ? ptx::ex2(m[k] - mn) : 1.f;
                     m[k] = live ? mn : m[k];
+                    lsum[k] *= alpha[k];
+                    rescale = rescale || alpha[k] != 1.f;
+                }
+                if (es_new != es) {
+                    es = es_new;
+                    pow2_from_exp(es + 2, sc, inv);
+                    lim = __uint_as_float((uint32_t)max(1, min(254, es + 127)) << 23);
+                }
+                if (i >= 1 && rescale) {
+                    // every output MMA so far is done (tile i's waits for this warp's weights)
+                    if (observe(i - 1)) {
+                        ptx::tc_fence_after();
+                        float ov[16];
+                        ptx::tmem_ld16(tmem + kColO + 16 * hh + lane_base, ov);
+                        uint32_t ou[16];
+#pragma unroll
+                        for (int c = 0; c < 16; ++c)
+                            ou[c] = __float_as_uint(ov[c] * (alpha[c & 3] * shift));
+                        tmem_st16(tmem + kColO + 16 * hh + lane_base, ou);
+                        ptx::tmem_wait_st();
+                        ptx::tc_fence_before();
+                    } else {
+                        carried = false;
+                    }
                 }
             }
-            float smax = sm.red[sb][0][kHH];
-#pragma unroll
-            for (int w = 1; w < 4; ++w) smax = fmaxf(smax, sm.red[sb][w][kHH]);
-            // weights <= 4 and row scales < 2^es: 2^(6 - es) keeps every weight term below 256
-            const int es = (int)((__float_as_uint(smax) >> 23) & 0xFFu) - 126;
-            float sc, inv;
-            pow2_from_exp(es + 2, sc, inv);
             const float sts = st * sc;
             float x[kHH];
 #pragma unroll
             for (int k = 0; k < kHH; ++k) {
                 const float p = kHH * hh + k < G ? ptx::ex2(s_k[k] - m[k]) : 0.f;
-                lsum[k] = fmaf(lsum[k], alpha[k], p);
+                lsum[k] += p;
                 x[k] = p * sts;
             }
             // W row of token t: 3 E4M3 terms of this warp's 4 heads, one 16-byte block. Each
@@ -664,13 +698,24 @@ __global__ void __launch_bounds__(kThreads, 2)
             ptx::fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&sm.p_full[sb]);
-
-            if (i >= 1) carried = correct(i - 1, alpha_prev, inv_prev);
-#pragma unroll
-            for (int k = 0; k < kHH; ++k) alpha_prev[k] = alpha[k];
-            inv_prev = inv;
         }
-        if (ok) carried = correct(n_tiles - 1, alpha_prev, inv_prev);
+        // O = (O_0 + O_1 / 16 + O_2 / 256) * inv once every output MMA is done
+        float o[kHH];
+#pragma unroll
+        for (int k = 0; k < kHH; ++k) o[k] = 0.f;
+        if (ok && carried) {
+            if (observe(n_tiles - 2) && observe(n_tiles - 1)) {
+                ptx::tc_fence_after();
+                float ov[16];
+                ptx::tmem_ld16(tmem + kColO + 16 * hh + lane_base, ov);
+                ptx::tc_fence_before();
+#pragma unroll
+                for (int k = 0; k < kHH; ++k)
+                    o[k] = fmaf(ov[8 + k], 1.f / 256.f, fmaf(ov[4 + k], 1.f / 16.f, ov[k])) * inv;
+            } else {
+                carried = false;
+            }
+        }
 
         // the epilogue's barrier (the row sums) settles the last waits
 #pragma unroll
