@@ -78,8 +78,9 @@ def measured_peaks():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-# the sources the decode kernel is compiled from
+# the sources each decode kernel is compiled from (traffic records are keyed to their hash)
 DECODE_SOURCES = ("kl_decode_tc.cu", "kl_internal.cuh", "kl_tc_ptx.cuh")
+FP8_SOURCES = ("kl_decode_fp8.cu", "kl_internal.cuh", "kl_tc_ptx.cuh")
 
 
 def kernel_source_digest(names=DECODE_SOURCES) -> str:
@@ -96,7 +97,7 @@ def recorded_traffic(workload: str, kernel: str):
     path = os.path.join(ROOT, "profiles", "dram_traffic.md")
     if not os.path.exists(path):
         return None
-    digest = kernel_source_digest()
+    digest = kernel_source_digest(FP8_SOURCES if kernel == "tensor-fp8" else DECODE_SOURCES)
     for line in open(path):
         m = re.match(r"\|\s*(\S+)\s*\|\s*(\S+)\s*\|\s*([0-9]+)\s*\|\s*([0-9a-f]+)\s*\|", line)
         if m and m.group(1) == workload and m.group(2) == kernel and m.group(4) == digest:

@@ -68,6 +68,7 @@ constexpr int kStages = 5;
 constexpr uint32_t kCodeBytes = kTile * kD;          // 16 KiB of codes per tile
 constexpr uint32_t kHalfBytes = 16384;               // one 64-column half of W^R (bf16)
 constexpr uint32_t kPBytes = kTile * kNP;            // weight operand: 4 KiB
+constexpr int kPBuf = 4;                             // weight operands in flight
 constexpr uint32_t kTmemCols = 128;
 constexpr uint32_t kColS = 0;                        // S[b]: columns 32 b .. 32 b + 31
 constexpr uint32_t kColO = 64;                       // O: columns 64 .. 95, summed over tiles
@@ -86,11 +87,11 @@ struct __align__(1024) Smem8 {
     // Weight terms, B operand of the output MMAs: [16 groups of 8 tokens][2 blocks of 16
     // columns][8 tokens][16 B], MN-major, no swizzle. During the routing prologue the first one
     // holds the query rows: [64-dim half][16 rows][128 B], K-major, 128B-swizzled.
-    uint8_t p[2][kPBytes];
+    uint8_t p[kPBuf][kPBytes];
     float scl[kStages][kTile];         // row scales of each stage's tile, token order
     float red[2][kComputeWarps][8];    // per warp: 4 head maxima (or row sums), the scale max
     uint64_t full[kStages], empty[kStages];
-    uint64_t s_full[2], s_empty[2], p_full[2], o_full[2];
+    uint64_t s_full[2], s_empty[2], p_full[kPBuf], o_full[kPBuf];
     uint64_t r_full, qt_full, drain, drain2;
     uint32_t tmem_base;
     int abort;
@@ -259,10 +260,11 @@ __global__ void __launch_bounds__(kThreads, 2)
         for (int i = 0; i < 2; ++i) {
             ptx::mbar_init(&sm.s_full[i], 1);
             ptx::mbar_init(&sm.s_empty[i], kComputeWarps);
-            ptx::mbar_init(&sm.p_full[i], kComputeWarps);
         }
-        ptx::mbar_init(&sm.o_full[0], 1);
-        ptx::mbar_init(&sm.o_full[1], 1);
+        for (int i = 0; i < kPBuf; ++i) {
+            ptx::mbar_init(&sm.p_full[i], kComputeWarps);
+            ptx::mbar_init(&sm.o_full[i], 1);
+        }
         ptx::mbar_init(&sm.r_full, 1);
         ptx::mbar_init(&sm.qt_full, kComputeWarps);
         ptx::mbar_init(&sm.drain, 1);
@@ -433,8 +435,8 @@ __global__ void __launch_bounds__(kThreads, 2)
             ptx::smem_desc(ptx::smem_addr(sm.codes[0]), 8192, 1024, ptx::kSwizzle128B);
         const uint64_t p_desc = ptx::smem_desc(ptx::smem_addr(sm.p[0]), 256, 128, ptx::kSwizzleNone);
         for (int j = 0; j < n_tiles; ++j) {
-            const int u = j + base, s = u % kStages, pb = j & 1;
-            if (!wait(&sm.p_full[pb], (j >> 1) & 1)) break;
+            const int u = j + base, s = u % kStages, pb = j % kPBuf;
+            if (!wait(&sm.p_full[pb], (j / kPBuf) & 1)) break;
             ptx::tc_fence_after();
             const int nvalid = min(kTile, t_end - (t_begin + j * kTile));
             const int ksteps = (nvalid + 31) >> 5;
@@ -444,7 +446,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                 for (int kk = 0; kk < ksteps; ++kk)
                     mma_f8(tmem + kColO, a0 + ((kk * 4096) >> 4), b0 + ((kk * 1024) >> 4), idesc_o,
                            (j > 0 || kk > 0) ? 1u : 0u);
-                ptx::mma_commit(&sm.o_full[pb]);   // one phase per tile of this parity
+                ptx::mma_commit(&sm.o_full[pb]);   // tile j: phase j / kPBuf of o_full[j % kPBuf]
                 ptx::mma_commit(&sm.empty[s]);     // the tile's last reader is done
             }
             __syncwarp();
@@ -534,17 +536,16 @@ __global__ void __launch_bounds__(kThreads, 2)
         // times sc = 2^(6 - es) and O times inv = 2^(es - 6) at the end.
         int es = -1000;
         float lim = 0.f, sc = 1.f, inv = 1.f;
-        // Completions of the output MMAs: tile j is phase j / 2 of o_full[j % 2]. Each barrier's
-        // phases are observed in order, and a warp observes tile i - 2 before it releases the
-        // weights of tile i, so no barrier runs more than one phase ahead of its observer and
-        // no phase is mistaken for a later one of the same parity.
-        int o_seen0 = 0, o_seen1 = 0;                  // phases observed on o_full[0], [1]
-        auto observe = [&](int j) -> bool {            // the output MMAs of tile j are done
-            if (j < 0) return true;
-            int &seen = (j & 1) ? o_seen1 : o_seen0;
-            while (seen <= (j >> 1)) {
-                if (!wait(&sm.o_full[j & 1], seen & 1)) return false;
-                ++seen;
+        // Completions of the output MMAs: tile j is phase j / kPBuf of o_full[j % kPBuf]. The
+        // tiles are observed in order, and a warp observes tile i - kPBuf (the last reader of
+        // the weight buffer it is about to fill) before it releases tile i, so no barrier runs
+        // more than one phase ahead of its observer and no phase is mistaken for a later one of
+        // the same parity.
+        int o_seen = 0;                                // tiles 0 .. o_seen - 1 observed
+        auto observe = [&](int j) -> bool {            // the output MMAs up to tile j are done
+            while (o_seen <= j) {
+                if (!wait(&sm.o_full[o_seen % kPBuf], (o_seen / kPBuf) & 1)) return false;
+                ++o_seen;
             }
             return true;
         };
@@ -557,10 +558,11 @@ __global__ void __launch_bounds__(kThreads, 2)
         for (int i = 0; ok && i < n_tiles; ++i) {
             const int u = i + base, s = u % kStages, sb = i & 1;
             // the stage's loads have landed (its scale row is read below), S is ready, and the
-            // output MMAs of tile i - 2 (the last reader of this weight buffer) are done
+            // output MMAs of tile i - kPBuf (the last reader of this weight buffer) are done
+            const int pb = i % kPBuf;
             bool ready = wait(&sm.full[s], (u / kStages) & 1);
             ready = ready && wait(&sm.s_full[sb], (i >> 1) & 1);
-            ready = ready && observe(i - 2);
+            ready = ready && observe(i - kPBuf);
             float sv[16];
             if (ready) {
                 ptx::tc_fence_after();
@@ -686,7 +688,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                 }
                 w[j] = c2[0] | (c2[1] << 16);
             }
-            *reinterpret_cast<uint4 *>(sm.p[sb] + (t >> 3) * 256 + hh * 128 + (t & 7) * 16) =
+            *reinterpret_cast<uint4 *>(sm.p[pb] + (t >> 3) * 256 + hh * 128 + (t & 7) * 16) =
                 make_uint4(w[0], w[1], w[2], 0u);
             // The output MMAs read whole 32-token steps of the tile: rows past the end of the
             // sequence hold stale bytes (possibly NaN codes), so zero them.
@@ -697,14 +699,14 @@ __global__ void __launch_bounds__(kThreads, 2)
             }
             ptx::fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(&sm.p_full[sb]);
+            if (lane == 0) ptx::mbar_arrive(&sm.p_full[pb]);
         }
         // O = (O_0 + O_1 / 16 + O_2 / 256) * inv once every output MMA is done
         float o[kHH];
 #pragma unroll
         for (int k = 0; k < kHH; ++k) o[k] = 0.f;
         if (ok && carried) {
-            if (observe(n_tiles - 2) && observe(n_tiles - 1)) {
+            if (observe(n_tiles - 1)) {
                 ptx::tc_fence_after();
                 float ov[16];
                 ptx::tmem_ld16(tmem + kColO + 16 * hh + lane_base, ov);
