@@ -52,12 +52,10 @@ namespace {
 
 constexpr int kD = 128;
 constexpr int kTile = 128;
-constexpr int kHH = 4;                      // heads per compute warp
 constexpr int kJq = 4;                      // E4M3 terms of the routed query
 constexpr int kJp = 3;                      // E4M3 terms of the weights
-constexpr int kNS = 32;                     // score MMA N: 2 x 16 columns
-constexpr int kNP = 32;                     // output MMA N: 2 x 16 columns (12 used each)
 constexpr int kNR = 16;                     // routing MMA N (query rows, padded)
+constexpr int kQuarters = 4;                // TMEM lane quarters (warps per head half)
 constexpr int kComputeWarps = 8;
 constexpr int kComputeThreads = kComputeWarps * 32;
 constexpr int kProducerWarp = 8;
@@ -67,7 +65,7 @@ constexpr int kThreads = 11 * 32;
 constexpr int kStages = 5;
 constexpr uint32_t kCodeBytes = kTile * kD;          // 16 KiB of codes per tile
 constexpr uint32_t kHalfBytes = 16384;               // one 64-column half of W^R (bf16)
-constexpr uint32_t kPBytes = kTile * kNP;            // weight operand: 4 KiB
+constexpr uint32_t kPBytes = 4096;                   // weight operand buffer (largest shape)
 constexpr int kPBuf = 4;                             // weight operands in flight
 constexpr uint32_t kTmemCols = 128;
 constexpr uint32_t kColS = 0;                        // S[b]: columns 32 b .. 32 b + 31
@@ -78,13 +76,26 @@ constexpr uint64_t kTimeoutNs = 1000000000ull;
 constexpr uint32_t kBarCompute = 1;
 constexpr uint32_t kBarComputeAnd = 2;
 
+// Operand shapes for KHH query heads per compute warp (4 when the group has 5..8 heads, 2 when
+// it has at most 4, so that no compute warp carries only padded heads). Head h = KHH hh + k
+// (hh = warp / 4) and term j sit in score column HS hh + KHH j + k and output column
+// HP hh + KHH j + k.
+template <int KHH>
+struct Fp8Shape {
+    static constexpr int NS = 8 * KHH;        // score MMA N: 4 query terms x 2 KHH heads
+    static constexpr int NP = 8 * KHH;        // output MMA N: 3 weight terms x 2 KHH heads, padded
+    static constexpr int HS = NS / 2;         // score columns of one warp
+    static constexpr int HP = NP / 2;         // output columns of one warp
+    static constexpr int GS = 8 * NP;         // weight operand: bytes per group of 8 tokens
+};
+
 struct __align__(1024) Smem8 {
     // Ring of code tiles as TMA lands them: [128 token rows][128 B], 128B-swizzled. Stages 0
     // and 1 first hold the two 64-column halves of W^R[g] (bf16) for the routing MMA.
     uint8_t codes[kStages][kCodeBytes];
-    // Query terms, B operand of the score MMAs: [32 rows n][128 dims], K-major, 128B-swizzled.
-    uint8_t qt[kNS * 128];
-    // Weight terms, B operand of the output MMAs: [16 groups of 8 tokens][2 blocks of 16
+    // Query terms, B operand of the score MMAs: [NS rows n][128 dims], K-major, 128B-swizzled.
+    uint8_t qt[32 * 128];
+    // Weight terms, B operand of the output MMAs: [16 groups of 8 tokens][NP / 16 blocks of 16
     // columns][8 tokens][16 B], MN-major, no swizzle. During the routing prologue the first one
     // holds the query rows: [64-dim half][16 rows][128 B], K-major, 128B-swizzled.
     uint8_t p[kPBuf][kPBytes];
@@ -174,8 +185,9 @@ __device__ __forceinline__ void pow2_from_exp(int e, float &sc, float &inv) {
 // Veltkamp split (c = x (2^20 + 1), hi = c - (c - x)), and below 2^-6, where the E4M3 values
 // are the multiples of 2^-9, by adding and subtracting 1.5 * 2^14 (whose spacing is 2^-9). The
 // result is an E4M3 value, so its code conversion is exact and x - hi is the exact residual.
-// (The small values matter: with a few large row scales in a tile, most weights sit far below
-// the tile's largest and would lose their residual without the second rounding.)
+// (The small values matter: the weight scale follows the largest row scale seen so far, so
+// most weights can sit far below it; leaving them whole to the later terms costs them too many
+// bits at this tolerance.)
 __device__ __forceinline__ float e4m3_round(float x) {
     // explicit roundings: the compiler must not fuse these into FMAs
     const float c = __fmul_rn(x, 1048577.f);
@@ -184,7 +196,7 @@ __device__ __forceinline__ float e4m3_round(float x) {
     return x < 0.015625f ? hs : hv;
 }
 
-// Byte offset of element (row n, column k) of the query-term operand: [48 rows][128 B],
+// Byte offset of element (row n, column k) of the query-term operand: [NS rows][128 B],
 // K-major, 128B-swizzled (8-row atoms of 1 KiB, 16-byte chunk index XOR row % 8).
 __device__ __forceinline__ uint32_t qt_offset(int n, int k) {
     return (n >> 3) * 1024 + (n & 7) * 128 + ((((k >> 4) ^ (n & 7))) << 4) + (k & 15);
@@ -219,6 +231,40 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&u)[16
         : "memory");
 }
 
+// 8 consecutive 32-bit columns of the thread's TMEM lane (load and wait in one statement).
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, float (&r)[8]) {
+    uint32_t u[8];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];\n\t"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(u[0]), "=r"(u[1]), "=r"(u[2]), "=r"(u[3]), "=r"(u[4]), "=r"(u[5]), "=r"(u[6]),
+          "=r"(u[7])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int i = 0; i < 8; ++i) r[i] = __uint_as_float(u[i]);
+}
+
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&u)[8]) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"r"(
+                     taddr),
+                 "r"(u[0]), "r"(u[1]), "r"(u[2]), "r"(u[3]), "r"(u[4]), "r"(u[5]), "r"(u[6]),
+                 "r"(u[7])
+                 : "memory");
+}
+
+// N (8 or 16) consecutive columns of the thread's TMEM lane.
+template <int N>
+__device__ __forceinline__ void tmem_ldn(uint32_t taddr, float (&r)[N]) {
+    if constexpr (N == 16) ptx::tmem_ld16(taddr, r);
+    else tmem_ld8(taddr, r);
+}
+template <int N>
+__device__ __forceinline__ void tmem_stn(uint32_t taddr, const uint32_t (&u)[N]) {
+    if constexpr (N == 16) tmem_st16(taddr, u);
+    else tmem_st8(taddr, u);
+}
+
 // Barrier `id` over `count` threads that also returns how many of them passed v = true.
 __device__ __forceinline__ uint32_t bar_popc(uint32_t id, uint32_t count, bool v) {
     uint32_t r;
@@ -232,11 +278,13 @@ __device__ __forceinline__ uint32_t bar_popc(uint32_t id, uint32_t count, bool v
     return r;
 }
 
+template <int KHH>
 __global__ void __launch_bounds__(kThreads, 2)
     decode_fp8_kernel(const __grid_constant__ CUtensorMap cmap,
                       const __grid_constant__ CUtensorMap wmap,
                       const __grid_constant__ CUtensorMap qmap, const DecodeArgs a,
                       const float *__restrict__ v_scales) {
+    using Sh = Fp8Shape<KHH>;
     extern __shared__ uint8_t smem_raw[];
     Smem8 &sm = *reinterpret_cast<Smem8 *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                            ~uintptr_t(1023));
@@ -402,7 +450,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
         ok = ok && wait(&sm.qt_full, 0);
         if (ok) ptx::tc_fence_after();
-        constexpr uint32_t idesc_s = idesc_f8(128, kNS, false, false);
+        constexpr uint32_t idesc_s = idesc_f8(128, Sh::NS, false, false);
         const uint64_t c_desc =
             ptx::smem_desc(ptx::smem_addr(sm.codes[0]), 16, 1024, ptx::kSwizzle128B);
         const uint64_t q_desc = ptx::smem_desc(ptx::smem_addr(sm.qt), 16, 1024, ptx::kSwizzle128B);
@@ -429,11 +477,12 @@ __global__ void __launch_bounds__(kThreads, 2)
     } else if (warp == kPvWarp) {
         // ------------------------------------------------------ output MMA issuer -------
         // A = C^T: the code tile read MN-major (8-token row groups 1 KiB apart); B = W:
-        // MN-major, no swizzle (16-column blocks 128 B apart, 8-token groups 256 B apart)
-        constexpr uint32_t idesc_o = idesc_f8(128, kNP, true, true);
+        // MN-major, no swizzle (16-column blocks 128 B apart, 8-token groups GS bytes apart)
+        constexpr uint32_t idesc_o = idesc_f8(128, Sh::NP, true, true);
         const uint64_t c_desc =
             ptx::smem_desc(ptx::smem_addr(sm.codes[0]), 8192, 1024, ptx::kSwizzle128B);
-        const uint64_t p_desc = ptx::smem_desc(ptx::smem_addr(sm.p[0]), 256, 128, ptx::kSwizzleNone);
+        const uint64_t p_desc =
+            ptx::smem_desc(ptx::smem_addr(sm.p[0]), Sh::GS, 128, ptx::kSwizzleNone);
         for (int j = 0; j < n_tiles; ++j) {
             const int u = j + base, s = u % kStages, pb = j % kPBuf;
             if (!wait(&sm.p_full[pb], (j / kPBuf) & 1)) break;
@@ -444,8 +493,8 @@ __global__ void __launch_bounds__(kThreads, 2)
                 const uint64_t a0 = c_desc + ((s * kCodeBytes) >> 4);
                 const uint64_t b0 = p_desc + ((pb * kPBytes) >> 4);
                 for (int kk = 0; kk < ksteps; ++kk)
-                    mma_f8(tmem + kColO, a0 + ((kk * 4096) >> 4), b0 + ((kk * 1024) >> 4), idesc_o,
-                           (j > 0 || kk > 0) ? 1u : 0u);
+                    mma_f8(tmem + kColO, a0 + ((kk * 4096) >> 4), b0 + ((kk * 4 * Sh::GS) >> 4),
+                           idesc_o, (j > 0 || kk > 0) ? 1u : 0u);
                 ptx::mma_commit(&sm.o_full[pb]);   // tile j: phase j / kPBuf of o_full[j % kPBuf]
                 ptx::mma_commit(&sm.empty[s]);     // the tile's last reader is done
             }
@@ -467,9 +516,9 @@ __global__ void __launch_bounds__(kThreads, 2)
         bool ok = true;
 
         // Routed query: from the routing MMA (TMEM), or the composed query itself.
-        float acc[kHH];
+        float acc[KHH];
 #pragma unroll
-        for (int k = 0; k < kHH; ++k) acc[k] = 0.f;
+        for (int k = 0; k < KHH; ++k) acc[k] = 0.f;
         if (route) {
             ok = ptx::bar_and(kBarComputeAnd, kComputeThreads, wait(&sm.r_full, 0));
             if (ok) {
@@ -477,47 +526,47 @@ __global__ void __launch_bounds__(kThreads, 2)
                 float rv[16];
                 ptx::tmem_ld16(tmem + kColR + lane_base, rv);
 #pragma unroll
-                for (int k = 0; k < kHH; ++k)
-                    acc[k] = kHH * hh + k < G ? (hh ? rv[kHH + k] : rv[k]) : 0.f;
+                for (int k = 0; k < KHH; ++k)
+                    acc[k] = KHH * hh + k < G ? (hh ? rv[KHH + k] : rv[k]) : 0.f;
                 ptx::tc_fence_before();
             }
         } else {
 #pragma unroll
-            for (int k = 0; k < kHH; ++k) {
-                const int h = kHH * hh + k;
+            for (int k = 0; k < KHH; ++k) {
+                const int h = KHH * hh + k;
                 acc[k] = h < G ? __uint_as_float((uint32_t)a.q[((size_t)b * geo.Hq + g * G + h) * kD + t] << 16)
                                : 0.f;
             }
         }
         // Query terms: per head, 2^(8 - e) over its largest |value|, then 6 E4M3 terms.
-        float invq[kHH];
+        float invq[KHH];
         if (ok) {
-            float v[kHH], av[kHH];
+            float v[KHH], av[KHH];
 #pragma unroll
-            for (int k = 0; k < kHH; ++k) {
+            for (int k = 0; k < KHH; ++k) {
                 v[k] = acc[k] * sl2;
                 av[k] = fabsf(v[k]);
             }
-            float wm[kHH];
+            float wm[KHH];
 #pragma unroll
-            for (int k = 0; k < kHH; ++k) wm[k] = warp_max(av[k]);
+            for (int k = 0; k < KHH; ++k) wm[k] = warp_max(av[k]);
             if (lane == 0) {
 #pragma unroll
-                for (int k = 0; k < kHH; ++k) sm.red[1][warp][k] = wm[k];
+                for (int k = 0; k < KHH; ++k) sm.red[1][warp][k] = wm[k];
             }
             ptx::bar_sync(kBarCompute, kComputeThreads);
 #pragma unroll
-            for (int k = 0; k < kHH; ++k) {
-                float amax = sm.red[1][kHH * hh][k];
+            for (int k = 0; k < KHH; ++k) {
+                float amax = sm.red[1][kQuarters * hh][k];
 #pragma unroll
-                for (int w = 1; w < 4; ++w) amax = fmaxf(amax, sm.red[1][kHH * hh + w][k]);
+                for (int w = 1; w < 4; ++w) amax = fmaxf(amax, sm.red[1][kQuarters * hh + w][k]);
                 float sc;
                 pow2_scale(amax, sc, invq[k]);
                 float x = v[k] * sc;
 #pragma unroll
                 for (int j = 0; j < kJq; ++j) {
                     const __nv_fp8_storage_t c = __nv_cvt_float_to_fp8(x, __NV_SATFINITE, __NV_E4M3);
-                    sm.qt[qt_offset(16 * hh + 4 * j + k, t)] = c;
+                    sm.qt[qt_offset(Sh::HS * hh + KHH * j + k, t)] = c;
                     x = (x - e4m3x2_to_float2((uint32_t)c).x) * 16.f;
                 }
             }
@@ -526,10 +575,14 @@ __global__ void __launch_bounds__(kThreads, 2)
             if (lane == 0) ptx::mbar_arrive(&sm.qt_full);
         }
 
-        float m[kHH], lsum[kHH];
+        // m: the reference maximum of each head (0 for padded heads, whose scores are -inf);
+        // thr = m + kLazy, the score that moves it (+inf for padded heads)
+        float m[KHH], thr[KHH], lsum[KHH];
 #pragma unroll
-        for (int k = 0; k < kHH; ++k) {
-            m[k] = -INFINITY;
+        for (int k = 0; k < KHH; ++k) {
+            const bool live = KHH * hh + k < G;
+            m[k] = live ? -INFINITY : 0.f;
+            thr[k] = live ? -INFINITY : INFINITY;
             lsum[k] = 0.f;
         }
         // Lazy weight scale: every row scale so far is below lim = 2^es; weights are taken
@@ -563,65 +616,64 @@ __global__ void __launch_bounds__(kThreads, 2)
             bool ready = wait(&sm.full[s], (u / kStages) & 1);
             ready = ready && wait(&sm.s_full[sb], (i >> 1) & 1);
             ready = ready && observe(i - kPBuf);
-            float sv[16];
+            float sv[Sh::HS];
             if (ready) {
                 ptx::tc_fence_after();
-                ptx::tmem_ld16(tmem + kColS + sb * 32 + 16 * hh + lane_base, sv);
+                tmem_ldn<Sh::HS>(tmem + kColS + sb * 32 + Sh::HS * hh + lane_base, sv);
                 ptx::tc_fence_before();
                 __syncwarp();
                 if (lane == 0) ptx::mbar_arrive(&sm.s_empty[sb]);
             } else {
 #pragma unroll
-                for (int c = 0; c < 16; ++c) sv[c] = 0.f;
+                for (int c = 0; c < Sh::HS; ++c) sv[c] = 0.f;
             }
 
             const int nvalid = min(kTile, t_end - (t_begin + i * kTile));
             const bool valid = t < nvalid;
             const float st = valid ? sm.scl[s][t] : 0.f;     // the row scale of token t
-            float s_k[kHH];
+            float s_k[KHH];
             bool grow = false;
 #pragma unroll
-            for (int k = 0; k < kHH; ++k) {
+            for (int k = 0; k < KHH; ++k) {
                 // sum of the term columns, 16^-j D_j, from the last term
-                const float d = fmaf(fmaf(fmaf(sv[12 + k], 1.f / 16.f, sv[8 + k]), 1.f / 16.f, sv[4 + k]),
+                const float d = fmaf(fmaf(fmaf(sv[3 * KHH + k], 1.f / 16.f, sv[2 * KHH + k]), 1.f / 16.f,
+                                          sv[KHH + k]),
                                      1.f / 16.f, sv[k]);
-                s_k[k] = (valid && kHH * hh + k < G) ? d * (invq[k] * st) : -INFINITY;
-                grow = grow || s_k[k] > m[k] + kLazy;
+                s_k[k] = (valid && KHH * hh + k < G) ? d * (invq[k] * st) : -INFINITY;
+                grow = grow || s_k[k] > thr[k];
             }
             // row scales are non-negative: their bits order as the values do
             const float smx = __uint_as_float(__reduce_max_sync(0xffffffffu, __float_as_uint(st)));
             grow = grow || smx >= lim;
-            if (lane == 0) sm.red[sb][warp][kHH] = smx;
+            if (lane == 0) sm.red[sb][warp][KHH] = smx;
             const bool fine = ready && carried;
-            float alpha[kHH];
+            float alpha[KHH];
 #pragma unroll
-            for (int k = 0; k < kHH; ++k) alpha[k] = 1.f;
+            for (int k = 0; k < KHH; ++k) alpha[k] = 1.f;
             if (bar_popc(kBarComputeAnd, kComputeThreads, grow || !fine) != 0) {
                 // move the references to the heads' running maxima and lim past the row scales
-                float wm[kHH];
+                float wm[KHH];
 #pragma unroll
-                for (int k = 0; k < kHH; ++k) wm[k] = warp_max(s_k[k]);
+                for (int k = 0; k < KHH; ++k) wm[k] = warp_max(s_k[k]);
                 if (lane == 0) {
 #pragma unroll
-                    for (int k = 0; k < kHH; ++k) sm.red[sb][warp][k] = wm[k];
+                    for (int k = 0; k < KHH; ++k) sm.red[sb][warp][k] = wm[k];
                 }
                 if (!ptx::bar_and(kBarComputeAnd, kComputeThreads, fine)) {
                     ok = false;
                     break;
                 }
-                float4 r = *reinterpret_cast<const float4 *>(&sm.red[sb][kHH * hh][0]);
-                float tmax[kHH] = {r.x, r.y, r.z, r.w};
+                float tmax[KHH];
 #pragma unroll
-                for (int w = 1; w < 4; ++w) {
-                    r = *reinterpret_cast<const float4 *>(&sm.red[sb][kHH * hh + w][0]);
-                    tmax[0] = fmaxf(tmax[0], r.x);
-                    tmax[1] = fmaxf(tmax[1], r.y);
-                    tmax[2] = fmaxf(tmax[2], r.z);
-                    tmax[3] = fmaxf(tmax[3], r.w);
+                for (int k = 0; k < KHH; ++k) {
+                    tmax[k] = sm.red[sb][kQuarters * hh][k];
+#pragma unroll
+                    for (int w = 1; w < kQuarters; ++w)
+                        tmax[k] = fmaxf(tmax[k], sm.red[sb][kQuarters * hh + w][k]);
                 }
-                float smax = sm.red[sb][0][kHH];
+                float smax = sm.red[sb][0][KHH];
 #pragma unroll
-                for (int w = 1; w < 4; ++w) smax = fmaxf(smax, sm.red[sb][w][kHH]);
+                for (int w = 1; w < 4; ++w) smax = fmaxf(smax, sm.red[sb][w][KHH]);
                 const int es_new =
                     smax > 0.f ? max(es, (int)((__float_as_uint(smax) >> 23) & 0xFFu) - 126) : es;
                 // O so far was taken with 2^(6 - es): bring it to 2^(6 - es_new)
@@ -629,11 +681,12 @@ __global__ void __launch_bounds__(kThreads, 2)
                                                                : 1.f;
                 bool rescale = shift != 1.f;
 #pragma unroll
-                for (int k = 0; k < kHH; ++k) {
-                    const bool live = kHH * hh + k < G;
+                for (int k = 0; k < KHH; ++k) {
+                    const bool live = KHH * hh + k < G;
                     const float mn = fmaxf(m[k], tmax[k]);
                     alpha[k] = live ? ptx::ex2(m[k] - mn) : 1.f;
                     m[k] = live ? mn : m[k];
+                    thr[k] = live ? mn + kLazy : thr[k];
                     lsum[k] *= alpha[k];
                     rescale = rescale || alpha[k] != 1.f;
                 }
@@ -646,13 +699,13 @@ __global__ void __launch_bounds__(kThreads, 2)
                     // every output MMA so far is done (tile i's waits for this warp's weights)
                     if (observe(i - 1)) {
                         ptx::tc_fence_after();
-                        float ov[16];
-                        ptx::tmem_ld16(tmem + kColO + 16 * hh + lane_base, ov);
-                        uint32_t ou[16];
+                        float ov[Sh::HP];
+                        tmem_ldn<Sh::HP>(tmem + kColO + Sh::HP * hh + lane_base, ov);
+                        uint32_t ou[Sh::HP];
 #pragma unroll
-                        for (int c = 0; c < 16; ++c)
-                            ou[c] = __float_as_uint(ov[c] * (alpha[c & 3] * shift));
-                        tmem_st16(tmem + kColO + 16 * hh + lane_base, ou);
+                        for (int c = 0; c < Sh::HP; ++c)
+                            ou[c] = __float_as_uint(ov[c] * (alpha[c % KHH] * shift));
+                        tmem_stn<Sh::HP>(tmem + kColO + Sh::HP * hh + lane_base, ou);
                         ptx::tmem_wait_st();
                         ptx::tc_fence_before();
                     } else {
@@ -661,21 +714,22 @@ __global__ void __launch_bounds__(kThreads, 2)
                 }
             }
             const float sts = st * sc;
-            float x[kHH];
+            float x[KHH];
 #pragma unroll
-            for (int k = 0; k < kHH; ++k) {
-                const float p = kHH * hh + k < G ? ptx::ex2(s_k[k] - m[k]) : 0.f;
+            for (int k = 0; k < KHH; ++k) {
+                const float p = ptx::ex2(s_k[k] - m[k]);       // 0 for padded heads
                 lsum[k] += p;
                 x[k] = p * sts;
             }
-            // W row of token t: 3 E4M3 terms of this warp's 4 heads, one 16-byte block. Each
-            // term but the last is the value rounded to E4M3; the residual times 16 goes on.
+            // W row of token t: 3 E4M3 terms of this warp's KHH heads (4 KHH bytes, zero
+            // padded). Each term but the last is the value rounded to E4M3; the exact residual
+            // times 16 goes on.
             uint32_t w[kJp];
 #pragma unroll
             for (int j = 0; j < kJp; ++j) {
-                uint32_t c2[2];
+                uint32_t c2[KHH / 2];
 #pragma unroll
-                for (int e = 0; e < 2; ++e) {
+                for (int e = 0; e < KHH / 2; ++e) {
                     float v0 = x[2 * e], v1 = x[2 * e + 1];
                     if (j + 1 < kJp) {
                         v0 = e4m3_round(v0);
@@ -686,10 +740,18 @@ __global__ void __launch_bounds__(kThreads, 2)
                     c2[e] = (uint32_t)__nv_cvt_float2_to_fp8x2(make_float2(v0, v1), __NV_SATFINITE,
                                                                 __NV_E4M3);
                 }
-                w[j] = c2[0] | (c2[1] << 16);
+                if constexpr (KHH == 4) w[j] = c2[0] | (c2[1] << 16);
+                else w[j] = c2[0];
             }
-            *reinterpret_cast<uint4 *>(sm.p[pb] + (t >> 3) * 256 + hh * 128 + (t & 7) * 16) =
-                make_uint4(w[0], w[1], w[2], 0u);
+            {
+                // the warp's first output column HP hh: 16-column block and byte within it
+                uint8_t *row = sm.p[pb] + (t >> 3) * Sh::GS + ((Sh::HP * hh) >> 4) * 128 +
+                               (t & 7) * 16 + ((Sh::HP * hh) & 15);
+                if constexpr (KHH == 4)
+                    *reinterpret_cast<uint4 *>(row) = make_uint4(w[0], w[1], w[2], 0u);
+                else
+                    *reinterpret_cast<uint2 *>(row) = make_uint2(w[0] | (w[1] << 16), w[2]);
+            }
             // The output MMAs read whole 32-token steps of the tile: rows past the end of the
             // sequence hold stale bytes (possibly NaN codes), so zero them.
             if (hh == 0 && !valid && t < ((nvalid + 31) & ~31)) {
@@ -702,18 +764,18 @@ __global__ void __launch_bounds__(kThreads, 2)
             if (lane == 0) ptx::mbar_arrive(&sm.p_full[pb]);
         }
         // O = (O_0 + O_1 / 16 + O_2 / 256) * inv once every output MMA is done
-        float o[kHH];
+        float o[KHH];
 #pragma unroll
-        for (int k = 0; k < kHH; ++k) o[k] = 0.f;
+        for (int k = 0; k < KHH; ++k) o[k] = 0.f;
         if (ok && carried) {
             if (observe(n_tiles - 1)) {
                 ptx::tc_fence_after();
-                float ov[16];
-                ptx::tmem_ld16(tmem + kColO + 16 * hh + lane_base, ov);
+                float ov[Sh::HP];
+                tmem_ldn<Sh::HP>(tmem + kColO + Sh::HP * hh + lane_base, ov);
                 ptx::tc_fence_before();
 #pragma unroll
-                for (int k = 0; k < kHH; ++k)
-                    o[k] = fmaf(ov[8 + k], 1.f / 256.f, fmaf(ov[4 + k], 1.f / 16.f, ov[k])) * inv;
+                for (int k = 0; k < KHH; ++k)
+                    o[k] = fmaf(ov[2 * KHH + k], 1.f / 256.f, fmaf(ov[KHH + k], 1.f / 16.f, ov[k])) * inv;
             } else {
                 carried = false;
             }
@@ -723,20 +785,20 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1)
 #pragma unroll
-            for (int k = 0; k < kHH; ++k) lsum[k] += __shfl_xor_sync(0xffffffffu, lsum[k], off);
+            for (int k = 0; k < KHH; ++k) lsum[k] += __shfl_xor_sync(0xffffffffu, lsum[k], off);
         const int rb = n_tiles & 1;
         if (lane == 0) {
 #pragma unroll
-            for (int k = 0; k < kHH; ++k) sm.red[rb][warp][k] = lsum[k];
+            for (int k = 0; k < KHH; ++k) sm.red[rb][warp][k] = lsum[k];
         }
         if (ptx::bar_and(kBarComputeAnd, kComputeThreads, ok && carried)) {
 #pragma unroll
-            for (int k = 0; k < kHH; ++k) {
-                const int h = kHH * hh + k;
+            for (int k = 0; k < KHH; ++k) {
+                const int h = KHH * hh + k;
                 if (h >= G) continue;
                 float lt = 0.f;
 #pragma unroll
-                for (int w = 0; w < 4; ++w) lt += sm.red[rb][kHH * hh + w][k];
+                for (int w = 0; w < 4; ++w) lt += sm.red[rb][kQuarters * hh + w][k];
                 const float val = o[k] / lt;
                 const size_t bh = (size_t)b * geo.Hq + g * G + h;
                 if (a.direct_out) {
@@ -858,6 +920,27 @@ bool encode2d(CUtensorMap *map, CUtensorMapDataType type, const void *base, uint
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The decode for one head count per compute warp: 2 for groups of up to 4 query heads, else 4.
+template <int KHH>
+cudaError_t launch_shape(const DecodeArgs &a, const CUtensorMap &cmap, const CUtensorMap &wmap,
+                         const CUtensorMap &qmap, const float *v_scales) {
+    const Geometry &g = a.geo;
+    const size_t smem = sizeof(Smem8) + 1024;
+    static bool configured = false;
+    if (!configured) {
+        cudaError_t e = cudaFuncSetAttribute(decode_fp8_kernel<KHH>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(g.S, g.Hkv, g.B);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = a.stream;
+    return cudaLaunchKernelEx(&cfg, decode_fp8_kernel<KHH>, cmap, wmap, qmap, a, v_scales);
+}
+
 }  // namespace
 
 cudaError_t launch_decode_fp8(const DecodeArgs &a, const float *v_scales) {
@@ -878,20 +961,8 @@ cudaError_t launch_decode_fp8(const DecodeArgs &a, const float *v_scales) {
                       64, (uint32_t)g.G, CU_TENSOR_MAP_SWIZZLE_128B))
             return cudaErrorInvalidValue;
     }
-    const size_t smem = sizeof(Smem8) + 1024;
-    static bool configured = false;
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(decode_fp8_kernel,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        configured = true;
-    }
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(g.S, g.Hkv, g.B);
-    cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = a.stream;
-    return cudaLaunchKernelEx(&cfg, decode_fp8_kernel, cmap, wmap, qmap, a, v_scales);
+    return g.G <= 2 * 2 ? launch_shape<2>(a, cmap, wmap, qmap, v_scales)
+                        : launch_shape<4>(a, cmap, wmap, qmap, v_scales);
 }
 
 cudaError_t launch_append_fp8(const Geometry &g, const uint16_t *v_new, const int32_t *block_table,
