@@ -56,6 +56,8 @@ def parse_args():
                    help="decode with the composed query q = x W^Q W^R (no W^R in the kernel)")
     p.add_argument("--fp8-cache", action="store_true",
                    help="FP8 (E4M3, per-row scale) value cache: quantizing append + FP8 decode")
+    p.add_argument("--num-seqs", type=int, default=0,
+                   help="override the workload's batch size (decode workloads; 0: as defined)")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=10.0)
     return p.parse_args()
@@ -273,6 +275,8 @@ def run_ours(args):
     wl = WORKLOADS[args.workload]
     if args.wr_per_query_head:
         wl = wl.with_(wr_per_query_head=True)
+    if args.num_seqs > 0:
+        wl = wl.with_(num_seqs=args.num_seqs)
     from paper_2606_21848_gb300.multi import job_throughput, max_over_ranks, replica_seed
     x = generate(wl, seed=replica_seed(wl.seed, rank))   # replicas: each rank its own batch
     if wl.q_len > 0:

@@ -181,19 +181,18 @@ __device__ __forceinline__ void pow2_from_exp(int e, float &sc, float &inv) {
     inv = __uint_as_float((uint32_t)(127 - 8 + e) << 23);
 }
 
-// x (0 <= x < 448) rounded to an E4M3 value on the FMA pipe: to 4 significant bits by a
-// Veltkamp split (c = x (2^20 + 1), hi = c - (c - x)), and below 2^-6, where the E4M3 values
-// are the multiples of 2^-9, by adding and subtracting 1.5 * 2^14 (whose spacing is 2^-9). The
-// result is an E4M3 value, so its code conversion is exact and x - hi is the exact residual.
-// (The small values matter: the weight scale follows the largest row scale seen so far, so
-// most weights can sit far below it; leaving them whole to the later terms costs them too many
-// bits at this tolerance.)
+// An E4M3 value next to x (0 <= x < 448), on the FMA pipe: x rounded to 4 significant bits by
+// a Veltkamp split (c = x (2^20 + 1), hv = c - (c - x)), then hv rounded to the multiples of 2^-9
+// by adding and subtracting 1.5 * 2^14 (whose spacing is 2^-9). Above 2^-6 hv is an E4M3 value
+// and already a multiple of 2^-9, so the second rounding keeps it; below, it lands on the E4M3
+// subnormals. The result is exactly representable, so its code conversion is exact, and x minus
+// it is exact and at most x / 16 + 2^-10. (The small values matter: the weight scale follows the
+// largest row scale seen so far, so many weights sit far below it.)
 __device__ __forceinline__ float e4m3_round(float x) {
     // explicit roundings: the compiler must not fuse these into FMAs
     const float c = __fmul_rn(x, 1048577.f);
     const float hv = __fsub_rn(c, __fsub_rn(c, x));
-    const float hs = __fsub_rn(__fadd_rn(x, 24576.f), 24576.f);
-    return x < 0.015625f ? hs : hv;
+    return __fsub_rn(__fadd_rn(hv, 24576.f), 24576.f);
 }
 
 // Byte offset of element (row n, column k) of the query-term operand: [NS rows][128 B],
@@ -278,7 +277,7 @@ __device__ __forceinline__ uint32_t bar_popc(uint32_t id, uint32_t count, bool v
     return r;
 }
 
-template <int KHH>
+template <int KHH, bool kAllLive>
 __global__ void __launch_bounds__(kThreads, 2)
     decode_fp8_kernel(const __grid_constant__ CUtensorMap cmap,
                       const __grid_constant__ CUtensorMap wmap,
@@ -286,6 +285,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                       const float *__restrict__ v_scales) {
     using Sh = Fp8Shape<KHH>;
     extern __shared__ uint8_t smem_raw[];
+    // kAllLive: the group has 2 KHH heads, so no compute warp holds a padded head
     Smem8 &sm = *reinterpret_cast<Smem8 *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                            ~uintptr_t(1023));
     const Geometry &geo = a.geo;
@@ -527,7 +527,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                 ptx::tmem_ld16(tmem + kColR + lane_base, rv);
 #pragma unroll
                 for (int k = 0; k < KHH; ++k)
-                    acc[k] = KHH * hh + k < G ? (hh ? rv[KHH + k] : rv[k]) : 0.f;
+                    acc[k] = (kAllLive || KHH * hh + k < G) ? (hh ? rv[KHH + k] : rv[k]) : 0.f;
                 ptx::tc_fence_before();
             }
         } else {
@@ -580,7 +580,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         float m[KHH], thr[KHH], lsum[KHH];
 #pragma unroll
         for (int k = 0; k < KHH; ++k) {
-            const bool live = KHH * hh + k < G;
+            const bool live = kAllLive || KHH * hh + k < G;
             m[k] = live ? -INFINITY : 0.f;
             thr[k] = live ? -INFINITY : INFINITY;
             lsum[k] = 0.f;
@@ -639,7 +639,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                 const float d = fmaf(fmaf(fmaf(sv[3 * KHH + k], 1.f / 16.f, sv[2 * KHH + k]), 1.f / 16.f,
                                           sv[KHH + k]),
                                      1.f / 16.f, sv[k]);
-                s_k[k] = (valid && KHH * hh + k < G) ? d * (invq[k] * st) : -INFINITY;
+                s_k[k] = (valid && (kAllLive || KHH * hh + k < G)) ? d * (invq[k] * st) : -INFINITY;
                 grow = grow || s_k[k] > thr[k];
             }
             // row scales are non-negative: their bits order as the values do
@@ -682,7 +682,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                 bool rescale = shift != 1.f;
 #pragma unroll
                 for (int k = 0; k < KHH; ++k) {
-                    const bool live = KHH * hh + k < G;
+                    const bool live = kAllLive || KHH * hh + k < G;
                     const float mn = fmaxf(m[k], tmax[k]);
                     alpha[k] = live ? ptx::ex2(m[k] - mn) : 1.f;
                     m[k] = live ? mn : m[k];
@@ -920,15 +920,16 @@ bool encode2d(CUtensorMap *map, CUtensorMapDataType type, const void *base, uint
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// The decode for one head count per compute warp: 2 for groups of up to 4 query heads, else 4.
-template <int KHH>
+// The decode for one head count per compute warp (2 for groups of up to 4 query heads, else 4)
+// and whether every compute warp's heads are real (groups of exactly 4 or 8).
+template <int KHH, bool kAllLive>
 cudaError_t launch_shape(const DecodeArgs &a, const CUtensorMap &cmap, const CUtensorMap &wmap,
                          const CUtensorMap &qmap, const float *v_scales) {
     const Geometry &g = a.geo;
     const size_t smem = sizeof(Smem8) + 1024;
     static bool configured = false;
     if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(decode_fp8_kernel<KHH>,
+        cudaError_t e = cudaFuncSetAttribute(decode_fp8_kernel<KHH, kAllLive>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         configured = true;
@@ -938,7 +939,7 @@ cudaError_t launch_shape(const DecodeArgs &a, const CUtensorMap &cmap, const CUt
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = a.stream;
-    return cudaLaunchKernelEx(&cfg, decode_fp8_kernel<KHH>, cmap, wmap, qmap, a, v_scales);
+    return cudaLaunchKernelEx(&cfg, decode_fp8_kernel<KHH, kAllLive>, cmap, wmap, qmap, a, v_scales);
 }
 
 }  // namespace
@@ -961,8 +962,10 @@ cudaError_t launch_decode_fp8(const DecodeArgs &a, const float *v_scales) {
                       64, (uint32_t)g.G, CU_TENSOR_MAP_SWIZZLE_128B))
             return cudaErrorInvalidValue;
     }
-    return g.G <= 2 * 2 ? launch_shape<2>(a, cmap, wmap, qmap, v_scales)
-                        : launch_shape<4>(a, cmap, wmap, qmap, v_scales);
+    if (g.G == 8) return launch_shape<4, true>(a, cmap, wmap, qmap, v_scales);
+    if (g.G == 4) return launch_shape<2, true>(a, cmap, wmap, qmap, v_scales);
+    return g.G < 4 ? launch_shape<2, false>(a, cmap, wmap, qmap, v_scales)
+                   : launch_shape<4, false>(a, cmap, wmap, qmap, v_scales);
 }
 
 cudaError_t launch_append_fp8(const Geometry &g, const uint16_t *v_new, const int32_t *block_table,
