@@ -280,35 +280,45 @@ kl_status kl_latent_decode(const kl_latent_shape *shape, const void *q, const vo
                            int32_t *err, kl_stream_t stream);
 
 /*
- * FP8 value cache: the low-precision value cache of the scope table (orthogonal to the paper's
- * method and compatible with it: the same value rows, stored in half the bytes). Each cached row
- * is D OCP FP8 E4M3 codes (1 sign, 4 exponent bits of bias 7, 3 mantissa bits; largest value
- * 448) and one fp32 scale, the row's values being scale * value(code):
- *   codes: [num_pages][Hkv][P][D] uint8,   scales: [num_pages][Hkv][P] fp32.
- * head_dim 128 only.
+ * FP8 value cache (not in the paper; §3 notes that the value-only cache is orthogonal to other
+ * cache-reduction methods, and a quantized cache is one): the same value rows stored in about
+ * half the bytes. Each cached row is D OCP FP8 E4M3 codes (1 sign, 4 exponent bits of bias 7,
+ * 3 mantissa bits; subnormals m/8 * 2^-6; largest finite value 448) and one fp32 scale, the
+ * row's values being scale * value(code):
+ *   codes: [num_pages][Hkv][P][D] uint8,   scales: [num_pages][Hkv][P] fp32,
+ * both caller-owned device memory, 16-byte aligned (KL_ERR_INVALID_ARG otherwise). head_dim 128
+ * only (KL_ERR_UNSUPPORTED otherwise). The library never writes the code 0x7F / 0xFF (NaN); a
+ * cache holding them yields NaN outputs.
  *
- * kl_append_v_fp8: quantize v_new[b][g] (bf16) into row positions[b] -- scale = max |v| / 448
- * in fp32, code_j = E4M3(v_j / scale) rounded to nearest even and saturating (an all-zero row
- * gets scale 0); position and page checks as in kl_append_v.
+ * kl_append_v_fp8: quantize v_new[b][g] (bf16, [B][Hkv][D]) into row positions[b] of sequence
+ * b -- scale = max |v| / 448 in fp32, code_j = E4M3(v_j / scale) rounded to nearest even and
+ * saturating (an all-zero row gets scale 0 and zero codes). A position outside the block table
+ * raises KL_FLAG_BAD_POSITION, a page id outside the pool KL_FLAG_BAD_PAGE, in *err; that row is
+ * skipped.
  */
 kl_status kl_append_v_fp8(const kl_shape *shape, const void *v_new, const int32_t *block_table,
                           const int32_t *positions, void *v_codes, float *v_scales, int32_t *err,
                           kl_stream_t stream);
 
-/* Quantize a whole bf16 value cache [num_pages][Hkv][P][128] into the FP8 layout, row by row,
- * with the arithmetic of kl_append_v_fp8 (e.g. to move an existing cache to FP8). */
+/* Quantize a whole bf16 value cache [num_pages][Hkv][P][128] (caller-owned device memory,
+ * 16-byte aligned) into the FP8 layout, row by row, with the arithmetic of kl_append_v_fp8 (e.g.
+ * to move an existing cache to FP8). The results are bit-identical to appending every row. */
 kl_status kl_quantize_cache_fp8(const kl_shape *shape, const void *v_cache, void *v_codes,
                                 float *v_scales, kl_stream_t stream);
 
 /*
- * kl_decode_attention_fp8: the keyless decode of kl_decode_attention over the FP8 cache (each
- * cached value is scale * value(code)), on the tensor cores: the codes are widened exactly to
- * half precision in shared memory, scores and outputs accumulate in fp32, the routed query and
- * the softmax weights enter as hi + lo half pairs. W^R per value head (wr_per_query_head = 0)
- * or w_r == NULL (composed query); at most 8 query heads per value head; page size a power of
- * two from 16 to 128; compute capability 10.3 (KL_ERR_UNSUPPORTED otherwise). num_splits,
- * workspace (kl_decode_workspace_size), out and flags as in kl_decode_attention; with more than
- * one split the states are merged by the combine kernel.
+ * kl_decode_attention_fp8: the keyless decode of kl_decode_attention (routing §2.2, one softmax
+ * over the cached value rows, each row serving score and output, §3) over the FP8 cache, each
+ * cached value being scale * value(code). On the tensor cores with E4M3 products straight on
+ * the stored codes and fp32 accumulation; the routed query and the softmax weights enter as
+ * sums of E4M3 terms (4 and 3 terms, about 16 and 12 significant bits), each row's scale
+ * multiplies its score and its weight. W^R per value head (wr_per_query_head = 0) or
+ * w_r == NULL (q is then the composed query); at most 8 query heads per value head; page size
+ * 16, 32, 64 or 128; compute capability 10.3 (KL_ERR_UNSUPPORTED otherwise). q, w_r, out,
+ * num_splits, the workspace (kl_decode_workspace_size of the same shape and split count), the
+ * output layout and the error flags are those of kl_decode_attention; with more than one split
+ * the split states are merged by the combine kernel in a second launch on the same stream.
+ * Returns after enqueueing; nothing is allocated or synchronized.
  */
 kl_status kl_decode_attention_fp8(const kl_shape *shape, const void *q, const void *w_r,
                                   const void *v_codes, const float *v_scales,
