@@ -1,5 +1,5 @@
 // Keyless decode over an FP8 value cache (E4M3 codes, one fp32 scale per cached row), on the
-// tensor cores for sm_103a; and the quantizing append.
+// tensor cores for sm_103a.
 //
 // Same method and split plan as the bf16 decode (routing q_r = q W^R, Section 2.2; one softmax
 // over the cached value rows, each row used for the score and for the output, Section 3). The
@@ -824,73 +824,6 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
 }
 
-// Quantizing append: one CTA per sequence, one warp per value head; lane j holds dims
-// 4j .. 4j + 3. scale = max |v| / 448 (fp32), code = E4M3(v / scale) rounded to nearest even,
-// saturating.
-__global__ void __launch_bounds__(256)
-    append_fp8_kernel(int Hkv, int P, int num_pages, int max_pages, const uint16_t *__restrict__ v_new,
-                      const int32_t *__restrict__ block_table, const int32_t *__restrict__ positions,
-                      uint8_t *__restrict__ codes, float *__restrict__ scales, int32_t *err) {
-    const int b = blockIdx.x, lane = threadIdx.x & 31;
-    const int pos = positions[b];
-    if (pos < 0 || pos >= max_pages * P) {
-        if (threadIdx.x == 0) raise_flag(err, KL_FLAG_BAD_POSITION);
-        return;
-    }
-    const int page = block_table[(size_t)b * max_pages + pos / P];
-    if (page < 0 || page >= num_pages) {
-        if (threadIdx.x == 0) raise_flag(err, KL_FLAG_BAD_PAGE);
-        return;
-    }
-    for (int g = threadIdx.x >> 5; g < Hkv; g += blockDim.x >> 5) {
-        const uint2 w = reinterpret_cast<const uint2 *>(v_new + ((size_t)b * Hkv + g) * kD)[lane];
-        const float v[4] = {bf16lo(w.x), bf16hi(w.x), bf16lo(w.y), bf16hi(w.y)};
-        float amax = fmaxf(fmaxf(fabsf(v[0]), fabsf(v[1])), fmaxf(fabsf(v[2]), fabsf(v[3])));
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
-        const float s = __fdiv_rn(amax, 448.0f);
-        uint32_t packed = 0;
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const uint32_t c = s > 0.f
-                                   ? (uint32_t)__nv_cvt_float_to_fp8(__fdiv_rn(v[e], s), __NV_SATFINITE, __NV_E4M3)
-                                   : 0u;
-            packed |= c << (8 * e);
-        }
-        const size_t row = ((size_t)page * Hkv + g) * P + pos % P;
-        reinterpret_cast<uint32_t *>(codes + row * kD)[lane] = packed;
-        if (lane == 0) scales[row] = s;
-    }
-}
-
-// Quantize a whole bf16 cache [rows][128] into codes [rows][128] and row scales [rows]: one warp
-// per row, the same arithmetic as the append.
-__global__ void __launch_bounds__(256)
-    quantize_rows_kernel(size_t rows, const uint16_t *__restrict__ v, uint8_t *__restrict__ codes,
-                         float *__restrict__ scales) {
-    const int lane = threadIdx.x & 31;
-    const size_t warps = (size_t)gridDim.x * (blockDim.x >> 5);
-    for (size_t row = (size_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); row < rows;
-         row += warps) {
-        const uint2 w = reinterpret_cast<const uint2 *>(v + row * kD)[lane];
-        const float x[4] = {bf16lo(w.x), bf16hi(w.x), bf16lo(w.y), bf16hi(w.y)};
-        float amax = fmaxf(fmaxf(fabsf(x[0]), fabsf(x[1])), fmaxf(fabsf(x[2]), fabsf(x[3])));
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
-        const float s = __fdiv_rn(amax, 448.0f);
-        uint32_t packed = 0;
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const uint32_t c = s > 0.f
-                                   ? (uint32_t)__nv_cvt_float_to_fp8(__fdiv_rn(x[e], s), __NV_SATFINITE, __NV_E4M3)
-                                   : 0u;
-            packed |= c << (8 * e);
-        }
-        reinterpret_cast<uint32_t *>(codes + row * kD)[lane] = packed;
-        if (lane == 0) scales[row] = s;
-    }
-}
-
 // ------------------------------------------------------------------------ host side ------
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -966,24 +899,6 @@ cudaError_t launch_decode_fp8(const DecodeArgs &a, const float *v_scales) {
     if (g.G == 4) return launch_shape<2, true>(a, cmap, wmap, qmap, v_scales);
     return g.G < 4 ? launch_shape<2, false>(a, cmap, wmap, qmap, v_scales)
                    : launch_shape<4, false>(a, cmap, wmap, qmap, v_scales);
-}
-
-cudaError_t launch_append_fp8(const Geometry &g, const uint16_t *v_new, const int32_t *block_table,
-                              const int32_t *positions, uint8_t *codes, float *scales, int32_t *err,
-                              cudaStream_t stream) {
-    if (g.B == 0) return cudaSuccess;
-    append_fp8_kernel<<<g.B, 256, 0, stream>>>(g.Hkv, g.P, g.num_pages, g.max_pages, v_new,
-                                               block_table, positions, codes, scales, err);
-    return cudaGetLastError();
-}
-
-cudaError_t launch_quantize_fp8(size_t rows, const uint16_t *v, uint8_t *codes, float *scales,
-                                cudaStream_t stream) {
-    if (rows == 0) return cudaSuccess;
-    const size_t blocks = (rows + 7) / 8;
-    const unsigned grid = (unsigned)(blocks < 65535 * 16 ? blocks : 65535 * 16);
-    quantize_rows_kernel<<<grid, 256, 0, stream>>>(rows, v, codes, scales);
-    return cudaGetLastError();
 }
 
 }  // namespace kl
