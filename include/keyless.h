@@ -85,7 +85,11 @@ typedef struct kl_decode_options {
      * state there -- partial_o [B][Hq][S][D] fp32 (normalized) and partial_ml [B][Hq][S][2]
      * fp32 ({m, l}, the layout kl_combine reads) -- and neither merges nor writes `out`
      * (which may be NULL); no workspace is needed. This exposes the states for a later
-     * kl_combine, e.g. after gathering the states of sequence shards from several devices. */
+     * kl_combine, e.g. after gathering the states of sequence shards from several devices.
+     * Split s holds tokens [s C, (s + 1) C) of every sequence, C = ceil(max_pages_per_seq * P
+     * / S) rounded up to a multiple of 128, with S = kl_decode_num_splits(shape, num_splits);
+     * a split past a sequence's end has m = -inf, l = 0 and a zero row. m is the split's largest
+     * score (natural-log units, scale included) and l = sum_t exp(s_t - m). */
     float *partial_o;
     float *partial_ml;
 } kl_decode_options;

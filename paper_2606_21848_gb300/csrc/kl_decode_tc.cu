@@ -1,7 +1,7 @@
 // Tensor-core split-sequence decode for sm_103a: TMA page gathers into a shared-memory ring,
 // tcgen05 MMAs with TMEM accumulators, warp-specialized roles.
 //
-// One CTA per (split, value head g, sequence b); head_dim 128, up to 8 query heads per value
+// One CTA per (run of splits, value head g, sequence b); head_dim 128, up to 8 query heads per value
 // group. The value-space routing (Section 2.2: q_r = q W^R) runs first, as tensor-core MMAs on
 // W^R tiles that stream through the ring, into a split-bf16 operand (q_r * scale * log2 e =
 // hi + lo, both bf16) for the G heads of the group.
@@ -100,6 +100,7 @@ struct __align__(1024) Smem {
     // During the routing prologue the first one holds the raw query, fp32 [k][8].
     uint8_t p[2][kTile * kN * 2];
     float red[2][kComputeWarps][kNG];
+    float lred[kComputeWarps][kNG];    // row sums of a split closed inside a CTA's run
     uint64_t full[Cfg<kStandard>::kStages], empty[Cfg<kStandard>::kStages];
     uint64_t s_full[2], s_empty[2], p_full[2], o_full[2], o_empty[2];
     uint64_t qr_full, q_ready, r_full, drain, drain2, merge_full;
@@ -305,7 +306,9 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int g, int n
     }
 }
 
-template <bool kStandard>
+// kPerSplit: the CTA runs several splits and writes a state for each (only when the caller
+// gets the split states, or the combine kernel merges them, and spc > 1).
+template <bool kStandard, bool kPerSplit>
 __global__ void __launch_bounds__(kThreads, 2)
     decode_tc_kernel(const __grid_constant__ CUtensorMap vmap,
                      const __grid_constant__ CUtensorMap kmap,
@@ -318,7 +321,10 @@ __global__ void __launch_bounds__(kThreads, 2)
                                    ~uintptr_t(1023));
 
     const Geometry &geo = a.geo;
-    const int split = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+    // A CTA runs geo.spc consecutive splits of one (b, g) (one split unless a launch of one CTA
+    // per split would not fit in one wave); it keeps one softmax state per split.
+    const int cta = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+    const int split0 = cta * geo.spc;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int G = geo.G;
 
@@ -338,7 +344,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     // entries, 32 pages per warp load, two batches.
     const int L_raw = a.seq_lens[b];
     const int pos_raw = a.v_new ? a.positions[b] : -1;
-    const int t_begin = split * geo.chunk;
+    const int t_begin = split0 * geo.chunk;
     const int first_page = t_begin / geo.P;
     const int32_t *bt = a.block_table + (size_t)b * geo.max_pages;
     int bt_cur = -1, bt_nxt = -1;
@@ -386,17 +392,17 @@ __global__ void __launch_bounds__(kThreads, 2)
 
     int L = L_raw;
     if (L < 0 || L > geo.max_pages * geo.P) {
-        if (tid == 0 && split == 0 && g == 0) raise_flag(a.err, KL_FLAG_BAD_LENGTH);
+        if (tid == 0 && cta == 0 && g == 0) raise_flag(a.err, KL_FLAG_BAD_LENGTH);
         L = 0;
     }
-    const int t_end = min(t_begin + geo.chunk, L);
+    const int t_end = min(t_begin + geo.spc * geo.chunk, L);
     const int n_tiles = t_end > t_begin ? (t_end - t_begin + kTile - 1) / kTile : 0;
 
-    // Fused append: the CTA whose split holds row positions[b] owns the current token's row.
+    // Fused append: the CTA whose splits hold row positions[b] owns the current token's row.
     const bool pos_ok = pos_raw >= 0 && pos_raw < geo.max_pages * geo.P;
-    if (a.v_new && !pos_ok && tid == 0 && split == 0 && g == 0)
+    if (a.v_new && !pos_ok && tid == 0 && cta == 0 && g == 0)
         raise_flag(a.err, KL_FLAG_BAD_POSITION);
-    const bool app_owner = a.v_new && pos_ok && pos_raw / geo.chunk == split;
+    const bool app_owner = a.v_new && pos_ok && pos_raw / (geo.chunk * geo.spc) == cta;
 
     // Empty split, no pipeline: in the split-state layout an empty state; otherwise the split
     // of a zero-length sequence writes the zero output, and the empty splits of a longer
@@ -416,7 +422,7 @@ __global__ void __launch_bounds__(kThreads, 2)
             for (int h = 0; h < G; ++h) {
                 const size_t bh = (size_t)b * geo.Hq + g * G + h;
                 if (a.merge_inside) {
-                    if (L == 0 && split == 0) {
+                    if (L == 0 && cta == 0) {
                         if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * kD + tid] = 0.f;
                         else static_cast<__nv_bfloat16 *>(a.out)[bh * kD + tid] = __float2bfloat16_rn(0.f);
                     }
@@ -424,11 +430,13 @@ __global__ void __launch_bounds__(kThreads, 2)
                     if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * kD + tid] = 0.f;
                     else static_cast<__nv_bfloat16 *>(a.out)[bh * kD + tid] = __float2bfloat16_rn(0.f);
                 } else {
-                    const size_t slot = bh * geo.S + split;
-                    a.part_o[slot * kD + tid] = 0.f;
-                    if (tid == 0) {
-                        a.part_ml[slot * 2] = -INFINITY;
-                        a.part_ml[slot * 2 + 1] = 0.f;
+                    for (int sp = split0; sp < min(split0 + geo.spc, geo.S); ++sp) {
+                        const size_t slot = bh * geo.S + sp;
+                        a.part_o[slot * kD + tid] = 0.f;
+                        if (tid == 0) {
+                            a.part_ml[slot * 2] = -INFINITY;
+                            a.part_ml[slot * 2 + 1] = 0.f;
+                        }
                     }
                 }
             }
@@ -732,11 +740,64 @@ __global__ void __launch_bounds__(kThreads, 2)
             return true;
         };
 
+        // Splits inside the CTA's run: tile i opens split split0 + i / tps. When the caller
+        // gets the split states (or the combine kernel merges them), each split starts from a
+        // fresh state (reference -inf, so the first alpha is 0 and its O starts over) and the
+        // closed split's state is written once its last O is in. When this kernel merges the
+        // splits itself, the run's splits are folded as they go: the online softmax simply
+        // continues across the boundary (the merge of adjacent states is associative), and
+        // the run leaves one state for the final merge.
+        const int tps = geo.chunk / kTile;
+        // The state of split sp from the running o, lsum and m (all of its O folded in).
+        auto emit_state = [&](int sp) {
+            float l[kNG];
+#pragma unroll
+            for (int h = 0; h < kNG; ++h) l[h] = lsum[h];
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1)
+#pragma unroll
+                for (int h = 0; h < kNG; ++h) l[h] += __shfl_xor_sync(0xffffffffu, l[h], off);
+            if (lane == 0) {
+#pragma unroll
+                for (int h = 0; h < kNG; ++h) sm.lred[warp][h] = l[h];
+            }
+            ptx::bar_sync(kBarCompute, kTile);
+#pragma unroll
+            for (int h = 0; h < kNG; ++h) {
+                if (h >= G) continue;
+                float lt = 0.f;
+#pragma unroll
+                for (int w = 0; w < kComputeWarps; ++w) lt += sm.lred[w][h];
+                const size_t slot = ((size_t)b * geo.Hq + g * G + h) * geo.S + sp;
+                a.part_o[slot * kD + t] = o[h] / lt;
+                if (t == 0) {
+                    a.part_ml[slot * 2] = m[h] * kLn2;
+                    a.part_ml[slot * 2 + 1] = lt;
+                }
+            }
+            ptx::bar_sync(kBarCompute, kTile);      // lred is free for the next split
+        };
+
         for (int i = 0; ok && i < n_tiles; ++i) {
             const int sb = i & 1;
             if (!ptx::bar_and(kBarComputeAnd, kTile, wait(&sm.s_full[sb], (i >> 1) & 1))) {
                 ok = false;
                 break;
+            }
+            const bool opens = kPerSplit && i > 0 && i % tps == 0;   // tile i opens a split
+            if (opens) {
+                // close the previous split: its last O, its state, then a fresh state
+                if (!correct(i - 1, alpha_prev)) {
+                    ok = false;
+                    break;
+                }
+                emit_state(split0 + i / tps - 1);
+#pragma unroll
+                for (int h = 0; h < kNG; ++h) {
+                    o[h] = 0.f;
+                    lsum[h] = 0.f;
+                    m[h] = -INFINITY;
+                }
             }
             ptx::tc_fence_after();
             float sv[16];
@@ -806,7 +867,7 @@ __global__ void __launch_bounds__(kThreads, 2)
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&sm.p_full[sb]);
 
-            if (i >= 1 && !correct(i - 1, alpha_prev)) { ok = false; break; }
+            if (i >= 1 && !opens && !correct(i - 1, alpha_prev)) { ok = false; break; }
             alpha_prev = alpha;
         }
         if (ok) ok = correct(n_tiles - 1, alpha_prev);
@@ -824,9 +885,11 @@ __global__ void __launch_bounds__(kThreads, 2)
             }
             ptx::bar_sync(kBarCompute, kTile);
             {
-                // splits of this (b, g) that hold tokens; one split writes the output itself
-                const int n_u = (L + geo.chunk - 1) / geo.chunk;
-                const bool write_out = a.direct_out || (a.merge_inside && n_u == 1);
+                // Merged here: one state per CTA run that holds tokens (slot cta; a single one
+                // writes the output itself). Otherwise: the state of the split closed last.
+                const int n_cta_u = (L + geo.chunk * geo.spc - 1) / (geo.chunk * geo.spc);
+                const int sp_last = a.merge_inside ? cta : split0 + (n_tiles - 1) / tps;
+                const bool write_out = a.direct_out || (a.merge_inside && n_cta_u == 1);
                 float lt[kNG];
 #pragma unroll
                 for (int h = 0; h < kNG; ++h) {
@@ -843,21 +906,32 @@ __global__ void __launch_bounds__(kThreads, 2)
                         if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * kD + t] = val;
                         else static_cast<__nv_bfloat16 *>(a.out)[bh * kD + t] = __float2bfloat16_rn(val);
                     } else {
-                        const size_t slot = bh * geo.S + split;
+                        const size_t slot = bh * geo.S + sp_last;
                         a.part_o[slot * kD + t] = val;
                         if (t == 0) {
                             a.part_ml[slot * 2] = m[h] * kLn2;
                             a.part_ml[slot * 2 + 1] = lt[h];
                         }
+                        // splits of the run past the sequence's end: empty states
+                        if (!a.merge_inside) {
+                            for (int sp = sp_last + 1; sp < min(split0 + geo.spc, geo.S); ++sp) {
+                                const size_t es = bh * geo.S + sp;
+                                a.part_o[es * kD + t] = 0.f;
+                                if (t == 0) {
+                                    a.part_ml[es * 2] = -INFINITY;
+                                    a.part_ml[es * 2 + 1] = 0.f;
+                                }
+                            }
+                        }
                     }
                 }
                 if (a.merge_inside && !write_out) {
-                    // The last split of (b, g) to finish merges the n_u states (as kl_combine).
+                    // The last CTA of (b, g) to finish merges the n_cta_u states (as kl_combine).
                     ptx::bar_sync(kBarCompute, kTile);
                     if (t == 0)
-                        sm.is_last = arrive_last(a.counters + (size_t)b * geo.Hkv + g, n_u) ? 1 : 0;
+                        sm.is_last = arrive_last(a.counters + (size_t)b * geo.Hkv + g, n_cta_u) ? 1 : 0;
                     ptx::bar_sync(kBarCompute, kTile);
-                    if (sm.is_last) merge_states(sm, a, b, g, n_u, t, warp, lane, wait);
+                    if (sm.is_last) merge_states(sm, a, b, g, n_cta_u, t, warp, lane, wait);
                 }
             }
         }
@@ -900,6 +974,26 @@ bool make_map(CUtensorMap *map, const void *base, uint64_t rows, uint32_t box_ro
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+template <bool kStandard, bool kPerSplit>
+cudaError_t launch_kernel(const DecodeArgs &la, const CUtensorMap &vmap, const CUtensorMap &kmap,
+                          const CUtensorMap &wmap, const CUtensorMap &qmap) {
+    const Geometry &g = la.geo;
+    const size_t smem = sizeof(Smem<kStandard>) + 1024;
+    static bool configured = false;
+    if (!configured) {
+        cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<kStandard, kPerSplit>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((g.S + g.spc - 1) / g.spc, g.Hkv, g.B);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = la.stream;
+    return cudaLaunchKernelEx(&cfg, decode_tc_kernel<kStandard, kPerSplit>, vmap, kmap, wmap, qmap, la);
+}
+
 template <bool kStandard>
 cudaError_t launch(const DecodeArgs &a) {
     const Geometry &g = a.geo;
@@ -917,20 +1011,18 @@ cudaError_t launch(const DecodeArgs &a) {
         if (!make_map(&wmap, a.w_r, hw * kD, kD)) return cudaErrorInvalidValue;
         if (!make_map(&qmap, a.q, (uint64_t)g.B * g.Hq, (uint32_t)g.G)) return cudaErrorInvalidValue;
     }
-    const size_t smem = sizeof(Smem<kStandard>) + 1024;
-    static bool configured = false;
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<kStandard>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        configured = true;
-    }
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(g.S, g.Hkv, g.B);
-    cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = a.stream;
-    return cudaLaunchKernelEx(&cfg, decode_tc_kernel<kStandard>, vmap, kmap, wmap, qmap, a);
+    // Splits per CTA: one, unless one CTA per split would overflow a wave of two CTAs per SM
+    // while the (b, g) units alone would not fill it (few long sequences split many ways): then
+    // the fewest consecutive splits per CTA that fit the wave.
+    DecodeArgs la = a;
+    const int64_t units = (int64_t)g.B * g.Hkv, slots = 2 * (int64_t)device_sm_count();
+    int spc = 1;
+    if (g.S > 1 && units < slots)
+        while ((int64_t)((g.S + spc - 1) / spc) * units > slots) ++spc;
+    la.geo.spc = spc;
+    const bool per_split = spc > 1 && !a.merge_inside && !a.direct_out;
+    return per_split ? launch_kernel<kStandard, true>(la, vmap, kmap, wmap, qmap)
+                     : launch_kernel<kStandard, false>(la, vmap, kmap, wmap, qmap);
 }
 
 }  // namespace

@@ -18,6 +18,7 @@ struct Geometry {
     float scale;       // lambda / sqrt(d_k)
     int S;             // split count
     int chunk;         // tokens per split (a multiple of 128)
+    int spc = 1;       // splits per CTA of the tensor-core decode (consecutive, same (b, g))
 };
 
 // Arguments of a decode launch (keyless or the standard K+V comparison).

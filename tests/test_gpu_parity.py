@@ -395,3 +395,46 @@ def test_composed_query_fused_step_appends_and_decodes():
     want = oracle.decode(bf16_bits(x["q"]), w_eye, cache, x["block_table"].numpy(),
                          x["seq_lens"].numpy(), scale=_gpu.default_scale(x))
     assert_parity(out.cpu().numpy(), want, "composed query, fused step")
+
+
+# ------------------------------------------------------------------ split-state outputs -----
+
+@pytest.mark.parametrize("splits", [3, 64])
+def test_split_states_match_oracle_partial_states(splits):
+    """The split states the caller asks for (partial_o / partial_ml): every split's normalized
+    output, largest score and exponent sum against the oracle's states of the same token
+    ranges, then their merge by kl_combine. At 64 splits of a 2-sequence, 8-value-head batch
+    one CTA runs several consecutive splits and writes a state at each split boundary."""
+    x = tiny(B=2, Hq=32, Hkv=8, D=128, P=16, lens=(2000, 4096), seed=23)
+    k = _kernel_or_skip("tensor", x)
+    g = to_dev(x)
+    sh = shape_of(x)
+    B, Hq, D = x["q"].shape
+    S = kl.kl_decode_num_splits(sh, splits)
+    lmax = x["block_table"].shape[1] * 16
+    chunk = -(-(-(-lmax // S)) // 128) * 128            # ceil(lmax / S), rounded up to 128
+    po = torch.full((B, Hq, S, D), float("nan"), dtype=torch.float32, device=_gpu.dev())
+    pml = torch.full((B, Hq, S, 2), float("nan"), dtype=torch.float32, device=_gpu.dev())
+    err = torch.zeros(1, dtype=torch.int32, device=_gpu.dev())
+    kl.kl_decode_attention_ex(sh, g["q"], g["w_r"], g["v_cache"], g["block_table"],
+                              g["seq_lens"], kl.decode_options(splits, k, po, pml), None,
+                              kl.KL_FP32, None, err)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    want_o, want_ml = oracle.decode_partial(bf16_bits(x["q"]), bf16_bits(x["w_r"]),
+                                            bf16_bits(x["v_cache"]), x["block_table"].numpy(),
+                                            x["seq_lens"].numpy(), scale=_gpu.default_scale(x),
+                                            chunk=chunk, num_splits=S)
+    got_o, got_ml = po.cpu().numpy().astype(np.float64), pml.cpu().numpy().astype(np.float64)
+    full = want_ml[..., 1] > 0
+    assert np.array_equal(got_ml[..., 1] > 0, full), "empty splits differ"
+    assert np.all(np.isneginf(got_ml[..., 0][~full])) and np.all(got_o[~full] == 0.0)
+    assert_parity(got_o[full], want_o[full], f"split states S={S}")
+    m_g, m_w = got_ml[..., 0][full], want_ml[..., 0][full]
+    assert np.all(np.abs(m_g - m_w) <= 1e-3 + 1e-4 * np.abs(m_w)), "largest scores differ"
+    l_g, l_w = got_ml[..., 1][full], want_ml[..., 1][full]
+    assert np.all(np.abs(l_g - l_w) <= 1e-3 * l_w), "exponent sums differ"
+    out = torch.empty(B, Hq, D, dtype=torch.float32, device=_gpu.dev())
+    kl.kl_combine(sh, po, pml, S, out, kl.KL_FP32)
+    torch.cuda.synchronize()
+    assert_parity(out.cpu().numpy(), oracle_decode(x, _gpu.default_scale(x)), "combined states")
