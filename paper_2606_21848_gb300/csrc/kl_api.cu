@@ -403,6 +403,22 @@ kl_status kl_decode_attention_fp8(const kl_shape *shape, const void *q, const vo
     if (g.G > 8 || g.wr_per_qh || !tc_supported(g, false)) return KL_ERR_UNSUPPORTED;
     if (g.P < 4) return KL_ERR_UNSUPPORTED;
     if (g.B == 0) return KL_OK;
+    // Runs of splits: when one CTA per split would overflow a wave of two CTAs per SM while the
+    // (b, g) units alone would not fill it, each CTA takes the fewest consecutive splits that
+    // fit and folds them as it goes (the online softmax continues across the boundary, the
+    // associative merge of adjacent states): the split chunk widens by that factor. The split
+    // states stay internal to this entry point (merged by the combine kernel).
+    {
+        const int64_t units = (int64_t)g.B * g.Hkv, slots = 2 * (int64_t)device_sm_count();
+        int spc = 1;
+        if (g.S > 1 && units < slots)
+            while ((int64_t)((g.S + spc - 1) / spc) * units > slots) ++spc;
+        if (spc > 1) {
+            const int64_t Lmax = (int64_t)g.max_pages * g.P;
+            g.chunk *= spc;
+            g.S = (int)((Lmax + g.chunk - 1) / g.chunk);
+        }
+    }
     if (!q || !v_codes || !v_scales || !block_table || !seq_lens || !out) return KL_ERR_INVALID_ARG;
     if (!aligned(q, 16) || !aligned(v_codes, 16) || !aligned(v_scales, 16) || !aligned(out, 16) ||
         (w_r && !aligned(w_r, 16)))
