@@ -230,6 +230,19 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int g, int n
     float *rows = reinterpret_cast<float *>(ring + table_bytes);           // [G][cap][128]
     const int cap = (int)((kRingBytes - table_bytes) / ((uint32_t)G * kD * sizeof(float)));
     const float2 *ml = reinterpret_cast<const float2 *>(a.part_ml);
+    // The first round's state rows go out at once, so that their copy overlaps the {m, l}
+    // loads and the weights (the ring is idle: every tile has been consumed).
+    auto issue_rows = [&](int c0, int nrow) {
+        if (t == 0) {
+            ptx::fence_proxy_async_global();
+            ptx::mbar_arrive_expect_tx(&sm.merge_full, (uint32_t)(G * nrow * kD * sizeof(float)));
+            for (int h = 0; h < G; ++h)
+                ptx::bulk_load(rows + (size_t)h * cap * kD,
+                               a.part_o + (((size_t)b * geo.Hq + g * G + h) * geo.S + c0) * kD,
+                               (uint32_t)(nrow * kD * sizeof(float)), &sm.merge_full);
+        }
+    };
+    issue_rows(0, min(cap, n_u));
     for (int i = t; i < G * n_u; i += kTile) {
         const int h = i / n_u, j = i - h * n_u;
         tab[i] = __ldcg(ml + ((size_t)b * geo.Hq + g * G + h) * geo.S + j);
@@ -263,14 +276,7 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int g, int n
         // every thread is done with the previous chunk (and the weights are written)
         ptx::fence_proxy_async_smem();
         ptx::bar_sync(kBarCompute, kTile);
-        if (t == 0) {
-            ptx::fence_proxy_async_global();
-            ptx::mbar_arrive_expect_tx(&sm.merge_full, (uint32_t)(G * nrow * kD * sizeof(float)));
-            for (int h = 0; h < G; ++h)
-                ptx::bulk_load(rows + (size_t)h * cap * kD,
-                               a.part_o + (((size_t)b * geo.Hq + g * G + h) * geo.S + c0) * kD,
-                               (uint32_t)(nrow * kD * sizeof(float)), &sm.merge_full);
-        }
+        if (c0 > 0) issue_rows(c0, nrow);
         if (!ptx::bar_and(kBarComputeAnd, kTile, wait(&sm.merge_full, round & 1))) return;
 #pragma unroll
         for (int pass = 0; pass < 2; ++pass) {
