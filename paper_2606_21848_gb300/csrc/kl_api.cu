@@ -101,7 +101,8 @@ kl_status decode_common(bool standard, const kl_shape *shape, const void *q, con
                         const int32_t *seq_lens, const kl_decode_options *opts, void *out,
                         kl_dtype out_dtype, void *workspace, size_t workspace_bytes,
                         int32_t *err, kl_stream_t stream, const void *v_new = nullptr,
-                        const int32_t *positions = nullptr, const float *q_routed = nullptr) {
+                        const int32_t *positions = nullptr, const float *q_routed = nullptr,
+                        bool pdl = false) {
     const int32_t ns = opts ? opts->num_splits : 0;
     const int32_t kernel = opts ? opts->kernel : KL_KERNEL_AUTO;
     if (ns < 0 || kernel < KL_KERNEL_AUTO || kernel > KL_KERNEL_SIMT) return KL_ERR_INVALID_ARG;
@@ -148,6 +149,7 @@ kl_status decode_common(bool standard, const kl_shape *shape, const void *q, con
     a.out_dtype = out_dtype;
     a.err = err;
     a.stream = reinterpret_cast<cudaStream_t>(stream);
+    a.pdl = pdl;
 
     bool use_tc = false;
     if (q_routed && !tc_supported(g, standard)) return KL_ERR_UNSUPPORTED;
@@ -487,15 +489,15 @@ kl_status kl_latent_decode(const kl_latent_shape *shape, const void *q, const vo
                                         shape->wr_per_query_head ? 1 : 0,
                                         static_cast<const uint16_t *>(q),
                                         static_cast<const uint16_t *>(w_r),
-                                        static_cast<const uint16_t *>(w_post), q_lat, s);
+                                        static_cast<const uint16_t *>(w_post), q_lat, err, s);
     if (e != cudaSuccess) return KL_ERR_CUDA;
     kl_decode_options o{num_splits, KL_KERNEL_TENSOR, nullptr, nullptr};
     st = decode_common(false, &p.dec, nullptr, nullptr, nullptr, v_lat, block_table, seq_lens, &o,
                        o_lat, KL_FP32, ws + p.dec_ws, workspace_bytes - p.dec_ws, err, stream,
-                       nullptr, nullptr, q_lat);
+                       nullptr, nullptr, q_lat, /*pdl=*/true);
     if (st != KL_OK) return st;
     return from_cuda(launch_latent_expand(B, Hq, D, r, o_lat, static_cast<const uint16_t *>(w_post),
-                                          out, out_dtype, s));
+                                          out, out_dtype, err, s));
 }
 
 int32_t kl_decode_kernel_available(const kl_shape *shape, int32_t kernel, int32_t standard) {

@@ -395,6 +395,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     ptx::tc_fence_before();
     __syncthreads();
     ptx::tc_fence_after();
+    if (a.pdl) grid_dep_launch();
 
     int L = L_raw;
     if (L < 0 || L > geo.max_pages * geo.P) {
@@ -685,6 +686,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                 ptx::fence_proxy_async_smem();
             }
         } else if (a.q_routed) {
+            if (a.pdl) grid_dep_wait();
 #pragma unroll
             for (int h = 0; h < kNG; ++h)
                 acc[h] = h < G ? a.q_routed[((size_t)b * geo.Hq + g * G + h) * kD + t] : 0.f;
@@ -997,6 +999,13 @@ cudaError_t launch_kernel(const DecodeArgs &la, const CUtensorMap &vmap, const C
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = la.stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    if (la.pdl) {
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+    }
     return cudaLaunchKernelEx(&cfg, decode_tc_kernel<kStandard, kPerSplit>, vmap, kmap, wmap, qmap, la);
 }
 

@@ -49,6 +49,11 @@ struct DecodeArgs {
     kl_dtype out_dtype;
     int32_t *err;
     cudaStream_t stream;
+    // Latent path: the launch is a programmatic dependent of the absorbed-query kernel ahead of
+    // it; the CTAs set up and start streaming cache tiles at once, the compute warps wait for
+    // that kernel (grid_dep_wait) before reading q_routed, and every CTA lets the expansion
+    // kernel behind it launch early (grid_dep_launch).
+    bool pdl = false;
 };
 
 // Arguments of a chunked-prefill launch (kl_prefill_attention). Sequence b's query rows are
@@ -76,6 +81,16 @@ __device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w &
 
 __device__ __forceinline__ void raise_flag(int32_t *err, int32_t bits) {
     if (err) atomicOr(err, bits);
+}
+
+// Programmatic dependent launch. A kernel launched with programmatic stream serialization may
+// start before the kernel ahead of it in the stream has finished: grid_dep_wait() blocks the
+// calling thread until that kernel has completed and its writes are visible (it returns at once
+// for an ordinary launch), and grid_dep_launch() lets such a follower start once every CTA of
+// the calling grid has signalled or exited.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
 // Launchers (each returns cudaGetLastError() of its launch).
@@ -119,12 +134,14 @@ cudaError_t launch_quantize_fp8(size_t rows, const uint16_t *v, uint8_t *codes, 
 
 // Latent value-only cache (head_dim D of queries and outputs, latent width r):
 // q_lat[b][h] = (q[b][h] W^R[w(h)]) W_post[h]^T and out[b][h] = o_lat[b][h] W_post[h].
+// Tensor-core kernels (D 64 or 128, r 128); the expansion is launched as a programmatic
+// dependent of the kernel ahead of it.
 cudaError_t launch_latent_query(int B, int Hq, int G, int D, int r, int wr_per_qh,
                                 const uint16_t *q, const uint16_t *w_r, const uint16_t *w_post,
-                                float *q_lat, cudaStream_t stream);
+                                float *q_lat, int32_t *err, cudaStream_t stream);
 cudaError_t launch_latent_expand(int B, int Hq, int D, int r, const float *o_lat,
                                  const uint16_t *w_post, void *out, kl_dtype out_dtype,
-                                 cudaStream_t stream);
+                                 int32_t *err, cudaStream_t stream);
 
 // Number of SMs of the current device (cached per device).
 int device_sm_count();

@@ -11,7 +11,7 @@ import torch
 
 import oracle
 import paper_2606_21848_gb300 as kl
-from paper_2606_21848_gb300.workloads import bf16_bits
+from paper_2606_21848_gb300.workloads import WORKLOADS, bf16_bits, generate
 from tests import _gpu
 from tests._gpu import assert_parity, to_dev
 from tests._inputs import tiny_latent
@@ -110,3 +110,48 @@ def test_latent_unsupported_shapes():
     with pytest.raises(kl.KLError) as e:
         run_latent(y)
     assert e.value.status == kl.KL_ERR_UNSUPPORTED
+
+
+def test_latent_two_sequence_blocks_with_a_ragged_tail():
+    """130 sequences: the projection kernels run two 128-sequence blocks, the second with two
+    rows (the rest of its TMA boxes read as zeros and are never stored)."""
+    lens = tuple(int(v) for v in np.random.default_rng(75).integers(0, 200, 130))
+    x = tiny_latent(B=130, Hq=8, Hl=2, D=128, r=128, P=16, lens=lens, seed=75)
+    got, err = run_latent(x)
+    assert err == 0
+    assert_parity(got.cpu().numpy(), oracle_latent(x, 1.0 / math.sqrt(128)), "130 sequences")
+
+
+@pytest.mark.parametrize("out_dtype", [kl.KL_BF16, kl.KL_FP32])
+def test_latent_head_dim_64_outputs(out_dtype):
+    """D 64: one 64-value half per query row, N = 64 expansion; bf16 rows are one 128-byte box,
+    fp32 rows two."""
+    x = tiny_latent(B=5, Hq=12, Hl=3, D=64, r=128, P=16, lens=(3, 250, 1, 77, 640), seed=76)
+    got, err = run_latent(x, out_dtype=out_dtype)
+    assert err == 0
+    want = oracle_latent(x, 1.0 / math.sqrt(128))
+    g = got.float().cpu().numpy().astype(np.float64)
+    rel = 1e-2 + (2.0 ** -8 if out_dtype == kl.KL_BF16 else 0.0)
+    assert not (np.abs(g - want) > 2e-3 + rel * np.abs(want)).any()
+
+
+@pytest.mark.slow
+def test_latent_serving_sampled_parity():
+    """The full latent serving workload (64 sequences of 8192 tokens, 32 query heads over 4
+    latent groups) in the bench's launch configuration; sampled heads against the oracle."""
+    wl = WORKLOADS["latent_serving"]
+    x = generate(wl)
+    got, err = run_latent(x, num_splits=max(wl.num_splits, 0), out_dtype=kl.KL_BF16)
+    assert err == 0
+    rng = np.random.default_rng(wl.seed)
+    B, Hq = wl.num_seqs, wl.num_q_heads
+    heads = [(int(b), int(h)) for b, h in zip(rng.integers(0, B, 40), rng.integers(0, Hq, 40))]
+    heads += [(B - 1, Hq - 1), (0, 0)]
+    want = oracle.latent_decode(bf16_bits(x["q"]), bf16_bits(x["w_r"]), bf16_bits(x["w_post"]),
+                                bf16_bits(x["v_lat"]), x["block_table"].numpy(),
+                                x["seq_lens"].numpy(), scale=1.0 / math.sqrt(wl.latent_dim),
+                                wr_per_query_head=bool(wl.wr_per_query_head), heads=heads)
+    g = got.float().cpu().numpy().astype(np.float64)
+    sampled = np.stack([g[b, h] for b, h in heads])
+    assert not (np.abs(sampled - want) > 2e-3 + (1e-2 + 2.0 ** -8) * np.abs(want)).any()
+    assert np.isfinite(g).all()
