@@ -512,6 +512,8 @@ __global__ void __launch_bounds__(kThreads, 2)
             }
             int page = __shfl_sync(0xffffffffu, bt_cur, ((p0 & 31) + lane) & 31);
             const bool exists = lane < ppt && p0 + lane < split_pages;
+            // with the ring full, a programmatic dependent sleeps until the routed queries exist
+            if (a.pdl && r == NS) grid_dep_wait();
             if (r >= NS && !wait(&sm.empty[s], ((r / NS) & 1) ^ 1)) break;
             const bool in_range = exists && page >= 0 && page < geo.num_pages;
             if (exists && !in_range) bad = true;
@@ -552,6 +554,8 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
     } else if (warp == kMmaWarp) {
         // ------------------------------------------------------- score MMA issuer -------
+        // (a programmatic dependent sleeps until the routed queries exist instead of polling)
+        if (a.pdl) grid_dep_wait();
         // Descriptors are formed once; a k step or a ring stage only moves the start address
         // (the low field, in 16-byte units; shared addresses stay below 256 KiB).
         constexpr uint32_t idesc_s = ptx::idesc_bf16(128, kN, false, false);
@@ -617,6 +621,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
     } else if (warp == kPvWarp) {
         // ------------------------------------------------------ output MMA issuer -------
+        if (a.pdl) grid_dep_wait();
         // A = V^T: MN-major SW128, 64-dim halves kHalfBytes apart (LBO), 8-token row groups
         //          1 KiB apart (SBO); 16 tokens per step.
         // B = P^T: MN-major, no swizzle; hi/lo blocks 128 B apart (SBO), 8-token groups 256 B

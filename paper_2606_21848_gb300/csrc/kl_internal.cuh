@@ -50,9 +50,9 @@ struct DecodeArgs {
     int32_t *err;
     cudaStream_t stream;
     // Latent path: the launch is a programmatic dependent of the absorbed-query kernel ahead of
-    // it; the CTAs set up and start streaming cache tiles at once, the compute warps wait for
-    // that kernel (grid_dep_wait) before reading q_routed, and every CTA lets the expansion
-    // kernel behind it launch early (grid_dep_launch).
+    // it; the CTAs set up and fill their ring of cache tiles at once, every role then sleeps in
+    // grid_dep_wait until that kernel has finished (the compute warps before reading q_routed),
+    // and every CTA lets the expansion kernel behind it launch early (grid_dep_launch).
     bool pdl = false;
 };
 

@@ -176,7 +176,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int h = blockIdx.x, b0 = blockIdx.y * kBM;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int nh = D / 64;                     // 64-value halves of a query row
-    grid_dep_launch();                         // the decode behind this kernel may set up
     setup(sm, warp);
     const uint32_t tmem = sm.tmem_base;
     uint8_t *const q_s = sm.stage, *const wr_s = sm.stage + 2 * kBox;
@@ -233,6 +232,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             __syncwarp();
         }
+        grid_dep_launch();
     } else {
         const int t = tid;                                   // row of the block = TMEM lane
         const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
@@ -261,6 +261,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         if (ok && lane == 0) ptx::mbar_arrive(&sm.a_ready);
         ok = ok && wait_bar(sm, &sm.d_full, 0, err);
+        // The decode behind this kernel may start setting up now, during the store: launched
+        // earlier, its CTAs slow this kernel's TMEM passes on the SMs they share.
+        grid_dep_launch();
         if (ok) {
             // Q* row t -> four 32-value boxes over Q and W^R (their MMAs have completed)
             ptx::tc_fence_after();
@@ -283,7 +286,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int c = 0; c < kR / 32; ++c)
                 ptx::tma_store_3d(&qlmap, sm.stage + c * kBox, 32 * c, h, b0);
             ptx::bulk_commit();
-            ptx::bulk_wait_all();
+            ptx::bulk_wait_read();
         }
     }
     teardown(sm, warp, lane);
@@ -409,7 +412,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int c = 0; c < D / box_cols; ++c)
                 ptx::tma_store_3d(&outmap, sm.stage + c * kBox, box_cols * c, h, b0);
             ptx::bulk_commit();
-            ptx::bulk_wait_all();
+            ptx::bulk_wait_read();
         }
     }
     teardown(sm, warp, lane);

@@ -98,9 +98,10 @@ __device__ __forceinline__ void bulk_commit() {
     asm volatile("cp.async.bulk.commit_group;" ::: "memory");
 }
 
-// Wait until every bulk group of this thread has completed (its writes performed).
-__device__ __forceinline__ void bulk_wait_all() {
-    asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+// Wait until every bulk group of this thread has finished reading its shared-memory source
+// (the global writes complete on their own; they are part of the grid's completion).
+__device__ __forceinline__ void bulk_wait_read() {
+    asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
 
 // 1-D bulk copy global -> shared of `bytes` (a multiple of 16; both addresses 16-byte aligned),
