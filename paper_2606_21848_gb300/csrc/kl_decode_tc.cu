@@ -15,14 +15,19 @@
 // routed query and of the softmax weights keeps about 16 significant bits where a plain bf16
 // operand would keep 8; the tensor cores have ample headroom for the doubled N.
 //
-// Roles (224 threads, two CTAs per SM):
-//   warps 0-3  compute: routing prologue; per tile read S from TMEM (thread = token), online
-//              softmax in base 2 (per-head running max across the CTA), write P^T to shared
-//              memory; read O from TMEM (thread = output dim) and accumulate with rescaling;
-//              epilogue writes the output or the split state, or merges the splits.
-//   warp 4     producer: block-table lookups and TMA loads of (page, head) tiles.
-//   warp 5     score-MMA issuer (one elected lane; also the routing MMA) and TMEM owner.
-//   warp 6     output-MMA issuer. Two issuing threads raise the SM's MMA issue rate (each
+// Roles (224 or 352 threads, two CTAs per SM):
+//   compute    routing prologue; per tile read S from TMEM (thread = token), online softmax in
+//              base 2 (per-head running max across the CTA), write P^T to shared memory; read
+//              O from TMEM (thread = output dim) and accumulate with rescaling; epilogue writes
+//              the output or the split state, or merges the splits. Groups of more than 4
+//              heads: warps 0-3, one per TMEM lane quarter, all 8 (padded) heads each. Groups
+//              of up to 4: warps 0-7, warps w and w + 4 sharing lane quarter w % 4 and 2 heads
+//              each, so the live heads alone are computed and a tile's softmax runs on two
+//              warps per SM sub-partition (6.7 % faster on the 4-head long-context decode; with
+//              8 heads, four per warp on eight warps, the 70B batch ran 2 % slower).
+//   next warp  producer: block-table lookups and TMA loads of (page, head) tiles.
+//   next       score-MMA issuer (one elected lane; also the routing MMA) and TMEM owner.
+//   last       output-MMA issuer. Two issuing threads raise the SM's MMA issue rate (each
 //              small-N tcgen05.mma costs tens of cycles to issue) and keep the output MMA of
 //              one tile from waiting behind the score MMA of the next.
 // Every wait is bounded (about one second); a wait that runs out raises KL_FLAG_TIMEOUT,
@@ -40,48 +45,73 @@ constexpr int kD = 128;
 constexpr int kTile = 128;                  // tokens per tile
 constexpr int kNG = 8;                      // query heads per value group (padded)
 constexpr int kN = 2 * kNG;                 // MMA N: hi and lo halves
-constexpr int kComputeWarps = 4;
-constexpr int kProducerWarp = 4;
-constexpr int kMmaWarp = 5;                 // score MMAs (and the routing MMA); owns TMEM
-constexpr int kPvWarp = 6;                  // output MMAs
-constexpr int kThreads = 7 * 32;
 constexpr uint32_t kTileBytes = kTile * kD * 2;   // 32 KiB per cache tile
 constexpr uint32_t kHalfBytes = kTileBytes / 2;   // one 64-dim half: 128 rows x 128 B
 constexpr uint32_t kTmemCols = 64;                // S: 2 x 16 columns, O: 2 x 16 columns
 constexpr uint32_t kTmemColsPq = 256;             // + one 16-column routing result per head
 constexpr uint64_t kTimeoutNs = 1000000000ull;
-// Named barriers of the 128 compute threads (id 0 is __syncthreads).
+// Warp roles for KH heads per compute warp: KH = 8, one compute warp per TMEM lane quarter;
+// KH = 2 (groups of up to 4 heads), two per quarter.
+template <int KH>
+struct Roles {
+    static constexpr int kComputeWarps = KH == 8 ? 4 : 8;
+    static constexpr int kComputeThreads = kComputeWarps * 32;
+    static constexpr int kProducerWarp = kComputeWarps;
+    static constexpr int kMmaWarp = kComputeWarps + 1;   // score MMAs (and routing); owns TMEM
+    static constexpr int kPvWarp = kComputeWarps + 2;    // output MMAs
+    static constexpr int kThreads = (kComputeWarps + 3) * 32;
+};
+// Named barriers of the compute threads (id 0 is __syncthreads).
 constexpr uint32_t kBarCompute = 1;       // plain sync
 constexpr uint32_t kBarComputeAnd = 2;    // sync + AND of a flag
 
-// Per-head maximum over the 32 lanes of a warp by transposed halving: after the three
-// exchange steps lane l holds one head, h(l) = 4 * bit4 + 2 * bit3 + bit2, reduced over the
-// lanes it shares with 3 others, then two more steps finish it. 9 shuffles instead of 40.
-__device__ __forceinline__ float warp_max8(const float (&x)[8], int lane) {
-    const bool b4 = lane & 16, b3 = lane & 8, b2 = lane & 4;
-    float a4[4], a2[2];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        const float send = b4 ? x[j] : x[j + 4];
-        const float keep = b4 ? x[j + 4] : x[j];
-        a4[j] = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, 16));
-    }
-#pragma unroll
-    for (int j = 0; j < 2; ++j) {
-        const float send = b3 ? a4[j] : a4[j + 2];
-        const float keep = b3 ? a4[j + 2] : a4[j];
-        a2[j] = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, 8));
-    }
+// Maximum over the 32 lanes of a warp of each of KH = 2 or 8 values by transposed halving:
+// each exchange step sends half of the lane's values and keeps the other half, so lane l ends
+// with the maximum of value e(l) = bit 4 of l (KH 2), or 4 bit4 + 2 bit3 + bit2 (KH 8: 9
+// shuffles instead of 40).
+template <int KH>
+__device__ __forceinline__ float warp_max_k(const float (&x)[KH], int lane) {
+    const bool b4 = lane & 16;
     float a1;
-    {
+    if constexpr (KH == 8) {
+        const bool b3 = lane & 8, b2 = lane & 4;
+        float a4[4], a2[2];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const float send = b4 ? x[j] : x[j + 4];
+            const float keep = b4 ? x[j + 4] : x[j];
+            a4[j] = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, 16));
+        }
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+            const float send = b3 ? a4[j] : a4[j + 2];
+            const float keep = b3 ? a4[j + 2] : a4[j];
+            a2[j] = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, 8));
+        }
         const float send = b2 ? a2[0] : a2[1];
         const float keep = b2 ? a2[1] : a2[0];
         a1 = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, 4));
+    } else {
+        static_assert(KH == 2, "two or eight heads per compute warp");
+        const float send = b4 ? x[0] : x[1];
+        const float keep = b4 ? x[1] : x[0];
+        a1 = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, 16));
+        a1 = fmaxf(a1, __shfl_xor_sync(0xffffffffu, a1, 8));
+        a1 = fmaxf(a1, __shfl_xor_sync(0xffffffffu, a1, 4));
     }
     a1 = fmaxf(a1, __shfl_xor_sync(0xffffffffu, a1, 2));
     a1 = fmaxf(a1, __shfl_xor_sync(0xffffffffu, a1, 1));
     return a1;
 }
+
+// Column base + h0 + e of a 16-column TMEM row [hi of heads 0-7 | lo of heads 0-7]: the upper
+// head block of a KH = 2 warp is picked with a select, so register arrays keep constant indices.
+template <int KH>
+__device__ __forceinline__ float head_col(const float (&v)[16], int base, bool hh, int e) {
+    if constexpr (KH == 8) return v[base + e];
+    else return hh ? v[base + KH + e] : v[base + e];
+}
+
 
 template <bool kStandard>
 struct Cfg {
@@ -99,8 +129,8 @@ struct __align__(1024) Smem {
     // P^T operands, no swizzle, MN-major: [16 groups of 8 tokens][hi | lo][8 tokens][16 B].
     // During the routing prologue the first one holds the raw query, fp32 [k][8].
     uint8_t p[2][kTile * kN * 2];
-    float red[2][kComputeWarps][kNG];
-    float lred[kComputeWarps][kNG];    // row sums of a split closed inside a CTA's run
+    float red[2][4][kNG];              // per lane quarter and head: tile maxima, row sums
+    float lred[4][kNG];                // row sums of a split closed inside a CTA's run
     uint64_t full[Cfg<kStandard>::kStages], empty[Cfg<kStandard>::kStages];
     uint64_t s_full[2], s_empty[2], p_full[2], o_full[2], o_empty[2];
     uint64_t qr_full, q_ready, r_full, drain, drain2, merge_full;
@@ -133,8 +163,9 @@ struct Waiter {
     }
 };
 
-struct Heads {
-    float v[8];
+template <int N>
+struct Vec {
+    float v[N];
 };
 
 __device__ __forceinline__ uint32_t pack_bf16(float lo_half, float hi_half) {
@@ -167,12 +198,15 @@ __device__ __forceinline__ bool arrive_last(unsigned int *counter, int n) {
 }
 
 // Merge of the n_u split states of (b, g) by the compute warps of the CTA that finished last
+// (t = the thread's index among them)
 // (kl_combine's formula). Up to eight splits: direct loads. More: the cache ring is idle by
 // now; the {m, l} table and the normalized weights go to its front, and TMA bulk copies bring
 // the state rows through the rest, folded by thread (head, 4 dims) from shared memory.
-template <typename SmemT, typename WaitT>
+template <int KH, typename SmemT, typename WaitT>
 __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int g, int n_u, int t,
                              int warp, int lane, const WaitT &wait) {
+    constexpr int kComputeWarps = Roles<KH>::kComputeWarps;
+    constexpr int kComputeThreads = Roles<KH>::kComputeThreads;
     const Geometry &geo = a.geo;
     const int G = geo.G;
     if (n_u <= 8) {
@@ -243,11 +277,11 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int g, int n
         }
     };
     issue_rows(0, min(cap, n_u));
-    for (int i = t; i < G * n_u; i += kTile) {
+    for (int i = t; i < G * n_u; i += kComputeThreads) {
         const int h = i / n_u, j = i - h * n_u;
         tab[i] = __ldcg(ml + ((size_t)b * geo.Hq + g * G + h) * geo.S + j);
     }
-    ptx::bar_sync(kBarCompute, kTile);
+    ptx::bar_sync(kBarCompute, kComputeThreads);
     for (int h = warp; h < G; h += kComputeWarps) {
         float M = -INFINITY;
         for (int j = lane; j < n_u; j += 32) {
@@ -268,16 +302,16 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int g, int n
         const float inv = z > 0.f ? 1.f / z : 0.f;
         for (int j = lane; j < n_u; j += 32) wt[h * n_u + j] *= inv;
     }
-    // thread t: head h = t / 32 (+ 4 for the second pass), dims 4 * (t % 32) .. + 3
+    // warp w: head w (+ kComputeWarps for a second pass), lane: dims 4 lane .. + 3
     float4 acc[2] = {make_float4(0.f, 0.f, 0.f, 0.f), make_float4(0.f, 0.f, 0.f, 0.f)};
     int round = 0;
     for (int c0 = 0; c0 < n_u; c0 += cap, ++round) {
         const int nrow = min(cap, n_u - c0);
         // every thread is done with the previous chunk (and the weights are written)
         ptx::fence_proxy_async_smem();
-        ptx::bar_sync(kBarCompute, kTile);
+        ptx::bar_sync(kBarCompute, kComputeThreads);
         if (c0 > 0) issue_rows(c0, nrow);
-        if (!ptx::bar_and(kBarComputeAnd, kTile, wait(&sm.merge_full, round & 1))) return;
+        if (!ptx::bar_and(kBarComputeAnd, kComputeThreads, wait(&sm.merge_full, round & 1))) return;
 #pragma unroll
         for (int pass = 0; pass < 2; ++pass) {
             const int h = warp + pass * kComputeWarps;
@@ -313,15 +347,21 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int g, int n
 }
 
 // kPerSplit: the CTA runs several splits and writes a state for each (only when the caller
-// gets the split states, or the combine kernel merges them, and spc > 1).
-template <bool kStandard, bool kPerSplit>
-__global__ void __launch_bounds__(kThreads, 2)
+// gets the split states, or the combine kernel merges them, and spc > 1). KH: heads per compute
+// warp (8, or 2 when G <= 4).
+template <bool kStandard, bool kPerSplit, int KH>
+__global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
     decode_tc_kernel(const __grid_constant__ CUtensorMap vmap,
                      const __grid_constant__ CUtensorMap kmap,
                      const __grid_constant__ CUtensorMap wmap,
                      const __grid_constant__ CUtensorMap qmap, const DecodeArgs a) {
     using S = Smem<kStandard>;
     constexpr int NS = Cfg<kStandard>::kStages;
+    constexpr int kComputeWarps = Roles<KH>::kComputeWarps;
+    constexpr int kComputeThreads = Roles<KH>::kComputeThreads;
+    constexpr int kProducerWarp = Roles<KH>::kProducerWarp;
+    constexpr int kMmaWarp = Roles<KH>::kMmaWarp;
+    constexpr int kPvWarp = Roles<KH>::kPvWarp;
     extern __shared__ uint8_t smem_raw[];
     S &sm = *reinterpret_cast<S *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                    ~uintptr_t(1023));
@@ -659,32 +699,40 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
     } else {
         // ------------------------------------------------------------------ compute -----
-        // (warps 0-3: the TMEM lane quarters 0-3)
-        const int t = tid;                                  // 0..127
-        const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+        // Warp w: TMEM lane quarter qd = w % 4 (thread t = 32 qd + lane is token t of a tile for
+        // S and P, output dim t for O) and the KH heads h0 .. h0 + KH - 1, h0 = KH (w / 4).
+        // Register arrays are indexed by constants only: the upper head block is picked with a
+        // select, never with a warp-dependent index.
+        const int qd = warp & 3;
+        const int t = qd * 32 + lane;
+        const bool hh = KH == 2 && warp >= 4;
+        const int h0 = hh ? KH : 0;
+        const uint32_t lane_base = (uint32_t)(qd * 32) << 16;
         float *qf = reinterpret_cast<float *>(sm.p[0]);     // [k][8] raw query (prologue only)
         const float sl2 = geo.scale * kLog2e;
         bool ok = true;
 
-        // Routing prologue: thread j obtains q_r[h][j] for the G heads in fp32 from the routing
+        // Routing prologue: thread t obtains q_r[h][t] for its heads in fp32 from the routing
         // MMAs in TMEM, from the caller's pre-routed queries, or the query itself (already
         // composed with W^R, or unrouted for the K+V comparison).
-        float acc[kNG];
+        float acc[KH];
 #pragma unroll
-        for (int h = 0; h < kNG; ++h) acc[h] = 0.f;
+        for (int e = 0; e < KH; ++e) acc[e] = 0.f;
         if (tc_route) {
             ok = wait(&sm.r_full, 0);
             if (ok) {
                 ptx::tc_fence_after();
                 if (route_pq) {
 #pragma unroll
-                    for (int h = 0; h < kNG; ++h)
-                        acc[h] = h < G ? ptx::tmem_ld1(tmem + 64 + 17 * h + lane_base) : 0.f;
+                    for (int e = 0; e < KH; ++e)
+                        acc[e] = h0 + e < G ? ptx::tmem_ld1(tmem + 64 + 17 * (h0 + e) + lane_base)
+                                            : 0.f;
                 } else {
                     float rv[16];
                     ptx::tmem_ld16(tmem + 2 * kN + lane_base, rv);
 #pragma unroll
-                    for (int h = 0; h < kNG; ++h) acc[h] = h < G ? rv[h] : 0.f;
+                    for (int e = 0; e < KH; ++e)
+                        acc[e] = h0 + e < G ? head_col<KH>(rv, 0, hh, e) : 0.f;
                 }
                 ptx::tc_fence_before();
                 // the q rows in the q_r buffer were read by the routing MMA; now overwrite them
@@ -693,10 +741,10 @@ __global__ void __launch_bounds__(kThreads, 2)
         } else if (a.q_routed) {
             if (a.pdl) grid_dep_wait();
 #pragma unroll
-            for (int h = 0; h < kNG; ++h)
-                acc[h] = h < G ? a.q_routed[((size_t)b * geo.Hq + g * G + h) * kD + t] : 0.f;
+            for (int e = 0; e < KH; ++e)
+                acc[e] = h0 + e < G ? a.q_routed[((size_t)b * geo.Hq + g * G + h0 + e) * kD + t] : 0.f;
         } else {
-            for (int i = t; i < kD * kNG; i += kTile) {
+            for (int i = tid; i < kD * kNG; i += kComputeThreads) {
                 const int k = i >> 3, h = i & 7;
                 qf[i] = h < G ? __uint_as_float(
                                     (uint32_t)a.q[((size_t)b * geo.Hq + g * G + h) * kD + k] << 16)
@@ -707,41 +755,60 @@ __global__ void __launch_bounds__(kThreads, 2)
             ok = wait(&sm.q_ready, 0);
             if (ok) {
 #pragma unroll
-                for (int h = 0; h < kNG; ++h) acc[h] = qf[t * kNG + h];
+                for (int e = 0; e < KH; ++e) acc[e] = qf[t * kNG + h0 + e];
             }
         }
         if (ok) {
-            // split-bf16 operand rows: n = h (hi), n = 8 + h (lo); column k = t
+            // split-bf16 operand rows: n = h (hi), n = 8 + h (lo); column k = t. With KH = 2
+            // the rows of heads 4-7 are zeros, written by the upper warps.
 #pragma unroll
-            for (int h = 0; h < kNG; ++h) {
-                const float v = acc[h] * sl2;
+            for (int e = 0; e < KH; ++e) {
+                const float v = acc[e] * sl2;
                 const __nv_bfloat16 hi = __float2bfloat16_rn(v);
                 const __nv_bfloat16 lo = __float2bfloat16_rn(v - __bfloat162float(hi));
-                *reinterpret_cast<__nv_bfloat16 *>(sm.qr + qr_offset(h, t)) = hi;
-                *reinterpret_cast<__nv_bfloat16 *>(sm.qr + qr_offset(kNG + h, t)) = lo;
+                *reinterpret_cast<__nv_bfloat16 *>(sm.qr + qr_offset(h0 + e, t)) = hi;
+                *reinterpret_cast<__nv_bfloat16 *>(sm.qr + qr_offset(kNG + h0 + e, t)) = lo;
+            }
+            if (KH == 2 && hh) {
+#pragma unroll
+                for (int h = 4; h < kNG; ++h) {
+                    *reinterpret_cast<uint16_t *>(sm.qr + qr_offset(h, t)) = 0;
+                    *reinterpret_cast<uint16_t *>(sm.qr + qr_offset(kNG + h, t)) = 0;
+                }
             }
             ptx::fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&sm.qr_full);
         }
 
-        // every decision below is taken by the four compute warps together
-        ok = ptx::bar_and(kBarComputeAnd, kTile, ok);
-
-        float m[kNG], lsum[kNG], o[kNG];
-        Heads alpha_prev;
+        // every decision below is taken by the compute warps together
+        ok = ptx::bar_and(kBarComputeAnd, kComputeThreads, ok);
+        if (KH == 2 && hh) {
+            // P^T columns of heads 4-7 (bytes 8-15 of a token's hi and lo rows) stay zero; the
+            // raw query in the first P buffer has been read by now
 #pragma unroll
-        for (int h = 0; h < kNG; ++h) {
-            m[h] = -INFINITY;
-            lsum[h] = 0.f;
-            o[h] = 0.f;
-            alpha_prev.v[h] = 0.f;
+            for (int pb = 0; pb < 2; ++pb) {
+                uint8_t *row = sm.p[pb] + (t >> 3) * 256 + (t & 7) * 16;
+                *reinterpret_cast<uint2 *>(row + 8) = make_uint2(0, 0);
+                *reinterpret_cast<uint2 *>(row + 128 + 8) = make_uint2(0, 0);
+            }
+        }
+
+        float m[KH], lsum[KH], o[KH];
+        Vec<KH> alpha_prev;
+#pragma unroll
+        for (int e = 0; e < KH; ++e) {
+            m[e] = -INFINITY;
+            lsum[e] = 0.f;
+            o[e] = 0.f;
+            alpha_prev.v[e] = 0.f;
         }
 
         // O accumulation of tile j: o = o * alpha_j + O_j (thread = output dim t).
-        auto correct = [&](int j, const Heads alpha) -> bool {
+        auto correct = [&](int j, const Vec<KH> alpha) -> bool {
             const int ob = j & 1;
-            if (!ptx::bar_and(kBarComputeAnd, kTile, wait(&sm.o_full[ob], (j >> 1) & 1))) return false;
+            if (!ptx::bar_and(kBarComputeAnd, kComputeThreads, wait(&sm.o_full[ob], (j >> 1) & 1)))
+                return false;
             ptx::tc_fence_after();
             float ov[16];
             ptx::tmem_ld16(tmem + 2 * kN + ob * kN + lane_base, ov);
@@ -749,7 +816,8 @@ __global__ void __launch_bounds__(kThreads, 2)
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&sm.o_empty[ob]);
 #pragma unroll
-            for (int h = 0; h < kNG; ++h) o[h] = fmaf(o[h], alpha.v[h], ov[h] + ov[kNG + h]);
+            for (int e = 0; e < KH; ++e)
+                o[e] = fmaf(o[e], alpha.v[e], head_col<KH>(ov, 0, hh, e) + head_col<KH>(ov, kNG, hh, e));
             return true;
         };
 
@@ -763,37 +831,36 @@ __global__ void __launch_bounds__(kThreads, 2)
         const int tps = geo.chunk / kTile;
         // The state of split sp from the running o, lsum and m (all of its O folded in).
         auto emit_state = [&](int sp) {
-            float l[kNG];
+            float l[KH];
 #pragma unroll
-            for (int h = 0; h < kNG; ++h) l[h] = lsum[h];
+            for (int e = 0; e < KH; ++e) l[e] = lsum[e];
 #pragma unroll
             for (int off = 16; off > 0; off >>= 1)
 #pragma unroll
-                for (int h = 0; h < kNG; ++h) l[h] += __shfl_xor_sync(0xffffffffu, l[h], off);
+                for (int e = 0; e < KH; ++e) l[e] += __shfl_xor_sync(0xffffffffu, l[e], off);
             if (lane == 0) {
 #pragma unroll
-                for (int h = 0; h < kNG; ++h) sm.lred[warp][h] = l[h];
+                for (int e = 0; e < KH; ++e) sm.lred[qd][h0 + e] = l[e];
             }
-            ptx::bar_sync(kBarCompute, kTile);
+            ptx::bar_sync(kBarCompute, kComputeThreads);
 #pragma unroll
-            for (int h = 0; h < kNG; ++h) {
+            for (int e = 0; e < KH; ++e) {
+                const int h = h0 + e;
                 if (h >= G) continue;
-                float lt = 0.f;
-#pragma unroll
-                for (int w = 0; w < kComputeWarps; ++w) lt += sm.lred[w][h];
+                const float lt = (sm.lred[0][h] + sm.lred[1][h]) + (sm.lred[2][h] + sm.lred[3][h]);
                 const size_t slot = ((size_t)b * geo.Hq + g * G + h) * geo.S + sp;
-                a.part_o[slot * kD + t] = o[h] / lt;
+                a.part_o[slot * kD + t] = o[e] / lt;
                 if (t == 0) {
-                    a.part_ml[slot * 2] = m[h] * kLn2;
+                    a.part_ml[slot * 2] = m[e] * kLn2;
                     a.part_ml[slot * 2 + 1] = lt;
                 }
             }
-            ptx::bar_sync(kBarCompute, kTile);      // lred is free for the next split
+            ptx::bar_sync(kBarCompute, kComputeThreads);      // lred is free for the next split
         };
 
         for (int i = 0; ok && i < n_tiles; ++i) {
             const int sb = i & 1;
-            if (!ptx::bar_and(kBarComputeAnd, kTile, wait(&sm.s_full[sb], (i >> 1) & 1))) {
+            if (!ptx::bar_and(kBarComputeAnd, kComputeThreads, wait(&sm.s_full[sb], (i >> 1) & 1))) {
                 ok = false;
                 break;
             }
@@ -806,10 +873,10 @@ __global__ void __launch_bounds__(kThreads, 2)
                 }
                 emit_state(split0 + i / tps - 1);
 #pragma unroll
-                for (int h = 0; h < kNG; ++h) {
-                    o[h] = 0.f;
-                    lsum[h] = 0.f;
-                    m[h] = -INFINITY;
+                for (int e = 0; e < KH; ++e) {
+                    o[e] = 0.f;
+                    lsum[e] = 0.f;
+                    m[e] = -INFINITY;
                 }
             }
             ptx::tc_fence_after();
@@ -821,58 +888,69 @@ __global__ void __launch_bounds__(kThreads, 2)
 
             const int nvalid = min(kTile, t_end - (t_begin + i * kTile));
             const bool valid = t < nvalid;
-            float s[kNG], mx[kNG];
+            float s[KH], mx[KH];
 #pragma unroll
-            for (int h = 0; h < kNG; ++h) {
-                s[h] = (valid && h < G) ? sv[h] + sv[kNG + h] : -INFINITY;
-                mx[h] = s[h];
+            for (int e = 0; e < KH; ++e) {
+                s[e] = (valid && h0 + e < G) ? head_col<KH>(sv, 0, hh, e) + head_col<KH>(sv, kNG, hh, e)
+                                             : -INFINITY;
+                mx[e] = s[e];
             }
-            // per-head maximum over the tile's 128 tokens: warp reduce, then across the 4 warps
+            // per-head maximum over the tile's 128 tokens: warp reduce, then across the 4
+            // lane quarters
             {
-                const float wm = warp_max8(mx, lane);
-                if ((lane & 3) == 0)
-                    sm.red[sb][warp][((lane >> 4) & 1) * 4 + ((lane >> 3) & 1) * 2 + ((lane >> 2) & 1)] = wm;
+                const float wm = warp_max_k<KH>(mx, lane);
+                if (KH == 8 && (lane & 3) == 0)
+                    sm.red[sb][qd][((lane >> 4) & 1) * 4 + ((lane >> 3) & 1) * 2 + ((lane >> 2) & 1)] = wm;
+                if (KH == 2 && (lane & 15) == 0) sm.red[sb][qd][h0 + ((lane >> 4) & 1)] = wm;
             }
-            ptx::bar_sync(kBarCompute, kTile);
-            Heads alpha;
-            float p[kNG];
+            ptx::bar_sync(kBarCompute, kComputeThreads);
+            Vec<KH> alpha;
+            float p[KH];
 #pragma unroll
-            for (int h = 0; h < kNG; ++h) {
+            for (int e = 0; e < KH; ++e) {
+                const int h = h0 + e;
                 float tmax = sm.red[sb][0][h];
 #pragma unroll
-                for (int w = 1; w < kComputeWarps; ++w) tmax = fmaxf(tmax, sm.red[sb][w][h]);
-                const float mn = fmaxf(m[h], tmax);
+                for (int q = 1; q < 4; ++q) tmax = fmaxf(tmax, sm.red[sb][q][h]);
+                const float mn = fmaxf(m[e], tmax);
                 const bool live = h < G;
-                alpha.v[h] = live ? exp2f(m[h] - mn) : 0.f;
-                p[h] = live ? exp2f(s[h] - mn) : 0.f;
-                lsum[h] = fmaf(lsum[h], alpha.v[h], p[h]);
-                m[h] = live ? mn : m[h];
+                alpha.v[e] = live ? exp2f(m[e] - mn) : 0.f;
+                p[e] = live ? exp2f(s[e] - mn) : 0.f;
+                lsum[e] = fmaf(lsum[e], alpha.v[e], p[e]);
+                m[e] = live ? mn : m[e];
             }
-            // P^T row of token t: hi and lo halves.
+            // P^T row of token t, this warp's heads: hi and lo halves.
             {
-                float r[kNG];
+                float r[KH];
 #pragma unroll
-                for (int h = 0; h < kNG; ++h)
-                    r[h] = p[h] - __bfloat162float(__float2bfloat16_rn(p[h]));
-                uint8_t *row = sm.p[sb] + (t >> 3) * 256 + (t & 7) * 16;
-                *reinterpret_cast<uint4 *>(row) =
-                    make_uint4(pack_bf16(p[0], p[1]), pack_bf16(p[2], p[3]),
-                               pack_bf16(p[4], p[5]), pack_bf16(p[6], p[7]));
-                *reinterpret_cast<uint4 *>(row + 128) =
-                    make_uint4(pack_bf16(r[0], r[1]), pack_bf16(r[2], r[3]),
-                               pack_bf16(r[4], r[5]), pack_bf16(r[6], r[7]));
+                for (int e = 0; e < KH; ++e) r[e] = p[e] - __bfloat162float(__float2bfloat16_rn(p[e]));
+                uint8_t *row = sm.p[sb] + (t >> 3) * 256 + (t & 7) * 16 + 2 * h0;
+                if constexpr (KH == 8) {
+                    *reinterpret_cast<uint4 *>(row) =
+                        make_uint4(pack_bf16(p[0], p[1]), pack_bf16(p[2], p[3]),
+                                   pack_bf16(p[4], p[5]), pack_bf16(p[6], p[7]));
+                    *reinterpret_cast<uint4 *>(row + 128) =
+                        make_uint4(pack_bf16(r[0], r[1]), pack_bf16(r[2], r[3]),
+                                   pack_bf16(r[4], r[5]), pack_bf16(r[6], r[7]));
+                } else {
+                    *reinterpret_cast<uint32_t *>(row) = pack_bf16(p[0], p[1]);
+                    *reinterpret_cast<uint32_t *>(row + 128) = pack_bf16(r[0], r[1]);
+                }
             }
-            // Rows past the end inside the last 16-token MMA step must be finite: zero them.
+            // Rows past the end inside the last 16-token MMA step must be finite: zero them
+            // (with two warps per lane quarter, each clears one 64-dim half).
             if (nvalid < kTile) {
                 const int st = (i + ro) % NS;
-                if (ptx::bar_and(kBarComputeAnd, kTile, wait(&sm.full[st], ((i + ro) / NS) & 1)) &&
+                if (ptx::bar_and(kBarComputeAnd, kComputeThreads,
+                                 wait(&sm.full[st], ((i + ro) / NS) & 1)) &&
                     t >= nvalid && t < ((nvalid + 15) & ~15)) {
-                    uint4 *r0 = reinterpret_cast<uint4 *>(sm.tiles[st][0] + t * 128);
+                    uint4 *r0 = reinterpret_cast<uint4 *>(sm.tiles[st][0] + (hh ? kHalfBytes : 0u) +
+                                                          t * 128);
                     uint4 *r1 = reinterpret_cast<uint4 *>(sm.tiles[st][0] + kHalfBytes + t * 128);
 #pragma unroll
                     for (int c = 0; c < 8; ++c) {
                         r0[c] = make_uint4(0, 0, 0, 0);
-                        r1[c] = make_uint4(0, 0, 0, 0);
+                        if (KH == 8) r1[c] = make_uint4(0, 0, 0, 0);
                     }
                 }
             }
@@ -890,30 +968,27 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
             for (int off = 16; off > 0; off >>= 1)
 #pragma unroll
-                for (int h = 0; h < kNG; ++h) lsum[h] += __shfl_xor_sync(0xffffffffu, lsum[h], off);
+                for (int e = 0; e < KH; ++e) lsum[e] += __shfl_xor_sync(0xffffffffu, lsum[e], off);
             const int rb = n_tiles & 1;   // red buffer not read by the last tile's exchange
             if (lane == 0) {
 #pragma unroll
-                for (int h = 0; h < kNG; ++h) sm.red[rb][warp][h] = lsum[h];
+                for (int e = 0; e < KH; ++e) sm.red[rb][qd][h0 + e] = lsum[e];
             }
-            ptx::bar_sync(kBarCompute, kTile);
+            ptx::bar_sync(kBarCompute, kComputeThreads);
             {
                 // Merged here: one state per CTA run that holds tokens (slot cta; a single one
                 // writes the output itself). Otherwise: the state of the split closed last.
                 const int n_cta_u = (L + geo.chunk * geo.spc - 1) / (geo.chunk * geo.spc);
                 const int sp_last = a.merge_inside ? cta : split0 + (n_tiles - 1) / tps;
                 const bool write_out = a.direct_out || (a.merge_inside && n_cta_u == 1);
-                float lt[kNG];
 #pragma unroll
-                for (int h = 0; h < kNG; ++h) {
-                    lt[h] = 0.f;
-#pragma unroll
-                    for (int w = 0; w < kComputeWarps; ++w) lt[h] += sm.red[rb][w][h];
-                }
-#pragma unroll
-                for (int h = 0; h < kNG; ++h) {
+                for (int e = 0; e < KH; ++e) {
+                    const int h = h0 + e;
                     if (h >= G) continue;
-                    const float val = o[h] / lt[h];
+                    float lt = 0.f;
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) lt += sm.red[rb][q][h];
+                    const float val = o[e] / lt;
                     const size_t bh = (size_t)b * geo.Hq + g * G + h;
                     if (write_out) {
                         if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * kD + t] = val;
@@ -922,8 +997,8 @@ __global__ void __launch_bounds__(kThreads, 2)
                         const size_t slot = bh * geo.S + sp_last;
                         a.part_o[slot * kD + t] = val;
                         if (t == 0) {
-                            a.part_ml[slot * 2] = m[h] * kLn2;
-                            a.part_ml[slot * 2 + 1] = lt[h];
+                            a.part_ml[slot * 2] = m[e] * kLn2;
+                            a.part_ml[slot * 2 + 1] = lt;
                         }
                         // splits of the run past the sequence's end: empty states
                         if (!a.merge_inside) {
@@ -940,11 +1015,11 @@ __global__ void __launch_bounds__(kThreads, 2)
                 }
                 if (a.merge_inside && !write_out) {
                     // The last CTA of (b, g) to finish merges the n_cta_u states (as kl_combine).
-                    ptx::bar_sync(kBarCompute, kTile);
-                    if (t == 0)
+                    ptx::bar_sync(kBarCompute, kComputeThreads);
+                    if (tid == 0)
                         sm.is_last = arrive_last(a.counters + (size_t)b * geo.Hkv + g, n_cta_u) ? 1 : 0;
-                    ptx::bar_sync(kBarCompute, kTile);
-                    if (sm.is_last) merge_states(sm, a, b, g, n_cta_u, t, warp, lane, wait);
+                    ptx::bar_sync(kBarCompute, kComputeThreads);
+                    if (sm.is_last) merge_states<KH>(sm, a, b, g, n_cta_u, tid, warp, lane, wait);
                 }
             }
         }
@@ -987,21 +1062,21 @@ bool make_map(CUtensorMap *map, const void *base, uint64_t rows, uint32_t box_ro
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <bool kStandard, bool kPerSplit>
+template <bool kStandard, bool kPerSplit, int KH>
 cudaError_t launch_kernel(const DecodeArgs &la, const CUtensorMap &vmap, const CUtensorMap &kmap,
                           const CUtensorMap &wmap, const CUtensorMap &qmap) {
     const Geometry &g = la.geo;
     const size_t smem = sizeof(Smem<kStandard>) + 1024;
     static bool configured = false;
     if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<kStandard, kPerSplit>,
+        cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<kStandard, kPerSplit, KH>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         configured = true;
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((g.S + g.spc - 1) / g.spc, g.Hkv, g.B);
-    cfg.blockDim = dim3(kThreads);
+    cfg.blockDim = dim3(Roles<KH>::kThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = la.stream;
     cudaLaunchAttribute attr[1];
@@ -1011,7 +1086,7 @@ cudaError_t launch_kernel(const DecodeArgs &la, const CUtensorMap &vmap, const C
         cfg.attrs = attr;
         cfg.numAttrs = 1;
     }
-    return cudaLaunchKernelEx(&cfg, decode_tc_kernel<kStandard, kPerSplit>, vmap, kmap, wmap, qmap, la);
+    return cudaLaunchKernelEx(&cfg, decode_tc_kernel<kStandard, kPerSplit, KH>, vmap, kmap, wmap, qmap, la);
 }
 
 template <bool kStandard>
@@ -1041,8 +1116,13 @@ cudaError_t launch(const DecodeArgs &a) {
         while ((int64_t)((g.S + spc - 1) / spc) * units > slots) ++spc;
     la.geo.spc = spc;
     const bool per_split = spc > 1 && !a.merge_inside && !a.direct_out;
-    return per_split ? launch_kernel<kStandard, true>(la, vmap, kmap, wmap, qmap)
-                     : launch_kernel<kStandard, false>(la, vmap, kmap, wmap, qmap);
+    // heads per compute warp: all 8 (padded) on four warps, or 2 on eight when the group has
+    // at most 4
+    if (g.G <= 4)
+        return per_split ? launch_kernel<kStandard, true, 2>(la, vmap, kmap, wmap, qmap)
+                         : launch_kernel<kStandard, false, 2>(la, vmap, kmap, wmap, qmap);
+    return per_split ? launch_kernel<kStandard, true, 8>(la, vmap, kmap, wmap, qmap)
+                     : launch_kernel<kStandard, false, 8>(la, vmap, kmap, wmap, qmap);
 }
 
 }  // namespace
