@@ -214,6 +214,68 @@ def cpu_oracle_rate(x, seconds: float, standard: bool):
     return seqs / el, seqs, el
 
 
+def _one_core_worker(sample, scale, standard, seconds, queue):
+    """Child process: the oracle with one OpenMP thread over the sample's sequences."""
+    import numpy as np
+
+    import oracle
+
+    q, w, v, bt, sl = sample
+    B, Hq = q.shape[0], q.shape[1]
+    seqs, t0, b = 0, time.perf_counter(), 0
+    while True:
+        heads = np.array([(b, h) for h in range(Hq)], np.int32)
+        if standard:
+            oracle.standard_decode(q, v, v, bt, sl, scale=scale, heads=heads)
+        else:
+            oracle.decode(q, w, v, bt, sl, scale=scale, heads=heads)
+        seqs += 1
+        b = (b + 1) % B
+        el = time.perf_counter() - t0
+        if el >= seconds:
+            break
+    queue.put((oracle.threads(), seqs, el))
+
+
+def cpu_oracle_one_core(x, seconds: float, standard: bool, max_seqs: int = 4):
+    """The oracle on one host core (OMP_NUM_THREADS=1) over the first `max_seqs` sequences,
+    gathered with their own pages; run in a spawned process (this one holds a CUDA context, and
+    the OpenMP thread count is fixed when the oracle library loads)."""
+    import multiprocessing as mp
+
+    import numpy as np
+
+    from paper_2606_21848_gb300.workloads import bf16_bits
+
+    n = min(max_seqs, x["q"].shape[0])
+    P = x["v_cache"].shape[2]
+    bt_all, sl = x["block_table"].numpy()[:n], x["seq_lens"].numpy()[:n].copy()
+    used = sorted({int(p) for b in range(n) for p in bt_all[b, :(int(sl[b]) + P - 1) // P]})
+    remap = {p: i for i, p in enumerate(used)}
+    bt = np.full_like(bt_all, -1)
+    for b in range(n):
+        for j in range((int(sl[b]) + P - 1) // P):
+            bt[b, j] = remap[int(bt_all[b, j])]
+    v = np.ascontiguousarray(bf16_bits(x["v_cache"])[used] if used else bf16_bits(x["v_cache"])[:1])
+    sample = (np.ascontiguousarray(bf16_bits(x["q"])[:n]), bf16_bits(x["w_r"]), v, bt, sl)
+    ctx = mp.get_context("spawn")
+    queue = ctx.Queue()
+    old = os.environ.get("OMP_NUM_THREADS")
+    os.environ["OMP_NUM_THREADS"] = "1"
+    try:
+        proc = ctx.Process(target=_one_core_worker,
+                           args=(sample, 1.0 / math.sqrt(x["q"].shape[2]), standard, seconds, queue))
+        proc.start()
+    finally:
+        if old is None:
+            del os.environ["OMP_NUM_THREADS"]
+        else:
+            os.environ["OMP_NUM_THREADS"] = old
+    cores, seqs, el = queue.get(timeout=seconds + 300)
+    proc.join(timeout=60)
+    return seqs / el, seqs, el, cores
+
+
 def run_reference(args):
     rank, world, local = dist_env()
     if rank != 0:
@@ -449,6 +511,10 @@ def run_ours(args):
         cpu = {"value": rate, "unit": "tokens/s", "cores": oracle.threads(), "kind": "oracle",
                "sample": f"{n} whole sequences of {wl.name} (all {Hq} heads, decode only, "
                          f"fp64) in {el:.1f}s"}
+        r1, n1, el1, c1 = cpu_oracle_one_core(x, min(args.cpu_seconds, 5.0), args.standard)
+        cpu["one_core"] = {"value": r1, "unit": "tokens/s", "cores": c1,
+                           "sample": f"{n1} whole sequences (the first 4 of the batch, round "
+                                     f"robin) in {el1:.1f}s"}
 
     kname = "tensor-fp8" if args.fp8_cache else "tensor" if tc else "simt"
     line = {

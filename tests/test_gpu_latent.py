@@ -155,3 +155,31 @@ def test_latent_serving_sampled_parity():
     sampled = np.stack([g[b, h] for b, h in heads])
     assert not (np.abs(sampled - want) > 2e-3 + (1e-2 + 2.0 ** -8) * np.abs(want)).any()
     assert np.isfinite(g).all()
+
+
+def test_latent_back_to_back_calls_with_different_queries():
+    """Two calls on one stream, same workspace, different queries, no synchronization between
+    them: the decode of each call must read that call's absorbed queries and its expansion that
+    call's decode output (a dependent launch that read too early would return the other call's
+    values)."""
+    x = tiny_latent(B=6, Hq=16, Hl=2, D=128, r=128, P=16, lens=(1500, 2048, 77, 900, 1, 3000),
+                    seed=77)
+    y = dict(x)
+    y["q"] = torch.randn(x["q"].shape, generator=torch.Generator().manual_seed(78)).to(torch.bfloat16)
+    g = to_dev(x)
+    q2 = y["q"].to(_gpu.dev())
+    sh = lshape(x)
+    ws = torch.zeros(kl.kl_latent_workspace_size(sh, 0), dtype=torch.uint8, device=_gpu.dev())
+    err = torch.zeros(1, dtype=torch.int32, device=_gpu.dev())
+    outs = []
+    for q in (g["q"], q2, g["q"], q2):
+        out = torch.empty(6, 16, 128, dtype=torch.float32, device=_gpu.dev())
+        kl.kl_latent_decode(sh, q, g["w_r"], g["w_post"], g["v_lat"], g["block_table"],
+                            g["seq_lens"], 0, out, kl.KL_FP32, ws, err)
+        outs.append(out)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    scale = 1.0 / math.sqrt(128)
+    want1, want2 = oracle_latent(x, scale), oracle_latent(y, scale)
+    for i, out in enumerate(outs):
+        assert_parity(out.cpu().numpy(), want1 if i % 2 == 0 else want2, f"call {i}")
