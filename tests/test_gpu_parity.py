@@ -106,9 +106,12 @@ def test_decode_matches_oracle(kname, si, splits):
     assert_parity(out.cpu().numpy(), want, f"{kname} {SHAPES[si]} S={splits}")
 
 
+# Group sizes 4 and 8 take the two compute-warp layouts of the tensor-core kernel (eight warps
+# of 2 heads, four warps of 8 heads).
 @pytest.mark.parametrize("kname", ["simt", "tensor"])
-def test_decode_per_query_head_routing(kname):
-    x = tiny(B=2, Hq=32, Hkv=8, D=128, P=16, lens=(260, 999), wr_per_query_head=True)
+@pytest.mark.parametrize("G", [4, 8])
+def test_decode_per_query_head_routing(kname, G):
+    x = tiny(B=2, Hq=8 * G, Hkv=8, D=128, P=16, lens=(260, 999), wr_per_query_head=True)
     k = _kernel_or_skip(kname, x)
     out, err = decode(to_dev(x), shape_of(x), kernel=k, num_splits=2)
     assert err == 0
@@ -282,8 +285,9 @@ def test_combine_matches_oracle():
 # ------------------------------------------------------------- standard K + V -----------
 
 @pytest.mark.parametrize("kname", ["simt", "tensor"])
-def test_standard_kv_decode_matches_oracle(kname):
-    x = tiny(B=3, Hq=32, Hkv=8, D=128, P=16, lens=(1, 300, 1111))
+@pytest.mark.parametrize("G", [4, 8])
+def test_standard_kv_decode_matches_oracle(kname, G):
+    x = tiny(B=3, Hq=8 * G, Hkv=8, D=128, P=16, lens=(1, 300, 1111))
     k = _kernel_or_skip(kname, x, standard=True)
     kc = torch.randn(x["v_cache"].shape, generator=torch.Generator().manual_seed(3)).to(torch.bfloat16)
     g = to_dev(x)
@@ -400,12 +404,13 @@ def test_composed_query_fused_step_appends_and_decodes():
 # ------------------------------------------------------------------ split-state outputs -----
 
 @pytest.mark.parametrize("splits", [3, 64])
-def test_split_states_match_oracle_partial_states(splits):
+@pytest.mark.parametrize("G", [4, 8])
+def test_split_states_match_oracle_partial_states(splits, G):
     """The split states the caller asks for (partial_o / partial_ml): every split's normalized
     output, largest score and exponent sum against the oracle's states of the same token
     ranges, then their merge by kl_combine. At 64 splits of a 2-sequence, 8-value-head batch
     one CTA runs several consecutive splits and writes a state at each split boundary."""
-    x = tiny(B=2, Hq=32, Hkv=8, D=128, P=16, lens=(2000, 4096), seed=23)
+    x = tiny(B=2, Hq=8 * G, Hkv=8, D=128, P=16, lens=(2000, 4096), seed=23)
     k = _kernel_or_skip("tensor", x)
     g = to_dev(x)
     sh = shape_of(x)
