@@ -842,8 +842,9 @@ def run_reference_latent(args, wl, x):
 
 
 def run_latent(args, wl, x, dev, rank, world):
-    """One latent decode step = kl_append_v of the current token's latent rows +
-    kl_latent_decode (absorbed query, tensor-core decode over the latent rows, expansion)."""
+    """One latent decode step = kl_latent_decode_step: the current token's latent rows appended
+    inside the tensor-core decode over the latent rows, between the absorbed-query and the
+    expansion kernels (three launches)."""
     import torch
 
     import paper_2606_21848_gb300 as kl
@@ -853,7 +854,7 @@ def run_latent(args, wl, x, dev, rank, world):
     num_pages, Hl, P, r = x["v_lat"].shape
     max_pages = x["block_table"].shape[1]
     lsh = kl.make_latent_shape(B, Hq, Hl, D, r, P, num_pages, max_pages, wl.wr_per_query_head)
-    ash = kl.make_shape(B, Hq, Hl, r, P, num_pages, max_pages)      # the append over latent rows
+    ash = kl.make_shape(B, Hq, Hl, r, P, num_pages, max_pages)      # the decode over latent rows
     splits_req = wl.num_splits if args.num_splits < 0 else args.num_splits
     S = kl.kl_decode_num_splits(ash, splits_req)
     g = {k: x[k].to(dev) for k in ("q", "w_r", "w_post", "v_lat", "block_table", "seq_lens",
@@ -871,19 +872,18 @@ def run_latent(args, wl, x, dev, rank, world):
 
     def step(d, ev=None):
         if ev: ev[0].record(stream)
-        kl.kl_append_v(ash, d["v_new"], d["block_table"], d["positions"], g["v_lat"], err, stream)
+        kl.kl_latent_decode_step(lsh, d["q"], g["w_r"], g["w_post"], d["v_new"], d["positions"],
+                                 g["v_lat"], d["block_table"], d["seq_lens"], splits_req, out,
+                                 kl.KL_BF16, ws, err, stream)
         if ev: ev[1].record(stream)
-        kl.kl_latent_decode(lsh, d["q"], g["w_r"], g["w_post"], g["v_lat"], d["block_table"],
-                            d["seq_lens"], splits_req, out, kl.KL_BF16, ws, err, stream)
-        if ev: ev[2].record(stream)
 
     E = lambda: torch.cuda.Event(enable_timing=True)
     for _ in range(args.warmup):
         flush_l2()
-        step(g, [E(), E(), E()])
+        step(g, [E(), E()])
     torch.cuda.synchronize()
     assert int(err.item()) == 0, f"device error flags {int(err.item())}"
-    evs = [[E(), E(), E()] for _ in range(args.steps)]
+    evs = [[E(), E()] for _ in range(args.steps)]
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
@@ -894,10 +894,9 @@ def run_latent(args, wl, x, dev, rank, world):
         torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
-    step_ms = statistics.mean(e[0].elapsed_time(e[2]) for e in evs)
-    app_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
-    dec_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
-    step_ms, app_ms, dec_ms = max_over_ranks([step_ms, app_ms, dec_ms], device=dev)
+    step_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+    step_ms, = max_over_ranks([step_ms], device=dev)
+    dec_ms = step_ms
     assert int(err.item()) == 0, f"device error flags {int(err.item())}"
     ab = latent_bytes(x)
     peak, peak_kind = measured_peaks()
@@ -956,16 +955,17 @@ def run_latent(args, wl, x, dev, rank, world):
                    "w_post": "per query head",
                    "l2": "flushed between timed steps (512 MiB write, then read back)",
                    "parallelism": f"replicas x{world}"},
-        "ms_breakdown": {"append": app_ms, "latent_decode": dec_ms},
-        "kernels_per_step": 4,
+        "ms_breakdown": {"latent_decode_step": step_ms},
+        "kernels_per_step": 3,
         "roofline": {"bound": "hbm", "achieved": dec_gbs, "peak": peak, "unit": "GB/s",
                      "frac": dec_gbs / peak, "peak_kind": peak_kind,
                      "pct_of_8tbs": 100.0 * dec_gbs / NOMINAL_HBM_GBS,
                      "algorithmic_bytes": ab["total"],
-                     "timed": "the kl_latent_decode call (absorbed query, decode, expansion)",
+                     "timed": "the kl_latent_decode_step call (absorbed query, decode with the "
+                              "fused append, expansion)",
                      "traffic": recorded_traffic(wl.name, "tensor"),
                      "traffic_of": "the decode kernel over the latent rows (ncu)"},
-        "gpu_launches": 4 * args.steps,
+        "gpu_launches": 3 * args.steps,
         "clocks": clk.summary(),
         "e2e": e2e,
         "cpu_baseline": cpu,

@@ -284,6 +284,23 @@ kl_status kl_latent_decode(const kl_latent_shape *shape, const void *q, const vo
                            int32_t *err, kl_stream_t stream);
 
 /*
+ * One decode step over a latent value-only cache: the current token's latent rows are appended
+ * (Section 3: the cache holds every row up to the current one) and the decode of
+ * kl_latent_decode runs over the n+1 rows -- kl_append_v into v_lat then kl_latent_decode,
+ * fused: the decode CTA whose split holds row positions[b] writes v_new[b][g] there before it
+ * reads that row. v_new: [B][Hl][r] bf16, 16-byte aligned; positions: [B] int32 (normally
+ * seq_lens[b] - 1); v_lat is written in place. A position outside the block table raises
+ * KL_FLAG_BAD_POSITION and a page id outside the pool KL_FLAG_BAD_PAGE in *err (that row is not
+ * written). Other arguments, layouts, workspace and flags as in kl_latent_decode.
+ */
+kl_status kl_latent_decode_step(const kl_latent_shape *shape, const void *q, const void *w_r,
+                                const void *w_post, const void *v_new, const int32_t *positions,
+                                void *v_lat, const int32_t *block_table, const int32_t *seq_lens,
+                                int32_t num_splits, void *out, kl_dtype out_dtype,
+                                void *workspace, size_t workspace_bytes, int32_t *err,
+                                kl_stream_t stream);
+
+/*
  * FP8 value cache (not in the paper; §3 notes that the value-only cache is orthogonal to other
  * cache-reduction methods, and a quantized cache is one): the same value rows stored in about
  * half the bytes. Each cached row is D OCP FP8 E4M3 codes (1 sign, 4 exponent bits of bias 7,

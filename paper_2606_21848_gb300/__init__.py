@@ -16,5 +16,6 @@ from ._lib import (  # noqa: F401
     kl_shape, kl_standard_decode, kl_status_string, load, make_shape,
     kl_append_v_chunk, kl_prefill_attention,
     kl_latent_shape, make_latent_shape, kl_latent_workspace_size, kl_latent_decode,
+    kl_latent_decode_step,
     kl_append_v_fp8, kl_decode_attention_fp8, kl_quantize_cache_fp8,
 )

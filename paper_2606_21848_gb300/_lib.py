@@ -88,6 +88,7 @@ def load() -> ctypes.CDLL:
         "kl_decode_attention_fp8": ([SH, P, P, P, P, P, P, I32, P, I32, P, SZ, P, P], I32),
         "kl_latent_workspace_size": ([LS, I32], SZ),
         "kl_latent_decode": ([LS, P, P, P, P, P, P, I32, P, I32, P, SZ, P, P], I32),
+        "kl_latent_decode_step": ([LS, P, P, P, P, P, P, P, P, I32, P, I32, P, SZ, P, P], I32),
         "kl_prefill_attention": ([SH, P, P, P, P, P, P, I32, I32, P, I32, P, P], I32),
         "kl_status_string": ([I32], ctypes.c_char_p),
     }
@@ -264,6 +265,15 @@ def kl_latent_decode(shape, q, w_r, w_post, v_lat, block_table, seq_lens, num_sp
                                    _p(block_table), _p(seq_lens), num_splits, _p(out), out_dtype,
                                    _p(workspace), _nbytes(workspace), _p(err), _stream(stream)),
            "kl_latent_decode")
+
+
+def kl_latent_decode_step(shape, q, w_r, w_post, v_new, positions, v_lat, block_table, seq_lens,
+                          num_splits, out, out_dtype, workspace, err=None, stream=None):
+    _check(load().kl_latent_decode_step(ctypes.byref(shape), _p(q), _p(w_r), _p(w_post), _p(v_new),
+                                        _p(positions), _p(v_lat), _p(block_table), _p(seq_lens),
+                                        num_splits, _p(out), out_dtype, _p(workspace),
+                                        _nbytes(workspace), _p(err), _stream(stream)),
+           "kl_latent_decode_step")
 
 
 def kl_decode_kernel_available(shape, kernel, standard=False) -> bool:

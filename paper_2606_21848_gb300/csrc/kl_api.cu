@@ -460,11 +460,16 @@ size_t kl_latent_workspace_size(const kl_latent_shape *shape, int32_t num_splits
     return latent_plan(shape, num_splits, &p) == KL_OK ? p.total : 0;
 }
 
-kl_status kl_latent_decode(const kl_latent_shape *shape, const void *q, const void *w_r,
-                           const void *w_post, const void *v_lat, const int32_t *block_table,
-                           const int32_t *seq_lens, int32_t num_splits, void *out,
-                           kl_dtype out_dtype, void *workspace, size_t workspace_bytes,
-                           int32_t *err, kl_stream_t stream) {
+}  // extern "C"
+
+namespace {
+
+// kl_latent_decode, with the fused append of kl_latent_decode_step when v_new is set.
+kl_status latent_decode(const kl_latent_shape *shape, const void *q, const void *w_r,
+                        const void *w_post, const void *v_lat, const int32_t *block_table,
+                        const int32_t *seq_lens, int32_t num_splits, void *out,
+                        kl_dtype out_dtype, void *workspace, size_t workspace_bytes, int32_t *err,
+                        kl_stream_t stream, const void *v_new, const int32_t *positions) {
     LatentPlan p;
     kl_status st = latent_plan(shape, num_splits, &p);
     if (st != KL_OK) return st;
@@ -494,10 +499,34 @@ kl_status kl_latent_decode(const kl_latent_shape *shape, const void *q, const vo
     kl_decode_options o{num_splits, KL_KERNEL_TENSOR, nullptr, nullptr};
     st = decode_common(false, &p.dec, nullptr, nullptr, nullptr, v_lat, block_table, seq_lens, &o,
                        o_lat, KL_FP32, ws + p.dec_ws, workspace_bytes - p.dec_ws, err, stream,
-                       nullptr, nullptr, q_lat, /*pdl=*/true);
+                       v_new, positions, q_lat, /*pdl=*/true);
     if (st != KL_OK) return st;
     return from_cuda(launch_latent_expand(B, Hq, D, r, o_lat, static_cast<const uint16_t *>(w_post),
                                           out, out_dtype, err, s));
+}
+
+}  // namespace
+
+extern "C" {
+
+kl_status kl_latent_decode(const kl_latent_shape *shape, const void *q, const void *w_r,
+                           const void *w_post, const void *v_lat, const int32_t *block_table,
+                           const int32_t *seq_lens, int32_t num_splits, void *out,
+                           kl_dtype out_dtype, void *workspace, size_t workspace_bytes,
+                           int32_t *err, kl_stream_t stream) {
+    return latent_decode(shape, q, w_r, w_post, v_lat, block_table, seq_lens, num_splits, out,
+                         out_dtype, workspace, workspace_bytes, err, stream, nullptr, nullptr);
+}
+
+kl_status kl_latent_decode_step(const kl_latent_shape *shape, const void *q, const void *w_r,
+                                const void *w_post, const void *v_new, const int32_t *positions,
+                                void *v_lat, const int32_t *block_table, const int32_t *seq_lens,
+                                int32_t num_splits, void *out, kl_dtype out_dtype,
+                                void *workspace, size_t workspace_bytes, int32_t *err,
+                                kl_stream_t stream) {
+    if (!v_new || !positions || !aligned(v_new, 16)) return KL_ERR_INVALID_ARG;
+    return latent_decode(shape, q, w_r, w_post, v_lat, block_table, seq_lens, num_splits, out,
+                         out_dtype, workspace, workspace_bytes, err, stream, v_new, positions);
 }
 
 int32_t kl_decode_kernel_available(const kl_shape *shape, int32_t kernel, int32_t standard) {

@@ -183,3 +183,39 @@ def test_latent_back_to_back_calls_with_different_queries():
     want1, want2 = oracle_latent(x, scale), oracle_latent(y, scale)
     for i, out in enumerate(outs):
         assert_parity(out.cpu().numpy(), want1 if i % 2 == 0 else want2, f"call {i}")
+
+
+def test_latent_decode_step_appends_then_decodes():
+    """kl_latent_decode_step: the current token's latent rows land bit-exactly where the oracle's
+    append puts them, the output matches the oracle over the appended cache, and it is
+    bit-identical to a separate kl_append_v followed by kl_latent_decode."""
+    x = tiny_latent(B=4, Hq=16, Hl=2, D=128, r=128, P=16, lens=(1, 40, 700, 1500), seed=79)
+    B, Hq, D = x["q"].shape
+    num_pages, Hl, P, r = x["v_lat"].shape
+    v_new = torch.randn(B, Hl, r, generator=torch.Generator().manual_seed(80)).to(torch.bfloat16)
+    positions = (x["seq_lens"] - 1).to(torch.int32)
+    sh = lshape(x)
+    ws = torch.zeros(max(256, kl.kl_latent_workspace_size(sh, 0)), dtype=torch.uint8,
+                     device=_gpu.dev())
+    err = torch.zeros(1, dtype=torch.int32, device=_gpu.dev())
+    g = to_dev(x)
+    vn, pos = v_new.to(_gpu.dev()), positions.to(_gpu.dev())
+    out = torch.empty(B, Hq, D, dtype=torch.float32, device=_gpu.dev())
+    kl.kl_latent_decode_step(sh, g["q"], g["w_r"], g["w_post"], vn, pos, g["v_lat"],
+                             g["block_table"], g["seq_lens"], 0, out, kl.KL_FP32, ws, err)
+    # the unfused pair on a second copy of the cache
+    v2 = to_dev(x)["v_lat"]
+    ash = kl.make_shape(B, Hq, Hl, r, P, num_pages, x["block_table"].shape[1])
+    kl.kl_append_v(ash, vn, g["block_table"], pos, v2, err)
+    out2 = torch.empty_like(out)
+    kl.kl_latent_decode(sh, g["q"], g["w_r"], g["w_post"], v2, g["block_table"], g["seq_lens"],
+                        0, out2, kl.KL_FP32, ws, err)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    want_cache = oracle.append(bf16_bits(x["v_lat"]), bf16_bits(v_new), x["block_table"].numpy(),
+                               positions.numpy())
+    assert np.array_equal(bf16_bits(g["v_lat"].cpu()), want_cache)
+    assert torch.equal(out, out2)
+    y = dict(x)
+    y["v_lat"] = torch.from_numpy(want_cache.view(np.int16)).view(torch.bfloat16)
+    assert_parity(out.cpu().numpy(), oracle_latent(y, 1.0 / math.sqrt(r)), "latent step")
