@@ -398,11 +398,9 @@ def run_ours(args):
     def decode_call(opts, o, w, d=None):
         d = d or g
         if args.fp8_cache:
-            kl.kl_append_v_fp8(sh, d["v_new"], d["block_table"], d["positions"], codes, scales,
-                               err, stream)
-            kl.kl_decode_attention_fp8(sh, d["q"], None if args.fused_query else g["w_r"], codes,
-                                       scales, d["block_table"], d["seq_lens"], S, o, kl.KL_BF16,
-                                       w, err, stream)
+            kl.kl_decode_step_fp8(sh, d["q"], None if args.fused_query else g["w_r"], d["v_new"],
+                                  d["positions"], codes, scales, d["block_table"], d["seq_lens"],
+                                  S, o, kl.KL_BF16, w, err, stream)
         elif args.standard:
             kl.kl_standard_decode(sh, g["q"], k_cache, g["v_cache"], g["block_table"],
                                   g["seq_lens"], opts, o, kl.KL_BF16, w, err, stream)
@@ -424,7 +422,7 @@ def run_ours(args):
             kl.kl_combine(sh, part_o, part_ml, S, out, kl.KL_BF16, stream)
         ev[2].record(stream)
 
-    launches_per_step = (2 + (S > 1)) if args.fp8_cache else 1 if one_kernel else 2
+    launches_per_step = (1 + (S > 1)) if args.fp8_cache else 1 if one_kernel else 2
     E = lambda: torch.cuda.Event(enable_timing=True)
     for _ in range(args.warmup):
         flush_l2()

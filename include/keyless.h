@@ -348,6 +348,21 @@ kl_status kl_decode_attention_fp8(const kl_shape *shape, const void *q, const vo
                                   void *workspace, size_t workspace_bytes, int32_t *err,
                                   kl_stream_t stream);
 
+/*
+ * One decode step over the FP8 cache: kl_append_v_fp8 of the current token's rows followed by
+ * kl_decode_attention_fp8 over the n+1 rows, fused -- the decode CTA whose split holds row
+ * positions[b] quantizes v_new[b][g] (bit-identical to kl_append_v_fp8) into the code and scale
+ * caches before it loads that row. v_new: [B][Hkv][D] bf16, 16-byte aligned; positions: [B]
+ * int32 (normally seq_lens[b] - 1); v_codes and v_scales are written in place. Flags as in
+ * kl_append_v_fp8 (that row is then not written) and kl_decode_attention_fp8; other arguments
+ * as in kl_decode_attention_fp8.
+ */
+kl_status kl_decode_step_fp8(const kl_shape *shape, const void *q, const void *w_r,
+                             const void *v_new, const int32_t *positions, void *v_codes,
+                             float *v_scales, const int32_t *block_table, const int32_t *seq_lens,
+                             int32_t num_splits, void *out, kl_dtype out_dtype, void *workspace,
+                             size_t workspace_bytes, int32_t *err, kl_stream_t stream);
+
 /* Size of the fixed device scratch that kl_decode_attention_noalloc uses (32 MiB). */
 #define KL_NOALLOC_SCRATCH_BYTES (32u * 1024u * 1024u)
 

@@ -17,5 +17,5 @@ from ._lib import (  # noqa: F401
     kl_append_v_chunk, kl_prefill_attention,
     kl_latent_shape, make_latent_shape, kl_latent_workspace_size, kl_latent_decode,
     kl_latent_decode_step,
-    kl_append_v_fp8, kl_decode_attention_fp8, kl_quantize_cache_fp8,
+    kl_append_v_fp8, kl_decode_attention_fp8, kl_decode_step_fp8, kl_quantize_cache_fp8,
 )

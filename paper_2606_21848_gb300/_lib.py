@@ -86,6 +86,7 @@ def load() -> ctypes.CDLL:
         "kl_append_v_fp8": ([SH, P, P, P, P, P, P, P], I32),
         "kl_quantize_cache_fp8": ([SH, P, P, P, P], I32),
         "kl_decode_attention_fp8": ([SH, P, P, P, P, P, P, I32, P, I32, P, SZ, P, P], I32),
+        "kl_decode_step_fp8": ([SH, P, P, P, P, P, P, P, P, I32, P, I32, P, SZ, P, P], I32),
         "kl_latent_workspace_size": ([LS, I32], SZ),
         "kl_latent_decode": ([LS, P, P, P, P, P, P, I32, P, I32, P, SZ, P, P], I32),
         "kl_latent_decode_step": ([LS, P, P, P, P, P, P, P, P, I32, P, I32, P, SZ, P, P], I32),
@@ -246,6 +247,15 @@ def kl_decode_attention_fp8(shape, q, w_r, v_codes, v_scales, block_table, seq_l
                                           _p(v_scales), _p(block_table), _p(seq_lens), num_splits,
                                           _p(out), out_dtype, _p(workspace), _nbytes(workspace),
                                           _p(err), _stream(stream)), "kl_decode_attention_fp8")
+
+
+def kl_decode_step_fp8(shape, q, w_r, v_new, positions, v_codes, v_scales, block_table, seq_lens,
+                       num_splits, out, out_dtype, workspace, err=None, stream=None):
+    _check(load().kl_decode_step_fp8(ctypes.byref(shape), _p(q), _p(w_r), _p(v_new), _p(positions),
+                                     _p(v_codes), _p(v_scales), _p(block_table), _p(seq_lens),
+                                     num_splits, _p(out), out_dtype, _p(workspace),
+                                     _nbytes(workspace), _p(err), _stream(stream)),
+           "kl_decode_step_fp8")
 
 
 def make_latent_shape(num_seqs, num_q_heads, num_latent_heads, head_dim, latent_dim, page_size,

@@ -391,12 +391,17 @@ kl_status kl_quantize_cache_fp8(const kl_shape *shape, const void *v_cache, void
                                          reinterpret_cast<cudaStream_t>(stream)));
 }
 
-kl_status kl_decode_attention_fp8(const kl_shape *shape, const void *q, const void *w_r,
-                                  const void *v_codes, const float *v_scales,
-                                  const int32_t *block_table, const int32_t *seq_lens,
-                                  int32_t num_splits, void *out, kl_dtype out_dtype,
-                                  void *workspace, size_t workspace_bytes, int32_t *err,
-                                  kl_stream_t stream) {
+}  // extern "C"
+
+namespace {
+
+// kl_decode_attention_fp8, with the fused quantizing append of kl_decode_step_fp8 when v_new
+// is set.
+kl_status decode_fp8(const kl_shape *shape, const void *q, const void *w_r, const void *v_codes,
+                     const float *v_scales, const int32_t *block_table, const int32_t *seq_lens,
+                     int32_t num_splits, void *out, kl_dtype out_dtype, void *workspace,
+                     size_t workspace_bytes, int32_t *err, kl_stream_t stream,
+                     const void *v_new, const int32_t *positions) {
     if (num_splits < 0) return KL_ERR_INVALID_ARG;
     if (out_dtype != KL_BF16 && out_dtype != KL_FP32) return KL_ERR_INVALID_ARG;
     Geometry g;
@@ -437,9 +442,11 @@ kl_status kl_decode_attention_fp8(const kl_shape *shape, const void *q, const vo
     a.v_cache = static_cast<const uint16_t *>(v_codes);
     a.block_table = block_table;
     a.seq_lens = seq_lens;
-    a.v_new = nullptr;
-    a.positions = nullptr;
+    a.v_new = static_cast<const uint16_t *>(v_new);
+    a.positions = positions;
     a.cache_rw = nullptr;
+    a.codes_rw = static_cast<uint8_t *>(const_cast<void *>(v_codes));
+    a.scales_rw = const_cast<float *>(v_scales);
     char *ws = static_cast<char *>(workspace);
     a.part_o = wl.total ? reinterpret_cast<float *>(ws + wl.part_o) : nullptr;
     a.part_ml = wl.total ? reinterpret_cast<float *>(ws + wl.part_ml) : nullptr;
@@ -453,6 +460,30 @@ kl_status kl_decode_attention_fp8(const kl_shape *shape, const void *q, const vo
     cudaError_t e = launch_decode_fp8(a, v_scales);
     if (e == cudaSuccess) e = finish_decode(a, false);
     return from_cuda(e);
+}
+
+}  // namespace
+
+extern "C" {
+
+kl_status kl_decode_attention_fp8(const kl_shape *shape, const void *q, const void *w_r,
+                                  const void *v_codes, const float *v_scales,
+                                  const int32_t *block_table, const int32_t *seq_lens,
+                                  int32_t num_splits, void *out, kl_dtype out_dtype,
+                                  void *workspace, size_t workspace_bytes, int32_t *err,
+                                  kl_stream_t stream) {
+    return decode_fp8(shape, q, w_r, v_codes, v_scales, block_table, seq_lens, num_splits, out,
+                      out_dtype, workspace, workspace_bytes, err, stream, nullptr, nullptr);
+}
+
+kl_status kl_decode_step_fp8(const kl_shape *shape, const void *q, const void *w_r,
+                             const void *v_new, const int32_t *positions, void *v_codes,
+                             float *v_scales, const int32_t *block_table, const int32_t *seq_lens,
+                             int32_t num_splits, void *out, kl_dtype out_dtype, void *workspace,
+                             size_t workspace_bytes, int32_t *err, kl_stream_t stream) {
+    if (!v_new || !positions || !aligned(v_new, 16)) return KL_ERR_INVALID_ARG;
+    return decode_fp8(shape, q, w_r, v_codes, v_scales, block_table, seq_lens, num_splits, out,
+                      out_dtype, workspace, workspace_bytes, err, stream, v_new, positions);
 }
 
 size_t kl_latent_workspace_size(const kl_latent_shape *shape, int32_t num_splits) {

@@ -44,6 +44,7 @@
 #include <cudaTypedefs.h>
 #include <math.h>
 
+#include "kl_fp8_quant.cuh"
 #include "kl_internal.cuh"
 #include "kl_tc_ptx.cuh"
 
@@ -297,6 +298,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int base = route ? 2 : 0;
 
     const int L_raw = a.seq_lens[b];
+    const int pos_raw = a.v_new ? a.positions[b] : -1;
     const int t_begin = split * geo.chunk;
     const int32_t *bt = a.block_table + (size_t)b * geo.max_pages;
 
@@ -343,7 +345,36 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int t_end = min(t_begin + geo.chunk, L);
     const int n_tiles = t_end > t_begin ? (t_end - t_begin + kTile - 1) / kTile : 0;
 
+    // Fused append (kl_decode_step_fp8): the CTA whose split holds row positions[b] quantizes
+    // v_new[b][g] into it before the loads of that row's tile (first, when the row lies past the
+    // sequence's end), with the arithmetic of kl_append_v_fp8.
+    const bool pos_ok = pos_raw >= 0 && pos_raw < geo.max_pages * geo.P;
+    if (a.v_new && !pos_ok && tid == 0 && split == 0 && g == 0)
+        raise_flag(a.err, KL_FLAG_BAD_POSITION);
+    const bool app_owner = a.v_new && pos_ok && pos_raw / geo.chunk == split;
+    // the row (page-checked), its codes for this lane and its scale; warp-uniform
+    auto quantize_new_row = [&](size_t &row, uint32_t &codes, float &scale) -> bool {
+        const int page = bt[pos_raw / geo.P];
+        if (page < 0 || page >= geo.num_pages) {
+            if (lane == 0) raise_flag(a.err, KL_FLAG_BAD_PAGE);
+            return false;
+        }
+        row = ((size_t)page * geo.Hkv + g) * geo.P + pos_raw % geo.P;
+        codes = quantize_row4(
+            reinterpret_cast<const uint2 *>(a.v_new + ((size_t)b * geo.Hkv + g) * kD)[lane], scale);
+        return true;
+    };
+
     if (n_tiles == 0) {
+        if (app_owner && warp == 0) {
+            size_t row;
+            uint32_t codes;
+            float scale;
+            if (quantize_new_row(row, codes, scale)) {
+                reinterpret_cast<uint32_t *>(a.codes_rw + row * kD)[lane] = codes;
+                if (lane == 0) a.scales_rw[row] = scale;
+            }
+        }
         // an empty split: zero output (direct) or an empty state
         if (tid < kD) {
             for (int h = 0; h < G; ++h) {
@@ -377,6 +408,12 @@ __global__ void __launch_bounds__(kThreads, 2)
         const uint32_t page_bytes = (uint32_t)P * 128u + (uint32_t)P * 4u;
         bool bad = false;
         int issued = 0;                                      // ring uses issued
+        int app_tile = -1;
+        size_t app_row = 0;
+        uint32_t app_codes = 0;
+        float app_scale = 0.f;
+        if (app_owner && quantize_new_row(app_row, app_codes, app_scale))
+            app_tile = pos_raw < t_end ? (pos_raw - t_begin) / kTile : 0;
         if (route) {
             if (lane == 0) {
                 // W^R[g] halves into stages 0 and 1 (MN-major A of the routing MMA); the
@@ -397,6 +434,12 @@ __global__ void __launch_bounds__(kThreads, 2)
             const bool exists = lane < ppt && p0 + lane < end_page;
             const int page = exists ? bt[p0 + lane] : -1;
             if (round >= 1 && !wait(&sm.empty[s], (round - 1) & 1)) break;
+            if (i == app_tile) {
+                reinterpret_cast<uint32_t *>(a.codes_rw + app_row * kD)[lane] = app_codes;
+                if (lane == 0) a.scales_rw[app_row] = app_scale;
+                ptx::fence_proxy_async_global();
+                __syncwarp();
+            }
             const bool in_range = exists && page >= 0 && page < geo.num_pages;
             if (exists && !in_range) bad = true;
             const unsigned mask = __ballot_sync(0xffffffffu, in_range);

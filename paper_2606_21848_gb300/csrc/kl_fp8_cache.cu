@@ -2,9 +2,7 @@
 // head) and the conversion of a whole bf16 cache. A row of 128 values becomes 128 OCP E4M3 codes
 // and one fp32 scale: scale = max |v| / 448 in fp32, code = E4M3(v / scale), rounded to nearest
 // even and saturating (the conversion intrinsic of cuda_fp8.h; an all-zero row gets scale 0).
-#include <cuda_fp8.h>
-
-#include "kl_internal.cuh"
+#include "kl_fp8_quant.cuh"
 
 namespace kl {
 namespace {
@@ -31,19 +29,8 @@ __global__ void __launch_bounds__(256)
     }
     for (int g = threadIdx.x >> 5; g < Hkv; g += blockDim.x >> 5) {
         const uint2 w = reinterpret_cast<const uint2 *>(v_new + ((size_t)b * Hkv + g) * kD)[lane];
-        const float v[4] = {bf16lo(w.x), bf16hi(w.x), bf16lo(w.y), bf16hi(w.y)};
-        float amax = fmaxf(fmaxf(fabsf(v[0]), fabsf(v[1])), fmaxf(fabsf(v[2]), fabsf(v[3])));
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
-        const float s = __fdiv_rn(amax, 448.0f);
-        uint32_t packed = 0;
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const uint32_t c = s > 0.f
-                                   ? (uint32_t)__nv_cvt_float_to_fp8(__fdiv_rn(v[e], s), __NV_SATFINITE, __NV_E4M3)
-                                   : 0u;
-            packed |= c << (8 * e);
-        }
+        float s;
+        const uint32_t packed = quantize_row4(w, s);
         const size_t row = ((size_t)page * Hkv + g) * P + pos % P;
         reinterpret_cast<uint32_t *>(codes + row * kD)[lane] = packed;
         if (lane == 0) scales[row] = s;
@@ -55,19 +42,8 @@ __global__ void __launch_bounds__(256)
 // reducing any of them, so that enough loads are in flight to keep HBM busy.
 __device__ __forceinline__ void quantize_row_regs(const uint2 w, int lane, uint8_t *__restrict__ codes,
                                                   float *__restrict__ scales, size_t row) {
-    const float x[4] = {bf16lo(w.x), bf16hi(w.x), bf16lo(w.y), bf16hi(w.y)};
-    float amax = fmaxf(fmaxf(fabsf(x[0]), fabsf(x[1])), fmaxf(fabsf(x[2]), fabsf(x[3])));
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
-    const float s = __fdiv_rn(amax, 448.0f);
-    uint32_t packed = 0;
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-        const uint32_t c = s > 0.f
-                               ? (uint32_t)__nv_cvt_float_to_fp8(__fdiv_rn(x[e], s), __NV_SATFINITE, __NV_E4M3)
-                               : 0u;
-        packed |= c << (8 * e);
-    }
+    float s;
+    const uint32_t packed = quantize_row4(w, s);
     reinterpret_cast<uint32_t *>(codes + row * kD)[lane] = packed;
     if (lane == 0) scales[row] = s;
 }

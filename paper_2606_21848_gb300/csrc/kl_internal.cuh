@@ -39,6 +39,10 @@ struct DecodeArgs {
     const uint16_t *v_new;            // [B][Hkv][D] bf16 or nullptr
     const int32_t *positions;         // [B]
     uint16_t *cache_rw;
+    // FP8 step (kl_decode_step_fp8): the row positions[b] of the code and scale caches receives
+    // v_new[b][g] quantized, in the same way, from the CTA whose split holds it.
+    uint8_t *codes_rw = nullptr;
+    float *scales_rw = nullptr;
     float *part_o;            // [B][Hq][S][D]   split states (unless direct_out)
     float *part_ml;           // [B][Hq][S][2]
     void *out;                // [B][Hq][D]

@@ -130,3 +130,43 @@ def test_fp8_unsupported_shapes():
     with pytest.raises(kl.KLError) as e:
         run_fp8(x, codes, scales)
     assert e.value.status == kl.KL_ERR_UNSUPPORTED
+
+
+@pytest.mark.parametrize("num_splits", [1, 3, 0])
+def test_fp8_decode_step_appends_then_decodes(num_splits):
+    """kl_decode_step_fp8: the current token's rows are quantized into the cache bit-exactly as
+    the oracle's append does it, the output matches the oracle's FP8 decode over the appended
+    cache, and it is bit-identical to kl_append_v_fp8 followed by kl_decode_attention_fp8. One
+    position lies past its sequence's end (it is written, and not attended)."""
+    x = tiny(B=4, Hq=32, Hkv=8, D=128, P=16, lens=(1, 130, 1000, 2049), seed=98)
+    codes, scales = fp8_cache(x)
+    B, Hq, D = x["q"].shape
+    v_new = torch.randn(B, 8, D, generator=torch.Generator().manual_seed(99)).to(torch.bfloat16)
+    positions = (x["seq_lens"] - 1).to(torch.int32)
+    positions[1] = 140                                     # past L = 130, inside its last page
+    g = to_dev(x)
+    sh = shape_of(x)
+    ws = torch.zeros(max(256, kl.kl_decode_workspace_size(sh, num_splits)), dtype=torch.uint8,
+                     device=_gpu.dev())
+    err = torch.zeros(1, dtype=torch.int32, device=_gpu.dev())
+    vn, pos = v_new.to(_gpu.dev()), positions.to(_gpu.dev())
+    c1, s1 = torch.from_numpy(codes).to(_gpu.dev()), torch.from_numpy(scales).to(_gpu.dev())
+    c2, s2 = c1.clone(), s1.clone()
+    out1 = torch.full((B, Hq, D), float("nan"), dtype=torch.float32, device=_gpu.dev())
+    out2 = torch.full_like(out1, float("nan"))
+    kl.kl_decode_step_fp8(sh, g["q"], g["w_r"], vn, pos, c1, s1, g["block_table"], g["seq_lens"],
+                          num_splits, out1, kl.KL_FP32, ws, err)
+    kl.kl_append_v_fp8(sh, vn, g["block_table"], pos, c2, s2, err)
+    kl.kl_decode_attention_fp8(sh, g["q"], g["w_r"], c2, s2, g["block_table"], g["seq_lens"],
+                               num_splits, out2, kl.KL_FP32, ws, err)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    want_c, want_s = oracle.append_fp8(codes, scales, bf16_bits(v_new), x["block_table"].numpy(),
+                                       positions.numpy())
+    assert np.array_equal(c1.cpu().numpy(), want_c)
+    assert np.array_equal(s1.cpu().numpy().view(np.uint32), want_s.view(np.uint32))
+    assert torch.equal(out1, out2)
+    want = oracle.decode_fp8(bf16_bits(x["q"]), bf16_bits(x["w_r"]), want_c, want_s,
+                             x["block_table"].numpy(), x["seq_lens"].numpy(),
+                             scale=1.0 / math.sqrt(128))
+    assert_parity(out1.cpu().numpy(), want, f"fp8 step S={num_splits}")
