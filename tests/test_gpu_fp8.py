@@ -170,3 +170,32 @@ def test_fp8_decode_step_appends_then_decodes(num_splits):
                              x["block_table"].numpy(), x["seq_lens"].numpy(),
                              scale=1.0 / math.sqrt(128))
     assert_parity(out1.cpu().numpy(), want, f"fp8 step S={num_splits}")
+
+
+def test_fp8_decode_step_flags_bad_position_and_page():
+    """A negative position raises KL_FLAG_BAD_POSITION and a row whose page id is -1 raises
+    KL_FLAG_BAD_PAGE; neither row is written, the valid sequence's row is."""
+    x = tiny(B=3, Hq=16, Hkv=4, D=128, P=16, lens=(40, 90, 130), seed=100)
+    codes, scales = fp8_cache(x)
+    B, Hq, D = x["q"].shape
+    v_new = torch.randn(B, 4, D, generator=torch.Generator().manual_seed(101)).to(torch.bfloat16)
+    positions = torch.tensor([39, -3, 129], dtype=torch.int32)
+    bt = x["block_table"].clone()
+    bt[2, 129 // 16] = -1                                  # page of sequence 2's new row
+    x["block_table"] = bt
+    g = to_dev(x)
+    sh = shape_of(x)
+    ws = torch.zeros(max(256, kl.kl_decode_workspace_size(sh, 1)), dtype=torch.uint8,
+                     device=_gpu.dev())
+    err = torch.zeros(1, dtype=torch.int32, device=_gpu.dev())
+    c, s = torch.from_numpy(codes).to(_gpu.dev()), torch.from_numpy(scales).to(_gpu.dev())
+    out = torch.empty(B, Hq, D, dtype=torch.float32, device=_gpu.dev())
+    kl.kl_decode_step_fp8(sh, g["q"], g["w_r"], v_new.to(_gpu.dev()), positions.to(_gpu.dev()), c, s,
+                          g["block_table"], g["seq_lens"], 1, out, kl.KL_FP32, ws, err)
+    torch.cuda.synchronize()
+    flags = int(err.item())
+    assert flags & kl.KL_FLAG_BAD_POSITION and flags & kl.KL_FLAG_BAD_PAGE
+    want_c, want_s = oracle.append_fp8(codes, scales, bf16_bits(v_new)[:1], bt.numpy()[:1],
+                                       positions.numpy()[:1])
+    assert np.array_equal(c.cpu().numpy(), want_c)
+    assert np.array_equal(s.cpu().numpy().view(np.uint32), want_s.view(np.uint32))
