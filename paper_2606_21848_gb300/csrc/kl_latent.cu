@@ -26,9 +26,11 @@
 // the O* rows from TMA boxes of the same layout.
 //
 // The three kernels overlap at their seams by programmatic dependent launch: the decode and the
-// expansion are launched as dependents of the kernel ahead of them, so the decode sets up and
-// starts streaming cache tiles while the absorbed queries are finished, and the expansion stages
-// W_post during the decode's tail; each waits for its predecessor only before reading its output.
+// expansion are launched as dependents of the kernel ahead of them. The query kernel lets the
+// decode launch once its MMAs are done, so the decode sets up and fills its ring of cache tiles
+// while the absorbed queries are stored; the decode lets the expansion launch at its set-up, so
+// the expansion stages W_post during the decode's tail. Each waits for its predecessor only
+// before reading that kernel's output.
 //
 // Roles (160 threads): warps 0-3 read and write the TMEM lanes (thread t = row t of the block);
 // warp 4 owns TMEM, issues the TMA copies and (one lane) the MMAs. Every wait is bounded (about
