@@ -34,13 +34,14 @@
 //              dim); epilogue (output row or split state). Two warps per lane quarter halve
 //              the per-thread work of a tile, which bounds the tile rate.
 //   warp 8     producer: W^R[g] (ring stages 0-1) and the group's query rows, then per tile the
-//              TMA loads of code pages and bulk copies of their scale rows
+//              TMA loads of code pages and bulk copies of their scale rows; for the decode step
+//              (kl_decode_step_fp8) it first quantizes the current token's row into the cache
+//              when that row falls in the CTA's split, before the loads of the row's tile
 //   warp 9     routing and score MMA issuer, TMEM owner
 //   warp 10    output MMA issuer; completion of a tile's output MMAs frees its ring stage
 // Every wait is bounded (about one second); a wait that runs out raises KL_FLAG_TIMEOUT and
 // every role leaves its loop, drains its copies and MMAs, and TMEM is freed.
 #include <cuda_fp16.h>
-#include <cuda_fp8.h>
 #include <cudaTypedefs.h>
 #include <math.h>
 
