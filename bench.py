@@ -257,17 +257,13 @@ def _one_core_worker(sample, scale, standard, seconds, queue):
     queue.put((oracle.threads(), seqs, el))
 
 
-def cpu_oracle_one_core(x, seconds: float, standard: bool, max_seqs: int = 4):
-    """The oracle on one host core (OMP_NUM_THREADS=1) over the first `max_seqs` sequences,
-    gathered with their own pages; run in a spawned process (this one holds a CUDA context, and
-    the OpenMP thread count is fixed when the oracle library loads)."""
-    import multiprocessing as mp
-
+def oracle_sample(x, n: int):
+    """The oracle's inputs (bf16 bits) for the batch's first n sequences over a compact pool of
+    only their own pages: (q, w_r, v_cache, block_table, seq_lens), block table renumbered."""
     import numpy as np
 
     from paper_2606_21848_gb300.workloads import bf16_bits
 
-    n = min(max_seqs, x["q"].shape[0])
     P = x["v_cache"].shape[2]
     bt_all, sl = x["block_table"].numpy()[:n], x["seq_lens"].numpy()[:n].copy()
     used = sorted({int(p) for b in range(n) for p in bt_all[b, :(int(sl[b]) + P - 1) // P]})
@@ -277,7 +273,16 @@ def cpu_oracle_one_core(x, seconds: float, standard: bool, max_seqs: int = 4):
         for j in range((int(sl[b]) + P - 1) // P):
             bt[b, j] = remap[int(bt_all[b, j])]
     v = np.ascontiguousarray(bf16_bits(x["v_cache"])[used] if used else bf16_bits(x["v_cache"])[:1])
-    sample = (np.ascontiguousarray(bf16_bits(x["q"])[:n]), bf16_bits(x["w_r"]), v, bt, sl)
+    return np.ascontiguousarray(bf16_bits(x["q"])[:n]), bf16_bits(x["w_r"]), v, bt, sl
+
+
+def cpu_oracle_one_core(x, seconds: float, standard: bool, max_seqs: int = 4):
+    """The oracle on one host core (OMP_NUM_THREADS=1) over the first `max_seqs` sequences,
+    gathered with their own pages; run in a spawned process (this one holds a CUDA context, and
+    the OpenMP thread count is fixed when the oracle library loads)."""
+    import multiprocessing as mp
+
+    sample = oracle_sample(x, min(max_seqs, x["q"].shape[0]))
     ctx = mp.get_context("spawn")
     queue = ctx.Queue()
     old = os.environ.get("OMP_NUM_THREADS")
