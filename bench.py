@@ -59,6 +59,8 @@ def parse_args():
     p.add_argument("--num-seqs", type=int, default=0,
                    help="override the workload's batch size (decode workloads; 0: as defined)")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-sweep", action="store_true",
+                   help="skip the other workloads (measured after the default line)")
     p.add_argument("--cpu-seconds", type=float, default=10.0)
     return p.parse_args()
 
@@ -301,45 +303,101 @@ def cpu_oracle_one_core(x, seconds: float, standard: bool, max_seqs: int = 4):
     return seqs / el, seqs, el, cores
 
 
+def reference_steps(run_unit, args):
+    """Time the oracle as the reference arm: `args.warmup` untimed steps, then `args.steps`
+    timed steps, each a bounded sample of the workload (the same number of units -- whole
+    sequences, or query rows -- handed to `run_unit(i)` round robin). The sample size is set
+    from the warm-up so that the timed steps together take about `args.cpu_seconds`.
+    Returns (units per second, measured ms per step, units per step, timed units)."""
+    i = 0
+    t0 = time.perf_counter()
+    for _ in range(max(1, args.warmup)):
+        run_unit(i)
+        i += 1
+    rate = max(1, args.warmup) / (time.perf_counter() - t0)
+    per_step = max(0.2, args.cpu_seconds / max(1, args.steps))
+    n = max(1, int(round(rate * per_step)))
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        for _ in range(n):
+            run_unit(i)
+            i += 1
+        times.append(time.perf_counter() - t0)
+    total = sum(times)
+    return n * args.steps / total, 1000.0 * total / args.steps, n, n * args.steps
+
+
 def run_reference(args):
     rank, world, local = dist_env()
     if rank != 0:
         return 0
-    from paper_2606_21848_gb300.workloads import WORKLOADS, generate
+    import numpy as np
+
+    from paper_2606_21848_gb300.workloads import WORKLOADS, bf16_bits, generate
 
     import oracle
-    wl = WORKLOADS[args.workload]
+    wl = workload_of(args)
     x = generate(wl)
     if wl.q_len > 0:
         return run_reference_prefill(args, wl, x)
     if wl.latent_dim > 0:
         return run_reference_latent(args, wl, x)
-    per_step = max(1.0, args.cpu_seconds / max(1, args.steps))
-    rates = []
-    total_seqs = 0
-    for i in range(args.warmup + args.steps):
-        r, n, _ = cpu_oracle_rate(x, per_step if i >= args.warmup else 0.0, args.standard)
-        if i >= args.warmup:
-            rates.append(r)
-            total_seqs += n
-    value = statistics.mean(rates)
+    q, w, v = bf16_bits(x["q"]), bf16_bits(x["w_r"]), bf16_bits(x["v_cache"])
+    bt, sl = x["block_table"].numpy(), x["seq_lens"].numpy()
+    B, Hq, D = x["q"].shape
+    scale = 1.0 / math.sqrt(D)
+    oracle.build()
+
+    def one_sequence(i):
+        heads = np.array([(i % B, h) for h in range(Hq)], np.int32)
+        if args.standard:
+            oracle.standard_decode(q, v, v, bt, sl, scale=scale, heads=heads)
+        else:
+            oracle.decode(q, w, v, bt, sl, scale=scale, heads=heads)
+
+    value, ms, n, total = reference_steps(one_sequence, args)
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": 1000.0 * wl.num_seqs / value, "higher_is_better": True,
+        "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": wl.name, "num_seqs": wl.num_seqs, "q_heads": wl.num_q_heads,
-                   "kv_heads": wl.num_kv_heads, "head_dim": wl.head_dim,
-                   "page_size": wl.page_size, "seq_len": wl.seq_len or list(wl.seq_len_range)},
+        "config": decode_config(wl, x, args, args.gpus),
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": oracle.threads(),
                          "kind": "oracle",
-                         "sample": f"{total_seqs} whole sequences (all heads, decode only) "
-                                   f"of {wl.name}, ~{per_step:.1f}s per step"},
+                         "sample": f"each step: {n} whole sequences (all {Hq} heads, decode "
+                                   f"only, fp64) of {wl.name}, round robin; {total} timed"},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
     return 0
+
+
+def workload_of(args):
+    """The selected workload with the command line's overrides."""
+    from paper_2606_21848_gb300.workloads import WORKLOADS
+    wl = WORKLOADS[args.workload]
+    if args.wr_per_query_head:
+        wl = wl.with_(wr_per_query_head=True)
+    if args.num_seqs > 0:
+        wl = wl.with_(num_seqs=args.num_seqs)
+    return wl
+
+
+def decode_config(wl, x, args, world) -> dict:
+    """The workload a decode line measures (the same keys and values for both arms)."""
+    B, Hq, D = x["q"].shape
+    Hkv, P = x["v_cache"].shape[1], x["v_cache"].shape[2]
+    return {"workload": wl.name, "num_seqs": B, "q_heads": Hq, "kv_heads": Hkv,
+            "head_dim": D, "page_size": P, "seq_len": wl.seq_len or list(wl.seq_len_range),
+            "context_tokens": int(x["seq_lens"].sum()),
+            "cache": "fp8 e4m3 + fp32 row scale" if args.fp8_cache else "bf16",
+            "decode": "standard K+V (comparison)" if args.standard else
+                      "keyless, composed query (x W^Q W^R)" if args.fused_query else "keyless",
+            "w_r": "per query head" if wl.wr_per_query_head else "per value head",
+            "l2": "GPU arm: flushed between timed steps (512 MiB write, then read back)",
+            "parallelism": f"replicas x{world}"}
 
 
 # ----------------------------------------------------------------------------- GPU arm --
@@ -359,11 +417,7 @@ def run_ours(args):
     dev = torch.device("cuda", local)
     kl.load()
 
-    wl = WORKLOADS[args.workload]
-    if args.wr_per_query_head:
-        wl = wl.with_(wr_per_query_head=True)
-    if args.num_seqs > 0:
-        wl = wl.with_(num_seqs=args.num_seqs)
+    wl = workload_of(args)
     from paper_2606_21848_gb300.multi import job_throughput, max_over_ranks, replica_seed
     x = generate(wl, seed=replica_seed(wl.seed, rank))   # replicas: each rank its own batch
     if wl.q_len > 0:
@@ -523,6 +577,12 @@ def run_ours(args):
         e2e = {"value": B * world / (e2e_ms / 1e3), "unit": "tokens/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms}
 
+    sweep = None
+    if (world == 1 and not args.no_sweep and args.workload == DEFAULT_WORKLOAD and
+            not (args.standard or args.fp8_cache or args.fused_query or args.wr_per_query_head
+                 or args.num_seqs or args.num_splits >= 0 or args.kernel != "auto")):
+        sweep = sweep_workloads(args, dev, stream, flush_l2, x, g, sh, mean_dec)
+
     if rank != 0:
         return 0
 
@@ -544,17 +604,8 @@ def run_ours(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": mean_step,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded; inputs resident in HBM)",
-        "config": {"workload": wl.name, "num_seqs": B, "q_heads": Hq, "kv_heads": Hkv,
-                   "head_dim": D, "page_size": P,
-                   "seq_len": wl.seq_len or list(wl.seq_len_range),
-                   "context_tokens": ab["tokens"], "num_splits": S, "kernel": kname,
-                   "cache": "fp8 e4m3 + fp32 row scale" if args.fp8_cache else "bf16",
-                   "decode": "standard K+V (comparison)" if args.standard else
-                             "keyless, composed query (x W^Q W^R)" if args.fused_query else
-                             "keyless",
-                   "w_r": "per query head" if wl.wr_per_query_head else "per value head",
-                   "l2": "flushed between timed steps (512 MiB write, then read back)",
-                   "parallelism": f"replicas x{world}"},
+        "config": decode_config(wl, x, args, world),
+        "launch": {"num_splits": S, "kernel": kname},
         "hbm_gbs_step": step_gbs,
         "pct_of_8tbs_step": 100.0 * step_gbs / NOMINAL_HBM_GBS,
         "ms_breakdown": {"decode": mean_dec, "combine": statistics.mean(comb_ms)},
@@ -569,10 +620,200 @@ def run_ours(args):
         "e2e": e2e,
         "cpu_baseline": cpu,
     }
+    if sweep is not None:
+        line.update(sweep)
     print(json.dumps(line), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()
     return 0
+
+
+def time_device(step, args, stream, flush_l2):
+    """Mean CUDA-event time (ms) of `step()` on `stream` over args.steps timed steps after
+    args.warmup untimed ones, L2 flushed before every step."""
+    import torch
+    E = lambda: torch.cuda.Event(enable_timing=True)
+    for _ in range(args.warmup):
+        flush_l2()
+        step()
+    torch.cuda.synchronize()
+    evs = [(E(), E()) for _ in range(args.steps)]
+    for a, b in evs:
+        flush_l2()
+        a.record(stream)
+        step()
+        b.record(stream)
+    torch.cuda.synchronize()
+    return statistics.mean(a.elapsed_time(b) for a, b in evs)
+
+
+def sweep_workloads(args, dev, stream, flush_l2, x70, g70, sh70, keyless_ms):
+    """The other workloads, measured in the same process with the same timing (L2 flushed
+    before every step, CUDA events on the launching stream): the four other decode workloads
+    (one step = kl_decode_step), the same-design K+V decode on the default batch against the
+    keyless decode of the same batch, the FP8 value cache on the default batch, the latent
+    value-only cache and the chunked prefill."""
+    import torch
+
+    import paper_2606_21848_gb300 as kl
+    from paper_2606_21848_gb300.workloads import ORDER, WORKLOADS, generate
+
+    peak, peak_kind = measured_peaks()
+    launches = 0
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+
+    def gbs_entry(ms, nbytes, B, extra):
+        gbs = nbytes / (ms / 1e3) / 1e9
+        e = {"ms": ms, "tokens_per_s": B / (ms / 1e3), "gb_s": gbs, "frac": gbs / peak,
+             "pct_of_8tbs": 100.0 * gbs / NOMINAL_HBM_GBS, "algorithmic_bytes": nbytes}
+        e.update(extra)
+        return e
+
+    workloads = {}
+    for name in ORDER:
+        if name == DEFAULT_WORKLOAD:
+            continue
+        wl = WORKLOADS[name]
+        x = generate(wl)
+        B, Hq, D = x["q"].shape
+        num_pages, Hkv, P, _ = x["v_cache"].shape
+        sh = kl.make_shape(B, Hq, Hkv, D, P, num_pages, x["block_table"].shape[1])
+        g = {k: x[k].to(dev) for k in ("q", "w_r", "v_cache", "block_table", "seq_lens",
+                                        "positions", "v_new")}
+        out = torch.empty(B, Hq, D, dtype=torch.bfloat16, device=dev)
+        plans = [("", wl.num_splits)] + ([("auto_plan", 0)] if wl.num_splits else [])
+        for suffix, req in plans:
+            S = kl.kl_decode_num_splits(sh, req)
+            ws = torch.zeros(max(256, kl.kl_decode_workspace_size(sh, req)), dtype=torch.uint8,
+                             device=dev)
+            opts = kl.decode_options(req)
+            tc = bool(kl.kl_decode_kernel_available(sh, kl.KL_KERNEL_TENSOR, False))
+
+            def step():
+                kl.kl_decode_step(sh, g["q"], g["w_r"], g["v_new"], g["positions"], g["v_cache"],
+                                  g["block_table"], g["seq_lens"], opts, out, kl.KL_BF16, ws, err,
+                                  stream)
+
+            ms = time_device(step, args, stream, flush_l2)
+            n_launch = 1 if (tc or S == 1) else 2
+            launches += n_launch * args.steps
+            ab = algorithmic_bytes(x, False)
+            workloads[name + ("_" + suffix if suffix else "")] = gbs_entry(
+                ms, ab["total"], B, {"num_splits": S, "kernel": "tensor" if tc else "simt",
+                                     "kernels_per_step": n_launch,
+                                     "context_tokens": ab["tokens"]})
+        del g, out, ws, x
+        torch.cuda.empty_cache()
+
+    # The K+V comparison: the same kernel reading a K tile and a V tile per 128 tokens, with
+    # K = V (W^R)^T so that it computes the same attention, against the keyless decode (without
+    # the append) of the same batch.
+    B, Hq, D = x70["q"].shape
+    Hkv = x70["v_cache"].shape[1]
+    out = torch.empty(B, Hq, D, dtype=torch.bfloat16, device=dev)
+    ws = torch.zeros(max(256, kl.kl_decode_workspace_size(sh70, 0)), dtype=torch.uint8, device=dev)
+    opts = kl.decode_options(0)
+    keyless_no_append = time_device(
+        lambda: kl.kl_decode_attention_ex(sh70, g70["q"], g70["w_r"], g70["v_cache"],
+                                          g70["block_table"], g70["seq_lens"], opts, out,
+                                          kl.KL_BF16, ws, err, stream), args, stream, flush_l2)
+    k_cache = torch.empty_like(g70["v_cache"])
+    for h in range(Hkv):
+        k_cache[:, h] = (g70["v_cache"][:, h].float() @ g70["w_r"][h].float().t()).to(torch.bfloat16)
+    standard = time_device(
+        lambda: kl.kl_standard_decode(sh70, g70["q"], k_cache, g70["v_cache"], g70["block_table"],
+                                      g70["seq_lens"], opts, out, kl.KL_BF16, ws, err, stream),
+        args, stream, flush_l2)
+    launches += 2 * args.steps
+    del k_cache
+    torch.cuda.empty_cache()
+    ab_k = algorithmic_bytes(x70, False)
+    ab_s = algorithmic_bytes(x70, True)
+    kv = {"workload": DEFAULT_WORKLOAD,
+          "keyless_decode": gbs_entry(keyless_no_append, ab_k["total"] - B * Hkv * D * 4, B, {"what": "kl_decode_attention (no append)"}),
+          "standard_kv_decode": gbs_entry(standard, ab_s["total"], B,
+                                          {"what": "kl_standard_decode, K = V (W^R)^T"}),
+          "time_ratio_standard_over_keyless": standard / keyless_no_append,
+          "cache_bytes_ratio": ab_s["cache"] / ab_k["cache"]}
+
+    # The FP8 value cache of the default batch (codes + one fp32 scale per row), quantized
+    # once on the GPU; one step = kl_decode_step_fp8 (the quantizing append inside the decode).
+    codes = torch.empty(g70["v_cache"].shape, dtype=torch.uint8, device=dev)
+    scales = torch.empty(g70["v_cache"].shape[:-1], dtype=torch.float32, device=dev)
+    kl.kl_quantize_cache_fp8(sh70, g70["v_cache"], codes, scales, stream)
+    S8 = kl.kl_decode_num_splits(sh70, 0)
+    ws8 = torch.zeros(max(256, kl.kl_decode_workspace_size(sh70, 0)), dtype=torch.uint8,
+                      device=dev)
+    fp8_ms = time_device(
+        lambda: kl.kl_decode_step_fp8(sh70, g70["q"], g70["w_r"], g70["v_new"], g70["positions"],
+                                      codes, scales, g70["block_table"], g70["seq_lens"], 0, out,
+                                      kl.KL_BF16, ws8, err, stream), args, stream, flush_l2)
+    launches += (1 + (S8 > 1)) * args.steps
+    del codes, scales, ws8
+    torch.cuda.empty_cache()
+    ab8 = algorithmic_bytes(x70, False, fp8=True)
+    fp8 = gbs_entry(fp8_ms, ab8["total"], B, {"workload": DEFAULT_WORKLOAD,
+                                              "what": "kl_decode_step_fp8",
+                                              "speedup_over_bf16_step": keyless_ms / fp8_ms})
+
+    # Latent value-only cache: one step = kl_latent_decode_step (three kernels).
+    wl = WORKLOADS["latent_serving"]
+    x = generate(wl)
+    B, Hq, D = x["q"].shape
+    num_pages, Hl, P, r = x["v_lat"].shape
+    lsh = kl.make_latent_shape(B, Hq, Hl, D, r, P, num_pages, x["block_table"].shape[1])
+    g = {k: x[k].to(dev) for k in ("q", "w_r", "w_post", "v_lat", "block_table", "seq_lens",
+                                    "positions", "v_new")}
+    lout = torch.empty(B, Hq, D, dtype=torch.bfloat16, device=dev)
+    lws = torch.zeros(kl.kl_latent_workspace_size(lsh, 0), dtype=torch.uint8, device=dev)
+    lat_ms = time_device(
+        lambda: kl.kl_latent_decode_step(lsh, g["q"], g["w_r"], g["w_post"], g["v_new"],
+                                         g["positions"], g["v_lat"], g["block_table"],
+                                         g["seq_lens"], 0, lout, kl.KL_BF16, lws, err, stream),
+        args, stream, flush_l2)
+    launches += 3 * args.steps
+    latent = gbs_entry(lat_ms, latent_bytes(x)["total"], B,
+                       {"workload": wl.name, "what": "kl_latent_decode_step"})
+    del g, lout, lws, x
+    torch.cuda.empty_cache()
+
+    # Chunked prefill: one step = kl_append_v_chunk + kl_prefill_attention; useful FLOPs of the
+    # prefill kernel against the measured bf16 peak.
+    wl = WORKLOADS["prefill_chunked_gqa"]
+    x = generate(wl)
+    T, Hq, D = x["q_chunk"].shape
+    B = x["seq_lens"].shape[0]
+    num_pages, Hkv, P, _ = x["v_cache"].shape
+    psh = kl.make_shape(B, Hq, Hkv, D, P, num_pages, x["block_table"].shape[1])
+    g = {k: x[k].to(dev) for k in ("q_chunk", "v_chunk", "w_r", "v_cache", "block_table",
+                                    "seq_lens", "cu_q")}
+    pout = torch.empty(T, Hq, D, dtype=torch.bfloat16, device=dev)
+    max_q = int(x["q_lens"].max())
+    pre_ms = time_device(
+        lambda: kl.kl_prefill_attention(psh, g["q_chunk"], g["w_r"], g["v_cache"],
+                                        g["block_table"], g["seq_lens"], g["cu_q"], T, max_q,
+                                        pout, kl.KL_BF16, err, stream), args, stream, flush_l2)
+    launches += args.steps
+    fl = prefill_flops(x)
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            tpeak = float(json.load(f)["bf16_tflops"])
+    except Exception:
+        tpeak = 1900.0
+    tfl = fl["total"] / (pre_ms / 1e3) / 1e12
+    prefill = {"workload": wl.name, "what": "kl_prefill_attention", "ms": pre_ms,
+               "query_tokens_per_s": T / (pre_ms / 1e3), "useful_tflops": tfl,
+               "frac_of_bf16_peak": tfl / tpeak, "bf16_peak_tflops": tpeak,
+               "note": "hi + lo bf16 operands issue twice the useful MMA work"}
+    del g, pout, x
+    torch.cuda.empty_cache()
+
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0, f"device error flags {int(err.item())} in the sweep"
+    return {"workloads": workloads, "kv_comparison": kv, "fp8_cache": fp8, "latent": latent,
+            "prefill": prefill, "sweep_gpu_launches": launches,
+            "sweep_timing": "each entry: mean of --steps CUDA-event-timed steps after --warmup, "
+                            "L2 flushed before every step, in this process"}
 
 
 # --------------------------------------------------------------------------- prefill ----
@@ -624,33 +865,53 @@ def cpu_oracle_prefill_rate(x, seconds: float):
 
 
 def run_reference_prefill(args, wl, x):
+    import numpy as np
+
     import oracle
-    per_step = max(1.0, args.cpu_seconds / max(1, args.steps))
-    rates, total = [], 0
-    for i in range(args.warmup + args.steps):
-        rt, n, _ = cpu_oracle_prefill_rate(x, per_step if i >= args.warmup else 0.0)
-        if i >= args.warmup:
-            rates.append(rt)
-            total += n
-    value = statistics.mean(rates)
-    T = int(x["cu_q"][-1])
+    from paper_2606_21848_gb300.workloads import bf16_bits
+
+    q, w, v = bf16_bits(x["q_chunk"]), bf16_bits(x["w_r"]), bf16_bits(x["v_cache"])
+    bt, sl, cu = x["block_table"].numpy(), x["seq_lens"].numpy(), x["cu_q"].numpy()
+    T, Hq, D = x["q_chunk"].shape
+    wr_pq = bool(wl.wr_per_query_head)
+    oracle.build()
+    stride = 7919                       # a fixed walk over the rows, early and late positions
+
+    def one_row(i):
+        sel = np.array([((i * stride) % T, h) for h in range(Hq)], np.int32)
+        oracle.prefill(q, w, v, bt, sl, cu, scale=1.0 / math.sqrt(D), wr_per_query_head=wr_pq,
+                       rows=sel)
+
+    value, ms, n, total = reference_steps(one_row, args)
+    B = x["seq_lens"].shape[0]
+    num_pages, Hkv, P, _ = x["v_cache"].shape
     line = {
         "impl": "reference", "metric": PREFILL_METRIC, "value": value, "unit": "tokens/s",
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": 1000.0 * T / value, "higher_is_better": True, "scaling": "weak",
+        "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": wl.name, "num_seqs": wl.num_seqs, "q_heads": wl.num_q_heads,
-                   "kv_heads": wl.num_kv_heads, "head_dim": wl.head_dim,
-                   "page_size": wl.page_size, "seq_len": wl.seq_len, "chunk": wl.q_len},
+        "config": prefill_config(wl, x, args.gpus),
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": oracle.threads(),
                          "kind": "oracle",
-                         "sample": f"{total} query rows (all heads) of {wl.name} on a fixed "
-                                   f"stride over the chunk, ~{per_step:.1f}s per step"},
+                         "sample": f"each step: {n} query rows (all {Hq} heads, fp64) of "
+                                   f"{wl.name} on a fixed stride over the chunk; {total} timed"},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
     return 0
+
+
+def prefill_config(wl, x, world) -> dict:
+    T, Hq, D = x["q_chunk"].shape
+    B = x["seq_lens"].shape[0]
+    Hkv, P = x["v_cache"].shape[1], x["v_cache"].shape[2]
+    return {"workload": wl.name, "num_seqs": B, "q_heads": Hq, "kv_heads": Hkv,
+            "head_dim": D, "page_size": P, "seq_len": wl.seq_len, "chunk": wl.q_len,
+            "query_rows": T, "visible_pairs": prefill_flops(x)["pairs"],
+            "w_r": "per query head" if wl.wr_per_query_head else "per value head",
+            "l2": "GPU arm: flushed between timed steps (512 MiB write, then read back)",
+            "parallelism": f"replicas x{world}"}
 
 
 def run_prefill(args, wl, x, dev, rank, world):
@@ -765,13 +1026,8 @@ def run_prefill(args, wl, x, dev, rank, world):
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded; inputs resident in HBM)",
-        "config": {"workload": wl.name, "num_seqs": B, "q_heads": Hq, "kv_heads": Hkv,
-                   "head_dim": D, "page_size": P, "seq_len": wl.seq_len, "chunk": wl.q_len,
-                   "query_rows": T, "visible_pairs": fl["pairs"],
-                   "w_r": "per query head" if wl.wr_per_query_head else "per value head",
-                   "operands": "hi + lo bf16 pairs (2x the attention MMA work)",
-                   "l2": "flushed between timed steps (512 MiB write, then read back)",
-                   "parallelism": f"replicas x{world}"},
+        "config": prefill_config(wl, x, world),
+        "operands": "hi + lo bf16 pairs (2x the attention MMA work)",
         "ms_breakdown": {"append": app_ms, "prefill": pre_ms},
         "tflops": tflops,
         "kernels_per_step": 2,
@@ -833,33 +1089,48 @@ def cpu_oracle_latent_rate(x, seconds: float):
 
 
 def run_reference_latent(args, wl, x):
+    import numpy as np
+
     import oracle
-    per_step = max(1.0, args.cpu_seconds / max(1, args.steps))
-    rates, total = [], 0
-    for i in range(args.warmup + args.steps):
-        rt, n, _ = cpu_oracle_latent_rate(x, per_step if i >= args.warmup else 0.0)
-        if i >= args.warmup:
-            rates.append(rt)
-            total += n
-    value = statistics.mean(rates)
+    from paper_2606_21848_gb300.workloads import bf16_bits
+    q, w, wp, v = (bf16_bits(x[k]) for k in ("q", "w_r", "w_post", "v_lat"))
+    bt, sl = x["block_table"].numpy(), x["seq_lens"].numpy()
+    B, Hq, D = x["q"].shape
+    r = x["v_lat"].shape[3]
+    oracle.build()
+
+    def one_sequence(i):
+        heads = np.array([(i % B, h) for h in range(Hq)], np.int32)
+        oracle.latent_decode(q, w, wp, v, bt, sl, scale=1.0 / math.sqrt(r), heads=heads)
+
+    value, ms, n, total = reference_steps(one_sequence, args)
     line = {
         "impl": "reference", "metric": LATENT_METRIC, "value": value, "unit": "tokens/s",
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": 1000.0 * wl.num_seqs / value, "higher_is_better": True,
+        "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": wl.name, "num_seqs": wl.num_seqs, "q_heads": wl.num_q_heads,
-                   "latent_heads": wl.num_kv_heads, "head_dim": wl.head_dim,
-                   "latent_dim": wl.latent_dim, "page_size": wl.page_size,
-                   "seq_len": wl.seq_len},
+        "config": latent_config(wl, x, args.gpus),
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": oracle.threads(),
                          "kind": "oracle",
-                         "sample": f"{total} whole sequences (all heads) of {wl.name}, "
-                                   f"~{per_step:.1f}s per step"},
+                         "sample": f"each step: {n} whole sequences (all {Hq} heads, fp64) of "
+                                   f"{wl.name}, round robin; {total} timed"},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
     return 0
+
+
+def latent_config(wl, x, world) -> dict:
+    B, Hq, D = x["q"].shape
+    num_pages, Hl, P, r = x["v_lat"].shape
+    return {"workload": wl.name, "num_seqs": B, "q_heads": Hq, "latent_heads": Hl,
+            "head_dim": D, "latent_dim": r, "page_size": P, "seq_len": wl.seq_len,
+            "context_tokens": int(x["seq_lens"].sum()),
+            "w_r": "per query head" if wl.wr_per_query_head else "per latent group",
+            "w_post": "per query head",
+            "l2": "GPU arm: flushed between timed steps (512 MiB write, then read back)",
+            "parallelism": f"replicas x{world}"}
 
 
 def run_latent(args, wl, x, dev, rank, world):
@@ -968,13 +1239,8 @@ def run_latent(args, wl, x, dev, rank, world):
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded; inputs resident in HBM)",
-        "config": {"workload": wl.name, "num_seqs": B, "q_heads": Hq, "latent_heads": Hl,
-                   "head_dim": D, "latent_dim": r, "page_size": P, "seq_len": wl.seq_len,
-                   "context_tokens": ab["tokens"], "num_splits": S,
-                   "w_r": "per query head" if wl.wr_per_query_head else "per latent group",
-                   "w_post": "per query head",
-                   "l2": "flushed between timed steps (512 MiB write, then read back)",
-                   "parallelism": f"replicas x{world}"},
+        "config": latent_config(wl, x, world),
+        "launch": {"num_splits": S},
         "ms_breakdown": {"latent_decode_step": step_ms},
         "kernels_per_step": 3,
         "roofline": {"bound": "hbm", "achieved": dec_gbs, "peak": peak, "unit": "GB/s",

@@ -375,7 +375,10 @@ kl_status kl_decode_step_fp8(const kl_shape *shape, const void *q, const void *w
  * The split states live in one fixed array of KL_NOALLOC_SCRATCH_BYTES in device memory,
  * which every GPU that loads the library holds until the process exits. The library looks
  * up that array's device address during the first call on each device (with that device
- * current); make that first call before any stream capture. Nothing is allocated and no
+ * current); make that first call before any stream capture. The address belongs to the CUDA
+ * context it was looked up in: the library records that context's unique id and looks the
+ * address up again when a call finds a different context current on the device (after
+ * cudaDeviceReset, for instance), so that call too is a first call. Nothing is allocated and no
  * allocating routine is called. Every call on a device shares the one array and leaves its
  * contents behind, so calls that may overlap on the GPU (different streams, or different
  * host threads without ordering) race and must be serialized by the caller. A shape and

@@ -23,7 +23,7 @@
  *   - decode over a latent value-only cache (Section 3, latent value-only cache paragraph);
  *   - the FP8 (E4M3, one fp32 scale per cached row) value cache: encoding, append, decode.
  *
- * Readings where the paper is silent (each is listed in the design notes):
+ * Readings taken where the paper is silent:
  *   - lambda / sqrt(d_k) is the caller's `scale`; lambda = 1 gives 1/sqrt(d_k);
  *   - query head h reads value head h / (Hq / Hkv) (contiguous groups);
  *   - W^R holds either Hkv matrices (indexed by value head) or Hq matrices (by query head);
@@ -545,8 +545,9 @@ int ko_latent_decode(int B, int Hq, int Hl, int D, int r, int P, int num_pages, 
 }
 
 /*
- * FP8 value cache (the low-precision value cache of the scope table: orthogonal to the method,
- * compatible with it). Values are stored as OCP FP8 E4M3 codes (1 sign bit, 4 exponent bits
+ * FP8 value cache. Section 3 states that the value-only cache is orthogonal to other
+ * KV-cache reduction methods, so it composes with a quantized cache; the paper fixes no format,
+ * and this one is the reading taken. Values are stored as OCP FP8 E4M3 codes (1 sign bit, 4 exponent bits
  * with bias 7, 3 mantissa bits; exponent field 0 encodes subnormals m/8 * 2^-6; the all-ones
  * exponent with all-ones mantissa is NaN; no infinities; largest finite value 448) with one
  * fp32 scale per cached row: v = scale * value(code).

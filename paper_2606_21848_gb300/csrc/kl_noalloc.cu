@@ -1,6 +1,8 @@
 // kl_decode_attention_noalloc: the keyless decode for callers that cannot allocate device
 // memory. The split states that kl_decode_attention keeps in a caller-provided workspace live
 // here in one fixed, file-scope device array instead.
+#include <cudaTypedefs.h>
+
 #include <mutex>
 
 #include "kl_internal.cuh"
@@ -15,21 +17,52 @@ static __device__ __align__(256) unsigned char g_split_scratch[kScratchBytes];
 
 constexpr int kMaxDevices = 64;
 std::mutex g_setup_mutex;
+// Per device: the device address of the scratch array and the id of the CUDA context it was
+// looked up in. The address belongs to the module loaded into that context, so a new context on
+// the device (after cudaDeviceReset, say) gets its own lookup.
 void *g_scratch_ptr[kMaxDevices] = {nullptr};
+unsigned long long g_scratch_ctx[kMaxDevices] = {0};
 
-// Device address of the scratch array on the current device, looked up once per device.
-// Host code cannot use the symbol itself as a device address.
+// The unique id of the calling thread's current context (0 if it cannot be read).
+unsigned long long current_context_id() {
+    static PFN_cuCtxGetCurrent_v4000 get_current = nullptr;
+    static PFN_cuCtxGetId_v12000 get_id = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) ==
+                cudaSuccess && q == cudaDriverEntryPointSuccess)
+            get_current = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(p);
+        p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess && q == cudaDriverEntryPointSuccess)
+            get_id = reinterpret_cast<PFN_cuCtxGetId_v12000>(p);
+    });
+    if (!get_current || !get_id) return 0;
+    CUcontext ctx = nullptr;
+    unsigned long long id = 0;
+    if (get_current(&ctx) != CUDA_SUCCESS || !ctx || get_id(ctx, &id) != CUDA_SUCCESS) return 0;
+    return id;
+}
+
+// Device address of the scratch array for the current device and context. Host code cannot
+// use the symbol itself as a device address: cudaGetSymbolAddress translates it, once per
+// device and context (the runtime makes the device's primary context current first).
 cudaError_t scratch_for_current_device(void **out) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
     std::lock_guard<std::mutex> lock(g_setup_mutex);
-    if (!g_scratch_ptr[dev]) {
+    const unsigned long long ctx = current_context_id();
+    if (!g_scratch_ptr[dev] || ctx == 0 || ctx != g_scratch_ctx[dev]) {
         void *p = nullptr;
         e = cudaGetSymbolAddress(&p, g_split_scratch);
         if (e != cudaSuccess) return e;
         g_scratch_ptr[dev] = p;
+        // the context id is read again after the lookup, which may have created the context
+        g_scratch_ctx[dev] = current_context_id();
     }
     *out = g_scratch_ptr[dev];
     return cudaSuccess;
@@ -57,7 +90,9 @@ extern "C" kl_status kl_decode_attention_noalloc(const kl_shape *shape, const vo
     const size_t o_bytes = round_up256(rows * shape->head_dim * sizeof(float));
     const size_t ml_bytes = round_up256(rows * 2 * sizeof(float));
     if (o_bytes + ml_bytes > kScratchBytes) return KL_ERR_WORKSPACE;
-    if (!out) return KL_ERR_INVALID_ARG;
+    // the decode below writes split states, not `out`, so `out` is checked here as
+    // kl_decode_attention checks it
+    if (!out || (reinterpret_cast<uintptr_t>(out) & 15u) != 0) return KL_ERR_INVALID_ARG;
 
     void *base = nullptr;
     if (scratch_for_current_device(&base) != cudaSuccess) return KL_ERR_CUDA;
