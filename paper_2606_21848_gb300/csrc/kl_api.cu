@@ -22,6 +22,7 @@ int device_sm_count() {
 namespace {
 
 constexpr int kChunkQuantum = 128;  // split boundaries fall on multiples of 128 tokens
+constexpr int kSimtMaxGroup = 8;    // query heads per value head of the CUDA-core kernel
 constexpr int kMaxSplits = 1024;
 
 bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
@@ -51,6 +52,8 @@ kl_status resolve(const kl_shape *s, int32_t num_splits, Geometry *g) {
     g->scale = s->scale > 0.f ? s->scale : 1.0f / sqrtf((float)s->head_dim);
     g->S = 1;
     g->chunk = 0;
+    g->nhb = (g->G + 7) / 8;
+    g->qbox = g->G < 8 ? g->G : 8;
     if (num_splits < 0) return KL_OK;
     if (num_splits > kMaxSplits) return KL_ERR_INVALID_ARG;
 
@@ -60,7 +63,7 @@ kl_status resolve(const kl_shape *s, int32_t num_splits, Geometry *g) {
         // As many splits as fit one wave of two CTAs per SM over the (value head, sequence)
         // units, and splits of at most 8192 tokens so that ragged batches balance; never
         // below 256 tokens per split.
-        const int64_t units = (int64_t)(g->B > 0 ? g->B : 1) * g->Hkv;
+        const int64_t units = (int64_t)(g->B > 0 ? g->B : 1) * g->Hkv * g->nhb;
         const int64_t slots = 2 * (int64_t)device_sm_count();
         const int64_t fill = units < slots ? slots / units : 1;
         const int64_t cap = (Lmax + 8191) / 8192;
@@ -82,7 +85,8 @@ struct WorkspaceLayout {
     size_t part_o, part_ml, counters, total;
 };
 
-// [B][Hq][S][D] fp32 states, [B][Hq][S][2] fp32 {m, l}, [B][Hkv] u32 merge counters.
+// [B][Hq][S][D] fp32 states, [B][Hq][S][2] fp32 {m, l}, [B][Hkv][nhb] u32 merge counters (one
+// per sequence and block of up to 8 query heads of a value head).
 WorkspaceLayout layout(const Geometry &g) {
     WorkspaceLayout w{0, 0, 0, 0};
     if (g.S <= 1) return w;
@@ -90,7 +94,7 @@ WorkspaceLayout layout(const Geometry &g) {
     w.part_o = 0;
     w.part_ml = round_up(rows * g.D * sizeof(float), 256);
     w.counters = w.part_ml + round_up(rows * 2 * sizeof(float), 256);
-    w.total = w.counters + round_up((size_t)g.B * g.Hkv * sizeof(unsigned int), 256);
+    w.total = w.counters + round_up((size_t)g.B * g.Hkv * g.nhb * sizeof(unsigned int), 256);
     return w;
 }
 
@@ -110,7 +114,6 @@ kl_status decode_common(bool standard, const kl_shape *shape, const void *q, con
     Geometry g;
     kl_status st = resolve(shape, ns, &g);
     if (st != KL_OK) return st;
-    if (g.G > 8) return KL_ERR_UNSUPPORTED;
     if (g.B == 0) return KL_OK;
     if ((!q && !q_routed) || !v_cache || !block_table || !seq_lens) return KL_ERR_INVALID_ARG;
     if (standard && !k_cache) return KL_ERR_INVALID_ARG;   // keyless: w_r == NULL = composed q
@@ -160,6 +163,8 @@ kl_status decode_common(bool standard, const kl_shape *shape, const void *q, con
     } else if (kernel == KL_KERNEL_AUTO) {
         use_tc = tc_supported(g, standard);
     }
+    // the CUDA-core kernel serves groups of up to 8 query heads
+    if (!use_tc && g.G > kSimtMaxGroup) return KL_ERR_UNSUPPORTED;
     a.merge_inside = use_tc && !states && tc_merge_inside(g, standard);
     cudaError_t e = use_tc ? launch_decode_tc(a, standard) : launch_decode_simt(a, standard);
     if (e == cudaSuccess) e = finish_decode(a, states);
@@ -407,7 +412,7 @@ kl_status decode_fp8(const kl_shape *shape, const void *q, const void *w_r, cons
     Geometry g;
     kl_status st = resolve(shape, num_splits, &g);
     if (st != KL_OK) return st;
-    if (g.G > 8 || g.wr_per_qh || !tc_supported(g, false)) return KL_ERR_UNSUPPORTED;
+    if (g.wr_per_qh || !tc_supported(g, false)) return KL_ERR_UNSUPPORTED;
     if (g.P < 4) return KL_ERR_UNSUPPORTED;
     if (g.B == 0) return KL_OK;
     // Runs of splits: when one CTA per split would overflow a wave of two CTAs per SM while the
@@ -416,7 +421,8 @@ kl_status decode_fp8(const kl_shape *shape, const void *q, const void *w_r, cons
     // associative merge of adjacent states): the split chunk widens by that factor. The split
     // states stay internal to this entry point (merged by the combine kernel).
     {
-        const int64_t units = (int64_t)g.B * g.Hkv, slots = 2 * (int64_t)device_sm_count();
+        const int64_t units = (int64_t)g.B * g.Hkv * g.nhb;
+        const int64_t slots = 2 * (int64_t)device_sm_count();
         int spc = 1;
         if (g.S > 1 && units < slots)
             while ((int64_t)((g.S + spc - 1) / spc) * units > slots) ++spc;
@@ -562,9 +568,12 @@ kl_status kl_latent_decode_step(const kl_latent_shape *shape, const void *q, con
 
 int32_t kl_decode_kernel_available(const kl_shape *shape, int32_t kernel, int32_t standard) {
     Geometry g;
-    if (resolve(shape, 1, &g) != KL_OK || g.G > 8) return 0;
-    if (kernel == KL_KERNEL_SIMT || kernel == KL_KERNEL_AUTO) return 1;
-    if (kernel == KL_KERNEL_TENSOR) return tc_supported(g, standard != 0) ? 1 : 0;
+    if (resolve(shape, 1, &g) != KL_OK) return 0;
+    const bool tc = tc_supported(g, standard != 0);
+    const bool simt = g.G <= kSimtMaxGroup;
+    if (kernel == KL_KERNEL_SIMT) return simt ? 1 : 0;
+    if (kernel == KL_KERNEL_AUTO) return (tc || simt) ? 1 : 0;
+    if (kernel == KL_KERNEL_TENSOR) return tc ? 1 : 0;
     return 0;
 }
 

@@ -291,9 +291,14 @@ __global__ void __launch_bounds__(kThreads, 2)
     Smem8 &sm = *reinterpret_cast<Smem8 *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                            ~uintptr_t(1023));
     const Geometry &geo = a.geo;
-    const int split = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+    // A group of more than 8 query heads is served by geo.nhb sibling CTAs, adjacent in
+    // blockIdx.x, each for up to 8 of its heads (the second and later reads of a page come
+    // from L2).
+    const int hb = blockIdx.x % geo.nhb, split = blockIdx.x / geo.nhb;
+    const int g = blockIdx.y, b = blockIdx.z;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int G = geo.G;
+    const int G = min(8, geo.G - 8 * hb);       // query heads of this CTA
+    const int qh0 = g * geo.G + 8 * hb;          // its first query head within the sequence
     const bool route = a.w_r != nullptr;      // W^R given; else q is the composed query
     // Ring uses: with routing, uses 0 and 1 are the W^R halves and tile i is use i + 2.
     const int base = route ? 2 : 0;
@@ -379,7 +384,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         // an empty split: zero output (direct) or an empty state
         if (tid < kD) {
             for (int h = 0; h < G; ++h) {
-                const size_t bh = (size_t)b * geo.Hq + g * G + h;
+                const size_t bh = (size_t)b * geo.Hq + qh0 + h;
                 if (a.direct_out) {
                     if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * kD + tid] = 0.f;
                     else static_cast<__nv_bfloat16 *>(a.out)[bh * kD + tid] = __float2bfloat16_rn(0.f);
@@ -419,10 +424,10 @@ __global__ void __launch_bounds__(kThreads, 2)
             if (lane == 0) {
                 // W^R[g] halves into stages 0 and 1 (MN-major A of the routing MMA); the
                 // group's query rows into the first weight buffer (K-major B)
-                ptx::mbar_arrive_expect_tx(&sm.full[0], kHalfBytes + 2u * (uint32_t)G * 128u);
+                ptx::mbar_arrive_expect_tx(&sm.full[0], kHalfBytes + 2u * (uint32_t)geo.qbox * 128u);
                 ptx::tma_load_2d(sm.codes[0], &wmap, &sm.full[0], 0, g * kD);
-                ptx::tma_load_2d(sm.p[0], &qmap, &sm.full[0], 0, b * geo.Hq + g * G);
-                ptx::tma_load_2d(sm.p[0] + kNR * 128, &qmap, &sm.full[0], 64, b * geo.Hq + g * G);
+                ptx::tma_load_2d(sm.p[0], &qmap, &sm.full[0], 0, b * geo.Hq + qh0);
+                ptx::tma_load_2d(sm.p[0] + kNR * 128, &qmap, &sm.full[0], 64, b * geo.Hq + qh0);
                 ptx::mbar_arrive_expect_tx(&sm.full[1], kHalfBytes);
                 ptx::tma_load_2d(sm.codes[1], &wmap, &sm.full[1], 64, g * kD);
             }
@@ -578,7 +583,7 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
             for (int k = 0; k < KHH; ++k) {
                 const int h = KHH * hh + k;
-                acc[k] = h < G ? __uint_as_float((uint32_t)a.q[((size_t)b * geo.Hq + g * G + h) * kD + t] << 16)
+                acc[k] = h < G ? __uint_as_float((uint32_t)a.q[((size_t)b * geo.Hq + qh0 + h) * kD + t] << 16)
                                : 0.f;
             }
         }
@@ -844,7 +849,7 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
                 for (int w = 0; w < 4; ++w) lt += sm.red[rb][kQuarters * hh + w][k];
                 const float val = o[k] / lt;
-                const size_t bh = (size_t)b * geo.Hq + g * G + h;
+                const size_t bh = (size_t)b * geo.Hq + qh0 + h;
                 if (a.direct_out) {
                     if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * kD + t] = val;
                     else static_cast<__nv_bfloat16 *>(a.out)[bh * kD + t] = __float2bfloat16_rn(val);
@@ -912,7 +917,7 @@ cudaError_t launch_shape(const DecodeArgs &a, const CUtensorMap &cmap, const CUt
         configured = true;
     }
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(g.S, g.Hkv, g.B);
+    cfg.gridDim = dim3(g.S * g.nhb, g.Hkv, g.B);
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = a.stream;
@@ -936,10 +941,12 @@ cudaError_t launch_decode_fp8(const DecodeArgs &a, const float *v_scales) {
                       kD * 2, 64, kD, CU_TENSOR_MAP_SWIZZLE_128B))
             return cudaErrorInvalidValue;
         if (!encode2d(&qmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.q, kD, (uint64_t)g.B * g.Hq, kD * 2,
-                      64, (uint32_t)g.G, CU_TENSOR_MAP_SWIZZLE_128B))
+                      64, (uint32_t)g.qbox, CU_TENSOR_MAP_SWIZZLE_128B))
             return cudaErrorInvalidValue;
     }
-    if (g.G == 8) return launch_shape<4, true>(a, cmap, wmap, qmap, v_scales);
+    // groups of more than 8 heads: blocks of 8 (and a last, smaller one)
+    if (g.G % 8 == 0) return launch_shape<4, true>(a, cmap, wmap, qmap, v_scales);
+    if (g.G > 8) return launch_shape<4, false>(a, cmap, wmap, qmap, v_scales);
     if (g.G == 4) return launch_shape<2, true>(a, cmap, wmap, qmap, v_scales);
     return g.G < 4 ? launch_shape<2, false>(a, cmap, wmap, qmap, v_scales)
                    : launch_shape<4, false>(a, cmap, wmap, qmap, v_scales);

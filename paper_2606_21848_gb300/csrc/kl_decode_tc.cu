@@ -43,7 +43,8 @@ namespace {
 
 constexpr int kD = 128;
 constexpr int kTile = 128;                  // tokens per tile
-constexpr int kNG = 8;                      // query heads per value group (padded)
+constexpr int kNG = 8;                      // query heads per CTA (padded)
+constexpr int kMaxGroup = 128;              // query heads per value head (16 CTAs of 8)
 constexpr int kN = 2 * kNG;                 // MMA N: hi and lo halves
 constexpr uint32_t kTileBytes = kTile * kD * 2;   // 32 KiB per cache tile
 constexpr uint32_t kHalfBytes = kTileBytes / 2;   // one 64-dim half: 128 rows x 128 B
@@ -203,18 +204,17 @@ __device__ __forceinline__ bool arrive_last(unsigned int *counter, int n) {
 // now; the {m, l} table and the normalized weights go to its front, and TMA bulk copies bring
 // the state rows through the rest, folded by thread (head, 4 dims) from shared memory.
 template <int KH, typename SmemT, typename WaitT>
-__device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int g, int n_u, int t,
-                             int warp, int lane, const WaitT &wait) {
+__device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int qh0, int G, int n_u,
+                             int t, int warp, int lane, const WaitT &wait) {
     constexpr int kComputeWarps = Roles<KH>::kComputeWarps;
     constexpr int kComputeThreads = Roles<KH>::kComputeThreads;
     const Geometry &geo = a.geo;
-    const int G = geo.G;
     if (n_u <= 8) {
         // Few splits: thread (head, 4 dims) loads its n_u {m, l} pairs and state rows at once
         // (one round trip) and folds them; no staging.
         const float2 *ml = reinterpret_cast<const float2 *>(a.part_ml);
         for (int h = warp; h < G; h += kComputeWarps) {
-            const size_t bh = (size_t)b * geo.Hq + g * G + h;
+            const size_t bh = (size_t)b * geo.Hq + qh0 + h;
             const float4 *po = reinterpret_cast<const float4 *>(a.part_o + bh * geo.S * kD) + lane;
             float2 v[8];
             float4 r[8];
@@ -272,14 +272,14 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int g, int n
             ptx::mbar_arrive_expect_tx(&sm.merge_full, (uint32_t)(G * nrow * kD * sizeof(float)));
             for (int h = 0; h < G; ++h)
                 ptx::bulk_load(rows + (size_t)h * cap * kD,
-                               a.part_o + (((size_t)b * geo.Hq + g * G + h) * geo.S + c0) * kD,
+                               a.part_o + (((size_t)b * geo.Hq + qh0 + h) * geo.S + c0) * kD,
                                (uint32_t)(nrow * kD * sizeof(float)), &sm.merge_full);
         }
     };
     issue_rows(0, min(cap, n_u));
     for (int i = t; i < G * n_u; i += kComputeThreads) {
         const int h = i / n_u, j = i - h * n_u;
-        tab[i] = __ldcg(ml + ((size_t)b * geo.Hq + g * G + h) * geo.S + j);
+        tab[i] = __ldcg(ml + ((size_t)b * geo.Hq + qh0 + h) * geo.S + j);
     }
     ptx::bar_sync(kBarCompute, kComputeThreads);
     for (int h = warp; h < G; h += kComputeWarps) {
@@ -335,7 +335,7 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int g, int n
     for (int pass = 0; pass < 2; ++pass) {
         const int h = warp + pass * kComputeWarps;
         if (h >= G) continue;
-        const size_t oi = ((size_t)b * geo.Hq + g * G + h) * kD + 4 * lane;
+        const size_t oi = ((size_t)b * geo.Hq + qh0 + h) * kD + 4 * lane;
         if (a.out_dtype == KL_FP32) {
             *reinterpret_cast<float4 *>(static_cast<float *>(a.out) + oi) = acc[pass];
         } else {
@@ -368,14 +368,19 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
 
     const Geometry &geo = a.geo;
     // A CTA runs geo.spc consecutive splits of one (b, g) (one split unless a launch of one CTA
-    // per split would not fit in one wave); it keeps one softmax state per split.
-    const int cta = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+    // per split would not fit in one wave); it keeps one softmax state per split. A group of
+    // more than 8 query heads is served by geo.nhb sibling CTAs, adjacent in blockIdx.x, each
+    // for up to 8 of its heads: the siblings read the same pages at about the same time, so
+    // the second and later reads of a page are served by L2.
+    const int hb = blockIdx.x % geo.nhb, cta = blockIdx.x / geo.nhb;
+    const int g = blockIdx.y, b = blockIdx.z;
     const int split0 = cta * geo.spc;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int G = geo.G;
+    const int G = min(kNG, geo.G - kNG * hb);    // query heads of this CTA
+    const int qh0 = g * geo.G + kNG * hb;         // its first query head within the sequence
 
     // The routing runs on the tensor cores: W^R[g] (one per value head) or the G matrices
-    // W^R[g G + h] (one per query head) arrive by TMA as ring positions 0 .. route_tiles - 1,
+    // W^R[qh0 + h] (one per query head) arrive by TMA as ring positions 0 .. route_tiles - 1,
     // with the group's query rows, and the cache tiles follow.
     // routing on the tensor cores unless the query arrives routed: pre-routed fp32 queries, or
     // the composed query q = x W^Q W^R of Section 2.1 (no W^R given)
@@ -467,7 +472,7 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
         }
         if (tid < kD) {
             for (int h = 0; h < G; ++h) {
-                const size_t bh = (size_t)b * geo.Hq + g * G + h;
+                const size_t bh = (size_t)b * geo.Hq + qh0 + h;
                 if (a.merge_inside) {
                     if (L == 0 && cta == 0) {
                         if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * kD + tid] = 0.f;
@@ -525,13 +530,13 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
             const int s = r % NS;
             if (r >= NS && !wait(&sm.empty[s], ((r / NS) & 1) ^ 1)) break;
             if (lane == 0) {
-                const int wrow = (route_pq ? g * G + r : g) * kD;
-                ptx::mbar_arrive_expect_tx(&sm.full[s], kTileBytes + (r == 0 ? 2u * (uint32_t)G * 128u : 0u));
+                const int wrow = (route_pq ? qh0 + r : g) * kD;
+                ptx::mbar_arrive_expect_tx(&sm.full[s], kTileBytes + (r == 0 ? 2u * (uint32_t)geo.qbox * 128u : 0u));
                 ptx::tma_load_2d(sm.tiles[s][0], &wmap, &sm.full[s], 0, wrow);
                 ptx::tma_load_2d(sm.tiles[s][0] + kHalfBytes, &wmap, &sm.full[s], 64, wrow);
                 if (r == 0) {
-                    ptx::tma_load_2d(sm.qr, &qmap, &sm.full[s], 0, b * geo.Hq + g * G);
-                    ptx::tma_load_2d(sm.qr + kN * 128, &qmap, &sm.full[s], 64, b * geo.Hq + g * G);
+                    ptx::tma_load_2d(sm.qr, &qmap, &sm.full[s], 0, b * geo.Hq + qh0);
+                    ptx::tma_load_2d(sm.qr + kN * 128, &qmap, &sm.full[s], 64, b * geo.Hq + qh0);
                 }
             }
             __syncwarp();
@@ -742,12 +747,12 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
             if (a.pdl) grid_dep_wait();
 #pragma unroll
             for (int e = 0; e < KH; ++e)
-                acc[e] = h0 + e < G ? a.q_routed[((size_t)b * geo.Hq + g * G + h0 + e) * kD + t] : 0.f;
+                acc[e] = h0 + e < G ? a.q_routed[((size_t)b * geo.Hq + qh0 + h0 + e) * kD + t] : 0.f;
         } else {
             for (int i = tid; i < kD * kNG; i += kComputeThreads) {
                 const int k = i >> 3, h = i & 7;
                 qf[i] = h < G ? __uint_as_float(
-                                    (uint32_t)a.q[((size_t)b * geo.Hq + g * G + h) * kD + k] << 16)
+                                    (uint32_t)a.q[((size_t)b * geo.Hq + qh0 + h) * kD + k] << 16)
                               : 0.f;
             }
             __syncwarp();
@@ -848,7 +853,7 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
                 const int h = h0 + e;
                 if (h >= G) continue;
                 const float lt = (sm.lred[0][h] + sm.lred[1][h]) + (sm.lred[2][h] + sm.lred[3][h]);
-                const size_t slot = ((size_t)b * geo.Hq + g * G + h) * geo.S + sp;
+                const size_t slot = ((size_t)b * geo.Hq + qh0 + h) * geo.S + sp;
                 a.part_o[slot * kD + t] = o[e] / lt;
                 if (t == 0) {
                     a.part_ml[slot * 2] = m[e] * kLn2;
@@ -989,7 +994,7 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
 #pragma unroll
                     for (int q = 0; q < 4; ++q) lt += sm.red[rb][q][h];
                     const float val = o[e] / lt;
-                    const size_t bh = (size_t)b * geo.Hq + g * G + h;
+                    const size_t bh = (size_t)b * geo.Hq + qh0 + h;
                     if (write_out) {
                         if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * kD + t] = val;
                         else static_cast<__nv_bfloat16 *>(a.out)[bh * kD + t] = __float2bfloat16_rn(val);
@@ -1017,9 +1022,10 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
                     // The last CTA of (b, g) to finish merges the n_cta_u states (as kl_combine).
                     ptx::bar_sync(kBarCompute, kComputeThreads);
                     if (tid == 0)
-                        sm.is_last = arrive_last(a.counters + (size_t)b * geo.Hkv + g, n_cta_u) ? 1 : 0;
+                        sm.is_last = arrive_last(
+                            a.counters + ((size_t)b * geo.Hkv + g) * geo.nhb + hb, n_cta_u) ? 1 : 0;
                     ptx::bar_sync(kBarCompute, kComputeThreads);
-                    if (sm.is_last) merge_states<KH>(sm, a, b, g, n_cta_u, tid, warp, lane, wait);
+                    if (sm.is_last) merge_states<KH>(sm, a, b, qh0, G, n_cta_u, tid, warp, lane, wait);
                 }
             }
         }
@@ -1075,7 +1081,7 @@ cudaError_t launch_kernel(const DecodeArgs &la, const CUtensorMap &vmap, const C
         configured = true;
     }
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((g.S + g.spc - 1) / g.spc, g.Hkv, g.B);
+    cfg.gridDim = dim3((g.S + g.spc - 1) / g.spc * g.nhb, g.Hkv, g.B);
     cfg.blockDim = dim3(Roles<KH>::kThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = la.stream;
@@ -1101,16 +1107,16 @@ cudaError_t launch(const DecodeArgs &a) {
         return cudaErrorInvalidValue;
     if (!kStandard && !a.q_routed && a.w_r) {
         // W^R [Hw * 128 rows (k)][128 (j)], Hw = Hkv or Hq, one box = one 64-column half of one
-        // matrix; q [B * Hq rows][128], one box = the G rows of one value group.
+        // matrix; q [B * Hq rows][128], one box = the up to 8 rows of one CTA's heads.
         const uint64_t hw = g.wr_per_qh ? (uint64_t)g.Hq : (uint64_t)g.Hkv;
         if (!make_map(&wmap, a.w_r, hw * kD, kD)) return cudaErrorInvalidValue;
-        if (!make_map(&qmap, a.q, (uint64_t)g.B * g.Hq, (uint32_t)g.G)) return cudaErrorInvalidValue;
+        if (!make_map(&qmap, a.q, (uint64_t)g.B * g.Hq, (uint32_t)a.geo.qbox)) return cudaErrorInvalidValue;
     }
     // Splits per CTA: one, unless one CTA per split would overflow a wave of two CTAs per SM
     // while the (b, g) units alone would not fill it (few long sequences split many ways): then
     // the fewest consecutive splits per CTA that fit the wave.
     DecodeArgs la = a;
-    const int64_t units = (int64_t)g.B * g.Hkv, slots = 2 * (int64_t)device_sm_count();
+    const int64_t units = (int64_t)g.B * g.Hkv * g.nhb, slots = 2 * (int64_t)device_sm_count();
     int spc = 1;
     if (g.S > 1 && units < slots)
         while ((int64_t)((g.S + spc - 1) / spc) * units > slots) ++spc;
@@ -1128,16 +1134,17 @@ cudaError_t launch(const DecodeArgs &a) {
 }  // namespace
 
 bool tc_merge_inside(const Geometry &g, bool standard) {
-    // the merging CTA keeps {m, l} and the weights of G * S states (12 B each) in its ring and
-    // streams the state rows (512 B) through the rest, at least one split per round
-    const size_t table = ((size_t)g.G * g.S * 12 + 1023) & ~(size_t)1023;
+    // the merging CTA keeps {m, l} and the weights of its heads' S states (12 B each) in its
+    // ring and streams the state rows (512 B) through the rest, at least one split per round
+    const size_t gc = g.G < kNG ? g.G : kNG;
+    const size_t table = (gc * g.S * 12 + 1023) & ~(size_t)1023;
     const size_t ring = standard ? sizeof(Smem<true>::tiles) : sizeof(Smem<false>::tiles);
-    return g.S > 1 && table + (size_t)g.G * kD * sizeof(float) <= ring;
+    return g.S > 1 && table + gc * kD * sizeof(float) <= ring;
 }
 
 bool tc_supported(const Geometry &g, bool standard) {
     (void)standard;
-    if (g.D != kD || g.G > kNG) return false;
+    if (g.D != kD || g.G > kMaxGroup) return false;
     if (g.P != 16 && g.P != 32 && g.P != 64 && g.P != 128) return false;
     if ((int64_t)g.num_pages * g.Hkv * g.P >= ((int64_t)1 << 31)) return false;
     int dev = 0, major = 0, minor = 0;

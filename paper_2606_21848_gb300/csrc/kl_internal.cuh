@@ -19,6 +19,8 @@ struct Geometry {
     int S;             // split count
     int chunk;         // tokens per split (a multiple of 128)
     int spc = 1;       // splits per CTA of the tensor-core decode (consecutive, same (b, g))
+    int nhb = 1;       // CTAs per (run of splits, b, g): blocks of up to 8 query heads
+    int qbox = 8;      // query rows per block: min(G, 8)
 };
 
 // Arguments of a decode launch (keyless or the standard K+V comparison).
@@ -49,7 +51,7 @@ struct DecodeArgs {
     bool direct_out;          // true: S == 1 and the CTA writes `out` itself (no split states)
     bool merge_inside;        // true: the last split of each (b, g) merges the split states
                               // into `out` (tensor-core kernel), using the workspace counters
-    unsigned int *counters;   // [B][Hkv] arrivals of the current call (zero between calls)
+    unsigned int *counters;   // [B][Hkv][nhb] arrivals of the current call (zero between calls)
     kl_dtype out_dtype;
     int32_t *err;
     cudaStream_t stream;
