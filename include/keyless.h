@@ -74,8 +74,9 @@ typedef struct kl_shape {
 /* Kernel family of the decode. */
 typedef enum kl_kernel {
     KL_KERNEL_AUTO = 0,   /* tensor-core kernel where supported, else the CUDA-core one */
-    KL_KERNEL_TENSOR = 1, /* tcgen05 + TMA kernel (head_dim 128, group size <= 8) */
-    KL_KERNEL_SIMT = 2    /* CUDA-core kernel (any supported shape) */
+    KL_KERNEL_TENSOR = 1, /* tcgen05 + TMA kernel (head_dim 128; a group of more than 8 query
+                           * heads is served by CTAs of up to 8 heads each, group size <= 128) */
+    KL_KERNEL_SIMT = 2    /* CUDA-core kernel (group size <= 8) */
 } kl_kernel;
 
 typedef struct kl_decode_options {
@@ -119,8 +120,8 @@ kl_status kl_append_v(const kl_shape *shape, const void *v_new, const int32_t *b
  * Bytes of device workspace kl_decode_attention / kl_decode_step / kl_standard_decode need for
  * `num_splits` (0 = the automatic choice); 0 when no workspace is needed (one split). Returns
  * 0 on invalid shapes. The workspace holds the split states and, for the tensor-core kernel,
- * one merge counter per (sequence, value head): it must be zero-filled (cudaMemsetAsync)
- * before its first use. Every call leaves the counters at zero again, so the workspace can
+ * one merge counter per sequence, value head and block of up to 8 of its query heads: it must
+ * be zero-filled (cudaMemsetAsync) before its first use. Every call leaves the counters at zero again, so the workspace can
  * be reused across calls and shapes -- except after a call that raised KL_FLAG_TIMEOUT,
  * which may leave counters behind: zero the workspace again then. Calls that share a
  * workspace must not overlap on the GPU.
@@ -334,7 +335,8 @@ kl_status kl_quantize_cache_fp8(const kl_shape *shape, const void *v_cache, void
  * the stored codes and fp32 accumulation; the routed query and the softmax weights enter as
  * sums of E4M3 terms (4 and 3 terms, about 16 and 12 significant bits), each row's scale
  * multiplies its score and its weight. W^R per value head (wr_per_query_head = 0) or
- * w_r == NULL (q is then the composed query); at most 8 query heads per value head; page size
+ * w_r == NULL (q is then the composed query); a group of more than 8 query heads is served by
+ * CTAs of up to 8 heads each (group size <= 128); page size
  * 16, 32, 64 or 128; compute capability 10.3 (KL_ERR_UNSUPPORTED otherwise). q, w_r, out,
  * num_splits, the workspace (kl_decode_workspace_size of the same shape and split count), the
  * output layout and the error flags are those of kl_decode_attention; with more than one split
@@ -397,6 +399,21 @@ kl_status kl_decode_attention_noalloc(const kl_shape *shape, const void *q, cons
  * library; the paper has no counterpart.
  */
 int32_t kl_decode_kernel_available(const kl_shape *shape, int32_t kernel, int32_t standard);
+
+/*
+ * Failure detection of the decodes: every wait of a tensor-core decode CTA on its own pipeline
+ * (a copy landing, an MMA finishing, another role's hand-off) gives up after a time limit, about
+ * one second by default. A CTA whose wait runs out raises KL_FLAG_TIMEOUT, leaves its loops,
+ * waits (with the full default bound) for the copies and MMAs it has in flight, frees its tensor
+ * memory and exits, so that the call returns and the context stays usable; its outputs are then
+ * undefined, and a workspace it used must be zero-filled again before the next call. This sets
+ * that limit, in nanoseconds, for every decode launched afterwards by kl_decode_attention(_ex),
+ * kl_decode_step, kl_standard_decode, kl_decode_attention_noalloc, the latent decodes and the FP8
+ * decodes, process-wide; 0 restores the default. Returns the limit in force before the call. A
+ * small value makes the waits run out on purpose: this is how the timeout path is tested. The
+ * paper has no counterpart.
+ */
+uint64_t kl_set_wait_timeout_ns(uint64_t ns);
 
 /* Static description of a status code. */
 const char *kl_status_string(kl_status status);

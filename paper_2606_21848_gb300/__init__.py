@@ -18,4 +18,5 @@ from ._lib import (  # noqa: F401
     kl_latent_shape, make_latent_shape, kl_latent_workspace_size, kl_latent_decode,
     kl_latent_decode_step,
     kl_append_v_fp8, kl_decode_attention_fp8, kl_decode_step_fp8, kl_quantize_cache_fp8,
+    kl_set_wait_timeout_ns,
 )

@@ -91,6 +91,7 @@ def load() -> ctypes.CDLL:
         "kl_latent_decode": ([LS, P, P, P, P, P, P, I32, P, I32, P, SZ, P, P], I32),
         "kl_latent_decode_step": ([LS, P, P, P, P, P, P, P, P, I32, P, I32, P, SZ, P, P], I32),
         "kl_prefill_attention": ([SH, P, P, P, P, P, P, I32, I32, P, I32, P, P], I32),
+        "kl_set_wait_timeout_ns": ([ctypes.c_uint64], ctypes.c_uint64),
         "kl_status_string": ([I32], ctypes.c_char_p),
     }
     for name, (args, res) in sig.items():
@@ -288,6 +289,11 @@ def kl_latent_decode_step(shape, q, w_r, w_post, v_new, positions, v_lat, block_
 
 def kl_decode_kernel_available(shape, kernel, standard=False) -> bool:
     return bool(load().kl_decode_kernel_available(ctypes.byref(shape), kernel, int(standard)))
+
+
+def kl_set_wait_timeout_ns(ns: int) -> int:
+    """Set the decodes' pipeline-wait limit (ns; 0 = the default); returns the previous one."""
+    return int(load().kl_set_wait_timeout_ns(int(ns)))
 
 
 def kl_status_string(status: int) -> str:

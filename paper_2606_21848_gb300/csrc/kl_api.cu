@@ -3,9 +3,20 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "kl_internal.cuh"
 
 namespace kl {
+
+namespace {
+std::atomic<uint64_t> g_wait_ns{0};   // 0: the default
+}  // namespace
+
+uint64_t current_wait_ns() {
+    const uint64_t v = g_wait_ns.load(std::memory_order_relaxed);
+    return v ? v : kDefaultWaitNs;
+}
 
 int device_sm_count() {
     static int cache[64] = {0};
@@ -153,6 +164,7 @@ kl_status decode_common(bool standard, const kl_shape *shape, const void *q, con
     a.err = err;
     a.stream = reinterpret_cast<cudaStream_t>(stream);
     a.pdl = pdl;
+    a.wait_ns = current_wait_ns();
 
     bool use_tc = false;
     if (q_routed && !tc_supported(g, standard)) return KL_ERR_UNSUPPORTED;
@@ -463,6 +475,7 @@ kl_status decode_fp8(const kl_shape *shape, const void *q, const void *w_r, cons
     a.out_dtype = out_dtype;
     a.err = err;
     a.stream = reinterpret_cast<cudaStream_t>(stream);
+    a.wait_ns = current_wait_ns();
     cudaError_t e = launch_decode_fp8(a, v_scales);
     if (e == cudaSuccess) e = finish_decode(a, false);
     return from_cuda(e);
@@ -575,6 +588,11 @@ int32_t kl_decode_kernel_available(const kl_shape *shape, int32_t kernel, int32_
     if (kernel == KL_KERNEL_AUTO) return (tc || simt) ? 1 : 0;
     if (kernel == KL_KERNEL_TENSOR) return tc ? 1 : 0;
     return 0;
+}
+
+uint64_t kl_set_wait_timeout_ns(uint64_t ns) {
+    const uint64_t old = g_wait_ns.exchange(ns, std::memory_order_relaxed);
+    return old ? old : kDefaultWaitNs;
 }
 
 const char *kl_status_string(kl_status s) {

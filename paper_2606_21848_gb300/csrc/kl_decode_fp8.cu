@@ -74,7 +74,7 @@ constexpr uint32_t kColS = 0;                        // S[b]: columns 32 b .. 32
 constexpr uint32_t kColO = 64;                       // O: columns 64 .. 95, summed over tiles
 constexpr uint32_t kColR = 96;                       // routing result: 96 .. 111
 constexpr float kLazy = 2.f;                         // reference slack (base 2): weights <= 4
-constexpr uint64_t kTimeoutNs = 1000000000ull;
+constexpr uint64_t kTimeoutNs = kDefaultWaitNs;   // bound of the drains
 constexpr uint32_t kBarCompute = 1;
 constexpr uint32_t kBarComputeAnd = 2;
 
@@ -125,9 +125,12 @@ __device__ __forceinline__ bool mbar_wait_sleep(uint64_t *bar, uint32_t parity) 
     return ok != 0;
 }
 
+// Warp-collective bounded wait (as in the bf16 decode): false when the CTA is aborting or the
+// wait ran out (`limit` ns, about 1 s unless the library's limit was lowered).
 struct Waiter {
     volatile int *abort;
     int32_t *err;
+    uint64_t limit;
     __device__ bool operator()(uint64_t *bar, uint32_t parity) const {
         bool ok = ptx::mbar_try_wait(bar, parity);
         if (!ok) {
@@ -135,7 +138,7 @@ struct Waiter {
             while (true) {
                 if (mbar_wait_sleep(bar, parity)) { ok = true; break; }
                 if (*abort) break;
-                if (ptx::globaltimer() - t0 > kTimeoutNs) {
+                if (ptx::globaltimer() - t0 > limit) {
                     *abort = 1;
                     raise_flag(err, KL_FLAG_TIMEOUT);
                     break;
@@ -403,7 +406,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
 
     const uint32_t tmem = sm.tmem_base;
-    const Waiter wait{&sm.abort, a.err};
+    const Waiter wait{&sm.abort, a.err, a.wait_ns};
 
     if (warp == kProducerWarp) {
         // ------------------------------------------------------------------ producer ----
@@ -460,13 +463,12 @@ __global__ void __launch_bounds__(kThreads, 2)
             issued = u + 1;
         }
         if (__any_sync(0xffffffffu, bad) && lane == 0) raise_flag(a.err, KL_FLAG_BAD_PAGE);
-        if (sm.abort) {
-            // the most recent use of every stage may still have copies in flight
-            for (int v = max(0, issued - kStages); v < issued; ++v) {
-                const uint64_t t0 = ptx::globaltimer();
-                while (!ptx::mbar_try_wait(&sm.full[v % kStages], (v / kStages) & 1) &&
-                       ptx::globaltimer() - t0 < kTimeoutNs) {
-                }
+        // the most recent use of every stage may still have copies in flight: they land before
+        // the CTA's shared memory goes away, also when a consumer gives up after this loop
+        for (int v = max(0, issued - kStages); v < issued; ++v) {
+            const uint64_t t0 = ptx::globaltimer();
+            while (!ptx::mbar_try_wait(&sm.full[v % kStages], (v / kStages) & 1) &&
+                   ptx::globaltimer() - t0 < kTimeoutNs) {
             }
         }
     } else if (warp == kMmaWarp) {

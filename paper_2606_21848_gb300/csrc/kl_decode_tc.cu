@@ -50,7 +50,7 @@ constexpr uint32_t kTileBytes = kTile * kD * 2;   // 32 KiB per cache tile
 constexpr uint32_t kHalfBytes = kTileBytes / 2;   // one 64-dim half: 128 rows x 128 B
 constexpr uint32_t kTmemCols = 64;                // S: 2 x 16 columns, O: 2 x 16 columns
 constexpr uint32_t kTmemColsPq = 256;             // + one 16-column routing result per head
-constexpr uint64_t kTimeoutNs = 1000000000ull;
+constexpr uint64_t kTimeoutNs = kDefaultWaitNs;   // bound of the drains
 // Warp roles for KH heads per compute warp: KH = 8, one compute warp per TMEM lane quarter;
 // KH = 2 (groups of up to 4 heads), two per quarter.
 template <int KH>
@@ -141,11 +141,12 @@ struct __align__(1024) Smem {
 };
 
 // Warp-collective bounded wait: every lane of the warp calls it in uniform control flow and
-// gets the same answer. False when this CTA is aborting or the wait ran out (about 1 s), in
-// which case the caller leaves its loop.
+// gets the same answer. False when this CTA is aborting or the wait ran out (`limit` ns, about
+// 1 s unless the library's limit was lowered), in which case the caller leaves its loop.
 struct Waiter {
     volatile int *abort;
     int32_t *err;
+    uint64_t limit;
     __device__ bool operator()(uint64_t *bar, uint32_t parity) const {
         bool ok = ptx::mbar_try_wait(bar, parity);
         if (!ok) {
@@ -153,7 +154,7 @@ struct Waiter {
             while (true) {
                 if (ptx::mbar_try_wait(bar, parity)) { ok = true; break; }
                 if (*abort) break;
-                if (ptx::globaltimer() - t0 > kTimeoutNs) {
+                if (ptx::globaltimer() - t0 > limit) {
                     *abort = 1;
                     raise_flag(err, KL_FLAG_TIMEOUT);
                     break;
@@ -311,7 +312,14 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int qh0, int
         ptx::fence_proxy_async_smem();
         ptx::bar_sync(kBarCompute, kComputeThreads);
         if (c0 > 0) issue_rows(c0, nrow);
-        if (!ptx::bar_and(kBarComputeAnd, kComputeThreads, wait(&sm.merge_full, round & 1))) return;
+        if (!ptx::bar_and(kBarComputeAnd, kComputeThreads, wait(&sm.merge_full, round & 1))) {
+            // gave up: this round's copies must still land before the CTA's shared memory goes
+            const uint64_t t0 = ptx::globaltimer();
+            while (!ptx::mbar_try_wait(&sm.merge_full, round & 1) &&
+                   ptx::globaltimer() - t0 < kTimeoutNs) {
+            }
+            return;
+        }
 #pragma unroll
         for (int pass = 0; pass < 2; ++pass) {
             const int h = warp + pass * kComputeWarps;
@@ -498,7 +506,7 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
     }
 
     const uint32_t tmem = sm.tmem_base;
-    const Waiter wait{&sm.abort, a.err};
+    const Waiter wait{&sm.abort, a.err, a.wait_ns};
 
     if (warp == kProducerWarp) {
         // ------------------------------------------------------------------ producer ----
@@ -586,16 +594,13 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
             issued = r + 1;
         }
         if (__any_sync(0xffffffffu, bad) && lane == 0) raise_flag(a.err, KL_FLAG_BAD_PAGE);
-        // Drain: copies still in flight must land before the CTA's shared memory goes away.
-        if (sm.abort) {
-            const Waiter drain_wait{&sm.abort, a.err};
-            for (int i = max(0, issued - NS); i < issued; ++i) {
-                const uint64_t t0 = ptx::globaltimer();
-                while (!ptx::mbar_try_wait(&sm.full[i % NS], (i / NS) & 1) &&
-                       ptx::globaltimer() - t0 < kTimeoutNs) {
-                }
+        // Drain: copies still in flight must land before the CTA's shared memory goes away,
+        // also when a consumer gives up after this loop has ended (at once when they landed).
+        for (int i = max(0, issued - NS); i < issued; ++i) {
+            const uint64_t t0 = ptx::globaltimer();
+            while (!ptx::mbar_try_wait(&sm.full[i % NS], (i / NS) & 1) &&
+                   ptx::globaltimer() - t0 < kTimeoutNs) {
             }
-            (void)drain_wait;
         }
     } else if (warp == kMmaWarp) {
         // ------------------------------------------------------- score MMA issuer -------

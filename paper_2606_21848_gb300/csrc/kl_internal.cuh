@@ -11,6 +11,10 @@ namespace kl {
 
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
+constexpr uint64_t kDefaultWaitNs = 1000000000ull;   // about one second
+
+// The pipeline-wait limit in force (kl_set_wait_timeout_ns; the default unless set).
+uint64_t current_wait_ns();
 
 // Geometry of one decode call, resolved on the host.
 struct Geometry {
@@ -55,6 +59,9 @@ struct DecodeArgs {
     kl_dtype out_dtype;
     int32_t *err;
     cudaStream_t stream;
+    // Limit of each pipeline wait of the tensor-core decodes (ns); the drains of a CTA that gave
+    // up keep the full default so that its copies and MMAs complete before it exits.
+    uint64_t wait_ns = kDefaultWaitNs;
     // Latent path: the launch is a programmatic dependent of the absorbed-query kernel ahead of
     // it; the CTAs set up and fill their ring of cache tiles at once, every role then sleeps in
     // grid_dep_wait until that kernel has finished (the compute warps before reading q_routed),

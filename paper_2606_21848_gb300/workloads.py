@@ -93,6 +93,17 @@ WORKLOADS: dict[str, Workload] = {
 
 ORDER = ["tiny_mha", "small_gqa", "long_context", "ragged_serving", "high_concurrency_70b"]
 
+# Groups of more than 8 query heads per value head (Section 3, multi-query and grouped-query
+# attention): all 32 heads of a sequence on one value head (MQA), and 128 query heads over 8
+# value heads (groups of 16).
+WORKLOADS.update({
+    "mqa_group32": Workload("mqa_group32", 256, 32, 1, 128, 16, seq_len=8192,
+                            wr_std=math.sqrt(1 / 128), seed=8),
+    "gqa_group16": Workload("gqa_group16", 64, 128, 8, 128, 32, seq_len=8192,
+                            wr_std=math.sqrt(1 / 128), seed=9),
+})
+LARGE_GROUPS = ["mqa_group32", "gqa_group16"]
+
 # Prefill workloads (chunked prefill, the step before decode): a whole 32K-token prompt with
 # the paper's Qwen2-1.5B attention (12 query heads, 2 value heads, head dim 128, W^R per query
 # head, trained at 32,768 tokens), and a serving-style chunk of 512 new tokens on an
