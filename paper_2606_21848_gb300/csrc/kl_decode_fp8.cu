@@ -132,11 +132,15 @@ struct Waiter {
     int32_t *err;
     uint64_t limit;
     __device__ bool operator()(uint64_t *bar, uint32_t parity) const {
-        bool ok = ptx::mbar_try_wait(bar, parity);
+        const bool exact = limit < kPollNs;     // poll without the blocking forms
+        bool ok = exact ? ptx::mbar_test_wait(bar, parity) : ptx::mbar_try_wait(bar, parity);
         if (!ok) {
             const uint64_t t0 = ptx::globaltimer();
             while (true) {
-                if (mbar_wait_sleep(bar, parity)) { ok = true; break; }
+                if (exact ? ptx::mbar_test_wait(bar, parity) : mbar_wait_sleep(bar, parity)) {
+                    ok = true;
+                    break;
+                }
                 if (*abort) break;
                 if (ptx::globaltimer() - t0 > limit) {
                     *abort = 1;

@@ -147,12 +147,15 @@ struct Waiter {
     volatile int *abort;
     int32_t *err;
     uint64_t limit;
+    __device__ bool poll(uint64_t *bar, uint32_t parity) const {
+        return limit < kPollNs ? ptx::mbar_test_wait(bar, parity) : ptx::mbar_try_wait(bar, parity);
+    }
     __device__ bool operator()(uint64_t *bar, uint32_t parity) const {
-        bool ok = ptx::mbar_try_wait(bar, parity);
+        bool ok = poll(bar, parity);
         if (!ok) {
             const uint64_t t0 = ptx::globaltimer();
             while (true) {
-                if (ptx::mbar_try_wait(bar, parity)) { ok = true; break; }
+                if (poll(bar, parity)) { ok = true; break; }
                 if (*abort) break;
                 if (ptx::globaltimer() - t0 > limit) {
                     *abort = 1;
