@@ -75,6 +75,7 @@ constexpr uint32_t kColO = 64;                       // O: columns 64 .. 95, sum
 constexpr uint32_t kColR = 96;                       // routing result: 96 .. 111
 constexpr float kLazy = 2.f;                         // reference slack (base 2): weights <= 4
 constexpr uint64_t kTimeoutNs = kDefaultWaitNs;   // bound of the drains
+constexpr uint32_t kSleepHintNs = 20000u;         // suspend hint of a wait that did not finish at once
 constexpr uint32_t kBarCompute = 1;
 constexpr uint32_t kBarComputeAnd = 2;
 
@@ -110,34 +111,26 @@ struct __align__(1024) Smem8 {
     int abort;
 };
 
-// mbarrier.try_wait with a suspend-time hint: a thread whose phase is not complete sleeps in
-// the instruction (it wakes when the phase completes or the hint runs out) instead of spinning
-// and taking issue slots from the warps that share its scheduler.
-__device__ __forceinline__ bool mbar_wait_sleep(uint64_t *bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}\n"
-        : "=r"(ok)
-        : "r"(ptx::smem_addr(bar)), "r"(parity), "r"(20000u)
-        : "memory");
-    return ok != 0;
-}
-
 // Warp-collective bounded wait (as in the bf16 decode): false when the CTA is aborting or the
 // wait ran out (`limit` ns, about 1 s unless the library's limit was lowered).
+// A thread whose phase is not complete sleeps in the try_wait (it wakes when the phase
+// completes or the hint runs out) instead of spinning and taking issue slots from the warps
+// that share its scheduler.
+// The first poll is the plain try_wait (a hinted first poll wakes later when the phase
+// completes: 4 % on the 70B batch); kExact (limits below kExactWaitNs) polls with the
+// non-blocking test_wait, so that short limits hold exactly.
+template <bool kExact>
 struct Waiter {
     volatile int *abort;
     int32_t *err;
     uint64_t limit;
     __device__ bool operator()(uint64_t *bar, uint32_t parity) const {
-        const bool exact = limit < kPollNs;     // poll without the blocking forms
-        bool ok = exact ? ptx::mbar_test_wait(bar, parity) : ptx::mbar_try_wait(bar, parity);
+        bool ok = kExact ? ptx::mbar_test_wait(bar, parity) : ptx::mbar_try_wait(bar, parity);
         if (!ok) {
             const uint64_t t0 = ptx::globaltimer();
             while (true) {
-                if (exact ? ptx::mbar_test_wait(bar, parity) : mbar_wait_sleep(bar, parity)) {
+                if (kExact ? ptx::mbar_test_wait(bar, parity)
+                           : ptx::mbar_try_wait_hint(bar, parity, kSleepHintNs)) {
                     ok = true;
                     break;
                 }
@@ -286,7 +279,7 @@ __device__ __forceinline__ uint32_t bar_popc(uint32_t id, uint32_t count, bool v
     return r;
 }
 
-template <int KHH, bool kAllLive>
+template <int KHH, bool kAllLive, bool kExact>
 __global__ void __launch_bounds__(kThreads, 2)
     decode_fp8_kernel(const __grid_constant__ CUtensorMap cmap,
                       const __grid_constant__ CUtensorMap wmap,
@@ -410,7 +403,8 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
 
     const uint32_t tmem = sm.tmem_base;
-    const Waiter wait{&sm.abort, a.err, a.wait_ns};
+    int issued = 0;                 // ring uses whose copies the producer issued
+    const Waiter<kExact> wait{&sm.abort, a.err, a.wait_ns};
 
     if (warp == kProducerWarp) {
         // ------------------------------------------------------------------ producer ----
@@ -420,7 +414,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         const int end_page = (t_end + P - 1) / P;
         const uint32_t page_bytes = (uint32_t)P * 128u + (uint32_t)P * 4u;
         bool bad = false;
-        int issued = 0;                                      // ring uses issued
+        issued = 0;
         int app_tile = -1;
         size_t app_row = 0;
         uint32_t app_codes = 0;
@@ -467,14 +461,7 @@ __global__ void __launch_bounds__(kThreads, 2)
             issued = u + 1;
         }
         if (__any_sync(0xffffffffu, bad) && lane == 0) raise_flag(a.err, KL_FLAG_BAD_PAGE);
-        // the most recent use of every stage may still have copies in flight: they land before
-        // the CTA's shared memory goes away, also when a consumer gives up after this loop
-        for (int v = max(0, issued - kStages); v < issued; ++v) {
-            const uint64_t t0 = ptx::globaltimer();
-            while (!ptx::mbar_try_wait(&sm.full[v % kStages], (v / kStages) & 1) &&
-                   ptx::globaltimer() - t0 < kTimeoutNs) {
-            }
-        }
+
     } else if (warp == kMmaWarp) {
         // ------------------------------------------------- routing and score MMA issuer ----
         bool ok = true;
@@ -877,6 +864,17 @@ __global__ void __launch_bounds__(kThreads, 2)
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tmem, kTmemCols);
     }
+    // A CTA that gave up (every role has left its loop by now, so the flag is final): the most
+    // recent use of every stage may still have copies in flight; they land before its shared
+    // memory goes away.
+    if (warp == kProducerWarp && sm.abort) {
+        for (int v = max(0, issued - kStages); v < issued; ++v) {
+            const uint64_t t0 = ptx::globaltimer();
+            while (!ptx::mbar_try_wait(&sm.full[v % kStages], (v / kStages) & 1) &&
+                   ptx::globaltimer() - t0 < kTimeoutNs) {
+            }
+        }
+    }
 }
 
 // ------------------------------------------------------------------------ host side ------
@@ -910,14 +908,14 @@ bool encode2d(CUtensorMap *map, CUtensorMapDataType type, const void *base, uint
 
 // The decode for one head count per compute warp (2 for groups of up to 4 query heads, else 4)
 // and whether every compute warp's heads are real (groups of exactly 4 or 8).
-template <int KHH, bool kAllLive>
+template <int KHH, bool kAllLive, bool kExact>
 cudaError_t launch_shape(const DecodeArgs &a, const CUtensorMap &cmap, const CUtensorMap &wmap,
                          const CUtensorMap &qmap, const float *v_scales) {
     const Geometry &g = a.geo;
     const size_t smem = sizeof(Smem8) + 1024;
     static bool configured = false;
     if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(decode_fp8_kernel<KHH, kAllLive>,
+        cudaError_t e = cudaFuncSetAttribute(decode_fp8_kernel<KHH, kAllLive, kExact>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         configured = true;
@@ -927,7 +925,20 @@ cudaError_t launch_shape(const DecodeArgs &a, const CUtensorMap &cmap, const CUt
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = a.stream;
-    return cudaLaunchKernelEx(&cfg, decode_fp8_kernel<KHH, kAllLive>, cmap, wmap, qmap, a, v_scales);
+    return cudaLaunchKernelEx(&cfg, decode_fp8_kernel<KHH, kAllLive, kExact>, cmap, wmap, qmap, a,
+                              v_scales);
+}
+
+template <bool kExact>
+cudaError_t launch_waits(const DecodeArgs &a, const CUtensorMap &cmap, const CUtensorMap &wmap,
+                         const CUtensorMap &qmap, const float *v_scales) {
+    const Geometry &g = a.geo;
+    // groups of more than 8 heads: blocks of 8 (and a last, smaller one)
+    if (g.G % 8 == 0) return launch_shape<4, true, kExact>(a, cmap, wmap, qmap, v_scales);
+    if (g.G > 8) return launch_shape<4, false, kExact>(a, cmap, wmap, qmap, v_scales);
+    if (g.G == 4) return launch_shape<2, true, kExact>(a, cmap, wmap, qmap, v_scales);
+    return g.G < 4 ? launch_shape<2, false, kExact>(a, cmap, wmap, qmap, v_scales)
+                   : launch_shape<4, false, kExact>(a, cmap, wmap, qmap, v_scales);
 }
 
 }  // namespace
@@ -950,12 +961,9 @@ cudaError_t launch_decode_fp8(const DecodeArgs &a, const float *v_scales) {
                       64, (uint32_t)g.qbox, CU_TENSOR_MAP_SWIZZLE_128B))
             return cudaErrorInvalidValue;
     }
-    // groups of more than 8 heads: blocks of 8 (and a last, smaller one)
-    if (g.G % 8 == 0) return launch_shape<4, true>(a, cmap, wmap, qmap, v_scales);
-    if (g.G > 8) return launch_shape<4, false>(a, cmap, wmap, qmap, v_scales);
-    if (g.G == 4) return launch_shape<2, true>(a, cmap, wmap, qmap, v_scales);
-    return g.G < 4 ? launch_shape<2, false>(a, cmap, wmap, qmap, v_scales)
-                   : launch_shape<4, false>(a, cmap, wmap, qmap, v_scales);
+    // exact short waits only when the limit asks for them
+    return a.wait_ns < kExactWaitNs ? launch_waits<true>(a, cmap, wmap, qmap, v_scales)
+                                      : launch_waits<false>(a, cmap, wmap, qmap, v_scales);
 }
 
 }  // namespace kl

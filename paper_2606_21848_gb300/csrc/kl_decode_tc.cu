@@ -143,12 +143,17 @@ struct __align__(1024) Smem {
 // Warp-collective bounded wait: every lane of the warp calls it in uniform control flow and
 // gets the same answer. False when this CTA is aborting or the wait ran out (`limit` ns, about
 // 1 s unless the library's limit was lowered), in which case the caller leaves its loop.
+// The try_wait may suspend the thread for a hardware-defined time before it returns false;
+// kExact (limits below kExactWaitNs) polls with the non-blocking test_wait instead, so that
+// short limits hold exactly.
+template <bool kExact>
 struct Waiter {
     volatile int *abort;
     int32_t *err;
     uint64_t limit;
     __device__ bool poll(uint64_t *bar, uint32_t parity) const {
-        return limit < kPollNs ? ptx::mbar_test_wait(bar, parity) : ptx::mbar_try_wait(bar, parity);
+        if constexpr (kExact) return ptx::mbar_test_wait(bar, parity);
+        else return ptx::mbar_try_wait(bar, parity);
     }
     __device__ bool operator()(uint64_t *bar, uint32_t parity) const {
         bool ok = poll(bar, parity);
@@ -360,7 +365,7 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int qh0, int
 // kPerSplit: the CTA runs several splits and writes a state for each (only when the caller
 // gets the split states, or the combine kernel merges them, and spc > 1). KH: heads per compute
 // warp (8, or 2 when G <= 4).
-template <bool kStandard, bool kPerSplit, int KH>
+template <bool kStandard, bool kPerSplit, int KH, bool kExact>
 __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
     decode_tc_kernel(const __grid_constant__ CUtensorMap vmap,
                      const __grid_constant__ CUtensorMap kmap,
@@ -509,7 +514,8 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
     }
 
     const uint32_t tmem = sm.tmem_base;
-    const Waiter wait{&sm.abort, a.err, a.wait_ns};
+    int issued = 0;                 // ring uses whose copies the producer issued
+    const Waiter<kExact> wait{&sm.abort, a.err, a.wait_ns};
 
     if (warp == kProducerWarp) {
         // ------------------------------------------------------------------ producer ----
@@ -518,7 +524,7 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
         const int end_page = (t_end + P - 1) / P;
         const uint32_t page_bytes = (uint32_t)P * 128u;   // one half of one page
         bool bad = false;
-        int issued = 0;
+        issued = 0;
         // The new token's row (fused append), 8 bytes per lane, written just before the loads of
         // the tile that holds it (or first, when it lies past the sequence's end).
         int app_tile = -1;
@@ -597,14 +603,7 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
             issued = r + 1;
         }
         if (__any_sync(0xffffffffu, bad) && lane == 0) raise_flag(a.err, KL_FLAG_BAD_PAGE);
-        // Drain: copies still in flight must land before the CTA's shared memory goes away,
-        // also when a consumer gives up after this loop has ended (at once when they landed).
-        for (int i = max(0, issued - NS); i < issued; ++i) {
-            const uint64_t t0 = ptx::globaltimer();
-            while (!ptx::mbar_try_wait(&sm.full[i % NS], (i / NS) & 1) &&
-                   ptx::globaltimer() - t0 < kTimeoutNs) {
-            }
-        }
+
     } else if (warp == kMmaWarp) {
         // ------------------------------------------------------- score MMA issuer -------
         // (a programmatic dependent sleeps until the routed queries exist instead of polling)
@@ -1045,6 +1044,16 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tmem, tmem_cols);
     }
+    // A CTA that gave up (every role has left its loop by now, so the flag is final): the cache
+    // copies still in flight land before its shared memory goes away.
+    if (warp == kProducerWarp && sm.abort) {
+        for (int i = max(0, issued - NS); i < issued; ++i) {
+            const uint64_t t0 = ptx::globaltimer();
+            while (!ptx::mbar_try_wait(&sm.full[i % NS], (i / NS) & 1) &&
+                   ptx::globaltimer() - t0 < kTimeoutNs) {
+            }
+        }
+    }
 }
 
 // ------------------------------------------------------------------------ host side ------
@@ -1076,14 +1085,14 @@ bool make_map(CUtensorMap *map, const void *base, uint64_t rows, uint32_t box_ro
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <bool kStandard, bool kPerSplit, int KH>
+template <bool kStandard, bool kPerSplit, int KH, bool kExact>
 cudaError_t launch_kernel(const DecodeArgs &la, const CUtensorMap &vmap, const CUtensorMap &kmap,
                           const CUtensorMap &wmap, const CUtensorMap &qmap) {
     const Geometry &g = la.geo;
     const size_t smem = sizeof(Smem<kStandard>) + 1024;
     static bool configured = false;
     if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<kStandard, kPerSplit, KH>,
+        cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<kStandard, kPerSplit, KH, kExact>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         configured = true;
@@ -1100,7 +1109,15 @@ cudaError_t launch_kernel(const DecodeArgs &la, const CUtensorMap &vmap, const C
         cfg.attrs = attr;
         cfg.numAttrs = 1;
     }
-    return cudaLaunchKernelEx(&cfg, decode_tc_kernel<kStandard, kPerSplit, KH>, vmap, kmap, wmap, qmap, la);
+    return cudaLaunchKernelEx(&cfg, decode_tc_kernel<kStandard, kPerSplit, KH, kExact>, vmap, kmap,
+                              wmap, qmap, la);
+}
+
+template <bool kStandard, int KH, bool kExact>
+cudaError_t launch_waits(const DecodeArgs &la, bool per_split, const CUtensorMap &vmap,
+                         const CUtensorMap &kmap, const CUtensorMap &wmap, const CUtensorMap &qmap) {
+    return per_split ? launch_kernel<kStandard, true, KH, kExact>(la, vmap, kmap, wmap, qmap)
+                     : launch_kernel<kStandard, false, KH, kExact>(la, vmap, kmap, wmap, qmap);
 }
 
 template <bool kStandard>
@@ -1131,12 +1148,13 @@ cudaError_t launch(const DecodeArgs &a) {
     la.geo.spc = spc;
     const bool per_split = spc > 1 && !a.merge_inside && !a.direct_out;
     // heads per compute warp: all 8 (padded) on four warps, or 2 on eight when the group has
-    // at most 4
+    // at most 4; exact short waits only when the limit asks for them
+    const bool exact = a.wait_ns < kExactWaitNs;
     if (g.G <= 4)
-        return per_split ? launch_kernel<kStandard, true, 2>(la, vmap, kmap, wmap, qmap)
-                         : launch_kernel<kStandard, false, 2>(la, vmap, kmap, wmap, qmap);
-    return per_split ? launch_kernel<kStandard, true, 8>(la, vmap, kmap, wmap, qmap)
-                     : launch_kernel<kStandard, false, 8>(la, vmap, kmap, wmap, qmap);
+        return exact ? launch_waits<kStandard, 2, true>(la, per_split, vmap, kmap, wmap, qmap)
+                     : launch_waits<kStandard, 2, false>(la, per_split, vmap, kmap, wmap, qmap);
+    return exact ? launch_waits<kStandard, 8, true>(la, per_split, vmap, kmap, wmap, qmap)
+                 : launch_waits<kStandard, 8, false>(la, per_split, vmap, kmap, wmap, qmap);
 }
 
 }  // namespace

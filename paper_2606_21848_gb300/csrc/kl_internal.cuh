@@ -12,9 +12,9 @@ namespace kl {
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr uint64_t kDefaultWaitNs = 1000000000ull;   // about one second
-// Wait limits below this are kept exactly: such waits poll without the hardware's blocking
-// try_wait, whose own suspend time may be longer than the limit.
-constexpr uint64_t kPollNs = 100000ull;
+// Wait limits below this are kept exactly: the decodes are then launched in a variant whose
+// waits poll without suspending (a suspended try_wait can outlast such a limit).
+constexpr uint64_t kExactWaitNs = 100000ull;
 
 // The pipeline-wait limit in force (kl_set_wait_timeout_ns; the default unless set).
 uint64_t current_wait_ns();
