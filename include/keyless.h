@@ -74,8 +74,9 @@ typedef struct kl_shape {
 /* Kernel family of the decode. */
 typedef enum kl_kernel {
     KL_KERNEL_AUTO = 0,   /* tensor-core kernel where supported, else the CUDA-core one */
-    KL_KERNEL_TENSOR = 1, /* tcgen05 + TMA kernel (head_dim 128; a group of more than 8 query
-                           * heads is served by CTAs of up to 8 heads each, group size <= 128) */
+    KL_KERNEL_TENSOR = 1, /* tcgen05 + TMA kernel (head_dim 128 or 64; a group of more than 8
+                           * query heads is served by CTAs of up to 8 heads each, group size
+                           * <= 128) */
     KL_KERNEL_SIMT = 2    /* CUDA-core kernel (group size <= 8) */
 } kl_kernel;
 

@@ -424,7 +424,7 @@ kl_status decode_fp8(const kl_shape *shape, const void *q, const void *w_r, cons
     Geometry g;
     kl_status st = resolve(shape, num_splits, &g);
     if (st != KL_OK) return st;
-    if (g.wr_per_qh || !tc_supported(g, false)) return KL_ERR_UNSUPPORTED;
+    if (g.D != 128 || g.wr_per_qh || !tc_supported(g, false)) return KL_ERR_UNSUPPORTED;
     if (g.P < 4) return KL_ERR_UNSUPPORTED;
     if (g.B == 0) return KL_OK;
     // Runs of splits: when one CTA per split would overflow a wave of two CTAs per SM while the

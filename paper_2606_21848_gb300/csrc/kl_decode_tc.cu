@@ -218,20 +218,22 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int qh0, int
     constexpr int kComputeWarps = Roles<KH>::kComputeWarps;
     constexpr int kComputeThreads = Roles<KH>::kComputeThreads;
     const Geometry &geo = a.geo;
+    const int D = geo.D;                 // a state row holds D floats: lanes below D / 4 fold them
+    const bool lane_live = lane < D / 4;
     if (n_u <= 8) {
         // Few splits: thread (head, 4 dims) loads its n_u {m, l} pairs and state rows at once
         // (one round trip) and folds them; no staging.
         const float2 *ml = reinterpret_cast<const float2 *>(a.part_ml);
         for (int h = warp; h < G; h += kComputeWarps) {
             const size_t bh = (size_t)b * geo.Hq + qh0 + h;
-            const float4 *po = reinterpret_cast<const float4 *>(a.part_o + bh * geo.S * kD) + lane;
+            const float4 *po = reinterpret_cast<const float4 *>(a.part_o + bh * geo.S * D) + lane;
             float2 v[8];
             float4 r[8];
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
                 if (j < n_u) {
                     v[j] = __ldcg(ml + bh * geo.S + j);
-                    r[j] = __ldcg(po + (size_t)j * (kD / 4));
+                    r[j] = lane_live ? __ldcg(po + (size_t)j * (D / 4)) : make_float4(0.f, 0.f, 0.f, 0.f);
                 }
             }
             float M = -INFINITY;
@@ -253,7 +255,8 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int qh0, int
             }
             const float inv = z > 0.f ? 1.f / z : 0.f;
             acc.x *= inv; acc.y *= inv; acc.z *= inv; acc.w *= inv;
-            const size_t oi = bh * kD + 4 * lane;
+            const size_t oi = bh * D + 4 * lane;
+            if (!lane_live) continue;
             if (a.out_dtype == KL_FP32) {
                 *reinterpret_cast<float4 *>(static_cast<float *>(a.out) + oi) = acc;
             } else {
@@ -271,18 +274,18 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int qh0, int
     float *wt = reinterpret_cast<float *>(tab + G * n_u);                  // [G][n_u] weights
     const uint32_t table_bytes = ((uint32_t)G * n_u * 12u + 1023u) & ~1023u;
     float *rows = reinterpret_cast<float *>(ring + table_bytes);           // [G][cap][128]
-    const int cap = (int)((kRingBytes - table_bytes) / ((uint32_t)G * kD * sizeof(float)));
+    const int cap = (int)((kRingBytes - table_bytes) / ((uint32_t)G * D * sizeof(float)));
     const float2 *ml = reinterpret_cast<const float2 *>(a.part_ml);
     // The first round's state rows go out at once, so that their copy overlaps the {m, l}
     // loads and the weights (the ring is idle: every tile has been consumed).
     auto issue_rows = [&](int c0, int nrow) {
         if (t == 0) {
             ptx::fence_proxy_async_global();
-            ptx::mbar_arrive_expect_tx(&sm.merge_full, (uint32_t)(G * nrow * kD * sizeof(float)));
+            ptx::mbar_arrive_expect_tx(&sm.merge_full, (uint32_t)(G * nrow * D * sizeof(float)));
             for (int h = 0; h < G; ++h)
-                ptx::bulk_load(rows + (size_t)h * cap * kD,
-                               a.part_o + (((size_t)b * geo.Hq + qh0 + h) * geo.S + c0) * kD,
-                               (uint32_t)(nrow * kD * sizeof(float)), &sm.merge_full);
+                ptx::bulk_load(rows + (size_t)h * cap * D,
+                               a.part_o + (((size_t)b * geo.Hq + qh0 + h) * geo.S + c0) * D,
+                               (uint32_t)(nrow * D * sizeof(float)), &sm.merge_full);
         }
     };
     issue_rows(0, min(cap, n_u));
@@ -331,14 +334,14 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int qh0, int
 #pragma unroll
         for (int pass = 0; pass < 2; ++pass) {
             const int h = warp + pass * kComputeWarps;
-            if (h >= G) continue;
-            const float4 *po = reinterpret_cast<const float4 *>(rows + (size_t)h * cap * kD) + lane;
+            if (h >= G || !lane_live) continue;
+            const float4 *po = reinterpret_cast<const float4 *>(rows + (size_t)h * cap * D) + lane;
             const float *w = wt + h * n_u + c0;
 #pragma unroll 4
             for (int j = 0; j < nrow; ++j) {
                 const float wj = w[j];
                 if (wj != 0.f) {
-                    const float4 v = po[(size_t)j * (kD / 4)];
+                    const float4 v = po[(size_t)j * (D / 4)];
                     acc[pass].x = fmaf(wj, v.x, acc[pass].x);
                     acc[pass].y = fmaf(wj, v.y, acc[pass].y);
                     acc[pass].z = fmaf(wj, v.z, acc[pass].z);
@@ -350,8 +353,8 @@ __device__ void merge_states(SmemT &sm, const DecodeArgs &a, int b, int qh0, int
 #pragma unroll
     for (int pass = 0; pass < 2; ++pass) {
         const int h = warp + pass * kComputeWarps;
-        if (h >= G) continue;
-        const size_t oi = ((size_t)b * geo.Hq + qh0 + h) * kD + 4 * lane;
+        if (h >= G || !lane_live) continue;
+        const size_t oi = ((size_t)b * geo.Hq + qh0 + h) * D + 4 * lane;
         if (a.out_dtype == KL_FP32) {
             *reinterpret_cast<float4 *>(static_cast<float *>(a.out) + oi) = acc[pass];
         } else {
@@ -394,6 +397,10 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int G = min(kNG, geo.G - kNG * hb);    // query heads of this CTA
     const int qh0 = g * geo.G + kNG * hb;         // its first query head within the sequence
+    // Head dim of the rows in HBM: 128, or 64. A 64-dim row lands in the first 64-dim half of
+    // its tile row; the second halves, the rows past 64 of a W^R tile and the second half of the
+    // query operand are zero for the whole launch, so the 128-dim MMAs give the 64-dim products.
+    const int D = geo.D;
 
     // The routing runs on the tensor cores: W^R[g] (one per value head) or the G matrices
     // W^R[qh0 + h] (one per query head) arrive by TMA as ring positions 0 .. route_tiles - 1,
@@ -445,6 +452,15 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
         ptx::tmem_alloc(&sm.tmem_base, tmem_cols);
         ptx::tmem_relinquish();
     }
+    if (D != kD) {
+        // zeros under the halves that TMA never writes (the ring and the query operand); the
+        // fence orders these writes before the copies and MMAs issued after the barrier below
+        uint4 *z = reinterpret_cast<uint4 *>(&sm.tiles[0][0][0]);
+        for (uint32_t i = tid; i < sizeof(sm.tiles) / 16; i += blockDim.x) z[i] = make_uint4(0, 0, 0, 0);
+        uint4 *zq = reinterpret_cast<uint4 *>(sm.qr);
+        for (uint32_t i = tid; i < sizeof(sm.qr) / 16; i += blockDim.x) zq[i] = make_uint4(0, 0, 0, 0);
+        ptx::fence_proxy_async_smem();
+    }
     if (warp == kProducerWarp && lane == 0) {
         ptx::prefetch_tensormap(&vmap);
         if (kStandard) ptx::prefetch_tensormap(&kmap);
@@ -479,28 +495,31 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
         if (app_owner && warp == 0) {
             const int page = bt[pos_raw / geo.P];
             if (page >= 0 && page < geo.num_pages) {
-                const size_t off = (((size_t)page * geo.Hkv + g) * geo.P + pos_raw % geo.P) * kD;
-                reinterpret_cast<uint2 *>(a.cache_rw + off)[lane] =
-                    reinterpret_cast<const uint2 *>(a.v_new + ((size_t)b * geo.Hkv + g) * kD)[lane];
+                const size_t off = (((size_t)page * geo.Hkv + g) * geo.P + pos_raw % geo.P) * D;
+                const uint16_t *src = a.v_new + ((size_t)b * geo.Hkv + g) * D;
+                if (D == kD)
+                    reinterpret_cast<uint2 *>(a.cache_rw + off)[lane] = reinterpret_cast<const uint2 *>(src)[lane];
+                else
+                    reinterpret_cast<uint32_t *>(a.cache_rw + off)[lane] = reinterpret_cast<const uint32_t *>(src)[lane];
             } else if (lane == 0) {
                 raise_flag(a.err, KL_FLAG_BAD_PAGE);
             }
         }
-        if (tid < kD) {
+        if (tid < D) {
             for (int h = 0; h < G; ++h) {
                 const size_t bh = (size_t)b * geo.Hq + qh0 + h;
                 if (a.merge_inside) {
                     if (L == 0 && cta == 0) {
-                        if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * kD + tid] = 0.f;
-                        else static_cast<__nv_bfloat16 *>(a.out)[bh * kD + tid] = __float2bfloat16_rn(0.f);
+                        if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * D + tid] = 0.f;
+                        else static_cast<__nv_bfloat16 *>(a.out)[bh * D + tid] = __float2bfloat16_rn(0.f);
                     }
                 } else if (a.direct_out) {
-                    if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * kD + tid] = 0.f;
-                    else static_cast<__nv_bfloat16 *>(a.out)[bh * kD + tid] = __float2bfloat16_rn(0.f);
+                    if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * D + tid] = 0.f;
+                    else static_cast<__nv_bfloat16 *>(a.out)[bh * D + tid] = __float2bfloat16_rn(0.f);
                 } else {
                     for (int sp = split0; sp < min(split0 + geo.spc, geo.S); ++sp) {
                         const size_t slot = bh * geo.S + sp;
-                        a.part_o[slot * kD + tid] = 0.f;
+                        a.part_o[slot * D + tid] = 0.f;
                         if (tid == 0) {
                             a.part_ml[slot * 2] = -INFINITY;
                             a.part_ml[slot * 2 + 1] = 0.f;
@@ -534,8 +553,10 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
             const int page = bt[pos_raw / P];
             if (page >= 0 && page < geo.num_pages) {
                 app_tile = pos_raw < t_end ? (pos_raw - t_begin) / kTile : 0;
-                app_off = (((size_t)page * geo.Hkv + g) * P + pos_raw % P) * kD;
-                app_val = reinterpret_cast<const uint2 *>(a.v_new + ((size_t)b * geo.Hkv + g) * kD)[lane];
+                app_off = (((size_t)page * geo.Hkv + g) * P + pos_raw % P) * D;
+                const uint16_t *src = a.v_new + ((size_t)b * geo.Hkv + g) * D;
+                app_val = D == kD ? reinterpret_cast<const uint2 *>(src)[lane]
+                                  : make_uint2(reinterpret_cast<const uint32_t *>(src)[lane], 0u);
             } else if (lane == 0) {
                 raise_flag(a.err, KL_FLAG_BAD_PAGE);
             }
@@ -547,13 +568,16 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
             const int s = r % NS;
             if (r >= NS && !wait(&sm.empty[s], ((r / NS) & 1) ^ 1)) break;
             if (lane == 0) {
-                const int wrow = (route_pq ? qh0 + r : g) * kD;
-                ptx::mbar_arrive_expect_tx(&sm.full[s], kTileBytes + (r == 0 ? 2u * (uint32_t)geo.qbox * 128u : 0u));
+                // W^R: two 64-column halves of 128 rows, or (head dim 64) one box of 64 x 64
+                const int wrow = (route_pq ? qh0 + r : g) * D;
+                const uint32_t halves = (uint32_t)D / 64u;
+                ptx::mbar_arrive_expect_tx(&sm.full[s], (D == kD ? kTileBytes : 64u * 128u) +
+                                                            (r == 0 ? halves * (uint32_t)geo.qbox * 128u : 0u));
                 ptx::tma_load_2d(sm.tiles[s][0], &wmap, &sm.full[s], 0, wrow);
-                ptx::tma_load_2d(sm.tiles[s][0] + kHalfBytes, &wmap, &sm.full[s], 64, wrow);
+                if (D == kD) ptx::tma_load_2d(sm.tiles[s][0] + kHalfBytes, &wmap, &sm.full[s], 64, wrow);
                 if (r == 0) {
                     ptx::tma_load_2d(sm.qr, &qmap, &sm.full[s], 0, b * geo.Hq + qh0);
-                    ptx::tma_load_2d(sm.qr + kN * 128, &qmap, &sm.full[s], 64, b * geo.Hq + qh0);
+                    if (D == kD) ptx::tma_load_2d(sm.qr + kN * 128, &qmap, &sm.full[s], 64, b * geo.Hq + qh0);
                 }
             }
             __syncwarp();
@@ -580,24 +604,25 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
             const bool in_range = exists && page >= 0 && page < geo.num_pages;
             if (exists && !in_range) bad = true;
             if (i == app_tile) {
-                reinterpret_cast<uint2 *>(a.cache_rw + app_off)[lane] = app_val;
+                if (D == kD) reinterpret_cast<uint2 *>(a.cache_rw + app_off)[lane] = app_val;
+                else reinterpret_cast<uint32_t *>(a.cache_rw + app_off)[lane] = app_val.x;
                 ptx::fence_proxy_async_global();
                 __syncwarp();
             }
             const unsigned mask = __ballot_sync(0xffffffffu, in_range);
             if (lane == 0)
-                ptx::mbar_arrive_expect_tx(&sm.full[s], __popc(mask) * page_bytes * 2u *
+                ptx::mbar_arrive_expect_tx(&sm.full[s], __popc(mask) * page_bytes * ((uint32_t)D / 64u) *
                                                             Cfg<kStandard>::kTilesPerStage);
             __syncwarp();
             if (in_range) {
                 const int row = (page * geo.Hkv + g) * P;
                 uint8_t *dst = sm.tiles[s][0] + lane * page_bytes;
                 ptx::tma_load_2d(dst, &vmap, &sm.full[s], 0, row);
-                ptx::tma_load_2d(dst + kHalfBytes, &vmap, &sm.full[s], 64, row);
+                if (D == kD) ptx::tma_load_2d(dst + kHalfBytes, &vmap, &sm.full[s], 64, row);
                 if constexpr (kStandard) {
                     uint8_t *kd = sm.tiles[s][1] + lane * page_bytes;
                     ptx::tma_load_2d(kd, &kmap, &sm.full[s], 0, row);
-                    ptx::tma_load_2d(kd + kHalfBytes, &kmap, &sm.full[s], 64, row);
+                    if (D == kD) ptx::tma_load_2d(kd + kHalfBytes, &kmap, &sm.full[s], 64, row);
                 }
             }
             issued = r + 1;
@@ -754,13 +779,13 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
             if (a.pdl) grid_dep_wait();
 #pragma unroll
             for (int e = 0; e < KH; ++e)
-                acc[e] = h0 + e < G ? a.q_routed[((size_t)b * geo.Hq + qh0 + h0 + e) * kD + t] : 0.f;
+                acc[e] = h0 + e < G && t < D ? a.q_routed[((size_t)b * geo.Hq + qh0 + h0 + e) * D + t] : 0.f;
         } else {
             for (int i = tid; i < kD * kNG; i += kComputeThreads) {
                 const int k = i >> 3, h = i & 7;
-                qf[i] = h < G ? __uint_as_float(
-                                    (uint32_t)a.q[((size_t)b * geo.Hq + qh0 + h) * kD + k] << 16)
-                              : 0.f;
+                qf[i] = h < G && k < D ? __uint_as_float(
+                                             (uint32_t)a.q[((size_t)b * geo.Hq + qh0 + h) * D + k] << 16)
+                                       : 0.f;
             }
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&sm.q_ready);
@@ -861,7 +886,7 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
                 if (h >= G) continue;
                 const float lt = (sm.lred[0][h] + sm.lred[1][h]) + (sm.lred[2][h] + sm.lred[3][h]);
                 const size_t slot = ((size_t)b * geo.Hq + qh0 + h) * geo.S + sp;
-                a.part_o[slot * kD + t] = o[e] / lt;
+                if (t < D) a.part_o[slot * D + t] = o[e] / lt;
                 if (t == 0) {
                     a.part_ml[slot * 2] = m[e] * kLn2;
                     a.part_ml[slot * 2 + 1] = lt;
@@ -1003,11 +1028,12 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
                     const float val = o[e] / lt;
                     const size_t bh = (size_t)b * geo.Hq + qh0 + h;
                     if (write_out) {
-                        if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * kD + t] = val;
-                        else static_cast<__nv_bfloat16 *>(a.out)[bh * kD + t] = __float2bfloat16_rn(val);
+                        if (t >= D) continue;
+                        if (a.out_dtype == KL_FP32) static_cast<float *>(a.out)[bh * D + t] = val;
+                        else static_cast<__nv_bfloat16 *>(a.out)[bh * D + t] = __float2bfloat16_rn(val);
                     } else {
                         const size_t slot = bh * geo.S + sp_last;
-                        a.part_o[slot * kD + t] = val;
+                        if (t < D) a.part_o[slot * D + t] = val;
                         if (t == 0) {
                             a.part_ml[slot * 2] = m[e] * kLn2;
                             a.part_ml[slot * 2 + 1] = lt;
@@ -1016,7 +1042,7 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
                         if (!a.merge_inside) {
                             for (int sp = sp_last + 1; sp < min(split0 + geo.spc, geo.S); ++sp) {
                                 const size_t es = bh * geo.S + sp;
-                                a.part_o[es * kD + t] = 0.f;
+                                if (t < D) a.part_o[es * D + t] = 0.f;
                                 if (t == 0) {
                                     a.part_ml[es * 2] = -INFINITY;
                                     a.part_ml[es * 2 + 1] = 0.f;
@@ -1071,13 +1097,13 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     return fn;
 }
 
-// 2-D bf16 tensor map over `rows` rows of 128 dims (256-byte rows), box = 64 dims x box_rows
+// 2-D bf16 tensor map over `rows` rows of `dim` (128 or 64) dims, box = 64 dims x box_rows
 // (one 128-byte swizzle span), 128-byte swizzle.
-bool make_map(CUtensorMap *map, const void *base, uint64_t rows, uint32_t box_rows) {
+bool make_map(CUtensorMap *map, const void *base, int dim, uint64_t rows, uint32_t box_rows) {
     auto fn = encode_fn();
     if (!fn) return false;
-    const cuuint64_t dims[2] = {(cuuint64_t)kD, (cuuint64_t)rows};
-    const cuuint64_t strides[1] = {(cuuint64_t)kD * 2};
+    const cuuint64_t dims[2] = {(cuuint64_t)dim, (cuuint64_t)rows};
+    const cuuint64_t strides[1] = {(cuuint64_t)dim * 2};
     const cuuint32_t box[2] = {64, box_rows};
     const cuuint32_t estr[2] = {1, 1};
     return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides,
@@ -1126,16 +1152,17 @@ cudaError_t launch(const DecodeArgs &a) {
     // cache viewed as [num_pages * Hkv * P rows][128]; one box = one page of one head
     const uint64_t cache_rows = (uint64_t)g.num_pages * g.Hkv * g.P;
     CUtensorMap vmap, kmap, wmap, qmap;
-    if (!make_map(&vmap, a.v_cache, cache_rows, (uint32_t)g.P)) return cudaErrorInvalidValue;
+    if (!make_map(&vmap, a.v_cache, g.D, cache_rows, (uint32_t)g.P)) return cudaErrorInvalidValue;
     kmap = wmap = qmap = vmap;
-    if (kStandard && !make_map(&kmap, a.k_cache, cache_rows, (uint32_t)g.P))
+    if (kStandard && !make_map(&kmap, a.k_cache, g.D, cache_rows, (uint32_t)g.P))
         return cudaErrorInvalidValue;
     if (!kStandard && !a.q_routed && a.w_r) {
         // W^R [Hw * 128 rows (k)][128 (j)], Hw = Hkv or Hq, one box = one 64-column half of one
         // matrix; q [B * Hq rows][128], one box = the up to 8 rows of one CTA's heads.
         const uint64_t hw = g.wr_per_qh ? (uint64_t)g.Hq : (uint64_t)g.Hkv;
-        if (!make_map(&wmap, a.w_r, hw * kD, kD)) return cudaErrorInvalidValue;
-        if (!make_map(&qmap, a.q, (uint64_t)g.B * g.Hq, (uint32_t)a.geo.qbox)) return cudaErrorInvalidValue;
+        if (!make_map(&wmap, a.w_r, g.D, hw * g.D, (uint32_t)g.D)) return cudaErrorInvalidValue;
+        if (!make_map(&qmap, a.q, g.D, (uint64_t)g.B * g.Hq, (uint32_t)a.geo.qbox))
+            return cudaErrorInvalidValue;
     }
     // Splits per CTA: one, unless one CTA per split would overflow a wave of two CTAs per SM
     // while the (b, g) units alone would not fill it (few long sequences split many ways): then
@@ -1170,7 +1197,7 @@ bool tc_merge_inside(const Geometry &g, bool standard) {
 
 bool tc_supported(const Geometry &g, bool standard) {
     (void)standard;
-    if (g.D != kD || g.G > kMaxGroup) return false;
+    if ((g.D != kD && g.D != 64) || g.G > kMaxGroup) return false;
     if (g.P != 16 && g.P != 32 && g.P != 64 && g.P != 128) return false;
     if ((int64_t)g.num_pages * g.Hkv * g.P >= ((int64_t)1 << 31)) return false;
     int dev = 0, major = 0, minor = 0;
