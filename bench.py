@@ -656,7 +656,7 @@ def sweep_workloads(args, dev, stream, flush_l2, x70, g70, sh70, keyless_ms):
     import torch
 
     import paper_2606_21848_gb300 as kl
-    from paper_2606_21848_gb300.workloads import LARGE_GROUPS, ORDER, WORKLOADS, generate
+    from paper_2606_21848_gb300.workloads import EXTRA, ORDER, WORKLOADS, generate
 
     peak, peak_kind = measured_peaks()
     launches = 0
@@ -670,7 +670,7 @@ def sweep_workloads(args, dev, stream, flush_l2, x70, g70, sh70, keyless_ms):
         return e
 
     workloads = {}
-    for name in ORDER + LARGE_GROUPS:
+    for name in ORDER + EXTRA:
         if name == DEFAULT_WORKLOAD:
             continue
         wl = WORKLOADS[name]

@@ -104,6 +104,14 @@ WORKLOADS.update({
 })
 LARGE_GROUPS = ["mqa_group32", "gqa_group16"]
 
+# Head dim 64 (GPT-2's head layout, the paper's main experiments): 16 heads of 64 dims, multi-head
+# (one value head per query head), batch 32 at 8192 tokens -- 512 MiB of cached values.
+WORKLOADS.update({
+    "mha_d64": Workload("mha_d64", 32, 16, 16, 64, 16, seq_len=8192, wr_std=math.sqrt(1 / 64),
+                        seed=10),
+})
+EXTRA = LARGE_GROUPS + ["mha_d64"]
+
 # Prefill workloads (chunked prefill, the step before decode): a whole 32K-token prompt with
 # the paper's Qwen2-1.5B attention (12 query heads, 2 value heads, head dim 128, W^R per query
 # head, trained at 32,768 tokens), and a serving-style chunk of 512 new tokens on an
