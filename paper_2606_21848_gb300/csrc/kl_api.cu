@@ -65,6 +65,9 @@ kl_status resolve(const kl_shape *s, int32_t num_splits, Geometry *g) {
     g->chunk = 0;
     g->nhb = (g->G + 7) / 8;
     g->qbox = g->G < 8 ? g->G : 8;
+    // head dim 64: a tensor-core CTA takes two value heads (even Hkv, groups of up to 4)
+    g->vpc = (g->D == 64 && g->Hkv % 2 == 0 && g->G <= 4) ? 2 : 1;
+    if (g->vpc == 2) g->qbox = 2 * g->G;
     if (num_splits < 0) return KL_OK;
     if (num_splits > kMaxSplits) return KL_ERR_INVALID_ARG;
 
@@ -74,7 +77,7 @@ kl_status resolve(const kl_shape *s, int32_t num_splits, Geometry *g) {
         // As many splits as fit one wave of two CTAs per SM over the (value head, sequence)
         // units, and splits of at most 8192 tokens so that ragged batches balance; never
         // below 256 tokens per split.
-        const int64_t units = (int64_t)(g->B > 0 ? g->B : 1) * g->Hkv * g->nhb;
+        const int64_t units = (int64_t)(g->B > 0 ? g->B : 1) * (g->Hkv / g->vpc) * g->nhb;
         const int64_t slots = 2 * (int64_t)device_sm_count();
         const int64_t fill = units < slots ? slots / units : 1;
         const int64_t cap = (Lmax + 8191) / 8192;

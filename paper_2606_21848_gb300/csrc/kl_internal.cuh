@@ -27,7 +27,9 @@ struct Geometry {
     int chunk;         // tokens per split (a multiple of 128)
     int spc = 1;       // splits per CTA of the tensor-core decode (consecutive, same (b, g))
     int nhb = 1;       // CTAs per (run of splits, b, g): blocks of up to 8 query heads
-    int qbox = 8;      // query rows per block: min(G, 8)
+    int qbox = 8;      // query rows of one CTA: min(G, 8), or 2 G with two value heads
+    int vpc = 1;       // value heads per CTA of the tensor-core decode: 2 at head dim 64 (the
+                       // two heads' rows side by side in one 128-wide tile), else 1
 };
 
 // Arguments of a decode launch (keyless or the standard K+V comparison).

@@ -1,6 +1,10 @@
 """GPU parity of the tensor-core decode at head dim 64 (GPT-2's head layout, the paper's main
 experiments in Section 5): every cached row read once for score and output, against the fp64
 oracle at |gpu - oracle| <= 2e-3 + 1e-2 |oracle|, appended rows and permutations bit-exact.
+
+With an even number of value heads and groups of up to 4 query heads, one CTA takes two value
+heads side by side in its 128-wide tiles (block-diagonal routing); otherwise a 64-dim row fills
+half of a zero-padded tile. Both layouts are covered below.
 """
 from __future__ import annotations
 
@@ -31,6 +35,7 @@ SHAPES = [
     dict(B=3, Hq=32, Hkv=8, D=64, P=32, lens=(0, 129, 2000)),     # GQA 4, P 32
     dict(B=2, Hq=64, Hkv=8, D=64, P=16, lens=(700, 1500)),        # GQA 8
     dict(B=1, Hq=16, Hkv=1, D=64, P=64, lens=(3000,)),            # MQA, group 16 (two CTAs)
+    dict(B=2, Hq=6, Hkv=3, D=64, P=16, lens=(800, 5)),            # odd value-head count
 ]
 
 
