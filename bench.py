@@ -83,8 +83,9 @@ def measured_peaks():
 
 
 # the sources each decode kernel is compiled from (traffic records are keyed to their hash)
-DECODE_SOURCES = ("kl_decode_tc.cu", "kl_internal.cuh", "kl_tc_ptx.cuh")
-FP8_SOURCES = ("kl_decode_fp8.cu", "kl_internal.cuh", "kl_tc_ptx.cuh")
+DECODE_SOURCES = ("kl_decode_tc.cu", "kl_decode_tc64.cu", "kl_decode_tc_kernel.cuh",
+                  "kl_internal.cuh", "kl_tc_ptx.cuh")
+FP8_SOURCES = ("kl_decode_fp8.cu", "kl_fp8_quant.cuh", "kl_internal.cuh", "kl_tc_ptx.cuh")
 
 
 def kernel_source_digest(names=DECODE_SOURCES) -> str:
@@ -701,7 +702,9 @@ def sweep_workloads(args, dev, stream, flush_l2, x70, g70, sh70, keyless_ms):
             workloads[name + ("_" + suffix if suffix else "")] = gbs_entry(
                 ms, ab["total"], B, {"num_splits": S, "kernel": "tensor" if tc else "simt",
                                      "kernels_per_step": n_launch,
-                                     "context_tokens": ab["tokens"]})
+                                     "context_tokens": ab["tokens"],
+                                     "traffic": None if suffix else
+                                     recorded_traffic(name, "tensor" if tc else "simt")})
         del g, out, ws, x
         torch.cuda.empty_cache()
 
@@ -754,7 +757,9 @@ def sweep_workloads(args, dev, stream, flush_l2, x70, g70, sh70, keyless_ms):
     ab8 = algorithmic_bytes(x70, False, fp8=True)
     fp8 = gbs_entry(fp8_ms, ab8["total"], B, {"workload": DEFAULT_WORKLOAD,
                                               "what": "kl_decode_step_fp8",
-                                              "speedup_over_bf16_step": keyless_ms / fp8_ms})
+                                              "speedup_over_bf16_step": keyless_ms / fp8_ms,
+                                              "traffic": recorded_traffic(DEFAULT_WORKLOAD,
+                                                                          "tensor-fp8")})
 
     # Latent value-only cache: one step = kl_latent_decode_step (three kernels).
     wl = WORKLOADS["latent_serving"]
