@@ -57,6 +57,7 @@ constexpr uint32_t kHalfBytes = kTileBytes / 2;   // one 64-dim half: 128 rows x
 constexpr uint32_t kTmemCols = 64;                // S: 2 x 16 columns, O: 2 x 16 columns
 constexpr uint32_t kTmemColsPq = 256;             // + one 16-column routing result per head
 constexpr uint64_t kTimeoutNs = kDefaultWaitNs;   // bound of the drains
+constexpr float kLazy = 2.f;                      // reference slack (base 2): weights <= 4
 // Warp roles for KH heads per compute warp: KH = 8, one compute warp per TMEM lane quarter;
 // KH = 2 (groups of up to 4 heads), two per quarter.
 template <int KH>
@@ -138,6 +139,7 @@ struct __align__(1024) Smem {
     uint8_t p[2][kTile * kN * 2];
     float red[2][4][kNG];              // per lane quarter and head: tile maxima, row sums
     float lred[4][kNG];                // row sums of a split closed inside a CTA's run
+    float mred[4][kNG];                // per lane quarter and head: largest score of a state
     uint64_t full[Cfg<kStandard>::kStages], empty[Cfg<kStandard>::kStages];
     uint64_t s_full[2], s_empty[2], p_full[2], o_full[2], o_empty[2];
     uint64_t qr_full, q_ready, r_full, drain, drain2, merge_full;
@@ -888,15 +890,34 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
             }
         }
 
-        float m[KH], lsum[KH], o[KH];
+        // Lazy reference: a tile's weights are 2^(s - m) with the head's current reference m,
+        // which moves to the running maximum (rescaling the running sums) only when a score
+        // passes thr = m + kLazy, so the weights stay at most 2^kLazy and most tiles need one
+        // vote of the compute warps instead of an exchange of their maxima. mx holds the
+        // thread's largest score of the current state, so that a state written out carries
+        // its true largest score.
+        float m[KH], thr[KH], mx[KH], lsum[KH], o[KH];
         Vec<KH> alpha_prev;
 #pragma unroll
         for (int e = 0; e < KH; ++e) {
             m[e] = -INFINITY;
+            thr[e] = -INFINITY;
+            mx[e] = -INFINITY;
             lsum[e] = 0.f;
             o[e] = 0.f;
             alpha_prev.v[e] = 0.f;
         }
+        // The CTA's largest score of each head of the current state into sm.mred (the caller's
+        // next CTA barrier makes it visible).
+        auto head_max = [&]() {
+            float x[KH];
+#pragma unroll
+            for (int e = 0; e < KH; ++e) x[e] = mx[e];
+            const float wm = warp_max_k<KH>(x, lane);
+            if (KH == 8 && (lane & 3) == 0)
+                sm.mred[qd][((lane >> 4) & 1) * 4 + ((lane >> 3) & 1) * 2 + ((lane >> 2) & 1)] = wm;
+            if (KH == 2 && (lane & 15) == 0) sm.mred[qd][h0 + ((lane >> 4) & 1)] = wm;
+        };
 
         // O accumulation of tile j: o = o * alpha_j + O_j (thread = output dim t).
         auto correct = [&](int j, const Vec<KH> alpha) -> bool {
@@ -936,6 +957,7 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
 #pragma unroll
                 for (int e = 0; e < KH; ++e) sm.lred[qd][h0 + e] = l[e];
             }
+            head_max();
             ptx::bar_sync(kBarCompute, kComputeThreads);
 #pragma unroll
             for (int e = 0; e < KH; ++e) {
@@ -946,8 +968,11 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
                 const int dd = t - dim0(h);
                 if (dd >= 0 && dd < D) a.part_o[slot * D + dd] = o[e] / lt;
                 if (t == 0) {
-                    a.part_ml[slot * 2] = m[e] * kLn2;
-                    a.part_ml[slot * 2 + 1] = lt;
+                    // the state with its largest score M: l = sum 2^(s - M) = lt 2^(m - M)
+                    const float M = fmaxf(fmaxf(sm.mred[0][h], sm.mred[1][h]),
+                                          fmaxf(sm.mred[2][h], sm.mred[3][h]));
+                    a.part_ml[slot * 2] = M * kLn2;
+                    a.part_ml[slot * 2 + 1] = lt * exp2f(m[e] - M);
                 }
             }
             ptx::bar_sync(kBarCompute, kComputeThreads);      // lred is free for the next split
@@ -972,6 +997,8 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
                     o[e] = 0.f;
                     lsum[e] = 0.f;
                     m[e] = -INFINITY;
+                    thr[e] = -INFINITY;
+                    mx[e] = -INFINITY;
                 }
             }
             ptx::tc_fence_after();
@@ -983,36 +1010,50 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
 
             const int nvalid = min(kTile, t_end - (t_begin + i * kTile));
             const bool valid = t < nvalid;
-            float s[KH], mx[KH];
+            float s[KH];
+            bool grow = false;
 #pragma unroll
             for (int e = 0; e < KH; ++e) {
                 s[e] = (valid && h0 + e < G) ? head_col<KH>(sv, 0, hh, e) + head_col<KH>(sv, kNG, hh, e)
                                              : -INFINITY;
-                mx[e] = s[e];
+                grow = grow || s[e] > thr[e];
+                mx[e] = fmaxf(mx[e], s[e]);
             }
-            // per-head maximum over the tile's 128 tokens: warp reduce, then across the 4
-            // lane quarters
-            {
-                const float wm = warp_max_k<KH>(mx, lane);
+            Vec<KH> alpha;
+#pragma unroll
+            for (int e = 0; e < KH; ++e) alpha.v[e] = 1.f;
+            // (a state's first tile always sets the reference: no vote)
+            const bool first = i == 0 || (kPerSplit && i % tps == 0);
+            if (first || ptx::bar_popc(kBarComputeAnd, kComputeThreads, grow) != 0) {
+                // a score passed its reference: the per-head maximum over the tile's 128 tokens
+                // (warp reduce, then across the 4 lane quarters) becomes the reference
+                float x[KH];
+#pragma unroll
+                for (int e = 0; e < KH; ++e) x[e] = s[e];
+                const float wm = warp_max_k<KH>(x, lane);
                 if (KH == 8 && (lane & 3) == 0)
                     sm.red[sb][qd][((lane >> 4) & 1) * 4 + ((lane >> 3) & 1) * 2 + ((lane >> 2) & 1)] = wm;
                 if (KH == 2 && (lane & 15) == 0) sm.red[sb][qd][h0 + ((lane >> 4) & 1)] = wm;
+                ptx::bar_sync(kBarCompute, kComputeThreads);
+#pragma unroll
+                for (int e = 0; e < KH; ++e) {
+                    const int h = h0 + e;
+                    float tmax = sm.red[sb][0][h];
+#pragma unroll
+                    for (int q = 1; q < 4; ++q) tmax = fmaxf(tmax, sm.red[sb][q][h]);
+                    const bool live = h < G;
+                    const float mn = fmaxf(m[e], tmax);
+                    alpha.v[e] = live ? exp2f(m[e] - mn) : 0.f;
+                    lsum[e] *= alpha.v[e];
+                    m[e] = live ? mn : m[e];
+                    thr[e] = live ? mn + kLazy : thr[e];
+                }
             }
-            ptx::bar_sync(kBarCompute, kComputeThreads);
-            Vec<KH> alpha;
             float p[KH];
 #pragma unroll
             for (int e = 0; e < KH; ++e) {
-                const int h = h0 + e;
-                float tmax = sm.red[sb][0][h];
-#pragma unroll
-                for (int q = 1; q < 4; ++q) tmax = fmaxf(tmax, sm.red[sb][q][h]);
-                const float mn = fmaxf(m[e], tmax);
-                const bool live = h < G;
-                alpha.v[e] = live ? exp2f(m[e] - mn) : 0.f;
-                p[e] = live ? exp2f(s[e] - mn) : 0.f;
-                lsum[e] = fmaf(lsum[e], alpha.v[e], p[e]);
-                m[e] = live ? mn : m[e];
+                p[e] = h0 + e < G ? exp2f(s[e] - m[e]) : 0.f;
+                lsum[e] += p[e];
             }
             // P^T row of token t, this warp's heads: hi and lo halves.
             {
@@ -1069,6 +1110,11 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
 #pragma unroll
                 for (int e = 0; e < KH; ++e) sm.red[rb][qd][h0 + e] = lsum[e];
             }
+            // States that leave the kernel (for the caller or the combine kernel) carry their
+            // true largest score; the merge inside the kernel takes any reference (l = sum
+            // 2^(s - m) for the m it is given), so its states keep the lazy one.
+            const bool exact_m = !a.direct_out && !a.merge_inside;
+            if (exact_m) head_max();
             ptx::bar_sync(kBarCompute, kComputeThreads);
             {
                 // Merged here: one state per CTA run that holds tokens (slot cta; a single one
@@ -1095,8 +1141,13 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
                         const size_t slot = bh * geo.S + sp_last;
                         if (mine) a.part_o[slot * D + dd] = val;
                         if (t == 0) {
-                            a.part_ml[slot * 2] = m[e] * kLn2;
-                            a.part_ml[slot * 2 + 1] = lt;
+                            // the state with its largest score M (l = lt 2^(m - M)), or with the
+                            // lazy reference m for the merge inside the kernel
+                            const float M = exact_m ? fmaxf(fmaxf(sm.mred[0][h], sm.mred[1][h]),
+                                                            fmaxf(sm.mred[2][h], sm.mred[3][h]))
+                                                    : m[e];
+                            a.part_ml[slot * 2] = M * kLn2;
+                            a.part_ml[slot * 2 + 1] = exact_m ? lt * exp2f(m[e] - M) : lt;
                         }
                         // splits of the run past the sequence's end: empty states
                         if (!a.merge_inside) {

@@ -162,6 +162,19 @@ __device__ __forceinline__ void bar_sync(uint32_t id, uint32_t count) {
 
 // Barrier `id` over `count` threads that also returns the AND of `v` over them, so that a
 // decision (e.g. to leave a loop) is taken by all of them together.
+// Barrier `id` over `count` threads that also returns how many of them passed v = true.
+__device__ __forceinline__ uint32_t bar_popc(uint32_t id, uint32_t count, bool v) {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "bar.red.popc.u32 %0, %2, %3, p;\n\t}\n"
+        : "=r"(r)
+        : "r"((uint32_t)v), "r"(id), "r"(count)
+        : "memory");
+    return r;
+}
+
 __device__ __forceinline__ bool bar_and(uint32_t id, uint32_t count, bool v) {
     uint32_t r;
     asm volatile(
