@@ -83,7 +83,8 @@ def measured_peaks():
 
 
 # the sources each decode kernel is compiled from (traffic records are keyed to their hash)
-DECODE_SOURCES = ("kl_decode_tc.cu", "kl_decode_tc64.cu", "kl_decode_tc_kernel.cuh",
+DECODE_SOURCES = ("kl_decode_tc.cu", "kl_decode_tc64.cu", "kl_decode_tc_groups.cu",
+                  "kl_decode_tc_kernel.cuh",
                   "kl_internal.cuh", "kl_tc_ptx.cuh")
 FP8_SOURCES = ("kl_decode_fp8.cu", "kl_fp8_quant.cuh", "kl_internal.cuh", "kl_tc_ptx.cuh")
 

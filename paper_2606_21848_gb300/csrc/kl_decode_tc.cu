@@ -1,6 +1,7 @@
 // Tensor-core split-sequence decode: the host-side plan (tensor maps, splits per CTA, heads per
-// compute warp) and the head-dim-128 kernels; the kernel itself is in kl_decode_tc_kernel.cuh,
-// the head-dim-64 kernels in kl_decode_tc64.cu.
+// compute warp) and the head-dim-128 kernels of groups of up to 8 heads; the kernel itself is in
+// kl_decode_tc_kernel.cuh, the head-dim-64 kernels in kl_decode_tc64.cu, those of larger groups
+// in kl_decode_tc_groups.cu.
 #include "kl_decode_tc_kernel.cuh"
 
 namespace kl {
@@ -16,7 +17,8 @@ cudaError_t launch_waits(const DecodeArgs &la, bool per_split, const CUtensorMap
 
 template <bool kStandard>
 cudaError_t launch(const DecodeArgs &a) {
-    const Geometry &g = a.geo;
+    DecodeArgs la = a;
+    const Geometry &g = la.geo;
     // cache viewed as [num_pages * Hkv * P rows][128]; one box = one page of one head
     const uint64_t cache_rows = (uint64_t)g.num_pages * g.Hkv * g.P;
     CUtensorMap vmap, kmap, wmap, qmap;
@@ -29,13 +31,12 @@ cudaError_t launch(const DecodeArgs &a) {
         // matrix; q [B * Hq rows][128], one box = the up to 8 rows of one CTA's heads.
         const uint64_t hw = g.wr_per_qh ? (uint64_t)g.Hq : (uint64_t)g.Hkv;
         if (!make_map(&wmap, a.w_r, g.D, hw * g.D, (uint32_t)g.D)) return cudaErrorInvalidValue;
-        if (!make_map(&qmap, a.q, g.D, (uint64_t)g.B * g.Hq, (uint32_t)a.geo.qbox))
+        if (!make_map(&qmap, a.q, g.D, (uint64_t)g.B * g.Hq, (uint32_t)g.qbox))
             return cudaErrorInvalidValue;
     }
     // Splits per CTA: one, unless one CTA per split would overflow a wave of two CTAs per SM
     // while the (b, g) units alone would not fill it (few long sequences split many ways): then
     // the fewest consecutive splits per CTA that fit the wave.
-    DecodeArgs la = a;
     const int64_t units = (int64_t)g.B * (g.Hkv / g.vpc) * g.nhb;
     const int64_t slots = 2 * (int64_t)device_sm_count();
     int spc = 1;
@@ -43,9 +44,12 @@ cudaError_t launch(const DecodeArgs &a) {
         while ((int64_t)((g.S + spc - 1) / spc) * units > slots) ++spc;
     la.geo.spc = spc;
     const bool per_split = spc > 1 && !a.merge_inside && !a.direct_out;
-    // heads per compute warp: all 8 (padded) on four warps, or 2 on eight when the group has
-    // at most 4; exact short waits only when the limit asks for them
+    // heads per compute warp: all 8 (padded) on four warps; 4 on eight for the sibling CTAs
+    // of larger groups (head dim 128); 2 on eight when the group has at most 4. Exact short
+    // waits only when the limit asks for them.
     const bool exact = a.wait_ns < kExactWaitNs;
+    if (g.nhb > 1 && g.D == 128)
+        return launch_tc_groups(la, per_split, kStandard, exact, vmap, kmap, wmap, qmap);
     if (g.vpc * (g.G < kNG ? g.G : kNG) <= 4)
         return exact ? launch_waits<kStandard, 2, true>(la, per_split, vmap, kmap, wmap, qmap)
                      : launch_waits<kStandard, 2, false>(la, per_split, vmap, kmap, wmap, qmap);

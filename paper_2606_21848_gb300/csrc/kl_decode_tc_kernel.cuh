@@ -1,8 +1,9 @@
 // Tensor-core split-sequence decode for sm_103a: TMA page gathers into a shared-memory ring,
 // tcgen05 MMAs with TMEM accumulators, warp-specialized roles.
 //
-// One CTA per (run of splits, value head g, sequence b); head_dim 128, up to 8 query heads per value
-// group. The value-space routing (Section 2.2: q_r = q W^R) runs first, as tensor-core MMAs on
+// One CTA per (run of splits, value head g, sequence b, block of up to 8 of the group's query
+// heads: groups of more than 8 heads run ceil(G / 8) sibling CTAs that read the same pages);
+// head_dim 128 or 64. The value-space routing (Section 2.2: q_r = q W^R) runs first, as tensor-core MMAs on
 // W^R tiles that stream through the ring, into a split-bf16 operand (q_r * scale * log2 e =
 // hi + lo, both bf16) for the G heads of the group.
 // Then each 128-token tile of cached value rows V_t [128 x 128] (Section 3) is used twice by
@@ -17,14 +18,16 @@
 //
 // Roles (224 or 352 threads, two CTAs per SM):
 //   compute    routing prologue; per tile read S from TMEM (thread = token), online softmax in
-//              base 2 (per-head running max across the CTA), write P^T to shared memory; read
-//              O from TMEM (thread = output dim) and accumulate with rescaling; epilogue writes
-//              the output or the split state, or merges the splits. Groups of more than 4
-//              heads: warps 0-3, one per TMEM lane quarter, all 8 (padded) heads each. Groups
-//              of up to 4: warps 0-7, warps w and w + 4 sharing lane quarter w % 4 and 2 heads
-//              each, so the live heads alone are computed and a tile's softmax runs on two
-//              warps per SM sub-partition (6.7 % faster on the 4-head long-context decode; with
-//              8 heads, four per warp on eight warps, the 70B batch ran 2 % slower).
+//              base 2 against a lazy per-head reference (moved only when a score passes it by
+//              more than 2), write P^T to shared memory; read O from TMEM (thread = output dim)
+//              and accumulate with rescaling; epilogue writes the output or the split state, or
+//              merges the splits. Groups of 5-8 heads: warps 0-3, one per TMEM lane quarter, all
+//              8 (padded) heads each (KH 8; the 70B batch is HBM-bound there and ran 2 % slower
+//              on eight warps). Sibling CTAs of larger groups, whose tiles are computed once per
+//              sibling and so bound by the compute warps: warps 0-7, warps w and w + 4 sharing
+//              lane quarter w % 4 with 4 heads each (KH 4), twice the warps to hide each one's
+//              latencies. Groups of up to 4: the same eight warps with 2 heads each (KH 2), so
+//              the live heads alone are computed (6.7 % faster on the 4-head long context).
 //   next warp  producer: block-table lookups and TMA loads of (page, head) tiles.
 //   next       score-MMA issuer (one elected lane; also the routing MMA) and TMEM owner.
 //   last       output-MMA issuer. Two issuing threads raise the SM's MMA issue rate (each
@@ -34,8 +37,9 @@
 // makes every role leave its loop, drains outstanding copies and MMAs and frees TMEM.
 //
 // This header holds the kernel template and its launch for one head dim; kl_decode_tc.cu
-// instantiates head dim 128 and the host-side plan, kl_decode_tc64.cu head dim 64, so that the
-// two compile in parallel.
+// instantiates head dim 128 and the host-side plan, kl_decode_tc64.cu head dim 64 and
+// kl_decode_tc_groups.cu the CTAs of groups of more than 8 heads, so that they compile in
+// parallel.
 #pragma once
 
 #include <cudaTypedefs.h>
@@ -59,7 +63,8 @@ constexpr uint32_t kTmemColsPq = 256;             // + one 16-column routing res
 constexpr uint64_t kTimeoutNs = kDefaultWaitNs;   // bound of the drains
 constexpr float kLazy = 2.f;                      // reference slack (base 2): weights <= 4
 // Warp roles for KH heads per compute warp: KH = 8, one compute warp per TMEM lane quarter;
-// KH = 2 (groups of up to 4 heads), two per quarter.
+// KH = 4 (the CTAs of groups of more than 8 heads) and KH = 2 (groups of up to 4 heads), two
+// per quarter, the second of them taking the upper head block.
 template <int KH>
 struct Roles {
     static constexpr int kComputeWarps = KH == 8 ? 4 : 8;
@@ -73,10 +78,10 @@ struct Roles {
 constexpr uint32_t kBarCompute = 1;       // plain sync
 constexpr uint32_t kBarComputeAnd = 2;    // sync + AND of a flag
 
-// Maximum over the 32 lanes of a warp of each of KH = 2 or 8 values by transposed halving:
+// Maximum over the 32 lanes of a warp of each of KH = 2, 4 or 8 values by transposed halving:
 // each exchange step sends half of the lane's values and keeps the other half, so lane l ends
-// with the maximum of value e(l) = bit 4 of l (KH 2), or 4 bit4 + 2 bit3 + bit2 (KH 8: 9
-// shuffles instead of 40).
+// with the maximum of value e(l) = max_head<KH>(l): bit 4 of l (KH 2), 2 bit4 + bit3 (KH 4),
+// 4 bit4 + 2 bit3 + bit2 (KH 8: 9 shuffles instead of 40).
 template <int KH>
 __device__ __forceinline__ float warp_max_k(const float (&x)[KH], int lane) {
     const bool b4 = lane & 16;
@@ -99,8 +104,21 @@ __device__ __forceinline__ float warp_max_k(const float (&x)[KH], int lane) {
         const float send = b2 ? a2[0] : a2[1];
         const float keep = b2 ? a2[1] : a2[0];
         a1 = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, 4));
+    } else if constexpr (KH == 4) {
+        const bool b3 = lane & 8;
+        float a2[2];
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+            const float send = b4 ? x[j] : x[j + 2];
+            const float keep = b4 ? x[j + 2] : x[j];
+            a2[j] = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, 16));
+        }
+        const float send = b3 ? a2[0] : a2[1];
+        const float keep = b3 ? a2[1] : a2[0];
+        a1 = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, 8));
+        a1 = fmaxf(a1, __shfl_xor_sync(0xffffffffu, a1, 4));
     } else {
-        static_assert(KH == 2, "two or eight heads per compute warp");
+        static_assert(KH == 2, "two, four or eight heads per compute warp");
         const float send = b4 ? x[0] : x[1];
         const float keep = b4 ? x[1] : x[0];
         a1 = fmaxf(keep, __shfl_xor_sync(0xffffffffu, send, 16));
@@ -112,8 +130,40 @@ __device__ __forceinline__ float warp_max_k(const float (&x)[KH], int lane) {
     return a1;
 }
 
+// The head (of the warp's KH) whose maximum lane l holds after warp_max_k, and whether l is
+// the first lane that holds it (the one that publishes it).
+template <int KH>
+__device__ __forceinline__ int max_head(int lane) {
+    if constexpr (KH == 8) return ((lane >> 4) & 1) * 4 + ((lane >> 3) & 1) * 2 + ((lane >> 2) & 1);
+    else if constexpr (KH == 4) return ((lane >> 4) & 1) * 2 + ((lane >> 3) & 1);
+    else return (lane >> 4) & 1;
+}
+template <int KH>
+__device__ __forceinline__ bool max_writer(int lane) {
+    return (lane & (32 / KH - 1)) == 0;
+}
+
+// The hi and lo columns of the warp's KH heads h0 .. h0 + KH - 1 in a 16-column TMEM row
+// [hi of heads 0-7 | lo of heads 0-7] at column address `row` (lane base included): one load
+// of the whole row for KH 8, two runs of KH columns otherwise.
+template <int KH>
+__device__ __forceinline__ void tmem_ld_heads(uint32_t row, int h0, float (&hi)[KH], float (&lo)[KH]) {
+    if constexpr (KH == 8) {
+        float v[16];
+        ptx::tmem_ld16(row, v);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            hi[e] = v[e];
+            lo[e] = v[8 + e];
+        }
+    } else {
+        ptx::tmem_ld_two<KH>(row + h0, row + kNG + h0, hi, lo);
+    }
+}
+
 // Column base + h0 + e of a 16-column TMEM row [hi of heads 0-7 | lo of heads 0-7]: the upper
-// head block of a KH = 2 warp is picked with a select, so register arrays keep constant indices.
+// head block of a KH = 2 or 4 warp is picked with a select, so register arrays keep constant
+// indices.
 template <int KH>
 __device__ __forceinline__ float head_col(const float (&v)[16], int base, bool hh, int e) {
     if constexpr (KH == 8) return v[base + e];
@@ -185,6 +235,16 @@ template <int N>
 struct Vec {
     float v[N];
 };
+
+// The split-bf16 form of two values a and b: hi = their bf16 roundings, lo = the bf16 roundings
+// of the remainders, each pair packed as a | b << 16 (a + b keeps about 16 significant bits).
+__device__ __forceinline__ void split_bf16x2(float a, float b, uint32_t &hi, uint32_t &lo) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+    hi = *reinterpret_cast<const uint32_t *>(&h);
+    const float ha = __uint_as_float(hi << 16), hb = __uint_as_float(hi & 0xffff0000u);
+    const __nv_bfloat162 l = __floats2bfloat162_rn(a - ha, b - hb);
+    lo = *reinterpret_cast<const uint32_t *>(&l);
+}
 
 __device__ __forceinline__ uint32_t pack_bf16(float lo_half, float hi_half) {
     const uint32_t a = __bfloat16_as_ushort(__float2bfloat16_rn(lo_half));
@@ -793,7 +853,7 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
         // select, never with a warp-dependent index.
         const int qd = warp & 3;
         const int t = qd * 32 + lane;
-        const bool hh = KH == 2 && warp >= 4;
+        const bool hh = KH != 8 && warp >= 4;
         const int h0 = hh ? KH : 0;
         const uint32_t lane_base = (uint32_t)(qd * 32) << 16;
         float *qf = reinterpret_cast<float *>(sm.p[0]);     // [k][8] raw query (prologue only)
@@ -896,12 +956,11 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
         // vote of the compute warps instead of an exchange of their maxima. mx holds the
         // thread's largest score of the current state, so that a state written out carries
         // its true largest score.
-        float m[KH], thr[KH], mx[KH], lsum[KH], o[KH];
+        float m[KH], mx[KH], lsum[KH], o[KH];
         Vec<KH> alpha_prev;
 #pragma unroll
         for (int e = 0; e < KH; ++e) {
             m[e] = -INFINITY;
-            thr[e] = -INFINITY;
             mx[e] = -INFINITY;
             lsum[e] = 0.f;
             o[e] = 0.f;
@@ -914,9 +973,7 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
 #pragma unroll
             for (int e = 0; e < KH; ++e) x[e] = mx[e];
             const float wm = warp_max_k<KH>(x, lane);
-            if (KH == 8 && (lane & 3) == 0)
-                sm.mred[qd][((lane >> 4) & 1) * 4 + ((lane >> 3) & 1) * 2 + ((lane >> 2) & 1)] = wm;
-            if (KH == 2 && (lane & 15) == 0) sm.mred[qd][h0 + ((lane >> 4) & 1)] = wm;
+            if (max_writer<KH>(lane)) sm.mred[qd][h0 + max_head<KH>(lane)] = wm;
         };
 
         // O accumulation of tile j: o = o * alpha_j + O_j (thread = output dim t).
@@ -925,14 +982,14 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
             if (!ptx::bar_and(kBarComputeAnd, kComputeThreads, wait(&sm.o_full[ob], (j >> 1) & 1)))
                 return false;
             ptx::tc_fence_after();
-            float ov[16];
-            ptx::tmem_ld16(tmem + 2 * kN + ob * kN + lane_base, ov);
+            float ohi[KH], olo[KH];
+            tmem_ld_heads<KH>(tmem + 2 * kN + ob * kN + lane_base, h0, ohi, olo);
             ptx::tc_fence_before();
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&sm.o_empty[ob]);
 #pragma unroll
             for (int e = 0; e < KH; ++e)
-                o[e] = fmaf(o[e], alpha.v[e], head_col<KH>(ov, 0, hh, e) + head_col<KH>(ov, kNG, hh, e));
+                o[e] = fmaf(o[e], alpha.v[e], ohi[e] + olo[e]);
             return true;
         };
 
@@ -997,26 +1054,30 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
                     o[e] = 0.f;
                     lsum[e] = 0.f;
                     m[e] = -INFINITY;
-                    thr[e] = -INFINITY;
                     mx[e] = -INFINITY;
                 }
             }
             ptx::tc_fence_after();
-            float sv[16];
-            ptx::tmem_ld16(tmem + sb * kN + lane_base, sv);
+            float shi[KH], slo[KH];
+            tmem_ld_heads<KH>(tmem + sb * kN + lane_base, h0, shi, slo);
             ptx::tc_fence_before();
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&sm.s_empty[sb]);
 
+            // A padded head (h >= G) has a zero query row: its scores are 0, it follows the
+            // same steps as a live head with finite values and is never written out.
             const int nvalid = min(kTile, t_end - (t_begin + i * kTile));
-            const bool valid = t < nvalid;
             float s[KH];
             bool grow = false;
 #pragma unroll
+            for (int e = 0; e < KH; ++e) s[e] = shi[e] + slo[e];
+            if (nvalid < kTile && t >= nvalid) {
+#pragma unroll
+                for (int e = 0; e < KH; ++e) s[e] = -INFINITY;      // tokens past the end
+            }
+#pragma unroll
             for (int e = 0; e < KH; ++e) {
-                s[e] = (valid && h0 + e < G) ? head_col<KH>(sv, 0, hh, e) + head_col<KH>(sv, kNG, hh, e)
-                                             : -INFINITY;
-                grow = grow || s[e] > thr[e];
+                grow = grow || s[e] - m[e] > kLazy;
                 mx[e] = fmaxf(mx[e], s[e]);
             }
             Vec<KH> alpha;
@@ -1031,9 +1092,7 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
 #pragma unroll
                 for (int e = 0; e < KH; ++e) x[e] = s[e];
                 const float wm = warp_max_k<KH>(x, lane);
-                if (KH == 8 && (lane & 3) == 0)
-                    sm.red[sb][qd][((lane >> 4) & 1) * 4 + ((lane >> 3) & 1) * 2 + ((lane >> 2) & 1)] = wm;
-                if (KH == 2 && (lane & 15) == 0) sm.red[sb][qd][h0 + ((lane >> 4) & 1)] = wm;
+                if (max_writer<KH>(lane)) sm.red[sb][qd][h0 + max_head<KH>(lane)] = wm;
                 ptx::bar_sync(kBarCompute, kComputeThreads);
 #pragma unroll
                 for (int e = 0; e < KH; ++e) {
@@ -1041,36 +1100,33 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
                     float tmax = sm.red[sb][0][h];
 #pragma unroll
                     for (int q = 1; q < 4; ++q) tmax = fmaxf(tmax, sm.red[sb][q][h]);
-                    const bool live = h < G;
                     const float mn = fmaxf(m[e], tmax);
-                    alpha.v[e] = live ? exp2f(m[e] - mn) : 0.f;
+                    alpha.v[e] = ptx::ex2(m[e] - mn);             // 0 for the first tile
                     lsum[e] *= alpha.v[e];
-                    m[e] = live ? mn : m[e];
-                    thr[e] = live ? mn + kLazy : thr[e];
+                    m[e] = mn;
                 }
             }
             float p[KH];
 #pragma unroll
             for (int e = 0; e < KH; ++e) {
-                p[e] = h0 + e < G ? exp2f(s[e] - m[e]) : 0.f;
+                p[e] = ptx::ex2(s[e] - m[e]);       // 0 past the end (s = -inf)
                 lsum[e] += p[e];
             }
             // P^T row of token t, this warp's heads: hi and lo halves.
             {
-                float r[KH];
+                uint32_t ph[KH / 2], pl[KH / 2];
 #pragma unroll
-                for (int e = 0; e < KH; ++e) r[e] = p[e] - __bfloat162float(__float2bfloat16_rn(p[e]));
+                for (int e = 0; e < KH / 2; ++e) split_bf16x2(p[2 * e], p[2 * e + 1], ph[e], pl[e]);
                 uint8_t *row = sm.p[sb] + (t >> 3) * 256 + (t & 7) * 16 + 2 * h0;
                 if constexpr (KH == 8) {
-                    *reinterpret_cast<uint4 *>(row) =
-                        make_uint4(pack_bf16(p[0], p[1]), pack_bf16(p[2], p[3]),
-                                   pack_bf16(p[4], p[5]), pack_bf16(p[6], p[7]));
-                    *reinterpret_cast<uint4 *>(row + 128) =
-                        make_uint4(pack_bf16(r[0], r[1]), pack_bf16(r[2], r[3]),
-                                   pack_bf16(r[4], r[5]), pack_bf16(r[6], r[7]));
+                    *reinterpret_cast<uint4 *>(row) = make_uint4(ph[0], ph[1], ph[2], ph[3]);
+                    *reinterpret_cast<uint4 *>(row + 128) = make_uint4(pl[0], pl[1], pl[2], pl[3]);
+                } else if constexpr (KH == 4) {
+                    *reinterpret_cast<uint2 *>(row) = make_uint2(ph[0], ph[1]);
+                    *reinterpret_cast<uint2 *>(row + 128) = make_uint2(pl[0], pl[1]);
                 } else {
-                    *reinterpret_cast<uint32_t *>(row) = pack_bf16(p[0], p[1]);
-                    *reinterpret_cast<uint32_t *>(row + 128) = pack_bf16(r[0], r[1]);
+                    *reinterpret_cast<uint32_t *>(row) = ph[0];
+                    *reinterpret_cast<uint32_t *>(row + 128) = pl[0];
                 }
             }
             // Rows past the end inside the last 16-token MMA step must be finite: zero them
@@ -1263,6 +1319,11 @@ cudaError_t launch_dim(const DecodeArgs &la, bool per_split, const CUtensorMap &
 // The head-dim-64 launches (kl_decode_tc64.cu): K+V comparison or keyless, KH heads per compute
 // warp (2 or 8), exact short waits or not.
 cudaError_t launch_tc_head64(const DecodeArgs &la, bool per_split, bool standard, int KH, bool exact,
+                             const CUtensorMap &vmap, const CUtensorMap &kmap,
+                             const CUtensorMap &wmap, const CUtensorMap &qmap);
+// The head-dim-128 launches of groups of more than 8 heads (kl_decode_tc_groups.cu): K+V
+// comparison or keyless, 4 heads per compute warp, exact short waits or not.
+cudaError_t launch_tc_groups(const DecodeArgs &la, bool per_split, bool standard, bool exact,
                              const CUtensorMap &vmap, const CUtensorMap &kmap,
                              const CUtensorMap &wmap, const CUtensorMap &qmap);
 

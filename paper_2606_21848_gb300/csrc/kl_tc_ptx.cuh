@@ -263,6 +263,37 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&r)[16]) {
     for (int i = 0; i < 16; ++i) r[i] = __uint_as_float(u[i]);
 }
 
+// Two runs of N (2 or 4) consecutive 32-bit columns of the thread's TMEM lane, at column
+// addresses a and b, both loaded before the one wait.
+template <int N>
+__device__ __forceinline__ void tmem_ld_two(uint32_t a, uint32_t b, float (&x)[N], float (&y)[N]) {
+    uint32_t u[N], v[N];
+    if constexpr (N == 4) {
+        asm volatile(
+            "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0, %1, %2, %3}, [%8];\n\t"
+            "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%4, %5, %6, %7}, [%9];\n\t"
+            "tcgen05.wait::ld.sync.aligned;"
+            : "=r"(u[0]), "=r"(u[1]), "=r"(u[2]), "=r"(u[3]), "=r"(v[0]), "=r"(v[1]), "=r"(v[2]),
+              "=r"(v[3])
+            : "r"(a), "r"(b)
+            : "memory");
+    } else {
+        static_assert(N == 2, "runs of 2 or 4 columns");
+        asm volatile(
+            "tcgen05.ld.sync.aligned.32x32b.x2.b32 {%0, %1}, [%4];\n\t"
+            "tcgen05.ld.sync.aligned.32x32b.x2.b32 {%2, %3}, [%5];\n\t"
+            "tcgen05.wait::ld.sync.aligned;"
+            : "=r"(u[0]), "=r"(u[1]), "=r"(v[0]), "=r"(v[1])
+            : "r"(a), "r"(b)
+            : "memory");
+    }
+#pragma unroll
+    for (int i = 0; i < N; ++i) {
+        x[i] = __uint_as_float(u[i]);
+        y[i] = __uint_as_float(v[i]);
+    }
+}
+
 // One 32-bit column of the thread's TMEM lane (load and wait in one statement).
 __device__ __forceinline__ float tmem_ld1(uint32_t taddr) {
     uint32_t u;

@@ -1,10 +1,11 @@
 """GPU parity of groups of more than 8 query heads per value head (the multi-query and
 grouped-query layouts of Section 3: every head of a group reads the same cached value rows).
 
-The tensor-core decodes serve such a group with sibling CTAs of up to 8 heads each; every
-floating-point output is checked against the fp64 oracle at |gpu - oracle| <= 2e-3 + 1e-2
-|oracle|, the appended rows bit-exact. The CUDA-core kernel serves groups of up to 8 heads and
-must reject larger ones without launching.
+The tensor-core decodes serve such a group with sibling CTAs of up to 8 heads each (the bf16
+decode puts 4 heads on each of their eight compute warps); every floating-point output is
+checked against the fp64 oracle at |gpu - oracle| <= 2e-3 + 1e-2 |oracle|, the appended rows
+bit-exact. The CUDA-core kernel serves groups of up to 8 heads and must reject larger ones
+without launching.
 """
 from __future__ import annotations
 
@@ -35,6 +36,8 @@ SHAPES = [
     dict(B=2, Hq=128, Hkv=8, D=128, P=32, lens=(1000, 257)),      # GQA 16 (128 / 8)
     dict(B=3, Hq=24, Hkv=2, D=128, P=16, lens=(0, 700, 129)),     # group 12: blocks of 8 and 4
     dict(B=1, Hq=64, Hkv=2, D=128, P=64, lens=(2222,)),           # group 32, P 64
+    dict(B=2, Hq=48, Hkv=2, D=128, P=32, lens=(1500, 64)),        # group 24: three blocks of 8
+    dict(B=3, Hq=20, Hkv=1, D=128, P=16, lens=(900, 0, 3000)),    # group 20: 8, 8 and 4, MQA
 ]
 
 
@@ -57,6 +60,24 @@ def test_large_group_many_splits_merge_in_kernel():
         out, err = decode(to_dev(x), shape_of(x), num_splits=s)
         assert err == 0
         assert_parity(out.cpu().numpy(), want, f"S={s}")
+
+
+def test_large_group_composed_query():
+    """No W^R: the query already is the composed x W^Q W^R (three sibling CTAs)."""
+    x = tiny(B=2, Hq=24, Hkv=1, D=128, P=16, lens=(700, 1900), seed=52)
+    g = to_dev(x)
+    sh = shape_of(x)
+    out = torch.full((2, 24, 128), float("nan"), dtype=torch.float32, device=_gpu.dev())
+    err = torch.zeros(1, dtype=torch.int32, device=_gpu.dev())
+    ws = torch.zeros(max(256, kl.kl_decode_workspace_size(sh, 3)), dtype=torch.uint8,
+                     device=_gpu.dev())
+    kl.kl_decode_attention_ex(sh, g["q"], None, g["v_cache"], g["block_table"], g["seq_lens"],
+                              kl.decode_options(3, kl.KL_KERNEL_TENSOR), out, kl.KL_FP32, ws, err)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    y = dict(x)
+    y["w_r"] = torch.eye(128, dtype=torch.float32).expand(1, 128, 128).contiguous().to(torch.bfloat16)
+    assert_parity(out.cpu().numpy(), oracle_decode(y, _gpu.default_scale(x)), "composed query")
 
 
 def test_large_group_per_query_head_routing():
