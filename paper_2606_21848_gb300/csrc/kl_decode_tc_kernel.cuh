@@ -61,7 +61,7 @@ constexpr uint32_t kHalfBytes = kTileBytes / 2;   // one 64-dim half: 128 rows x
 constexpr uint32_t kTmemCols = 64;                // S: 2 x 16 columns, O: 2 x 16 columns
 constexpr uint32_t kTmemColsPq = 256;             // + one 16-column routing result per head
 constexpr uint64_t kTimeoutNs = kDefaultWaitNs;   // bound of the drains
-constexpr float kLazy = 2.f;                      // reference slack (base 2): weights <= 4
+constexpr float kLazyW = 4.f;                     // reference slack: weights 2^(s - m) <= 4
 // Warp roles for KH heads per compute warp: KH = 8, one compute warp per TMEM lane quarter;
 // KH = 4 (the CTAs of groups of more than 8 heads) and KH = 2 (groups of up to 4 heads), two
 // per quarter, the second of them taking the upper head block.
@@ -951,11 +951,12 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
         }
 
         // Lazy reference: a tile's weights are 2^(s - m) with the head's current reference m,
-        // which moves to the running maximum (rescaling the running sums) only when a score
-        // passes thr = m + kLazy, so the weights stay at most 2^kLazy and most tiles need one
-        // vote of the compute warps instead of an exchange of their maxima. mx holds the
-        // thread's largest score of the current state, so that a state written out carries
-        // its true largest score.
+        // which moves to the running maximum (rescaling the running sums) only when a weight
+        // passes kLazyW (a score passes m + 2), so the weights stay at most 4 and most tiles need
+        // one vote of the compute warps instead of an exchange of their maxima. When the state
+        // leaves the kernel (exact_m), mx holds the thread's largest score of it, so that the
+        // state carries its true largest score.
+        const bool exact_m = !a.direct_out && !a.merge_inside;
         float m[KH], mx[KH], lsum[KH], o[KH];
         Vec<KH> alpha_prev;
 #pragma unroll
@@ -1068,18 +1069,24 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
             // same steps as a live head with finite values and is never written out.
             const int nvalid = min(kTile, t_end - (t_begin + i * kTile));
             float s[KH];
-            bool grow = false;
 #pragma unroll
             for (int e = 0; e < KH; ++e) s[e] = shi[e] + slo[e];
             if (nvalid < kTile && t >= nvalid) {
 #pragma unroll
                 for (int e = 0; e < KH; ++e) s[e] = -INFINITY;      // tokens past the end
             }
+            if (exact_m) {
 #pragma unroll
-            for (int e = 0; e < KH; ++e) {
-                grow = grow || s[e] - m[e] > kLazy;
-                mx[e] = fmaxf(mx[e], s[e]);
+                for (int e = 0; e < KH; ++e) mx[e] = fmaxf(mx[e], s[e]);
             }
+            // the weights against the current references (0 past the end: s = -inf)
+            float p[KH];
+#pragma unroll
+            for (int e = 0; e < KH; ++e) p[e] = ptx::ex2(s[e] - m[e]);
+            float pmax = p[0];
+#pragma unroll
+            for (int e = 1; e < KH; ++e) pmax = fmaxf(pmax, p[e]);
+            const bool grow = pmax > kLazyW;
             Vec<KH> alpha;
 #pragma unroll
             for (int e = 0; e < KH; ++e) alpha.v[e] = 1.f;
@@ -1104,14 +1111,11 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
                     alpha.v[e] = ptx::ex2(m[e] - mn);             // 0 for the first tile
                     lsum[e] *= alpha.v[e];
                     m[e] = mn;
+                    p[e] = ptx::ex2(s[e] - mn);
                 }
             }
-            float p[KH];
 #pragma unroll
-            for (int e = 0; e < KH; ++e) {
-                p[e] = ptx::ex2(s[e] - m[e]);       // 0 past the end (s = -inf)
-                lsum[e] += p[e];
-            }
+            for (int e = 0; e < KH; ++e) lsum[e] += p[e];
             // P^T row of token t, this warp's heads: hi and lo halves.
             {
                 uint32_t ph[KH / 2], pl[KH / 2];
@@ -1169,7 +1173,6 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
             // States that leave the kernel (for the caller or the combine kernel) carry their
             // true largest score; the merge inside the kernel takes any reference (l = sum
             // 2^(s - m) for the m it is given), so its states keep the lazy one.
-            const bool exact_m = !a.direct_out && !a.merge_inside;
             if (exact_m) head_max();
             ptx::bar_sync(kBarCompute, kComputeThreads);
             {
