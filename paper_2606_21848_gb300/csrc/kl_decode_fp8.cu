@@ -73,7 +73,7 @@ constexpr uint32_t kTmemCols = 128;
 constexpr uint32_t kColS = 0;                        // S[b]: columns 32 b .. 32 b + 31
 constexpr uint32_t kColO = 64;                       // O: columns 64 .. 95, summed over tiles
 constexpr uint32_t kColR = 96;                       // routing result: 96 .. 111
-constexpr float kLazy = 2.f;                         // reference slack (base 2): weights <= 4
+constexpr float kLazyW = 4.f;                        // reference slack: weights 2^(s - m) <= 4
 constexpr uint64_t kTimeoutNs = kDefaultWaitNs;   // bound of the drains
 constexpr uint32_t kSleepHintNs = 20000u;         // suspend hint of a wait that did not finish at once
 constexpr uint32_t kBarCompute = 1;
@@ -618,13 +618,12 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
 
         // m: the reference maximum of each head (0 for padded heads, whose scores are -inf);
-        // thr = m + kLazy, the score that moves it (+inf for padded heads)
-        float m[KHH], thr[KHH], lsum[KHH];
+        // a weight 2^(s - m) past kLazyW moves it
+        float m[KHH], lsum[KHH];
 #pragma unroll
         for (int k = 0; k < KHH; ++k) {
             const bool live = kAllLive || KHH * hh + k < G;
             m[k] = live ? -INFINITY : 0.f;
-            thr[k] = live ? -INFINITY : INFINITY;
             lsum[k] = 0.f;
         }
         // Lazy weight scale: every row scale so far is below lim = 2^es; weights are taken
@@ -672,18 +671,29 @@ __global__ void __launch_bounds__(kThreads, 2)
 
             const int nvalid = min(kTile, t_end - (t_begin + i * kTile));
             const bool valid = t < nvalid;
-            const float st = valid ? sm.scl[s][t] : 0.f;     // the row scale of token t
+            float st = sm.scl[s][t];                      // the row scale of token t
+            if (nvalid < kTile && !valid) st = 0.f;       // (stale bytes past the end)
             float s_k[KHH];
-            bool grow = false;
 #pragma unroll
             for (int k = 0; k < KHH; ++k) {
                 // sum of the term columns, 16^-j D_j, from the last term
                 const float d = fmaf(fmaf(fmaf(sv[3 * KHH + k], 1.f / 16.f, sv[2 * KHH + k]), 1.f / 16.f,
                                           sv[KHH + k]),
                                      1.f / 16.f, sv[k]);
-                s_k[k] = (valid && (kAllLive || KHH * hh + k < G)) ? d * (invq[k] * st) : -INFINITY;
-                grow = grow || s_k[k] > thr[k];
+                s_k[k] = (kAllLive || KHH * hh + k < G) ? d * (invq[k] * st) : -INFINITY;
             }
+            if (nvalid < kTile && !valid) {
+#pragma unroll
+                for (int k = 0; k < KHH; ++k) s_k[k] = -INFINITY;
+            }
+            // the weights against the current references; a weight past kLazyW moves them
+            float p_k[KHH];
+#pragma unroll
+            for (int k = 0; k < KHH; ++k) p_k[k] = ptx::ex2(s_k[k] - m[k]);   // 0 for padded heads
+            float pmax = p_k[0];
+#pragma unroll
+            for (int k = 1; k < KHH; ++k) pmax = fmaxf(pmax, p_k[k]);
+            bool grow = pmax > kLazyW;
             // row scales are non-negative: their bits order as the values do
             const float smx = __uint_as_float(__reduce_max_sync(0xffffffffu, __float_as_uint(st)));
             grow = grow || smx >= lim;
@@ -728,7 +738,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                     const float mn = fmaxf(m[k], tmax[k]);
                     alpha[k] = live ? ptx::ex2(m[k] - mn) : 1.f;
                     m[k] = live ? mn : m[k];
-                    thr[k] = live ? mn + kLazy : thr[k];
+                    p_k[k] = ptx::ex2(s_k[k] - m[k]);
                     lsum[k] *= alpha[k];
                     rescale = rescale || alpha[k] != 1.f;
                 }
@@ -759,7 +769,7 @@ __global__ void __launch_bounds__(kThreads, 2)
             float x[KHH];
 #pragma unroll
             for (int k = 0; k < KHH; ++k) {
-                const float p = ptx::ex2(s_k[k] - m[k]);       // 0 for padded heads
+                const float p = p_k[k];
                 lsum[k] += p;
                 x[k] = p * sts;
             }
