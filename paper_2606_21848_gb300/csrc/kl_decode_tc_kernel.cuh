@@ -549,10 +549,52 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
             ptx::prefetch_tensormap(&qmap);
         }
     }
+    // Ring position r < route_tiles: W^R as the MN-major A operand [j half][128 k rows][128 B];
+    // position 0 also brings the group's query rows as the K-major B operand (rows 0..G-1 of
+    // the q_r buffer). Issued by the producer warp.
+    auto issue_route = [&](int r) {
+        const int s = r % NS;
+        if (lane == 0) {
+            // W^R: two 64-column halves of 128 rows; or (head dim 64) one box of 64 x 64 at
+            // the top left, and with two value heads the second head's box at the bottom
+            // right (rows and columns 64-127; per query head: the box of the head's half).
+            // The query rows go to both 64-dim halves of the operand when two heads share
+            // the tile (each head keeps its own half of the result).
+            const int wrow = (route_pq ? qh0 + r : g) * D;
+            const bool two_q = D == kD || pair;
+            const int nbox = D == kD ? 2 : (pair && !route_pq) ? 2 : 1;
+            const uint32_t w_off = pair && route_pq && r >= geo.G ? kHalfBytes + 64u * 128u : 0u;
+            ptx::mbar_arrive_expect_tx(&sm.full[s], (D == kD ? kTileBytes : (uint32_t)nbox * 64u * 128u) +
+                                                        (r == 0 ? (two_q ? 2u : 1u) * (uint32_t)geo.qbox * 128u : 0u));
+            if (D == kD) {
+                ptx::tma_load_2d(sm.tiles[s][0], &wmap, &sm.full[s], 0, wrow);
+                ptx::tma_load_2d(sm.tiles[s][0] + kHalfBytes, &wmap, &sm.full[s], 64, wrow);
+            } else {
+                ptx::tma_load_2d(sm.tiles[s][0] + w_off, &wmap, &sm.full[s], 0, wrow);
+                if (nbox == 2)
+                    ptx::tma_load_2d(sm.tiles[s][0] + kHalfBytes + 64u * 128u, &wmap, &sm.full[s], 0,
+                                     wrow + D);
+            }
+            if (r == 0) {
+                ptx::tma_load_2d(sm.qr, &qmap, &sm.full[s], 0, b * geo.Hq + qh0);
+                if (two_q)
+                    ptx::tma_load_2d(sm.qr + kN * 128, &qmap, &sm.full[s], D == kD ? 64 : 0,
+                                     b * geo.Hq + qh0);
+            }
+        }
+        __syncwarp();
+    };
+
     ptx::tc_fence_before();
     __syncthreads();
     ptx::tc_fence_after();
     if (a.pdl) grid_dep_launch();
+    // The routing loads that fit the ring depend on nothing the CTA still reads (the length,
+    // the block table), so they go out at once: the routed query is then ready about when
+    // the first cache tile lands.
+    const int early_route = route_tiles < NS ? route_tiles : NS;
+    if (warp == kProducerWarp)
+        for (int r = 0; r < early_route; ++r) issue_route(r);
 
     int L = L_raw;
     if (L < 0 || L > geo.max_pages * geo.P) {
@@ -610,6 +652,14 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
             }
         }
         if (warp == kMmaWarp) ptx::tmem_dealloc(sm.tmem_base, tmem_cols);
+        // the routing loads issued at the start land before the shared memory goes away
+        if (warp == kProducerWarp) {
+            for (int r = 0; r < early_route; ++r) {
+                const uint64_t t0 = ptx::globaltimer();
+                while (!ptx::mbar_try_wait(&sm.full[r], 0) && ptx::globaltimer() - t0 < kTimeoutNs) {
+                }
+            }
+        }
         return;
     }
 
@@ -647,41 +697,13 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
                 raise_flag(a.err, KL_FLAG_BAD_PAGE);
             }
         }
-        // Ring positions 0 .. route_tiles - 1: the W^R matrices as the MN-major A operand
-        // [j half][128 k rows][128 B]; position 0 also brings the group's query rows as the
-        // K-major B operand (rows 0..G-1 of the q_r buffer).
+        // Ring positions 0 .. route_tiles - 1: the W^R matrices (the first early_route of them
+        // went out at the start).
         for (int r = 0; r < route_tiles; ++r) {
-            const int s = r % NS;
-            if (r >= NS && !wait(&sm.empty[s], ((r / NS) & 1) ^ 1)) break;
-            if (lane == 0) {
-                // W^R: two 64-column halves of 128 rows; or (head dim 64) one box of 64 x 64 at
-                // the top left, and with two value heads the second head's box at the bottom
-                // right (rows and columns 64-127; per query head: the box of the head's half).
-                // The query rows go to both 64-dim halves of the operand when two heads share
-                // the tile (each head keeps its own half of the result).
-                const int wrow = (route_pq ? qh0 + r : g) * D;
-                const bool two_q = D == kD || pair;
-                const int nbox = D == kD ? 2 : (pair && !route_pq) ? 2 : 1;
-                const uint32_t w_off = pair && route_pq && r >= geo.G ? kHalfBytes + 64u * 128u : 0u;
-                ptx::mbar_arrive_expect_tx(&sm.full[s], (D == kD ? kTileBytes : (uint32_t)nbox * 64u * 128u) +
-                                                            (r == 0 ? (two_q ? 2u : 1u) * (uint32_t)geo.qbox * 128u : 0u));
-                if (D == kD) {
-                    ptx::tma_load_2d(sm.tiles[s][0], &wmap, &sm.full[s], 0, wrow);
-                    ptx::tma_load_2d(sm.tiles[s][0] + kHalfBytes, &wmap, &sm.full[s], 64, wrow);
-                } else {
-                    ptx::tma_load_2d(sm.tiles[s][0] + w_off, &wmap, &sm.full[s], 0, wrow);
-                    if (nbox == 2)
-                        ptx::tma_load_2d(sm.tiles[s][0] + kHalfBytes + 64u * 128u, &wmap, &sm.full[s], 0,
-                                         wrow + D);
-                }
-                if (r == 0) {
-                    ptx::tma_load_2d(sm.qr, &qmap, &sm.full[s], 0, b * geo.Hq + qh0);
-                    if (two_q)
-                        ptx::tma_load_2d(sm.qr + kN * 128, &qmap, &sm.full[s], D == kD ? 64 : 0,
-                                         b * geo.Hq + qh0);
-                }
+            if (r >= early_route) {
+                if (r >= NS && !wait(&sm.empty[r % NS], ((r / NS) & 1) ^ 1)) break;
+                issue_route(r);
             }
-            __syncwarp();
             issued = r + 1;
         }
         // Block-table entries of the split, 32 pages per warp load, one batch ahead (the
