@@ -106,6 +106,40 @@ def test_large_group_split_states():
     assert_parity(out.cpu().numpy(), oracle_decode(x, _gpu.default_scale(x)), "states merged")
 
 
+def test_large_group_split_states_several_per_cta():
+    """The most splits of one sequence (235 of 128 tokens): two sibling CTAs per split would
+    overflow a wave, so each CTA runs two consecutive splits and writes a state for each; every
+    state against the oracle's, and their merge against the whole decode."""
+    x = tiny(B=1, Hq=16, Hkv=1, D=128, P=16, lens=(30000,), seed=53)
+    g = to_dev(x)
+    sh = shape_of(x)
+    S = kl.kl_decode_num_splits(sh, 1000)
+    B, Hq, D = x["q"].shape
+    po = torch.full((B, Hq, S, D), float("nan"), dtype=torch.float32, device=_gpu.dev())
+    pml = torch.full((B, Hq, S, 2), float("nan"), dtype=torch.float32, device=_gpu.dev())
+    err = torch.zeros(1, dtype=torch.int32, device=_gpu.dev())
+    kl.kl_decode_attention_ex(sh, g["q"], g["w_r"], g["v_cache"], g["block_table"], g["seq_lens"],
+                              kl.decode_options(1000, kl.KL_KERNEL_TENSOR, po, pml), None,
+                              kl.KL_FP32, None, err)
+    out = torch.full((B, Hq, D), float("nan"), dtype=torch.float32, device=_gpu.dev())
+    kl.kl_combine(sh, po, pml, S, out, kl.KL_FP32)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    assert_parity(out.cpu().numpy(), oracle_decode(x, _gpu.default_scale(x)), "states merged")
+    lmax = x["block_table"].shape[1] * 16
+    chunk = -(-(-(-lmax // S)) // 128) * 128        # ceil(lmax / S), rounded up to 128
+    want_o, want_ml = oracle.decode_partial(bf16_bits(x["q"]), bf16_bits(x["w_r"]),
+                                            bf16_bits(x["v_cache"]), x["block_table"].numpy(),
+                                            x["seq_lens"].numpy(), scale=_gpu.default_scale(x),
+                                            chunk=chunk, num_splits=S)
+    got_o, got_ml = po.cpu().numpy().astype(np.float64), pml.cpu().numpy().astype(np.float64)
+    full = want_ml[..., 1] > 0
+    assert np.array_equal(got_ml[..., 1] > 0, full), "empty splits differ"
+    assert_parity(got_o[full], want_o[full], f"split states S={S}")
+    m_g, m_w = got_ml[..., 0][full], want_ml[..., 0][full]
+    assert np.all(np.abs(m_g - m_w) <= 1e-3 + 1e-4 * np.abs(m_w)), "largest scores differ"
+
+
 @pytest.mark.parametrize("splits", [1, 3, 0])
 def test_large_group_fused_step(splits):
     x = tiny(B=2, Hq=128, Hkv=8, D=128, P=16, lens=(700, 1290), seed=50)

@@ -50,7 +50,7 @@ def test_wait_limit_setting_round_trips():
 
 
 @pytest.mark.parametrize("splits", [1, 4, 40])
-@pytest.mark.parametrize("Hq", [32, 64])
+@pytest.mark.parametrize("Hq", [32, 64, 128])
 def test_bf16_decode_times_out_then_recovers(splits, Hq):
     x = tiny(B=2, Hq=Hq, Hkv=8, D=128, P=16, lens=(5000, 3000), seed=71)
     g = to_dev(x)
