@@ -120,12 +120,15 @@ kl_status kl_append_v(const kl_shape *shape, const void *v_new, const int32_t *b
 /*
  * Bytes of device workspace kl_decode_attention / kl_decode_step / kl_standard_decode need for
  * `num_splits` (0 = the automatic choice); 0 when no workspace is needed (one split). Returns
- * 0 on invalid shapes. The workspace holds the split states and, for the tensor-core kernel,
- * one merge counter per sequence, value head and block of up to 8 of its query heads: it must
- * be zero-filled (cudaMemsetAsync) before its first use. Every call leaves the counters at zero again, so the workspace can
- * be reused across calls and shapes -- except after a call that raised KL_FLAG_TIMEOUT,
- * which may leave counters behind: zero the workspace again then. Calls that share a
- * workspace must not overlap on the GPU.
+ * 0 on invalid shapes. The workspace holds, for the tensor-core kernel, one merge counter per
+ * sequence, value head and block of up to 8 of its query heads, then the split states. It must
+ * be zero-filled (cudaMemsetAsync) before its first use; every call leaves its counters at zero
+ * again. The counters occupy a fixed front region of 64 KiB for every shape with at most 16384
+ * of them (larger shapes extend it), where no split state is ever written, so the workspace
+ * serves any sequence of calls and shapes -- batch sizes and split counts that change from
+ * call to call included -- except after a call that raised KL_FLAG_TIMEOUT, which may leave
+ * counters behind, or a switch from a shape with more than 16384 counters: zero the workspace
+ * again then. Calls that share a workspace must not overlap on the GPU.
  */
 size_t kl_decode_workspace_size(const kl_shape *shape, int32_t num_splits);
 
@@ -263,7 +266,8 @@ typedef struct {
 } kl_latent_shape;
 
 /* Bytes of device workspace kl_latent_decode needs for `num_splits` (0 = automatic); 0 on an
- * invalid or unsupported shape. Same zero-fill contract as kl_decode_workspace_size. */
+ * invalid or unsupported shape. Same zero-fill contract as kl_decode_workspace_size (its merge
+ * counters sit in the same front region). */
 size_t kl_latent_workspace_size(const kl_latent_shape *shape, int32_t num_splits);
 
 /*

@@ -99,16 +99,22 @@ struct WorkspaceLayout {
     size_t part_o, part_ml, counters, total;
 };
 
-// [B][Hq][S][D] fp32 states, [B][Hq][S][2] fp32 {m, l}, [B][Hkv][nhb] u32 merge counters (one
-// per sequence and block of up to 8 query heads of a value head).
+// [B][Hkv][nhb] u32 merge counters (one per sequence and block of up to 8 query heads of a
+// value head) in a region of at least kCounterFloor counters at the front, then [B][Hq][S][D]
+// fp32 states and [B][Hq][S][2] fp32 {m, l}. Every shape with at most kCounterFloor counters
+// keeps them in the same region, which no split state ever covers, so the counters that a call
+// leaves at zero stay zero whatever shape uses the workspace next.
+constexpr size_t kCounterFloor = 16384;
 WorkspaceLayout layout(const Geometry &g) {
     WorkspaceLayout w{0, 0, 0, 0};
     if (g.S <= 1) return w;
     const size_t rows = (size_t)g.B * g.Hq * g.S;
-    w.part_o = 0;
-    w.part_ml = round_up(rows * g.D * sizeof(float), 256);
-    w.counters = w.part_ml + round_up(rows * 2 * sizeof(float), 256);
-    w.total = w.counters + round_up((size_t)g.B * g.Hkv * g.nhb * sizeof(unsigned int), 256);
+    const size_t counters = (size_t)g.B * g.Hkv * g.nhb;
+    w.counters = 0;
+    w.part_o = round_up((counters > kCounterFloor ? counters : kCounterFloor) * sizeof(unsigned int),
+                        256);
+    w.part_ml = w.part_o + round_up(rows * g.D * sizeof(float), 256);
+    w.total = w.part_ml + round_up(rows * 2 * sizeof(float), 256);
     return w;
 }
 
@@ -191,7 +197,7 @@ kl_status decode_common(bool standard, const kl_shape *shape, const void *q, con
 cudaError_t finish_decode(const DecodeArgs &a, bool states_requested) {
     if (a.direct_out || a.merge_inside || states_requested) return cudaSuccess;
     return launch_combine(a.geo.B, a.geo.Hq, a.geo.D, a.geo.S, a.part_o, a.part_ml, a.out,
-                          a.out_dtype, a.stream);
+                          a.out_dtype, a.stream, true);
 }
 
 }  // namespace kl
@@ -369,10 +375,14 @@ kl_status latent_plan(const kl_latent_shape *s, int32_t num_splits, LatentPlan *
     if (st != KL_OK) return st;
     if (g.G > 8) return KL_ERR_UNSUPPORTED;
     const size_t rows = (size_t)s->num_seqs * s->num_q_heads * s->latent_dim * sizeof(float);
-    p->q_lat = 0;
-    p->o_lat = round_up(rows, 256);
-    p->dec_ws = p->o_lat + round_up(rows, 256);
-    p->total = p->dec_ws + layout(g).total;
+    // the decode's part first, so that its merge counters sit in the same front region as
+    // those of every other decode sharing the workspace (reserved even when S = 1)
+    const size_t dec = layout(g).total;
+    const size_t floor_bytes = kCounterFloor * sizeof(unsigned int);
+    p->dec_ws = 0;
+    p->q_lat = round_up(dec > floor_bytes ? dec : floor_bytes, 256);
+    p->o_lat = p->q_lat + round_up(rows, 256);
+    p->total = p->o_lat + round_up(rows, 256);
     return KL_OK;
 }
 

@@ -342,6 +342,9 @@ __global__ void __launch_bounds__(kThreads, 2)
     ptx::tc_fence_before();
     __syncthreads();
     ptx::tc_fence_after();
+    // the combine of the split states, launched behind as a programmatic dependent, may start
+    // setting up once every CTA is here
+    grid_dep_launch();
 
     int L = L_raw;
     if (L < 0 || L > geo.max_pages * geo.P) {

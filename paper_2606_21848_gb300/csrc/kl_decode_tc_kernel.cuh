@@ -588,7 +588,9 @@ __global__ void __launch_bounds__(Roles<KH>::kThreads, 2)
     ptx::tc_fence_before();
     __syncthreads();
     ptx::tc_fence_after();
-    if (a.pdl) grid_dep_launch();
+    // a kernel launched behind this one as a programmatic dependent (the combine of the split
+    // states, the latent expansion) may start setting up once every CTA is here
+    grid_dep_launch();
     // The routing loads that fit the ring depend on nothing the CTA still reads (the length,
     // the block table), so they go out at once: the routed query is then ready about when
     // the first cache tile lands.

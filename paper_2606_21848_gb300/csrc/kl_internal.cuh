@@ -117,9 +117,11 @@ cudaError_t launch_append(const Geometry &g, const uint16_t *v_new, const int32_
                           cudaStream_t stream);
 cudaError_t launch_route(const Geometry &g, const uint16_t *q, const uint16_t *w_r, float *q_r,
                          cudaStream_t stream);
+// dependent: launched as a programmatic dependent of the decode just before it in the stream
+// (it starts once every decode CTA has set up and waits for the decode to complete)
 cudaError_t launch_combine(int B, int Hq, int D, int S, const float *part_o,
                            const float *part_ml, void *out, kl_dtype out_dtype,
-                           cudaStream_t stream);
+                           cudaStream_t stream, bool dependent = false);
 cudaError_t launch_decode_simt(const DecodeArgs &a, bool standard);
 // Merges the split states of a finished decode into `out` unless it wrote `out` directly or
 // the caller asked for the states.

@@ -66,6 +66,9 @@ __global__ void __launch_bounds__(kCombineWarps * 32)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const size_t bh = (size_t)b * Hq + h;
     const float2 *ml = part_ml + bh * S;
+    // behind a decode as its programmatic dependent: the decode's states are complete and
+    // visible past this point (an ordinary launch returns at once)
+    grid_dep_wait();
 
     float M = -INFINITY;
     for (int s = tid; s < S; s += blockDim.x) {
@@ -144,13 +147,23 @@ cudaError_t launch_route(const Geometry &g, const uint16_t *q, const uint16_t *w
 
 cudaError_t launch_combine(int B, int Hq, int D, int S, const float *part_o,
                            const float *part_ml, void *out, kl_dtype out_dtype,
-                           cudaStream_t stream) {
+                           cudaStream_t stream, bool dependent) {
     if (B == 0) return cudaSuccess;
     if (S > kCombineMaxSplits) return cudaErrorInvalidValue;
-    combine_kernel<<<dim3(Hq, B), kCombineWarps * 32, 0, stream>>>(Hq, D, S, part_o,
-                                                 reinterpret_cast<const float2 *>(part_ml), out,
-                                                 out_dtype == KL_FP32);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(Hq, B);
+    cfg.blockDim = dim3(kCombineWarps * 32);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    if (dependent) {
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+    }
+    return cudaLaunchKernelEx(&cfg, combine_kernel, Hq, D, S, part_o,
+                              reinterpret_cast<const float2 *>(part_ml), out,
+                              (int)(out_dtype == KL_FP32));
 }
 
 }  // namespace kl
