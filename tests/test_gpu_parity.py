@@ -163,6 +163,19 @@ def test_split_counts_agree(kname):
         assert_parity(out.cpu().numpy(), want, f"{kname} S={s}")
 
 
+@pytest.mark.parametrize("splits", [9, 17, 100, 1000])
+def test_many_split_states_merged_in_the_kernel(splits):
+    """One long sequence over one value head, so that every split is a CTA of its own: 9, 17,
+    100 and the most (157 splits of 128 tokens) states, merged by the last CTA through the ring
+    in one or several rounds of bulk copies."""
+    x = tiny(B=1, Hq=4, Hkv=1, D=128, P=16, lens=(20000,), seed=24)
+    want = oracle_decode(x, _gpu.default_scale(x))
+    for _ in range(2):              # the counters are back at zero for the second call
+        out, err = decode(to_dev(x), shape_of(x), kernel=kl.KL_KERNEL_TENSOR, num_splits=splits)
+        assert err == 0
+        assert_parity(out.cpu().numpy(), want, f"S={splits}")
+
+
 @pytest.mark.parametrize("kname", ["simt", "tensor"])
 def test_workspace_reused_across_calls_and_shapes(kname):
     """One workspace, zero-filled once, serves repeated calls and different shapes -- batch
