@@ -926,13 +926,12 @@ cudaError_t launch_shape(const DecodeArgs &a, const CUtensorMap &cmap, const CUt
                          const CUtensorMap &qmap, const float *v_scales) {
     const Geometry &g = a.geo;
     const size_t smem = sizeof(Smem8) + 1024;
-    static bool configured = false;
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(decode_fp8_kernel<KHH, kAllLive, kExact>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        configured = true;
-    }
+    static PerDeviceOnce once;
+    const cudaError_t e = once.run([&] {
+        return cudaFuncSetAttribute(decode_fp8_kernel<KHH, kAllLive, kExact>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    });
+    if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(g.S * g.nhb, g.Hkv, g.B);
     cfg.blockDim = dim3(kThreads);

@@ -1310,13 +1310,12 @@ cudaError_t launch_kernel(const DecodeArgs &la, const CUtensorMap &vmap, const C
                           const CUtensorMap &wmap, const CUtensorMap &qmap) {
     const Geometry &g = la.geo;
     const size_t smem = sizeof(Smem<kStandard>) + 1024;
-    static bool configured = false;
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<kStandard, kPerSplit, KH, kExact, kD64>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        configured = true;
-    }
+    static PerDeviceOnce once;
+    const cudaError_t e = once.run([&] {
+        return cudaFuncSetAttribute(decode_tc_kernel<kStandard, kPerSplit, KH, kExact, kD64>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    });
+    if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((g.S + g.spc - 1) / g.spc * g.nhb, g.Hkv / g.vpc, g.B);
     cfg.blockDim = dim3(Roles<KH>::kThreads);

@@ -5,6 +5,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "keyless.h"
 
 namespace kl {
@@ -165,5 +167,22 @@ cudaError_t launch_latent_expand(int B, int Hq, int D, int r, const float *o_lat
 
 // Number of SMs of the current device (cached per device).
 int device_sm_count();
+
+// A launch site's one-time set-up of its kernel (a function attribute, which belongs to the
+// function on the current device): run once per device (ordinals below 64; others every time).
+struct PerDeviceOnce {
+    std::atomic<uint64_t> done{0};
+    template <typename F>
+    cudaError_t run(F &&setup) {
+        int dev = 0;
+        cudaError_t e = cudaGetDevice(&dev);
+        if (e != cudaSuccess) return e;
+        const uint64_t bit = dev >= 0 && dev < 64 ? 1ull << dev : 0ull;
+        if (bit && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+        e = setup();
+        if (e == cudaSuccess && bit) done.fetch_or(bit, std::memory_order_release);
+        return e;
+    }
+};
 
 }  // namespace kl

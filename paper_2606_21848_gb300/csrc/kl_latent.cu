@@ -467,12 +467,11 @@ bool matrix_map(CUtensorMap *map, const void *base, uint64_t rows, int cols, int
 constexpr size_t kSmemBytes = sizeof(LatentSmem) + 1024;
 
 template <typename Kernel>
-cudaError_t configure(Kernel kernel, bool &done) {
-    if (done) return cudaSuccess;
-    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kSmemBytes);
-    if (e == cudaSuccess) done = true;
-    return e;
+cudaError_t configure(Kernel kernel, PerDeviceOnce &once) {
+    return once.run([&] {
+        return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)kSmemBytes);
+    });
 }
 
 }  // namespace
@@ -489,8 +488,8 @@ cudaError_t launch_latent_query(int B, int Hq, int G, int D, int r, int wr_per_q
         !matrix_map(&wpmap, w_post, (uint64_t)Hq * kR, D, kR) ||
         !rows_map(&qlmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, q_lat, B, Hq, kR, 32))
         return cudaErrorInvalidValue;
-    static bool configured = false;
-    cudaError_t e = configure(latent_query_kernel, configured);
+    static PerDeviceOnce once;
+    cudaError_t e = configure(latent_query_kernel, once);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(Hq, (B + kBM - 1) / kBM);
@@ -513,8 +512,8 @@ cudaError_t launch_latent_expand(int B, int Hq, int D, int r, const float *o_lat
         !rows_map(&outmap, fp32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
                   fp32 ? 4 : 2, out, B, Hq, D, fp32 ? 32 : 64))
         return cudaErrorInvalidValue;
-    static bool configured = false;
-    cudaError_t e = configure(latent_expand_kernel, configured);
+    static PerDeviceOnce once;
+    cudaError_t e = configure(latent_expand_kernel, once);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(Hq, (B + kBM - 1) / kBM);

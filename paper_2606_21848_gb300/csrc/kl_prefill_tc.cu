@@ -624,13 +624,12 @@ cudaError_t launch_prefill_tc(const PrefillArgs &a) {
         if (!encode(&qmap, a.q, 3, dims, strides, box)) return cudaErrorInvalidValue;
     }
     const size_t smem = sizeof(PrefillSmem) + 1024;
-    static bool configured = false;
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(prefill_tc_kernel,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        configured = true;
-    }
+    static PerDeviceOnce once;
+    const cudaError_t e = once.run([&] {
+        return cudaFuncSetAttribute(prefill_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)smem);
+    });
+    if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(g.Hq, g.B, (a.max_q + kBM - 1) / kBM);
     cfg.blockDim = dim3(kThreads);
