@@ -810,7 +810,8 @@ def sweep_workloads(args, dev, stream, flush_l2, x70, g70, sh70, keyless_ms):
     prefill = {"workload": wl.name, "what": "kl_prefill_attention", "ms": pre_ms,
                "query_tokens_per_s": T / (pre_ms / 1e3), "useful_tflops": tfl,
                "frac_of_bf16_peak": tfl / tpeak, "bf16_peak_tflops": tpeak,
-               "note": "hi + lo bf16 operands issue twice the useful MMA work"}
+               "note": "scores from hi + lo bf16 query operands, output from fp16 weights and "
+                       "values: 1.5x the useful MMA work issued"}
     del g, pout, x
     torch.cuda.empty_cache()
 
@@ -1033,7 +1034,8 @@ def run_prefill(args, wl, x, dev, rank, world):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded; inputs resident in HBM)",
         "config": prefill_config(wl, x, world),
-        "operands": "hi + lo bf16 pairs (2x the attention MMA work)",
+        "operands": "scores: hi + lo bf16 query against the bf16 tile; output: fp16 weights "
+                    "against the tile converted to fp16 (1.5x the attention MMA work)",
         "ms_breakdown": {"append": app_ms, "prefill": pre_ms},
         "tflops": tflops,
         "kernels_per_step": 2,

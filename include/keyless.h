@@ -56,6 +56,8 @@ typedef enum kl_status {
 #define KL_FLAG_BAD_POSITION 0x2 /* append position outside [0, max_pages_per_seq * P) */
 #define KL_FLAG_BAD_LENGTH 0x4   /* seq_len outside [0, max_pages_per_seq * P] */
 #define KL_FLAG_TIMEOUT 0x8      /* a bounded pipeline wait gave up (output invalid) */
+#define KL_FLAG_RANGE 0x10       /* a non-finite output of kl_prefill_attention (a cached value
+                                    beyond its fp16 range, or a non-finite input) */
 
 typedef enum kl_dtype { KL_BF16 = 0, KL_FP32 = 1 } kl_dtype;
 
@@ -238,7 +240,12 @@ kl_status kl_append_v_chunk(const kl_shape *shape, const void *v_new, const int3
  * kl_decode_attention; cu_q_lens: [B + 1] int32 on the device; max_q_len: a host-side bound on
  * every n_b (it sizes the grid; rows past it get no output). head_dim 128 only
  * (KL_ERR_UNSUPPORTED otherwise). Needs no workspace. Flags as in kl_append_v_chunk, and a bad
- * page id leaves the affected outputs unspecified.
+ * page id leaves the affected outputs unspecified. Precision: the scores are formed from the
+ * bf16 cache rows with the routed query carried to about 16 significant bits; the output sum
+ * takes the softmax weights and the cached values in fp16 (exact for bf16 values of magnitude
+ * 2^-14 to 65280, smaller ones to within 2^-25). A cached value of magnitude 65536 or more has
+ * no finite fp16 form: the outputs of the query rows whose 128-token cache tiles hold it come
+ * out non-finite, and any non-finite output raises KL_FLAG_RANGE.
  */
 kl_status kl_prefill_attention(const kl_shape *shape, const void *q, const void *w_r,
                                const void *v_cache, const int32_t *block_table,

@@ -9,7 +9,7 @@ from .builder import build  # noqa: F401
 from ._lib import (  # noqa: F401
     KL_BF16, KL_FP32, KL_KERNEL_AUTO, KL_KERNEL_SIMT, KL_KERNEL_TENSOR, KL_OK,
     KL_ERR_CUDA, KL_ERR_INVALID_ARG, KL_ERR_UNSUPPORTED, KL_ERR_WORKSPACE,
-    KL_FLAG_BAD_LENGTH, KL_FLAG_BAD_PAGE, KL_FLAG_BAD_POSITION, KL_FLAG_TIMEOUT,
+    KL_FLAG_BAD_LENGTH, KL_FLAG_BAD_PAGE, KL_FLAG_BAD_POSITION, KL_FLAG_RANGE, KL_FLAG_TIMEOUT,
     KLError, decode_options, kl_append_v, kl_combine, kl_decode_attention, kl_decode_attention_ex,
     kl_decode_attention_noalloc, kl_decode_kernel_available, kl_decode_step, KL_NOALLOC_SCRATCH_BYTES,
     kl_decode_num_splits, kl_decode_options, kl_decode_workspace_size, kl_route_query,

@@ -16,7 +16,7 @@ from . import builder as _build
 KL_OK, KL_ERR_INVALID_ARG, KL_ERR_UNSUPPORTED, KL_ERR_WORKSPACE, KL_ERR_CUDA = range(5)
 KL_BF16, KL_FP32 = 0, 1
 KL_KERNEL_AUTO, KL_KERNEL_TENSOR, KL_KERNEL_SIMT = 0, 1, 2
-KL_FLAG_BAD_PAGE, KL_FLAG_BAD_POSITION, KL_FLAG_BAD_LENGTH, KL_FLAG_TIMEOUT = 1, 2, 4, 8
+KL_FLAG_BAD_PAGE, KL_FLAG_BAD_POSITION, KL_FLAG_BAD_LENGTH, KL_FLAG_TIMEOUT, KL_FLAG_RANGE = 1, 2, 4, 8, 16
 KL_NOALLOC_SCRATCH_BYTES = 32 * 1024 * 1024
 
 HEADER = os.path.join(_build.INCLUDE, "keyless.h")

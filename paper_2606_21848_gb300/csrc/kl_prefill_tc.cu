@@ -7,27 +7,36 @@
 //
 //   routing  Q_r = Q . W^R[w(h)]                      M = 128 rows, N = 128, K = 128 (Section 2.2)
 //   scores   S   = Q_hi . V_t^T + Q_lo . V_t^T        M = 128 rows, N = 128 tokens, K = 2 x 128
-//   output   O  += P_hi . V_t + P_lo . V_t            M = 128 rows, N = 128 dims,  K = 2 x 128
+//   output   O  += P . V_t                             M = 128 rows, N = 128 dims,  K = 128
 //
 // Each cached tile V_t [128 tokens x 128 dims] arrives once by TMA (one box per page) and feeds
-// both products from the same shared-memory copy: as the K-major B operand of the score MMAs and
-// as the MN-major B operand of the output MMAs. Everything else lives in TMEM (512 columns, 128
-// each): S, the softmax weights P_hi | P_lo, O, and the routed query Q_hi | Q_lo. Q and P enter
-// the MMAs as A operands straight from TMEM, so the only operand the tensor cores read from
-// shared memory is the cache tile. The softmax copies S of tile t into registers and releases
-// it at once, so the score MMAs of tile t + 1 run during the softmax of tile t, and the output
-// MMAs of tile t during the softmax of tile t + 1 (P is rewritten only after they finish).
+// both products from the same shared-memory copy: as the K-major B operand of the score MMAs
+// (bf16, as it landed) and, once the softmax warps have converted it to fp16 in place, as the
+// MN-major B operand of the output MMAs. Everything else lives in TMEM (512 columns, 128 each):
+// two S buffers, O, and the routed query Q_hi | Q_lo. Q and P enter the MMAs as A operands
+// straight from TMEM, so the only operand the tensor cores read from shared memory is the cache
+// tile. Tile t's scores go to buffer t % 2 as soon as the output MMAs of tile t - 2 have read
+// that buffer, so the score MMAs of tile t + 1 run during the softmax of tile t and the softmax
+// of tile t + 1 finds its scores ready; the softmax writes tile t's weights P over the first 64
+// columns of tile t's own buffer, and the output MMAs of tile t run during the softmax of tile
+// t + 1.
 //
-// Precision: the routed query (times scale * log2 e) and the softmax weights are each carried as
-// a pair of bf16 operands, x = hi + lo, which keeps about 16 significant bits where one bf16
-// operand keeps 8. With one bf16 operand each, rows whose softmax mass sits on a few tokens (the
-// first positions of a prompt, peaked scores) miss |err| <= 2e-3 + 1e-2 |ref| by up to 7e-3; the
-// pair costs twice the tensor-core work of a plain bf16 attention.
+// Precision: the routed query (times scale * log2 e) is carried as a pair of bf16 operands,
+// x = hi + lo, about 16 significant bits where one bf16 operand keeps 8; the softmax weights
+// are one fp16 operand (11 bits) against the tile in fp16. A CPU replay of these roundings on
+// the parity cases (peaked rows at the start of a prompt, scores of tens of units, 1 % outlier
+// values x20) puts the worst error at 0.40 of |err| <= 2e-3 + 1e-2 |ref|; with one bf16 operand
+// for the weights it is 1.0-2.5 times the bound, with one fp16 operand for the query 2-5 times.
+// So each tile costs three 128 x 128 x 128 MMAs instead of the four of a pair on both sides.
+// bf16 values convert to fp16 exactly from 2^-14 to 65280 (smaller ones round to fp16's
+// subnormal grid, an absolute error below 2^-25); a cached value of magnitude 65536 or more has
+// no finite fp16 form and makes the outputs of the rows whose tiles hold it non-finite. The
+// epilogue raises KL_FLAG_RANGE for any non-finite output.
 //
 // Softmax (thread = query row = TMEM lane): scores arrive already scaled by scale * log2 e (the
 // routed query is scaled before its bf16 rounding), so p = 2^(s - m). The reference maximum m of
 // a row only moves when the tile maximum exceeds it by more than 8 (a factor 256): then the row's
-// O in TMEM and its running sum l are rescaled; otherwise p may reach 2^8, well inside bf16 and
+// O in TMEM and its running sum l are rescaled; otherwise p may reach 2^8, well inside fp16 and
 // fp32 range, and the final O / l is unchanged because O and l share the same reference.
 //
 // Roles (352 threads, one CTA per SM):
@@ -61,8 +70,9 @@ constexpr int kThreads = 11 * 32;
 constexpr uint32_t kTileBytes = kBN * kD * 2;     // 32 KiB
 constexpr uint32_t kHalfBytes = kTileBytes / 2;   // one 64-column half: 128 rows x 128 B
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColS = 0;                     // S: columns 0 .. 127
-constexpr uint32_t kColP = 128;                   // P_hi: 128 .. 191, P_lo: 192 .. 255
+constexpr uint32_t kColS = 0;                     // S of tile t: 128 t % 2 .. + 127 (then P of
+                                                  // tile t, fp16 pairs, in its first 64); the
+                                                  // routed query first lands in buffer 0
 constexpr uint32_t kColO = 256;                   // O: columns 256 .. 383
 constexpr uint32_t kColQ = 384;                   // Q_hi: 384 .. 447, Q_lo: 448 .. 511
 constexpr uint32_t kLoCols = 64;                  // hi -> lo of a packed bf16 operand
@@ -77,7 +87,7 @@ struct __align__(1024) PrefillSmem {
     // the cache tiles ([64-dim half][128 tokens][128 B]); all 128B-swizzled.
     uint8_t tiles[kStages][kTileBytes];
     uint64_t full[kStages], empty[kStages];
-    uint64_t s_full, s_free, p_full, pv_done;
+    uint64_t s_full[2], s_free[2], p_full, pv_done;
     uint64_t r_full, qr_ready, drain, drain2;
     float red[2][2][kBM];      // per-tile half-row maxima of the two warps of a pair (2 tiles)
     float lsum[2][kBM];        // the two warps' shares of the row sums, for the epilogue
@@ -122,6 +132,57 @@ __device__ __forceinline__ void split2(float x0, float x1, uint32_t &hi, uint32_
     lo = *reinterpret_cast<const uint32_t *>(&l);
 }
 
+// Instruction descriptor of kind::f16 with fp16 A and B (A and B formats 0), fp32 accumulator,
+// operand majorness (0 = K-major, 1 = MN-major), N and M.
+__host__ __device__ constexpr uint32_t idesc_f16(uint32_t M, uint32_t N, bool a_mn, bool b_mn) {
+    return (1u << 4) | ((a_mn ? 1u : 0u) << 15) | ((b_mn ? 1u : 0u) << 16) | ((N >> 3) << 17) |
+           ((M >> 4) << 24);
+}
+
+// max(a, b, c) in one instruction.
+__device__ __forceinline__ float max3(float a, float b, float c) {
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
+// Packed fp32 pair arithmetic (one instruction for two lanes of data).
+__device__ __forceinline__ float2 add2(float2 a, float2 b) {
+    float2 d;
+    asm("{\n\t.reg .b64 x, y, z;\n\t"
+        "mov.b64 x, {%2, %3};\n\tmov.b64 y, {%4, %5};\n\t"
+        "add.rn.f32x2 z, x, y;\n\tmov.b64 {%0, %1}, z;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return d;
+}
+__device__ __forceinline__ float2 sub2(float2 a, float2 b) {
+    float2 d;
+    asm("{\n\t.reg .b64 x, y, z;\n\t"
+        "mov.b64 x, {%2, %3};\n\tmov.b64 y, {%4, %5};\n\t"
+        "sub.rn.f32x2 z, x, y;\n\tmov.b64 {%0, %1}, z;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return d;
+}
+__device__ __forceinline__ float2 mul2(float2 a, float f) {
+    return make_float2(a.x * f, a.y * f);
+}
+
+// Two values as an fp16 pair (a in the low half), round to nearest even.
+__device__ __forceinline__ uint32_t pack_f16(float a, float b) {
+    uint32_t d;
+    asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(b), "f"(a));
+    return d;
+}
+
+__device__ __forceinline__ void ld_shared_v4(uint32_t addr, uint32_t (&v)[4]) {
+    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3])
+                 : "r"(addr)
+                 : "memory");
+}
+
 __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
                                              uint32_t d) {
     asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c),
@@ -162,10 +223,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             ptx::mbar_init(&sm.full[s], 1);
             ptx::mbar_init(&sm.empty[s], 1);
         }
-        // One completion per tile on each. Every wait names the completion it needs: MMAs
-        // that write different TMEM ranges are not assumed to complete in issue order.
-        ptx::mbar_init(&sm.s_full, 1);
-        ptx::mbar_init(&sm.s_free, kComputeWarps);
+        // One completion per tile on p_full and pv_done, one per tile of its buffer on
+        // s_full[b] (scores of tile t in buffer b = t % 2) and s_free[b] (the output MMAs of
+        // tile t have read buffer t % 2). Every wait names the completion it needs: MMAs that
+        // write different TMEM ranges are not assumed to complete in issue order.
+        for (int b2 = 0; b2 < 2; ++b2) {
+            ptx::mbar_init(&sm.s_full[b2], 1);
+            ptx::mbar_init(&sm.s_free[b2], 1);
+        }
         ptx::mbar_init(&sm.p_full, kComputeWarps);
         ptx::mbar_init(&sm.pv_done, 1);
         ptx::mbar_init(&sm.r_full, 1);
@@ -243,9 +308,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ---------------------------------------------------------------- MMA issuers ----
         // K-major SW128 operands step 32 B per 16 columns inside a 64-column half and jump a
         // half (kHalfBytes) every 4 steps; MN-major SW128 operands step 16 rows = 2 KiB; TMEM
-        // A operands step 8 columns (16 packed bf16).
+        // A operands step 8 columns (16 packed 16-bit values).
         constexpr uint32_t idesc_qk = ptx::idesc_bf16(128, 128, false, false);
-        constexpr uint32_t idesc_pv = ptx::idesc_bf16(128, 128, false, true);
+        constexpr uint32_t idesc_route = ptx::idesc_bf16(128, 128, false, true);
+        constexpr uint32_t idesc_pv = idesc_f16(128, 128, false, true);   // (mma_bf16_ts issues
+        // the kind::f16 MMA; this descriptor makes both of its operands fp16)
         const uint64_t q_desc = ptx::smem_desc(ptx::smem_addr(sm.q), 16, 1024, ptx::kSwizzle128B);
         const uint64_t k_desc = ptx::smem_desc(ptx::smem_addr(sm.tiles[0]), 16, 1024, ptx::kSwizzle128B);
         const uint64_t mn_desc =
@@ -263,7 +330,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int kk = 0; kk < kD / 16; ++kk)
                         ptx::mma_bf16(tmem + kColS, q_desc + kstep(kk), mn_desc + ((kk * 2048) >> 4),
-                                      idesc_pv, kk > 0);
+                                      idesc_route, kk > 0);
                     ptx::mma_commit(&sm.empty[0]);
                     ptx::mma_commit(&sm.r_full);
                 }
@@ -271,10 +338,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             ok = ok && wait(&sm.qr_ready, 0);
             for (int i = 0; ok && i < n_tiles; ++i) {
-                const int r = i + 1, s = r % kStages;
+                const int r = i + 1, s = r % kStages, sb = i & 1;
+                // the output MMAs of tile i - 2 have read buffer sb (its P); waited on before
+                // the tile, so that this is the buffer's next completion (the one after it
+                // needs tile i's scores)
+                if (i >= 2 && !wait(&sm.s_free[sb], ((i >> 1) - 1) & 1)) { ok = false; break; }
                 if (!wait(&sm.full[s], (r / kStages) & 1)) { ok = false; break; }
-                // the softmax has copied S of tile i - 1 out of TMEM
-                if (i >= 1 && !wait(&sm.s_free, (i - 1) & 1)) { ok = false; break; }
                 ptx::tc_fence_after();
                 if (lane == 0) {
                     // S = Q_hi . V_i^T + Q_lo . V_i^T: A = Q_r in TMEM, B = the tile
@@ -282,29 +351,30 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const uint64_t b0 = k_desc + ((s * kTileBytes) >> 4);
 #pragma unroll
                     for (int kk = 0; kk < 2 * kD / 16; ++kk)
-                        ptx::mma_bf16_ts(tmem + kColS,
+                        ptx::mma_bf16_ts(tmem + kColS + sb * 128u,
                                          tmem + kColQ + (kk >= 8 ? kLoCols : 0u) + (kk & 7) * 8,
                                          b0 + kstep(kk & 7), idesc_qk, kk > 0);
-                    ptx::mma_commit(&sm.s_full);
+                    ptx::mma_commit(&sm.s_full[sb]);
                 }
                 __syncwarp();
             }
         } else {
-            // the output MMAs of every tile: O += P_hi . V_j + P_lo . V_j; A = P in TMEM,
-            // B = the tile (N = dims, MN-major)
+            // the output MMAs of every tile: O += P . V_j, fp16; A = P in TMEM (the first 64
+            // columns of buffer j % 2), B = the tile (N = dims, MN-major), converted to fp16 by
+            // the softmax warps before they arrive on p_full
             for (int j = 0; j < n_tiles; ++j) {
                 const int s = (j + 1) % kStages;
                 if (!wait(&sm.p_full, j & 1)) { ok = false; break; }
                 ptx::tc_fence_after();
                 if (lane == 0) {
                     const uint64_t b0 = mn_desc + ((s * kTileBytes) >> 4);
-                    const uint32_t pa = tmem + kColP;
+                    const uint32_t pa = tmem + kColS + (j & 1) * 128u;
 #pragma unroll
-                    for (int kk = 0; kk < 2 * kBN / 16; ++kk)
-                        ptx::mma_bf16_ts(tmem + kColO, pa + (kk >= 8 ? kLoCols : 0u) + (kk & 7) * 8,
-                                         b0 + (((kk & 7) * 2048) >> 4), idesc_pv,
+                    for (int kk = 0; kk < kBN / 16; ++kk)
+                        ptx::mma_bf16_ts(tmem + kColO, pa + kk * 8, b0 + ((kk * 2048) >> 4), idesc_pv,
                                          (j > 0 || kk > 0) ? 1u : 0u);
                     ptx::mma_commit(&sm.empty[s]);
+                    ptx::mma_commit(&sm.s_free[j & 1]);
                     ptx::mma_commit(&sm.pv_done);
                 }
                 __syncwarp();
@@ -360,21 +430,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
 
         float m_ref = -INFINITY;   // reference maximum of the row (base 2), shared by the pair
-        float l = 0.f;             // this warp's share of sum 2^(s - m_ref)
+        // this warp's share of sum 2^(s - m_ref), in two packed pairs of partial sums
+        float2 la = make_float2(0.f, 0.f), lb = make_float2(0.f, 0.f);
         // Both warps of a pair run the same tiles and meet on exactly one pair barrier per
         // tile and one in the epilogue; a wait that fails only turns this warp's vote false, and
         // the pair leaves together at the next barrier.
         bool okl = ok;
         for (int i = 0; i < n_tiles; ++i) {
             const int t0 = i * kBN, rb = i & 1;
-            if (okl) okl = wait(&sm.s_full, i & 1);
+            const uint32_t sbuf = tmem + kColS + (uint32_t)rb * 128u;   // S, then P, of tile i
+            if (okl) okl = wait(&sm.s_full[rb], (i >> 1) & 1);
             float sv[64];
             float mp = -INFINITY;
             if (okl) {
                 ptx::tc_fence_after();
                 uint32_t u0[32], u1[32];
-                ptx::tmem_ld32(tmem + kColS + c0 + lane_base, u0);
-                ptx::tmem_ld32(tmem + kColS + c0 + 32 + lane_base, u1);
+                ptx::tmem_ld32(sbuf + c0 + lane_base, u0);
+                ptx::tmem_ld32(sbuf + c0 + 32 + lane_base, u1);
                 ptx::tmem_wait_ld();
                 ptx::reg_fence(u0);
                 ptx::reg_fence(u1);
@@ -383,10 +455,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                     sv[c] = __uint_as_float(u0[c]);
                     sv[32 + c] = __uint_as_float(u1[c]);
                 }
-                // S is in registers: the score MMAs of the next tile may overwrite it
-                ptx::tc_fence_before();
-                __syncwarp();
-                if (lane == 0) ptx::mbar_arrive(&sm.s_free);
                 // causal mask: token t0 + c0 + c is visible to the row when it is <= pos_r
                 if (t0 + c0 + 63 > pos0) {
                     const int lim = pos_r - t0 - c0;
@@ -396,16 +464,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-                for (int c = 0; c < 64; c += 4) {
-                    mx[0] = fmaxf(mx[0], sv[c]);
-                    mx[1] = fmaxf(mx[1], sv[c + 1]);
-                    mx[2] = fmaxf(mx[2], sv[c + 2]);
-                    mx[3] = fmaxf(mx[3], sv[c + 3]);
+                for (int c = 0; c < 64; c += 8) {
+                    mx[0] = max3(mx[0], sv[c], sv[c + 1]);
+                    mx[1] = max3(mx[1], sv[c + 2], sv[c + 3]);
+                    mx[2] = max3(mx[2], sv[c + 4], sv[c + 5]);
+                    mx[3] = max3(mx[3], sv[c + 6], sv[c + 7]);
                 }
-                mp = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+                mp = max3(mx[0], mx[1], fmaxf(mx[2], mx[3]));
                 sm.red[rb][hf][r] = mp;
             }
-            // the pair exchanges its half maxima (and leaves together on any failed wait)
+            // the pair exchanges its half maxima (and leaves together on any failed wait); past
+            // this barrier both warps hold their S in registers, so P may overwrite the buffer
             if (!ptx::bar_and(pair_bar, 64, okl)) {
                 okl = false;
                 break;
@@ -435,37 +504,53 @@ __global__ void __launch_bounds__(kThreads, 1)
                         ptx::tmem_wait_st();
                     }
                 }
-                l *= f;
+                la = mul2(la, f);
+                lb = mul2(lb, f);
                 m_ref = m_new;
             }
             const float mr = m_ref == -INFINITY ? 0.f : m_ref;
 
-            // this warp's 64 weights -> 32 packed columns of P_hi and of P_lo: computed in
-            // registers first, stored once the output MMAs of tile i - 1 have read the previous P
-            uint32_t ph[32], pl[32];
-            float ls[4] = {0.f, 0.f, 0.f, 0.f};
+            // this warp's 64 weights -> 32 packed fp16 columns of P (in pairs: s - m, 2^x, the
+            // running sums, the fp16 pack)
+            uint32_t ph[32];
 #pragma unroll
             for (int e = 0; e < 32; ++e) {
-                const float a0 = ptx::ex2(sv[2 * e] - mr), a1 = ptx::ex2(sv[2 * e + 1] - mr);
-                ls[(2 * e) & 3] += a0;
-                ls[(2 * e + 1) & 3] += a1;
-                split2(a0, a1, ph[e], pl[e]);
+                const float2 d = sub2(make_float2(sv[2 * e], sv[2 * e + 1]), make_float2(mr, mr));
+                const float2 pe = make_float2(ptx::ex2(d.x), ptx::ex2(d.y));
+                if (e & 1) lb = add2(lb, pe); else la = add2(la, pe);
+                ph[e] = pack_f16(pe.x, pe.y);
             }
-            l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
-            if (okl && i >= 1) okl = wait(&sm.pv_done, (i - 1) & 1);
+            // The score MMAs are done with tile i: this thread converts its cache row r,
+            // dims 64 hf .. + 63 (128 contiguous bytes whatever the swizzle), to fp16 in place
+            // for the output MMAs. Rows at or past the sequence's end (an unwritten page
+            // tail, or a page slot no TMA filled) become zeros instead, so that 0-weights
+            // never meet a non-finite value. The lanes start at different 16-byte chunks so
+            // that a warp's accesses spread over all banks.
             if (okl) {
-                ptx::tmem_st32(tmem + kColP + c0 / 2 + lane_base, ph);
-                ptx::tmem_st32(tmem + kColP + kLoCols + c0 / 2 + lane_base, pl);
-                ptx::tmem_wait_st();
-                // cache rows at or past the sequence's end (an unwritten page tail, or a page
-                // slot no TMA filled) become zeros, so that 0-weights never meet a non-finite
-                // value; each warp of the pair clears its own 64-dim half of the row
-                if (t0 + kBN > L && t0 + r >= L) {
-                    const uint32_t v_s = ptx::smem_addr(sm.tiles[(i + 1) % kStages]) +
-                                         hf * kHalfBytes + r * 128;
+                const uint32_t v_s = ptx::smem_addr(sm.tiles[(i + 1) % kStages]) +
+                                     hf * kHalfBytes + r * 128;
+                if (t0 + r < L) {
+#pragma unroll 4
+                    for (int c = 0; c < 8; ++c) {
+                        const uint32_t addr = v_s + ((c + lane) & 7) * 16;
+                        uint32_t w[4];
+                        ld_shared_v4(addr, w);
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            w[e] = pack_f16(__uint_as_float(w[e] << 16),
+                                            __uint_as_float(w[e] & 0xffff0000u));
+                        }
+                        st_shared_v4(addr, w[0], w[1], w[2], w[3]);
+                    }
+                } else {
 #pragma unroll
                     for (int c = 0; c < 8; ++c) st_shared_v4(v_s + c * 16, 0u, 0u, 0u, 0u);
                 }
+                // P over the first 64 columns of the buffer (the output MMAs of tile i - 2, the
+                // last reader of P there, finished before tile i's scores were written)
+                ptx::tmem_st32(sbuf + c0 / 2 + lane_base, ph);
+                ptx::tmem_wait_st();
+                // the converted tile (generic-proxy stores) is read next by the output MMAs
                 ptx::tc_fence_before();
                 ptx::fence_proxy_async_smem();
                 __syncwarp();
@@ -475,13 +560,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             // false at the next pair barrier (or the epilogue's), where the pair leaves together
         }
 
-        // Epilogue: out = O / l, this warp's 64 output dims; l is the pair's two shares.
+        // Epilogue: out = O / l, this warp's 64 output dims; l is the pair's two shares. A
+        // non-finite output (a cached value beyond fp16's range, or a non-finite input) raises
+        // KL_FLAG_RANGE.
+        const float l = (la.x + la.y) + (lb.x + lb.y);
         const bool oke = okl && wait(&sm.pv_done, (n_tiles - 1) & 1);
         sm.lsum[hf][r] = l;
         if (ptx::bar_and(pair_bar, 64, oke)) {
             ptx::tc_fence_after();
             const float lt = l + sm.lsum[hf ^ 1][r];
             const float inv = lt > 0.f ? 1.f / lt : 0.f;
+            float nf = 0.f;   // x * 0 is NaN exactly when x is not finite
             const size_t orow = ((size_t)(q0 + m0 + r) * geo.Hq + h) * kD + c0;
 #pragma unroll
             for (int c4 = 0; c4 < 2; ++c4) {
@@ -490,6 +579,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ptx::tmem_wait_ld();
                 ptx::reg_fence(u);
                 if (r < rows) {
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) nf = fmaf(__uint_as_float(u[e]), 0.f, nf);
                     if (a.out_dtype == KL_FP32) {
                         float4 *o = reinterpret_cast<float4 *>(static_cast<float *>(a.out) + orow + c4 * 32);
 #pragma unroll
@@ -510,6 +601,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
             }
+            if (__any_sync(0xffffffffu, nf != nf) && lane == 0) raise_flag(a.err, KL_FLAG_RANGE);
         }
     }
 

@@ -201,6 +201,38 @@ def test_bad_lengths_and_pages_raise_flags():
     assert err & kl.KL_FLAG_BAD_PAGE
 
 
+def test_outlier_values():
+    """1 % of the cached entries scaled x20 (the ragged serving recipe): the case where the fp16
+    weights of the output sum come closest to the bound."""
+    x = tiny_prefill(B=2, Hq=8, Hkv=2, D=128, P=16, lens=(700, 260), q_lens=(300, 260), seed=36)
+    v = x["v_cache"].float()
+    mask = torch.rand(v.shape, generator=torch.Generator().manual_seed(9)) < 0.01
+    x["v_cache"] = torch.where(mask, v * 20, v).to(torch.bfloat16)
+    got, err = run_prefill(x)
+    assert err == 0
+    assert_parity(got.cpu().numpy(), oracle_prefill(x, 1.0 / math.sqrt(128)), "outliers")
+
+
+def test_values_at_the_edge_of_fp16_and_beyond():
+    """The output sum carries the cached values in fp16: the largest bf16 value it holds (65280)
+    gives the oracle's answer, and a larger finite one (69632) makes outputs non-finite, which
+    raises KL_FLAG_RANGE."""
+    x = tiny_prefill(B=2, Hq=8, Hkv=2, D=128, P=16, lens=(300, 140), q_lens=(300, 140), seed=43)
+    page = int(x["block_table"][0, 2])
+    y = dict(x)
+    y["v_cache"] = x["v_cache"].clone()
+    y["v_cache"][page, 1, 5, 17] = -65280.0
+    y["v_cache"][page, 0, 9, 100] = 65280.0
+    got, err = run_prefill(y)
+    assert err == 0
+    assert_parity(got.cpu().numpy(), oracle_prefill(y, 1.0 / math.sqrt(128)), "65280")
+    z = dict(x)
+    z["v_cache"] = x["v_cache"].clone()
+    z["v_cache"][page, 0, 9, 100] = 69632.0
+    _, err = run_prefill(z)
+    assert err & kl.KL_FLAG_RANGE
+
+
 def test_head_dim_64_is_unsupported():
     x = tiny_prefill(B=1, Hq=4, Hkv=4, D=64, P=16, lens=(32,), q_lens=(32,), seed=42)
     with pytest.raises(kl.KLError) as e:
