@@ -197,6 +197,34 @@ __device__ __forceinline__ float e4m3_round(float x) {
     return __fsub_rn(__fadd_rn(hv, 24576.f), 24576.f);
 }
 
+// Packed fp32 pairs: one instruction applies the same IEEE round-to-nearest operation to both
+// lanes, so each lane's result is bit for bit that of the scalar operation.
+struct F2 {
+    float x, y;
+};
+__device__ __forceinline__ F2 f2(float a, float b) { return F2{a, b}; }
+#define KL_F2_OP(name, op)                                                                      \
+    __device__ __forceinline__ F2 name(F2 a, F2 b) {                                           \
+        F2 d;                                                                                  \
+        asm("{\n\t.reg .b64 x, y, z;\n\tmov.b64 x, {%2, %3};\n\tmov.b64 y, {%4, %5};\n\t" op \
+            " z, x, y;\n\tmov.b64 {%0, %1}, z;\n\t}"                                            \
+            : "=f"(d.x), "=f"(d.y)                                                             \
+            : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));                                         \
+        return d;                                                                              \
+    }
+KL_F2_OP(add2, "add.rn.f32x2")
+KL_F2_OP(sub2, "sub.rn.f32x2")
+KL_F2_OP(mul2, "mul.rn.f32x2")
+#undef KL_F2_OP
+__device__ __forceinline__ F2 fma2(F2 a, F2 b, F2 c) {
+    F2 d;
+    asm("{\n\t.reg .b64 x, y, z, w;\n\tmov.b64 x, {%2, %3};\n\tmov.b64 y, {%4, %5};\n\t"
+        "mov.b64 z, {%6, %7};\n\tfma.rn.f32x2 w, x, y, z;\n\tmov.b64 {%0, %1}, w;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+    return d;
+}
+
 // Byte offset of element (row n, column k) of the query-term operand: [NS rows][128 B],
 // K-major, 128B-swizzled (8-row atoms of 1 KiB, 16-byte chunk index XOR row % 8).
 __device__ __forceinline__ uint32_t qt_offset(int n, int k) {
@@ -678,12 +706,16 @@ __global__ void __launch_bounds__(kThreads, 2)
             if (nvalid < kTile && !valid) st = 0.f;       // (stale bytes past the end)
             float s_k[KHH];
 #pragma unroll
-            for (int k = 0; k < KHH; ++k) {
-                // sum of the term columns, 16^-j D_j, from the last term
-                const float d = fmaf(fmaf(fmaf(sv[3 * KHH + k], 1.f / 16.f, sv[2 * KHH + k]), 1.f / 16.f,
-                                          sv[KHH + k]),
-                                     1.f / 16.f, sv[k]);
-                s_k[k] = (kAllLive || KHH * hh + k < G) ? d * (invq[k] * st) : -INFINITY;
+            for (int k = 0; k < KHH; k += 2) {
+                // sum of the term columns, 16^-j D_j, from the last term (two heads at once)
+                const F2 s16 = f2(1.f / 16.f, 1.f / 16.f);
+                const F2 d = fma2(fma2(fma2(f2(sv[3 * KHH + k], sv[3 * KHH + k + 1]), s16,
+                                            f2(sv[2 * KHH + k], sv[2 * KHH + k + 1])),
+                                       s16, f2(sv[KHH + k], sv[KHH + k + 1])),
+                                  s16, f2(sv[k], sv[k + 1]));
+                const F2 sk = mul2(d, mul2(f2(invq[k], invq[k + 1]), f2(st, st)));
+                s_k[k] = (kAllLive || KHH * hh + k < G) ? sk.x : -INFINITY;
+                s_k[k + 1] = (kAllLive || KHH * hh + k + 1 < G) ? sk.y : -INFINITY;
             }
             if (nvalid < kTile && !valid) {
 #pragma unroll
@@ -692,7 +724,11 @@ __global__ void __launch_bounds__(kThreads, 2)
             // the weights against the current references; a weight past kLazyW moves them
             float p_k[KHH];
 #pragma unroll
-            for (int k = 0; k < KHH; ++k) p_k[k] = ptx::ex2(s_k[k] - m[k]);   // 0 for padded heads
+            for (int k = 0; k < KHH; k += 2) {   // 0 for padded heads
+                const F2 e = sub2(f2(s_k[k], s_k[k + 1]), f2(m[k], m[k + 1]));
+                p_k[k] = ptx::ex2(e.x);
+                p_k[k + 1] = ptx::ex2(e.y);
+            }
             float pmax = p_k[0];
 #pragma unroll
             for (int k = 1; k < KHH; ++k) pmax = fmaxf(pmax, p_k[k]);
@@ -769,12 +805,14 @@ __global__ void __launch_bounds__(kThreads, 2)
                 }
             }
             const float sts = st * sc;
-            float x[KHH];
+            F2 x[KHH / 2];
 #pragma unroll
-            for (int k = 0; k < KHH; ++k) {
-                const float p = p_k[k];
-                lsum[k] += p;
-                x[k] = p * sts;
+            for (int e = 0; e < KHH / 2; ++e) {
+                const F2 p = f2(p_k[2 * e], p_k[2 * e + 1]);
+                const F2 l = add2(f2(lsum[2 * e], lsum[2 * e + 1]), p);
+                lsum[2 * e] = l.x;
+                lsum[2 * e + 1] = l.y;
+                x[e] = mul2(p, f2(sts, sts));
             }
             // W row of token t: 3 E4M3 terms of this warp's KHH heads (4 KHH bytes, zero
             // padded). Each term but the last is the value rounded to E4M3; the exact residual
@@ -785,14 +823,14 @@ __global__ void __launch_bounds__(kThreads, 2)
                 uint32_t c2[KHH / 2];
 #pragma unroll
                 for (int e = 0; e < KHH / 2; ++e) {
-                    float v0 = x[2 * e], v1 = x[2 * e + 1];
+                    F2 v = x[e];
                     if (j + 1 < kJp) {
-                        v0 = e4m3_round(v0);
-                        v1 = e4m3_round(v1);
-                        x[2 * e] = (x[2 * e] - v0) * 16.f;
-                        x[2 * e + 1] = (x[2 * e + 1] - v1) * 16.f;
+                        // (scalar: the compiler may simplify c - (c - x) and (h + k) - k when
+                        // they are written with packed operations, which breaks the rounding)
+                        v = f2(e4m3_round(v.x), e4m3_round(v.y));
+                        x[e] = mul2(sub2(x[e], v), f2(16.f, 16.f));   // exact
                     }
-                    c2[e] = (uint32_t)__nv_cvt_float2_to_fp8x2(make_float2(v0, v1), __NV_SATFINITE,
+                    c2[e] = (uint32_t)__nv_cvt_float2_to_fp8x2(make_float2(v.x, v.y), __NV_SATFINITE,
                                                                 __NV_E4M3);
                 }
                 if constexpr (KHH == 4) w[j] = c2[0] | (c2[1] << 16);
