@@ -139,7 +139,7 @@ __host__ __device__ constexpr uint32_t idesc_f16(uint32_t M, uint32_t N, bool a_
            ((M >> 4) << 24);
 }
 
-// max(a, b, c) in one instruction.
+// max(a, b, c): the three-operand PTX max.
 __device__ __forceinline__ float max3(float a, float b, float c) {
     float d;
     asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
