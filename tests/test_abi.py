@@ -23,6 +23,21 @@ def test_every_declared_symbol_is_exported():
     assert not missing, missing
 
 
+def test_header_constants_match_the_binding():
+    """Every KL_* value the header defines (flags, statuses, dtypes, kernel choices) has the same
+    value in the Python binding, so a flag added to one side cannot drift from the other."""
+    import re
+    text = open(_lib.HEADER).read()
+    defined = {m.group(1): int(m.group(2), 0)
+               for m in re.finditer(r"#define\s+(KL_FLAG_\w+)\s+(0x[0-9a-fA-F]+|\d+)", text)}
+    for body in re.findall(r"typedef enum\s+\w*\s*\{(.*?)\}", text, re.S):
+        for m in re.finditer(r"(KL_\w+)\s*=\s*(\d+)", body):
+            defined[m.group(1)] = int(m.group(2))
+    assert {"KL_FLAG_RANGE", "KL_FLAG_TIMEOUT", "KL_ERR_CUDA", "KL_FP32"} <= set(defined)
+    wrong = {k: (v, getattr(_lib, k, None)) for k, v in defined.items() if getattr(_lib, k, None) != v}
+    assert not wrong, wrong
+
+
 def test_status_strings():
     assert kl.kl_status_string(kl.KL_OK) == "ok"
     assert "workspace" in kl.kl_status_string(kl.KL_ERR_WORKSPACE)
